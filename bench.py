@@ -1,0 +1,368 @@
+#!/usr/bin/env python3
+"""Benchmark of the SubZero+ weight path on GB300: ZO steps/s and weight-pass HBM GB/s.
+
+Default workload: the LLaMA-7B-shaped parameter set (224 bf16 matrices, 6.48 G
+parameters, r = 32, q = 4 queries, central differences -> 8 weight passes per
+step, subspace refresh every 25 steps).  One "step" is Alg. 3's iteration for
+every matrix: the 2q-1 perturbation passes, the subspace-Adam update fused with
+the last restore, and (when t mod F == 0) the batched QR refresh.  The losses
+the forward passes would produce are synthetic (2.0 + 0.01 N(0,1)); the weights
+are N(0, 0.02^2) bf16.  25.9 GB of weights per pass is far larger than the
+129 MB L2, so every pass streams from HBM.
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl reference] [--workload NAME]
+
+Prints ONE JSON line (rank 0).  For N > 1 launch with torch.distributed.run:
+each rank runs its own layer partition (matrix indices rank*n .. rank*n+n-1 of an
+N-times larger set) with no data-path collective; NCCL is used only for the
+barrier and the max over ranks of the timed region.
+"""
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "ZO weight-pass HBM GB/s (% of peak) and ZO steps/s at 7B shape, 1 GB300"
+FALLBACK_HBM_GBS = 6800.0
+
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of the weight-pass kernel,
+# from the ncu capture summarised under profiles/, keyed by the sha256 of the kernel
+# source it was taken on (reported as null once the source differs).
+TRAFFIC_BY_SOURCE = {}
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=25)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="llama7b_bf16_r32")
+    p.add_argument("--scheme", choices=["central", "forward"], default="central")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    return p.parse_args()
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for name in ("zo_wpass_fma.cu", "zo_wpass_tc.cu"):
+        path = os.path.join(ROOT, "paper_2608_15665_gb300", "csrc", name)
+        if os.path.exists(path):
+            h.update(open(path, "rb").read())
+    return h.hexdigest()[:16]
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="zo_clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for nm, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(nm)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------- oracle timing
+def oracle_sample_step_seconds(wl, scheme, sample=((0, 1024),), seed_shift=0):
+    """Time the fp64 oracle, as it stands, on a bounded sample of one step: for each
+    (matrix, n_rows) in ``sample``, the refresh of that matrix (Alg. 1 on its full m x r
+    and n x r panels) and every weight pass of the step (perturbations, estimator,
+    Adam, fused update) on n_rows of its rows (rows of W update independently).
+    Returns (step_seconds, refresh_seconds, sample_text) extrapolated to the workload:
+    passes by weight count, refresh by panel rows m + n."""
+    import numpy as np
+    import torch
+    from oracle import subzero
+    from paper_2608_15665_gb300 import workloads
+    t_pass = t_ref = 0.0
+    el_sample = uv_sample = 0
+    seed = wl.seed + seed_shift
+    for i, n_rows in sample:
+        m, n = wl.shapes[i]
+        rows = np.arange(min(n_rows, m))
+        W0 = workloads.init_weight(wl, i, "cpu")[: rows.size].to(torch.float64).numpy()
+        st = subzero.MatrixState(W0, wl.dtype, wl.r)
+        st.m = m                                   # the panels keep the matrix's full shape
+        t0 = time.perf_counter()
+        subzero.refresh(st, seed, i, 0, reset_moments=True)
+        t_ref += time.perf_counter() - t0
+        losses = workloads.loss_table(wl, scheme, steps=1)[0]
+        passes, restore = subzero.pass_plan(scheme, wl.q)
+        t0 = time.perf_counter()
+        for terms in passes:
+            C = subzero.perturb_coeff(seed, i, 0, wl.r, terms, wl.eps)
+            st.W = subzero.apply_pass(st.W, wl.dtype, st.U, st.V, C, rows=rows)
+        rho = subzero.rho_from_losses(losses, scheme, wl.eps, wl.q)
+        G = subzero.grad_G(seed, i, 0, wl.r, rho)
+        st.M, st.Vm, D, _, _ = subzero.adam(st.M, st.Vm, G, wl.beta1, wl.beta2, wl.eps_adam, 1)
+        C = subzero.step_coeff(D, wl.lr, wl.eps, restore, seed, i, 0, wl.r)
+        st.W = subzero.apply_pass(st.W, wl.dtype, st.U, st.V, C, rows=rows)
+        t_pass += time.perf_counter() - t0
+        el_sample += rows.size * n
+        uv_sample += m + n
+    step_s = t_pass * wl.params / el_sample
+    refresh_s = t_ref * sum(m + n for m, n in wl.shapes) / uv_sample
+    text = ("fp64 oracle, one step: all weight passes + estimator + Adam on "
+            + ", ".join(f"{r} rows of matrix {i} {wl.shapes[i][0]}x{wl.shapes[i][1]}" for i, r in sample)
+            + f" ({el_sample} of {wl.params} weights) and the refresh of those matrices; "
+            f"extrapolated by weight count (refresh by m+n, amortized over F={wl.F})")
+    return step_s, refresh_s, text
+
+
+def oracle_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [d.get("num_threads", 1) for d in threadpool_info() if d.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+def cpu_baseline(wl, scheme):
+    step_s, refresh_s, text = oracle_sample_step_seconds(wl, scheme, sample=((0, 1024), (4, 1024)))
+    per_step = step_s + refresh_s / wl.F
+    return {"value": 1.0 / per_step, "unit": "ZO steps/s", "cores": oracle_threads(),
+            "kind": "oracle", "sample": text}
+
+
+# --------------------------------------------------------------------------- reference arm
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2608_15665_gb300 import workloads
+    wl = workloads.get(args.workload)
+    times = []
+    for s in range(args.warmup + args.steps):
+        step_s, refresh_s, text = oracle_sample_step_seconds(wl, args.scheme, sample=((0, 512),),
+                                                             seed_shift=s)
+        if s >= args.warmup:
+            times.append(step_s + refresh_s / wl.F)
+    per_step = sum(times) / len(times)
+    value = 1.0 / per_step
+    passes = 2 * wl.q if args.scheme == "central" else wl.q + 1
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "ZO steps/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": per_step * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "matrices": wl.n_mats, "params": wl.params, "r": wl.r,
+                   "q": wl.q, "scheme": args.scheme, "passes_per_step": passes,
+                   "refresh_every": wl.F},
+        "cpu_baseline": {"value": value, "unit": "ZO steps/s", "cores": oracle_threads(),
+                         "kind": "oracle", "sample": text},
+        "e2e": {"value": value, "unit": "ZO steps/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------- our arm
+def run_ours(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl")
+
+    from paper_2608_15665_gb300 import build
+    build.build()
+    from paper_2608_15665_gb300 import binding as zb
+    from paper_2608_15665_gb300 import workloads
+    from paper_2608_15665_gb300.schedule import SubZeroPlus, step_plan
+
+    wl0 = workloads.get(args.workload)
+    wl = workloads.scaled(wl0, seed=wl0.seed + 7919 * rank) if rank else wl0
+    weights = [workloads.init_weight(wl, i, dev) for i in range(wl.n_mats)]
+    z = SubZeroPlus(weights, wl.r, wl.q, wl.seed, matrix_index_base=rank * wl.n_mats)
+    calls, (rq, rc) = step_plan(args.scheme, wl.q)
+    passes = len(calls) + 1
+    K, W = args.steps, args.warmup
+    table = workloads.loss_table(wl, args.scheme, steps=W + 2 * K)
+    table_dev = torch.from_numpy(table).to(dev)
+
+    def do_step(t, losses, gamma=None):
+        if t % wl.F == 0:
+            z.refresh(t // wl.F, reset_moments=(t == 0))
+        for (qa, ca), second in calls:
+            qb, cb = second if second is not None else (-1, 0.0)
+            z.perturb(t, qa, ca, qb, cb, wl.eps)
+        z.step(t, t + 1, losses, args.scheme, wl.eps, wl.lr, wl.beta1, wl.beta2, wl.eps_adam,
+               rq, rc, gamma_out=gamma)
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    for t in range(W):
+        do_step(t, table_dev[t])
+    barrier()
+    z.sync()
+
+    # ---- device-timed region: inputs resident in HBM ---------------------------------
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_TIMING, 1)
+    launches0 = zb.zo_kernel_launches(z.ctx)
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record()
+    for t in range(W, W + K):
+        do_step(t, table_dev[t])
+    ev1.record()
+    barrier()
+    clk = clocks.stop()
+    elapsed_ms = max_over_ranks(ev0.elapsed_time(ev1))
+    wpass_ms, wpass_n = zb.zo_get_timing(z.ctx)
+    launches = zb.zo_kernel_launches(z.ctx) - launches0
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_TIMING, 0)
+    path = zb.zo_wpass_path(z.ctx)
+    z.sync()
+
+    # ---- end to end through the public API with host buffers -------------------------
+    e2e = None
+    if not args.no_e2e:
+        host_losses = torch.from_numpy(table[W + K:W + 2 * K].copy()).pin_memory()
+        gamma = torch.zeros(wl.n_mats, dtype=torch.float32, device=dev)
+        gamma_host = torch.zeros(wl.n_mats, dtype=torch.float32).pin_memory()
+        barrier()
+        t0 = time.perf_counter()
+        for k, t in enumerate(range(W + K, W + 2 * K)):
+            do_step(t, host_losses[k].numpy(), gamma)
+            gamma_host.copy_(gamma)            # the step's result back on the host (syncs)
+        barrier()
+        e2e_s = max_over_ranks(time.perf_counter() - t0)
+        e2e = {"value": world * K / e2e_s, "unit": "ZO steps/s",
+               "h2d_bytes_per_step": int(table.shape[1] * 4),
+               "d2h_bytes_per_step": int(wl.n_mats * 4)}
+    z.sync()
+
+    value = world * K / (elapsed_ms / 1e3)
+    bytes_pass = wl.bytes_per_pass()
+    peak, peak_kind = measured_peaks()
+    avg_launch_s = (wpass_ms / wpass_n) / 1e3 if wpass_n else float("nan")
+    achieved = bytes_pass / avg_launch_s / 1e9
+    src = kernel_source_hash()
+    line = {
+        "metric": METRIC, "value": value, "unit": "ZO steps/s", "n_gpus": world, "steps": K,
+        "warmup": W, "ms_per_step": elapsed_ms / K, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": wl0.name, "matrices": wl.n_mats, "params": wl.params,
+                   "weights": "bf16 N(0,0.02^2)" if wl.dtype == "bf16" else "f32 N(0,0.02^2)",
+                   "r": wl.r, "q": wl.q, "scheme": args.scheme, "passes_per_step": passes,
+                   "refresh_every": wl.F, "refreshes_in_timed_region":
+                       sum(1 for t in range(W, W + K) if t % wl.F == 0),
+                   "l2": "inputs larger than L2 (%.1f GB of weights per pass)" % (bytes_pass / 2e9),
+                   "parallelism": f"layer partition x{world}" if world > 1 else "single GPU"},
+        "weight_pass_gbs": passes * bytes_pass * K / (elapsed_ms / 1e3) / 1e9,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "peak_kind": peak_kind,
+                     "traffic": TRAFFIC_BY_SOURCE.get(src),
+                     "kernel": "wpass_fma" if path == 1 else "wpass_tc",
+                     "algorithmic_bytes_per_launch": bytes_pass,
+                     "avg_launch_ms": avg_launch_s * 1e3, "launches_timed": wpass_n},
+        "clocks": clk,
+        "gpu_launches": int(launches),
+    }
+    if e2e:
+        line["e2e"] = e2e
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl0, args.scheme)
+    z.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

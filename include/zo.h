@@ -1,0 +1,215 @@
+/*
+ * zo.h -- C ABI of the SubZero+ subspace zeroth-order weight path on GB300 (sm_103a).
+ *
+ * SubZero+ (arXiv 2608.15665) fine-tunes every trainable matrix W_i (m_i x n_i)
+ * of a model with perturbations confined to a per-matrix subspace:
+ *   W_i <- W_i + eps * U_i Z_i V_i^T                      (Sec. 4.1, Eq. (4); Alg. 2)
+ * where U_i (m_i x r) and V_i (n_i x r) are Haar-distributed column-orthonormal
+ * bases refreshed every F steps (Sec. 4.3, Eq. (11); Alg. 1) and Z_i is an r x r
+ * Gaussian regenerated from a seed (App. A.1).  The q query losses give
+ *   Zbar_i = (1/q) sum_k rho_k Z_i^(k)                    (Eq. (6); Alg. 3)
+ * which drives an Adam optimizer on r x r moments       (Sec. 4.2, Eqs. (7)-(10))
+ * whose update W_i <- W_i - eta U_i D_i V_i^T is applied in the same pass as the
+ * restore of the last query.  The forward passes that produce the losses are the
+ * caller's; the losses enter this ABI as fp32 arrays.
+ *
+ * Conventions for every entry point
+ * ---------------------------------
+ * - All tensors (W, U, V, M, Vm, losses, gamma) are CALLER-OWNED device memory
+ *   unless an argument says "host".  The library allocates only its context:
+ *   a device copy of the matrix table, per-call coefficient/projection buffers
+ *   (O(sum_i r*(r + m_i + n_i)) floats) and the refresh workspace.  All are freed
+ *   by zo_destroy.
+ * - Every call is asynchronous on the stream given to zo_create (a cudaStream_t
+ *   passed as void*; NULL = legacy default stream).  Arguments are validated on the
+ *   host before anything is launched; a rejected call launches nothing and
+ *   leaves all buffers untouched.
+ * - Kernels that detect a problem at run time (an mbarrier wait that ran out of
+ *   iterations, an internal bound check) write a code to a device status word;
+ *   zo_sync_status() synchronises the stream and returns and clears it.
+ * - There is no CPU fallback: without a usable sm_103 device zo_create fails with
+ *   ZO_ERR_CUDA.
+ * - Layouts are row-major.  W_i has leading dimension ldw >= n (in elements);
+ *   U_i is m x r and V_i is n x r, both contiguous fp32; M_i and Vm_i are r x r
+ *   contiguous fp32.
+ * - Random numbers follow one counter-based contract shared by nothing but its
+ *   definition: Philox4x32-10 (Salmon et al., SC'11), key = (seed lo, seed hi),
+ *   counter = (e / 4, matrix index, t or refresh index j, tag << 24 | query k),
+ *   lane e % 4 for element e of a row-major buffer; u = ((x >> 8) + 1) * 2^-24;
+ *   Box-Muller on lane pairs (0,1), (2,3): z_a = sqrt(-2 ln u_a) cos(2 pi u_b),
+ *   z_b = sqrt(-2 ln u_a) sin(2 pi u_b).  Tags: 1 = Z, 2 = Omega_U, 3 = Omega_V.
+ */
+#ifndef SUBZERO_GB300_ZO_H
+#define SUBZERO_GB300_ZO_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define ZO_API __attribute__((visibility("default")))
+#else
+#define ZO_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum zo_status {
+  ZO_OK = 0,
+  ZO_ERR_INVALID_ARG = 1,   /* null pointer, bad enum, negative size, bad scalar */
+  ZO_ERR_SHAPE = 2,         /* r > min(m, n), r unsupported, ldw < n, sizes too large */
+  ZO_ERR_ALIGN = 3,         /* a buffer is not 16-byte aligned */
+  ZO_ERR_DTYPE = 4,         /* unknown weight dtype */
+  ZO_ERR_CUDA = 5,          /* a CUDA runtime call failed (message: zo_last_error) */
+  ZO_ERR_TIMEOUT = 6,       /* a bounded device-side wait ran out (zo_sync_status) */
+  ZO_ERR_UNSUPPORTED = 7,   /* valid request this build does not implement */
+  ZO_ERR_NOMEM = 8          /* workspace allocation failed */
+} zo_status;
+
+/* Weight storage dtypes. */
+enum { ZO_F32 = 0, ZO_BF16 = 1 };
+
+/* How zo_step turns the losses into rho_k. */
+enum {
+  ZO_SCHEME_CENTRAL = 0,  /* losses = [L+_0, L-_0, ..., L+_(q-1), L-_(q-1)]: rho_k = (L+_k - L-_k)/(2 eps), Eq. (3) */
+  ZO_SCHEME_FORWARD = 1,  /* losses = [l_0, l_1, ..., l_q]: rho_k = (l_(k+1) - l_0)/eps, Eq. (6), Alg. 3 */
+  ZO_SCHEME_DIRECT = 2    /* losses = [rho_0, ..., rho_(q-1)] given directly */
+};
+
+/* Optimizer applied in the subspace by zo_step. */
+enum {
+  ZO_OPT_ADAM = 0,        /* subspace Adam, Eqs. (7)-(10) */
+  ZO_OPT_SGD = 1          /* SubZero's subspace SGD (Sec. 3): D = Zbar, moments untouched */
+};
+
+/* Options for zo_set_option. */
+enum {
+  ZO_OPTION_WPASS_PATH = 0, /* 0 = automatic, 1 = fp32-FMA path, 2 = tcgen05 path */
+  ZO_OPTION_TIMING = 1      /* 1 = record CUDA events around every weight-pass launch */
+};
+
+/* One trainable matrix W_i with its projection bases and Adam moments. */
+typedef struct zo_matrix {
+  void* W;        /* device; m x n, row-major, leading dimension ldw elements, dtype below */
+  int64_t m;      /* rows (nn.Linear out_features) */
+  int64_t n;      /* columns (nn.Linear in_features) */
+  int64_t ldw;    /* leading dimension of W in elements, >= n */
+  int32_t dtype;  /* ZO_F32 or ZO_BF16 */
+  int32_t reserved;
+  float* U;       /* device; m x r fp32, written by zo_refresh / zo_init_subspace */
+  float* V;       /* device; n x r fp32, written by zo_refresh / zo_init_subspace */
+  float* M;       /* device; r x r fp32 first moment (Eq. (7)) */
+  float* Vm;      /* device; r x r fp32 second moment (Eq. (8)); named Vm to keep V for the basis */
+} zo_matrix;
+
+typedef struct zo_ctx zo_ctx;
+
+/*
+ * zo_create -- bind the caller's matrices into a context (Alg. 3 "Require" line).
+ *   mats[n_mats]: copied; the pointers inside must stay valid until zo_destroy.
+ *   r: subspace rank, 1 <= r <= min(m_i, n_i); this build supports r in {4, 8, 16, 32, 64}.
+ *   q: queries per step (K in the paper), 1 <= q <= 4096.
+ *   seed: 64-bit base seed of the Philox key.
+ *   matrix_index_base: matrix i of this table uses Philox matrix index base + i
+ *     (lets several contexts or ranks share one global numbering).
+ *   stream: cudaStream_t (void*) every later call launches on.
+ * Validates every matrix (non-null, 16-byte aligned, shapes, dtype), allocates
+ * the workspace and uploads the table.  On failure *out is NULL.
+ */
+ZO_API zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t r, int32_t q,
+                    uint64_t seed, uint32_t matrix_index_base, void* stream);
+
+/* zo_destroy -- synchronise the stream, free the context and its workspace.  NULL is a no-op. */
+ZO_API zo_status zo_destroy(zo_ctx* ctx);
+
+/*
+ * zo_refresh -- Alg. 1 (HaarProjMatrix) for every matrix at refresh index j
+ * (Alg. 3 calls it when t mod F == 0; j = t / F).  Draws Omega_U (m x r, tag 2)
+ * and Omega_V (n x r, tag 3) from the counter contract, takes their thin
+ * Householder QR and multiplies column c of Q by sgn(R_cc) (Eq. (11), sgn(0) = +1),
+ * writing U_i and V_i in place.  reset_moments != 0 also zeroes M_i and Vm_i.
+ */
+ZO_API zo_status zo_refresh(zo_ctx* ctx, uint32_t refresh_idx, int32_t reset_moments);
+
+/* zo_init_subspace -- the first lines of Alg. 3: M_i = Vm_i = 0 and U_i, V_i from
+ * Alg. 1 at refresh index refresh_idx (normally 0). */
+ZO_API zo_status zo_init_subspace(zo_ctx* ctx, uint32_t refresh_idx);
+
+/*
+ * zo_perturb -- one fused weight pass of Alg. 2 (PerturbParams) over all matrices:
+ *   W_i <- rnd(W_i + eps * U_i (ca Z_i^(qa) + cb Z_i^(qb)) V_i^T)
+ * with Z_i^(k) the step-t Gaussian of query k (tag 1).  qb = -1 drops the second
+ * term.  Two terms fuse the restore of one query with the perturbation of the
+ * next (e.g. ca = +1, cb = -1 gives W += eps U (Z_(k+1) - Z_k) V^T); the sum is
+ * formed in fp32 and W is rounded once (RNE) to its dtype.
+ * 0 <= qa, qb < q.
+ */
+ZO_API zo_status zo_perturb(zo_ctx* ctx, uint32_t t, int32_t qa, float ca, int32_t qb, float cb,
+                     float eps);
+
+/*
+ * zo_step -- the update of Alg. 3 for all matrices, fused with the final restore:
+ *   rho_k from the losses per `scheme` (Eq. (3) or Eq. (6)),
+ *   G_i = (1/q) sum_k rho_k Z_i^(k)                       (Eq. (6), Alg. 3)
+ *   ZO_OPT_ADAM: M_i, Vm_i updated in place (Eqs. (7)-(8)); with
+ *     bias corrections 1 - beta^adam_t (Eq. (9), adam_t >= 1 counts Adam updates
+ *     since the moments were zeroed), D_i = Mhat / (sqrt(Vhat) + eps_adam);
+ *   ZO_OPT_SGD: D_i = G_i (moments untouched; adam_t, betas ignored);
+ *   W_i <- rnd(W_i + U_i (-lr D_i + restore_coef * eps * Z_i^(restore_query)) V_i^T)
+ *     (Eq. (10) plus the restore; restore_query = -1 drops the restore term).
+ * losses: n_losses fp32 values (2q central, q+1 forward, q direct); device memory
+ *   unless losses_on_host != 0, in which case they are copied from host memory
+ *   before the launch (the host buffer may be reused when the call returns).
+ * gamma_out: NULL or device array of n_mats floats receiving ||G_i||_F (Sec. 4.1).
+ */
+ZO_API zo_status zo_step(zo_ctx* ctx, uint32_t t, int32_t adam_t, const float* losses, int32_t n_losses,
+                  int32_t losses_on_host, int32_t scheme, int32_t optimizer, float eps, float lr,
+                  float beta1, float beta2, float eps_adam, int32_t restore_query,
+                  float restore_coef, float* gamma_out);
+
+/* zo_sync_status -- synchronise the stream; return (and clear) the device status word. */
+ZO_API zo_status zo_sync_status(zo_ctx* ctx);
+
+/* zo_set_option -- see ZO_OPTION_*; returns ZO_ERR_INVALID_ARG for unknown options/values. */
+ZO_API zo_status zo_set_option(zo_ctx* ctx, int32_t option, int64_t value);
+
+/*
+ * zo_get_timing -- with ZO_OPTION_TIMING on, the summed device time (ms) and count of
+ * weight-pass kernel launches since the option was last set.  Synchronises the stream.
+ */
+ZO_API zo_status zo_get_timing(zo_ctx* ctx, double* total_ms, int64_t* launches);
+
+/* zo_wpass_path -- the weight-pass path the last zo_perturb / zo_step launched (1 = FMA, 2 = tcgen05). */
+ZO_API int32_t zo_wpass_path(const zo_ctx* ctx);
+
+/* zo_kernel_launches -- number of kernels this context has launched since zo_create. */
+ZO_API int64_t zo_kernel_launches(const zo_ctx* ctx);
+
+/*
+ * zo_philox_fill -- the raw integer stream of the counter contract:
+ *   out[4c + l] = Philox4x32-10(counter = (c, x1, x2, x3), key = seed)[l], 0 <= 4c + l < n_words.
+ * out: device uint32 array.  Asynchronous on `stream` (void* cudaStream_t).
+ */
+ZO_API zo_status zo_philox_fill(uint64_t seed, uint32_t x1, uint32_t x2, uint32_t x3, uint32_t* out,
+                         int64_t n_words, void* stream);
+
+/*
+ * zo_normal_fill -- the Gaussian stream of the contract (uniform + Box-Muller on
+ * lane pairs), elements 0..n-1, fp32, into device memory.  This is exactly how
+ * Z_i^(k) (x1 = i, x2 = t, x3 = 1 << 24 | k) and Omega (x2 = j, x3 = tag << 24)
+ * are drawn inside the other calls.
+ */
+ZO_API zo_status zo_normal_fill(uint64_t seed, uint32_t x1, uint32_t x2, uint32_t x3, float* out,
+                         int64_t n, void* stream);
+
+/* zo_status_string -- static description of a status code. */
+ZO_API const char* zo_status_string(int32_t status);
+
+/* zo_last_error -- last CUDA error text seen by this thread (static storage). */
+ZO_API const char* zo_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SUBZERO_GB300_ZO_H */

@@ -1,0 +1,562 @@
+// Host runtime and C ABI of the SubZero+ weight path (declared in include/zo.h).
+//
+// The context owns: a device copy of the matrix table, the per-pass coefficient
+// C_i (r x r) and projection P_i (r x n_i) buffers, the TSQR workspace of the
+// refresh, a loss staging buffer and a device status word.  Every call validates
+// its arguments on the host, then launches on the context's stream.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/zo.h"
+#include "zo_kernels.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+zo_status cuda_fail(cudaError_t e, const char* what) {
+  g_last_error = std::string(what) + ": " + cudaGetErrorString(e);
+  return ZO_ERR_CUDA;
+}
+
+#define ZO_CUDA(call, what)                                   \
+  do {                                                        \
+    cudaError_t _e = (call);                                  \
+    if (_e != cudaSuccess) return cuda_fail(_e, what);        \
+  } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool supported_rank(int32_t r) { return r == 4 || r == 8 || r == 16 || r == 32 || r == 64; }
+
+struct QrLevel {
+  std::vector<zo::QrBlock> up;    // all blocks of this level (tops included)
+  std::vector<zo::QrBlock> down;  // non-top blocks of this level
+};
+
+}  // namespace
+
+struct zo_ctx {
+  int device = 0;
+  cudaStream_t stream = nullptr;
+  int32_t n_mats = 0, r = 0, q = 0;
+  uint64_t seed = 0;
+  uint32_t base = 0;
+  std::vector<zo::MatDesc> h_mats;
+  zo::MatDesc* d_mats = nullptr;
+  int64_t* d_tile_prefix = nullptr;
+  int64_t n_tiles = 0;
+  int2* d_proj_units = nullptr;
+  int32_t n_proj_units = 0;
+  float* d_coeff_ws = nullptr;   // C_i and P_i
+  float* d_losses = nullptr;
+  int32_t max_losses = 0;
+  float* d_qr_ws = nullptr;      // TSQR stacks and tau
+  zo::QrBlock* d_qr_blocks = nullptr;
+  std::vector<int64_t> up_off, up_cnt, down_off, down_cnt;   // per level, into d_qr_blocks
+  uint32_t* d_status = nullptr;
+  int path_option = 0;
+  int last_path = 0;
+  int64_t launches = 0;          // kernels launched by this context
+  bool timing = false;
+  std::vector<cudaEvent_t> ev_start, ev_stop;
+  size_t ev_used = 0;
+  double timing_ms = 0.0;
+  int64_t timing_launches = 0;
+};
+
+namespace {
+
+void free_ctx(zo_ctx* c) {
+  if (!c) return;
+  cudaFree(c->d_mats);
+  cudaFree(c->d_tile_prefix);
+  cudaFree(c->d_proj_units);
+  cudaFree(c->d_coeff_ws);
+  cudaFree(c->d_losses);
+  cudaFree(c->d_qr_ws);
+  cudaFree(c->d_qr_blocks);
+  cudaFree(c->d_status);
+  for (auto e : c->ev_start) cudaEventDestroy(e);
+  for (auto e : c->ev_stop) cudaEventDestroy(e);
+  delete c;
+}
+
+zo_status validate_matrix(const zo_matrix& mt, int32_t r) {
+  if (!mt.W || !mt.U || !mt.V || !mt.M || !mt.Vm) {
+    g_last_error = "null buffer in zo_matrix";
+    return ZO_ERR_INVALID_ARG;
+  }
+  if (mt.dtype != ZO_F32 && mt.dtype != ZO_BF16) {
+    g_last_error = "unknown dtype";
+    return ZO_ERR_DTYPE;
+  }
+  if (mt.m < r || mt.n < r || mt.ldw < mt.n) {
+    g_last_error = "need r <= min(m, n) and ldw >= n";
+    return ZO_ERR_SHAPE;
+  }
+  // the Philox counter word addresses e / 4 of an m x r (or n x r) buffer in 32 bits
+  if (mt.m * (int64_t)r >= (int64_t(1) << 34) || mt.n * (int64_t)r >= (int64_t(1) << 34)) {
+    g_last_error = "matrix too large for the 32-bit counter word";
+    return ZO_ERR_SHAPE;
+  }
+  const int64_t esize = mt.dtype == ZO_BF16 ? 2 : 4;
+  if (!aligned16(mt.W) || (mt.ldw * esize) % 16 != 0 || !aligned16(mt.U) || !aligned16(mt.V) ||
+      !aligned16(mt.M) || !aligned16(mt.Vm)) {
+    g_last_error = "buffers must be 16-byte aligned and ldw*sizeof(dtype) a multiple of 16";
+    return ZO_ERR_ALIGN;
+  }
+  return ZO_OK;
+}
+
+// TSQR plan of one panel (rows x r) stored at `panel`; appends blocks per level and
+// returns the floats of workspace it needs (stacks + tau), assigning offsets from *ws.
+void plan_panel(float* panel, int64_t rows, int32_t r, uint32_t gidx, uint32_t tag, int32_t B,
+                std::vector<QrLevel>& levels, float* ws_base, int64_t* ws_off) {
+  float* storage = panel;
+  int64_t level_rows = rows;
+  for (int level = 0;; ++level) {
+    if ((int)levels.size() <= level) levels.emplace_back();
+    const int64_t nb = (level_rows + B - 1) / B;
+    float* stack = nullptr;
+    if (nb > 1) {
+      stack = ws_base ? ws_base + *ws_off : nullptr;
+      *ws_off += nb * (int64_t)r * r;
+    }
+    for (int64_t b = 0; b < nb; ++b) {
+      zo::QrBlock blk{};
+      blk.rows = storage ? storage + b * (int64_t)B * r : nullptr;
+      blk.n_real = (int32_t)std::min<int64_t>(B, level_rows - b * B);
+      blk.row0 = b * B;
+      blk.flags = (level == 0 ? zo::kQrLevel0 : 0) | (nb == 1 ? zo::kQrTop : 0);
+      blk.gidx = gidx;
+      blk.tag = tag;
+      blk.tau = ws_base ? ws_base + *ws_off : nullptr;
+      *ws_off += (r + 3) / 4 * 4;
+      if (nb > 1) {
+        blk.r_out = stack ? stack + b * (int64_t)r * r : nullptr;
+        blk.s_in = blk.r_out;
+      }
+      levels[level].up.push_back(blk);
+      if (nb > 1) levels[level].down.push_back(blk);
+    }
+    if (nb == 1) break;
+    storage = stack;
+    level_rows = nb * r;
+  }
+}
+
+zo_status record_start(zo_ctx* c) {
+  if (!c->timing) return ZO_OK;
+  if (c->ev_used == c->ev_start.size()) {
+    cudaEvent_t a, b;
+    ZO_CUDA(cudaEventCreate(&a), "cudaEventCreate");
+    ZO_CUDA(cudaEventCreate(&b), "cudaEventCreate");
+    c->ev_start.push_back(a);
+    c->ev_stop.push_back(b);
+  }
+  ZO_CUDA(cudaEventRecord(c->ev_start[c->ev_used], c->stream), "cudaEventRecord");
+  return ZO_OK;
+}
+
+zo_status record_stop(zo_ctx* c) {
+  if (!c->timing) return ZO_OK;
+  ZO_CUDA(cudaEventRecord(c->ev_stop[c->ev_used], c->stream), "cudaEventRecord");
+  ++c->ev_used;
+  return ZO_OK;
+}
+
+// Projection of C_i onto V_i and the weight pass, shared by zo_perturb and zo_step.
+zo_status run_weight_pass(zo_ctx* c) {
+  ZO_CUDA(zo::launch_project_fma(c->d_mats, c->d_proj_units, c->n_proj_units, c->r, c->stream),
+          "projection kernel");
+  ++c->launches;
+  zo_status st = record_start(c);
+  if (st != ZO_OK) return st;
+  ZO_CUDA(zo::launch_wpass_fma(c->d_mats, c->n_mats, c->d_tile_prefix, c->n_tiles, c->r, c->stream),
+          "weight-pass kernel");
+  ++c->launches;
+  c->last_path = 1;
+  return record_stop(c);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* zo_status_string(int32_t s) {
+  switch (s) {
+    case ZO_OK: return "ok";
+    case ZO_ERR_INVALID_ARG: return "invalid argument";
+    case ZO_ERR_SHAPE: return "unsupported or inconsistent shape";
+    case ZO_ERR_ALIGN: return "misaligned buffer";
+    case ZO_ERR_DTYPE: return "unknown dtype";
+    case ZO_ERR_CUDA: return "CUDA error";
+    case ZO_ERR_TIMEOUT: return "device-side wait timed out";
+    case ZO_ERR_UNSUPPORTED: return "unsupported request";
+    case ZO_ERR_NOMEM: return "out of device memory";
+    default: return "unknown status";
+  }
+}
+
+const char* zo_last_error(void) { return g_last_error.c_str(); }
+
+zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t r, int32_t q,
+                    uint64_t seed, uint32_t matrix_index_base, void* stream) {
+  if (!out) return ZO_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!mats || n_mats <= 0) {
+    g_last_error = "need at least one matrix";
+    return ZO_ERR_INVALID_ARG;
+  }
+  if (!supported_rank(r)) {
+    g_last_error = "rank r must be one of 4, 8, 16, 32, 64";
+    return ZO_ERR_SHAPE;
+  }
+  if (q < 1 || q > 4096) {
+    g_last_error = "q must be in [1, 4096]";
+    return ZO_ERR_INVALID_ARG;
+  }
+  for (int32_t i = 0; i < n_mats; ++i) {
+    zo_status st = validate_matrix(mats[i], r);
+    if (st != ZO_OK) return st;
+  }
+  int dev = 0;
+  ZO_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
+  cudaDeviceProp prop;
+  ZO_CUDA(cudaGetDeviceProperties(&prop, dev), "cudaGetDeviceProperties");
+  if (!(prop.major == 10 && prop.minor == 3)) {
+    g_last_error = "this library is built for sm_103a (GB300) only; found sm_" +
+                   std::to_string(prop.major) + std::to_string(prop.minor);
+    return ZO_ERR_CUDA;
+  }
+
+  zo_ctx* c = new zo_ctx();
+  c->device = dev;
+  c->stream = reinterpret_cast<cudaStream_t>(stream);
+  c->n_mats = n_mats;
+  c->r = r;
+  c->q = q;
+  c->seed = seed;
+  c->base = matrix_index_base;
+
+  // coefficient workspace: C_i (r*r) then P_i (r*n_i) per matrix
+  int64_t coeff_floats = 0;
+  std::vector<int64_t> c_off(n_mats), p_off(n_mats);
+  for (int32_t i = 0; i < n_mats; ++i) {
+    c_off[i] = coeff_floats;
+    coeff_floats += (int64_t)r * r;
+    p_off[i] = coeff_floats;
+    coeff_floats += ((int64_t)r * mats[i].n + 3) / 4 * 4;
+  }
+  auto fail = [&](zo_status st) {
+    free_ctx(c);
+    return st;
+  };
+  cudaError_t e = cudaMalloc(&c->d_coeff_ws, sizeof(float) * coeff_floats);
+  if (e != cudaSuccess) {
+    cuda_fail(e, "cudaMalloc(coefficient workspace)");
+    return fail(ZO_ERR_NOMEM);
+  }
+
+  // weight-pass tiles and projection units
+  std::vector<int64_t> prefix(n_mats + 1, 0);
+  std::vector<int2> units;
+  c->h_mats.resize(n_mats);
+  for (int32_t i = 0; i < n_mats; ++i) {
+    const zo_matrix& mt = mats[i];
+    zo::MatDesc d{};
+    d.W = mt.W;
+    d.m = mt.m;
+    d.n = mt.n;
+    d.ldw = mt.ldw;
+    d.dtype = mt.dtype;
+    d.gidx = matrix_index_base + (uint32_t)i;
+    d.U = mt.U;
+    d.V = mt.V;
+    d.M = mt.M;
+    d.Vm = mt.Vm;
+    d.C = c->d_coeff_ws + c_off[i];
+    d.P = c->d_coeff_ws + p_off[i];
+    const int tn = zo::fma_tile_cols(mt.dtype);
+    const int64_t tiles = ((mt.m + zo::kFmaTileRows - 1) / zo::kFmaTileRows) * ((mt.n + tn - 1) / tn);
+    d.tile0 = prefix[i];
+    prefix[i + 1] = prefix[i] + tiles;
+    for (int64_t j0 = 0; j0 < mt.n; j0 += 128) units.push_back(make_int2(i, (int)j0));
+    c->h_mats[i] = d;
+  }
+  c->n_tiles = prefix[n_mats];
+  c->n_proj_units = (int32_t)units.size();
+  if (c->n_tiles > 0x7FFFFFFF) {
+    g_last_error = "too many weight-pass tiles";
+    return fail(ZO_ERR_SHAPE);
+  }
+
+  // refresh plan (dry run for sizes, then the real pass with pointers)
+  const int32_t B = zo::qr_block_rows(r);
+  int64_t qr_floats = 0;
+  {
+    std::vector<QrLevel> dry;
+    for (int32_t i = 0; i < n_mats; ++i) {
+      plan_panel(nullptr, mats[i].m, r, 0, zo::kTagOmegaU, B, dry, nullptr, &qr_floats);
+      plan_panel(nullptr, mats[i].n, r, 0, zo::kTagOmegaV, B, dry, nullptr, &qr_floats);
+    }
+  }
+  e = cudaMalloc(&c->d_qr_ws, sizeof(float) * std::max<int64_t>(qr_floats, 4));
+  if (e != cudaSuccess) {
+    cuda_fail(e, "cudaMalloc(refresh workspace)");
+    return fail(ZO_ERR_NOMEM);
+  }
+  std::vector<QrLevel> levels;
+  int64_t off = 0;
+  for (int32_t i = 0; i < n_mats; ++i) {
+    plan_panel(mats[i].U, mats[i].m, r, matrix_index_base + (uint32_t)i, zo::kTagOmegaU, B, levels,
+               c->d_qr_ws, &off);
+    plan_panel(mats[i].V, mats[i].n, r, matrix_index_base + (uint32_t)i, zo::kTagOmegaV, B, levels,
+               c->d_qr_ws, &off);
+  }
+  std::vector<zo::QrBlock> all_blocks;
+  for (auto& lv : levels) {
+    c->up_off.push_back((int64_t)all_blocks.size());
+    c->up_cnt.push_back((int64_t)lv.up.size());
+    all_blocks.insert(all_blocks.end(), lv.up.begin(), lv.up.end());
+    c->down_off.push_back((int64_t)all_blocks.size());
+    c->down_cnt.push_back((int64_t)lv.down.size());
+    all_blocks.insert(all_blocks.end(), lv.down.begin(), lv.down.end());
+  }
+
+  c->max_losses = std::max(2 * q, q + 1);
+  e = cudaMalloc(&c->d_losses, sizeof(float) * c->max_losses);
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_mats, sizeof(zo::MatDesc) * n_mats);
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_tile_prefix, sizeof(int64_t) * (n_mats + 1));
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_proj_units, sizeof(int2) * std::max<size_t>(units.size(), 1));
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_qr_blocks, sizeof(zo::QrBlock) * std::max<size_t>(all_blocks.size(), 1));
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_status, sizeof(uint32_t));
+  if (e != cudaSuccess) {
+    cuda_fail(e, "cudaMalloc(context tables)");
+    return fail(ZO_ERR_NOMEM);
+  }
+  e = cudaMemcpy(c->d_mats, c->h_mats.data(), sizeof(zo::MatDesc) * n_mats, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(c->d_tile_prefix, prefix.data(), sizeof(int64_t) * (n_mats + 1), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !units.empty())
+    e = cudaMemcpy(c->d_proj_units, units.data(), sizeof(int2) * units.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !all_blocks.empty())
+    e = cudaMemcpy(c->d_qr_blocks, all_blocks.data(), sizeof(zo::QrBlock) * all_blocks.size(),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemset(c->d_status, 0, sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    cuda_fail(e, "zo_create upload");
+    return fail(ZO_ERR_CUDA);
+  }
+  *out = c;
+  return ZO_OK;
+}
+
+zo_status zo_destroy(zo_ctx* c) {
+  if (!c) return ZO_OK;
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  free_ctx(c);
+  if (e != cudaSuccess) return cuda_fail(e, "zo_destroy");
+  return ZO_OK;
+}
+
+zo_status zo_refresh(zo_ctx* c, uint32_t refresh_idx, int32_t reset_moments) {
+  if (!c) return ZO_ERR_INVALID_ARG;
+  const int n_levels = (int)c->up_off.size();
+  for (int lv = 0; lv < n_levels; ++lv) {
+    if (c->up_cnt[lv] == 0) continue;
+    ZO_CUDA(zo::launch_qr_up(c->d_qr_blocks + c->up_off[lv], (int32_t)c->up_cnt[lv], c->r, c->seed,
+                             refresh_idx, c->d_status, c->stream),
+            "refresh up-pass kernel");
+    ++c->launches;
+  }
+  for (int lv = n_levels - 1; lv >= 0; --lv) {
+    if (c->down_cnt[lv] == 0) continue;
+    ZO_CUDA(zo::launch_qr_down(c->d_qr_blocks + c->down_off[lv], (int32_t)c->down_cnt[lv], c->r,
+                               c->d_status, c->stream),
+            "refresh down-pass kernel");
+    ++c->launches;
+  }
+  if (reset_moments) {
+    ZO_CUDA(zo::launch_zero_moments(c->d_mats, c->n_mats, c->r, c->stream), "zero moments");
+    ++c->launches;
+  }
+  return ZO_OK;
+}
+
+zo_status zo_init_subspace(zo_ctx* c, uint32_t refresh_idx) {
+  return zo_refresh(c, refresh_idx, 1);
+}
+
+zo_status zo_perturb(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t qb, float cb, float eps) {
+  if (!c) return ZO_ERR_INVALID_ARG;
+  if (qa < 0 || qa >= c->q || qb < -1 || qb >= c->q || !std::isfinite(ca) || !std::isfinite(cb) ||
+      !std::isfinite(eps)) {
+    g_last_error = "zo_perturb: query index out of range or non-finite scalar";
+    return ZO_ERR_INVALID_ARG;
+  }
+  zo::CoeffParams p{};
+  p.mode = zo::kCoeffPerturb;
+  p.seed = c->seed;
+  p.t = t;
+  p.r = c->r;
+  p.q = c->q;
+  p.qa = qa;
+  p.qb = qb;
+  p.ca = ca;
+  p.cb = cb;
+  p.eps = eps;
+  ZO_CUDA(zo::launch_coeff(c->d_mats, c->n_mats, p, c->stream), "coefficient kernel");
+  ++c->launches;
+  return run_weight_pass(c);
+}
+
+zo_status zo_step(zo_ctx* c, uint32_t t, int32_t adam_t, const float* losses, int32_t n_losses,
+                  int32_t losses_on_host, int32_t scheme, int32_t optimizer, float eps, float lr,
+                  float beta1, float beta2, float eps_adam, int32_t restore_query,
+                  float restore_coef, float* gamma_out) {
+  if (!c || !losses) return ZO_ERR_INVALID_ARG;
+  int32_t want = -1;
+  if (scheme == ZO_SCHEME_CENTRAL) want = 2 * c->q;
+  else if (scheme == ZO_SCHEME_FORWARD) want = c->q + 1;
+  else if (scheme == ZO_SCHEME_DIRECT) want = c->q;
+  if (want < 0 || n_losses != want) {
+    g_last_error = "zo_step: unknown scheme or wrong number of losses";
+    return ZO_ERR_INVALID_ARG;
+  }
+  if (optimizer != ZO_OPT_ADAM && optimizer != ZO_OPT_SGD) {
+    g_last_error = "zo_step: unknown optimizer";
+    return ZO_ERR_INVALID_ARG;
+  }
+  if (restore_query < -1 || restore_query >= c->q || !std::isfinite(eps) || !std::isfinite(lr) ||
+      !std::isfinite(restore_coef) || (scheme != ZO_SCHEME_DIRECT && eps == 0.0f)) {
+    g_last_error = "zo_step: restore query out of range or bad scalar";
+    return ZO_ERR_INVALID_ARG;
+  }
+  double inv_bc1 = 1.0, inv_bc2 = 1.0;
+  if (optimizer == ZO_OPT_ADAM) {
+    if (adam_t < 1 || !(beta1 >= 0.0f && beta1 < 1.0f) || !(beta2 >= 0.0f && beta2 < 1.0f) ||
+        !(eps_adam >= 0.0f)) {
+      g_last_error = "zo_step: need adam_t >= 1, betas in [0, 1), eps_adam >= 0";
+      return ZO_ERR_INVALID_ARG;
+    }
+    inv_bc1 = 1.0 / (1.0 - std::pow((double)beta1, (double)adam_t));
+    inv_bc2 = 1.0 / (1.0 - std::pow((double)beta2, (double)adam_t));
+  }
+  const float* d_losses = losses;
+  if (losses_on_host) {
+    ZO_CUDA(cudaMemcpyAsync(c->d_losses, losses, sizeof(float) * n_losses, cudaMemcpyHostToDevice,
+                            c->stream),
+            "copy losses to device");
+    d_losses = c->d_losses;
+  }
+  zo::CoeffParams p{};
+  p.mode = zo::kCoeffStep;
+  p.seed = c->seed;
+  p.t = t;
+  p.r = c->r;
+  p.q = c->q;
+  p.eps = eps;
+  p.losses = d_losses;
+  p.n_losses = n_losses;
+  p.scheme = scheme;
+  p.optimizer = optimizer;
+  p.lr = lr;
+  p.beta1 = beta1;
+  p.beta2 = beta2;
+  p.eps_adam = eps_adam;
+  p.inv_bc1 = (float)inv_bc1;
+  p.inv_bc2 = (float)inv_bc2;
+  p.restore_query = restore_query;
+  p.restore_coef = restore_coef;
+  p.gamma_out = gamma_out;
+  ZO_CUDA(zo::launch_coeff(c->d_mats, c->n_mats, p, c->stream), "coefficient kernel");
+  ++c->launches;
+  return run_weight_pass(c);
+}
+
+zo_status zo_sync_status(zo_ctx* c) {
+  if (!c) return ZO_ERR_INVALID_ARG;
+  ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
+  uint32_t s = 0;
+  ZO_CUDA(cudaMemcpy(&s, c->d_status, sizeof(s), cudaMemcpyDeviceToHost), "read status");
+  if (s != 0) {
+    ZO_CUDA(cudaMemset(c->d_status, 0, sizeof(uint32_t)), "clear status");
+    g_last_error = s == zo::kDevTimeout ? "a device-side wait ran out" : "a device-side bound check failed";
+    return s == zo::kDevTimeout ? ZO_ERR_TIMEOUT : ZO_ERR_CUDA;
+  }
+  return ZO_OK;
+}
+
+zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
+  if (!c) return ZO_ERR_INVALID_ARG;
+  if (option == ZO_OPTION_WPASS_PATH) {
+    if (value < 0 || value > 2) return ZO_ERR_INVALID_ARG;
+    if (value == 2) {
+      g_last_error = "tcgen05 weight pass not available in this build";
+      return ZO_ERR_UNSUPPORTED;
+    }
+    c->path_option = (int)value;
+    return ZO_OK;
+  }
+  if (option == ZO_OPTION_TIMING) {
+    if (value != 0 && value != 1) return ZO_ERR_INVALID_ARG;
+    ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
+    c->timing = value != 0;
+    c->ev_used = 0;
+    c->timing_ms = 0.0;
+    c->timing_launches = 0;
+    return ZO_OK;
+  }
+  return ZO_ERR_INVALID_ARG;
+}
+
+zo_status zo_get_timing(zo_ctx* c, double* total_ms, int64_t* launches) {
+  if (!c || !total_ms || !launches) return ZO_ERR_INVALID_ARG;
+  ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
+  for (size_t k = 0; k < c->ev_used; ++k) {
+    float ms = 0.f;
+    ZO_CUDA(cudaEventElapsedTime(&ms, c->ev_start[k], c->ev_stop[k]), "cudaEventElapsedTime");
+    c->timing_ms += ms;
+    ++c->timing_launches;
+  }
+  c->ev_used = 0;
+  *total_ms = c->timing_ms;
+  *launches = c->timing_launches;
+  return ZO_OK;
+}
+
+int32_t zo_wpass_path(const zo_ctx* c) { return c ? c->last_path : 0; }
+
+int64_t zo_kernel_launches(const zo_ctx* c) { return c ? c->launches : 0; }
+
+zo_status zo_philox_fill(uint64_t seed, uint32_t x1, uint32_t x2, uint32_t x3, uint32_t* out,
+                         int64_t n_words, void* stream) {
+  if (n_words < 0 || (n_words > 0 && !out) || (n_words + 3) / 4 > (int64_t(1) << 32)) {
+    g_last_error = "zo_philox_fill: bad output or size";
+    return ZO_ERR_INVALID_ARG;
+  }
+  ZO_CUDA(zo::launch_philox_fill(seed, x1, x2, x3, out, n_words,
+                                 reinterpret_cast<cudaStream_t>(stream)),
+          "philox fill kernel");
+  return ZO_OK;
+}
+
+zo_status zo_normal_fill(uint64_t seed, uint32_t x1, uint32_t x2, uint32_t x3, float* out,
+                         int64_t n, void* stream) {
+  if (n < 0 || (n > 0 && !out) || (n + 3) / 4 > (int64_t(1) << 32)) {
+    g_last_error = "zo_normal_fill: bad output or size";
+    return ZO_ERR_INVALID_ARG;
+  }
+  ZO_CUDA(zo::launch_normal_fill(seed, x1, x2, x3, out, n, reinterpret_cast<cudaStream_t>(stream)),
+          "normal fill kernel");
+  return ZO_OK;
+}
+
+}  // extern "C"

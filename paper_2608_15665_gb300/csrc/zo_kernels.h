@@ -1,0 +1,72 @@
+// Host-side launchers of the SubZero+ kernels (internal to the library).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "zo_device.cuh"
+
+namespace zo {
+
+// ---- counter-based Gaussian contract (zo_rng.cu) ---------------------------
+cudaError_t launch_philox_fill(uint64_t seed, uint32_t x1, uint32_t x2, uint32_t x3, uint32_t* out,
+                               int64_t n_words, cudaStream_t s);
+cudaError_t launch_normal_fill(uint64_t seed, uint32_t x1, uint32_t x2, uint32_t x3, float* out,
+                               int64_t n, cudaStream_t s);
+
+// ---- per-pass coefficient C_i and projection P_i (zo_coeff.cu) ---------------
+enum CoeffMode : int32_t { kCoeffPerturb = 0, kCoeffStep = 1 };
+
+struct CoeffParams {
+  int32_t mode;
+  uint64_t seed;
+  uint32_t t;
+  int32_t r, q;
+  // perturb: C = eps (ca Z_qa + cb Z_qb)
+  int32_t qa, qb;
+  float ca, cb, eps;
+  // step: rho from losses, G, optimizer, C = -lr D + restore_coef eps Z_restore
+  const float* losses;
+  int32_t n_losses, scheme, optimizer;
+  float lr, beta1, beta2, eps_adam;
+  float inv_bc1, inv_bc2;   // 1 / (1 - beta^adam_t), formed on the host in double
+  int32_t restore_query;
+  float restore_coef;
+  float* gamma_out;
+};
+
+cudaError_t launch_coeff(const MatDesc* d_mats, int32_t n_mats, const CoeffParams& p,
+                         cudaStream_t s);
+
+// P_i = C_i V_i^T (r x n, fp32) for the FMA weight pass.  Work units are
+// (matrix, first column) pairs of 128 columns.
+cudaError_t launch_project_fma(const MatDesc* d_mats, const int2* d_units, int32_t n_units,
+                               int32_t r, cudaStream_t s);
+
+// Pt_i = V_i C_i^T (n x r) split into bf16 hi + lo for the tensor-core pass.
+cudaError_t launch_project_split(const MatDesc* d_mats, const int2* d_units, int32_t n_units,
+                                 int32_t r, cudaStream_t s);
+
+// U_i split into bf16 hi + lo (after a refresh) for the tensor-core pass.
+cudaError_t launch_split_u(const MatDesc* d_mats, const int2* d_units, int32_t n_units, int32_t r,
+                           cudaStream_t s);
+
+// ---- weight pass, fp32 FMA path (zo_wpass_fma.cu) ---------------------------
+constexpr int kFmaTileRows = 32;
+__host__ __device__ constexpr int fma_tile_cols(int32_t dtype) { return dtype == 1 ? 256 : 128; }
+
+cudaError_t launch_wpass_fma(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_tile_prefix,
+                             int64_t n_tiles, int32_t r, cudaStream_t s);
+
+// ---- weight pass, tcgen05 path (zo_wpass_tc.cu) --------------------------------
+bool wpass_tc_supported(int32_t r);
+
+// ---- refresh: batched TSQR + sign correction (zo_qr.cu) ------------------------
+int32_t qr_block_rows(int32_t r);
+cudaError_t launch_qr_up(const QrBlock* d_blocks, int32_t n_blocks, int32_t r, uint64_t seed,
+                         uint32_t refresh_idx, uint32_t* d_status, cudaStream_t s);
+cudaError_t launch_qr_down(const QrBlock* d_blocks, int32_t n_blocks, int32_t r,
+                           uint32_t* d_status, cudaStream_t s);
+cudaError_t launch_zero_moments(const MatDesc* d_mats, int32_t n_mats, int32_t r, cudaStream_t s);
+
+}  // namespace zo

@@ -30,3 +30,33 @@ def read_golden_rows(name):
 @pytest.fixture(scope="session")
 def golden():
     return read_golden_rows
+
+
+def ensure_library():
+    """Build libsubzero_zo.so in-tree if it is missing or stale (nvcc cross-compiles on CPU)."""
+    from paper_2608_15665_gb300 import build
+    return build.build()
+
+
+def cuda_available():
+    try:
+        import torch
+        return torch.cuda.is_available()
+    except Exception:
+        return False
+
+
+@pytest.fixture(scope="session")
+def lib():
+    ensure_library()
+    from paper_2608_15665_gb300 import binding
+    return binding
+
+
+@pytest.fixture(scope="session")
+def gpu(lib):
+    if not cuda_available():
+        pytest.fail("GPU test selected but no CUDA device is visible")
+    import torch
+    torch.cuda.init()
+    return torch.device("cuda:0")

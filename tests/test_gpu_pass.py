@@ -1,0 +1,162 @@
+"""Per-call GPU parity of the weight passes (zo_perturb, zo_step) against the oracle.
+
+Each test reads the library's state before a call (W, U, V, M, Vm), lets the
+oracle compute the call exactly in fp64 from that state, and compares:
+bf16 weights within 1 ulp of the oracle's rounded result, fp32 weights and the
+Adam moments within relative 1e-5 (floored at 1e-3 of the largest entry).
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from gpu_util import dtype_of, f32, make_weight, oracle_perturb, oracle_step, snapshot
+from parity import assert_rel, assert_weights
+
+pytestmark = pytest.mark.gpu
+
+# (r, [(m, n, dtype, ldw)]) -- several tiles in both directions plus ragged tails
+CASES = {
+    "r4": (4, [(300, 520, "bf16", None), (64, 1000, "f32", None), (8, 5120, "f32", None),
+               (5120, 8, "f32", None)]),
+    "r8": (8, [(300, 520, "bf16", None), (1030, 72, "bf16", None), (256, 256, "f32", None)]),
+    "r16": (16, [(300, 520, "bf16", 528), (130, 1000, "bf16", None), (100, 96, "f32", 100)]),
+    "r32": (32, [(300, 520, "bf16", None), (1030, 72, "bf16", 80), (64, 2048, "f32", None)]),
+    "r64": (64, [(300, 520, "bf16", None), (130, 1000, "bf16", None), (1030, 72, "f32", None)]),
+}
+
+
+def _build(gpu, case, seed, base=3):
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    r, spec = CASES[case]
+    weights = [make_weight(m, n, dt, 100 + k, gpu, ldw) for k, (m, n, dt, ldw) in enumerate(spec)]
+    z = SubZeroPlus(weights, r, 4, seed, matrix_index_base=base)
+    z.init_subspace(0)
+    return z, base
+
+
+@pytest.mark.parametrize("case", list(CASES))
+@pytest.mark.parametrize("eps", [1e-3, 1e-1])
+def test_perturb_pass_matches_oracle(lib, gpu, case, eps):
+    z, base = _build(gpu, case, seed=555)
+    calls = [(0, 1.0, -1, 0.0), (0, -2.0, -1, 0.0), (0, 1.0, 1, 1.0), (3, 1.0, 2, -1.0)]
+    for t, (qa, ca, qb, cb) in zip((0, 0, 7, 123456), calls):
+        before = snapshot(z)
+        z.perturb(t, qa, ca, qb, cb, eps)
+        after = snapshot(z)
+        terms = [(qa, ca)] + ([(qb, cb)] if qb >= 0 else [])
+        for i, W in enumerate(z.weights):
+            want = oracle_perturb(before, i, dtype_of(W), z.seed, base + i, t, z.r, terms, eps)
+            assert_weights(after["W"][i], want, dtype_of(W), f"{case} matrix {i} t={t}")
+    z.sync()
+    z.close()
+
+
+@pytest.mark.parametrize("case", ["r4", "r8", "r16", "r32", "r64"])
+@pytest.mark.parametrize("scheme", ["central", "forward", "direct"])
+def test_step_matches_oracle(lib, gpu, case, scheme):
+    z, base = _build(gpu, case, seed=777)
+    q, eps, lr, b1, b2, ea = z.q, 1e-3, 1e-2, 0.9, 0.95, 1e-8
+    n_losses = {"central": 2 * q, "forward": q + 1, "direct": q}[scheme]
+    restore = {"central": (q - 1, 1.0), "forward": (q - 1, -1.0), "direct": (-1, 0.0)}[scheme]
+    rs = np.random.default_rng(5)
+    gamma = torch.zeros(len(z.weights), dtype=torch.float32, device=gpu)
+    for step, t in enumerate((0, 1, 2)):
+        if scheme == "direct":
+            losses = (rs.standard_normal(n_losses) * 7.0).astype(np.float32)
+        else:
+            losses = (2.0 + 0.01 * rs.standard_normal(n_losses)).astype(np.float32)
+        before = snapshot(z)
+        z.step(t, step + 1, losses, scheme, eps, lr, b1, b2, ea, restore[0], restore[1],
+               gamma_out=gamma)
+        after = snapshot(z)
+        g = gamma.cpu().double().numpy()
+        rterms = [restore] if restore[0] >= 0 else []
+        for i, W in enumerate(z.weights):
+            Wo, Mo, Vmo, G = oracle_step(before, i, dtype_of(W), z.seed, base + i, t, z.r, q,
+                                         losses, scheme, eps, lr, b1, b2, ea, step + 1, rterms)
+            assert_rel(after["M"][i], Mo, f"M {case} {i}")
+            assert_rel(after["Vm"][i], Vmo, f"Vm {case} {i}")
+            assert_weights(after["W"][i], Wo, dtype_of(W), f"W {case} {i} step {step}")
+            assert abs(g[i] - np.linalg.norm(G)) <= 1e-5 * np.linalg.norm(G)
+    z.close()
+
+
+def test_sgd_step_matches_oracle_and_leaves_moments(lib, gpu):
+    z, base = _build(gpu, "r8", seed=31)
+    z.M[0].fill_(0.25)
+    losses = (2.0 + 0.01 * np.random.default_rng(1).standard_normal(2 * z.q)).astype(np.float32)
+    before = snapshot(z)
+    from paper_2608_15665_gb300 import binding as zb
+    z.step(4, 1, losses, "central", 1e-3, 1e-4, 0.9, 0.95, 1e-8, z.q - 1, 1.0,
+           optimizer=zb.ZO_OPT_SGD)
+    after = snapshot(z)
+    for i, W in enumerate(z.weights):
+        Wo, _, _, _ = oracle_step(before, i, dtype_of(W), z.seed, base + i, 4, z.r, z.q, losses,
+                                  "central", 1e-3, 1e-4, 0.9, 0.95, 1e-8, 1, [(z.q - 1, 1.0)],
+                                  optimizer="sgd")
+        assert_weights(after["W"][i], Wo, dtype_of(W), f"sgd W {i}")
+        assert np.array_equal(after["M"][i], before["M"][i])
+    z.close()
+
+
+def test_losses_from_device_memory(lib, gpu):
+    z, base = _build(gpu, "r16", seed=9)
+    losses = (2.0 + 0.01 * np.random.default_rng(2).standard_normal(2 * z.q)).astype(np.float32)
+    before = snapshot(z)
+    z.step(0, 1, torch.from_numpy(losses).to(gpu), "central", 1e-3, 1e-3, 0.9, 0.95, 1e-8,
+           z.q - 1, 1.0)
+    after = snapshot(z)
+    Wo, Mo, _, _ = oracle_step(before, 0, "bf16", z.seed, base, 0, z.r, z.q, losses, "central",
+                               1e-3, 1e-3, 0.9, 0.95, 1e-8, 1, [(z.q - 1, 1.0)])
+    assert_rel(after["M"][0], Mo, "M")
+    assert_weights(after["W"][0], Wo, "bf16", "W")
+    z.close()
+
+
+def test_same_calls_give_bit_identical_weights(lib, gpu):
+    outs = []
+    for _ in range(2):
+        z, _ = _build(gpu, "r32", seed=2024)
+        z.perturb(3, 0, 1.0, -1, 0.0, 1e-1)
+        z.perturb(3, 0, 1.0, 1, 1.0, 1e-1)
+        z.step(3, 1, np.full(2 * z.q, 2.0, np.float32) + np.arange(2 * z.q, dtype=np.float32) * 1e-3,
+               "central", 1e-1, 1e-2, 0.9, 0.95, 1e-8, z.q - 1, 1.0)
+        torch.cuda.synchronize()
+        outs.append([W.clone() for W in z.weights])
+        z.close()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+
+
+def test_padding_columns_beyond_n_are_untouched(lib, gpu):
+    # ldw > n: the bytes between n and ldw belong to the caller and must not change
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    buf = make_weight(200, 272, "bf16", 3, gpu)
+    view = buf[:, :264]
+    z = SubZeroPlus([view], 8, 2, 1)
+    z.init_subspace(0)
+    pad = buf[:, 264:].clone()
+    z.perturb(0, 0, 1.0, -1, 0.0, 1e-1)
+    torch.cuda.synchronize()
+    assert torch.equal(buf[:, 264:], pad)
+    z.close()
+
+
+def test_rejected_calls_launch_nothing(lib, gpu):
+    from paper_2608_15665_gb300 import binding as zb
+    z, _ = _build(gpu, "r8", seed=4)
+    before = snapshot(z)
+    with pytest.raises(zb.ZoError) as e:
+        z.perturb(0, 4, 1.0, -1, 0.0, 1e-3)          # qa == q
+    assert e.value.status == zb.ZO_ERR_INVALID_ARG
+    with pytest.raises(zb.ZoError):
+        z.step(0, 1, np.zeros(3, np.float32), "central", 1e-3, 1e-3, 0.9, 0.95, 1e-8, 3, 1.0)
+    with pytest.raises(zb.ZoError):
+        z.step(0, 0, np.zeros(8, np.float32), "central", 1e-3, 1e-3, 0.9, 0.95, 1e-8, 3, 1.0)
+    after = snapshot(z)
+    for k in ("W", "M", "Vm"):
+        for a, b in zip(before[k], after[k]):
+            assert np.array_equal(a, b)
+    z.sync()
+    z.close()

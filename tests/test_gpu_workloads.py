@@ -1,0 +1,129 @@
+"""Workload-level GPU parity: whole Alg. 3 trajectories on the small workloads, and
+per-call parity on sampled matrices / rows of the full-size workloads (each matrix's
+update depends only on its own state and the shared losses, so a sample is exact)."""
+
+import numpy as np
+import pytest
+import torch
+
+from gpu_util import dtype_of, f32, snapshot
+from oracle import haar, subzero
+from parity import UV_ABS, assert_rel, assert_weights, to_f64
+
+pytestmark = pytest.mark.gpu
+
+
+def _run_gpu_schedule(z, wl, scheme, T):
+    from paper_2608_15665_gb300 import workloads
+    table = workloads.loss_table(wl, scheme, steps=T)
+    for t in range(T):
+        if t % wl.F == 0:
+            z.refresh(t // wl.F, reset_moments=(t == 0))
+        z.run_step(t, t + 1, lambda tt, k: float(table[tt][k]), scheme, wl.eps, wl.lr, wl.beta1,
+                   wl.beta2, wl.eps_adam)
+    return table
+
+
+def _oracle_trajectory(wl, W0, i, table, scheme, T):
+    st = subzero.MatrixState(W0, wl.dtype, wl.r)
+    subzero.run_schedule(st, wl.seed, i, table, scheme, wl.q, T, wl.F, f32(wl.eps), f32(wl.lr),
+                         f32(wl.beta1), f32(wl.beta2), f32(wl.eps_adam))
+    return st
+
+
+@pytest.mark.parametrize("scheme", ["central", "forward"])
+def test_single256_trajectory(lib, gpu, scheme):
+    from paper_2608_15665_gb300 import workloads
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    wl = workloads.get("single256_f32_r8")
+    W0 = workloads.init_weight(wl, 0, "cpu")
+    z = SubZeroPlus([W0.clone().to(gpu)], wl.r, wl.q, wl.seed)
+    table = _run_gpu_schedule(z, wl, scheme, wl.steps)
+    s = snapshot(z)
+    st = _oracle_trajectory(wl, to_f64(W0), 0, table, scheme, wl.steps)
+    assert_rel(s["W"][0], st.W, "W after 10 steps")
+    assert_rel(s["M"][0], st.M, "M after 10 steps")
+    assert_rel(s["Vm"][0], st.Vm, "Vm after 10 steps")
+    assert np.max(np.abs(s["U"][0] - st.U)) <= UV_ABS
+    assert np.max(np.abs(s["V"][0] - st.V)) <= UV_ABS
+    # the weights did move: the update is not a no-op
+    assert np.max(np.abs(s["W"][0] - to_f64(W0))) > 1e-6
+    z.close()
+
+
+def test_lora_trajectory_on_sampled_matrices(lib, gpu):
+    from paper_2608_15665_gb300 import workloads
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    wl = workloads.get("lora_opt13b_f32_r4")
+    W0 = [workloads.init_weight(wl, i, "cpu") for i in range(wl.n_mats)]
+    z = SubZeroPlus([W.clone().to(gpu) for W in W0], wl.r, wl.q, wl.seed)
+    table = _run_gpu_schedule(z, wl, "central", wl.steps)
+    s = snapshot(z)
+    for i in (0, 1, 2, 3, 158, 159):
+        st = _oracle_trajectory(wl, to_f64(W0[i]), i, table, "central", wl.steps)
+        assert_rel(s["W"][i], st.W, f"LoRA matrix {i} after 200 steps")
+        assert_rel(s["M"][i], st.M, f"M {i}")
+        assert_rel(s["Vm"][i], st.Vm, f"Vm {i}")
+    z.close()
+
+
+FULL = [
+    ("opt1.3b_bf16_r16", (0, 4, 5, 143)),
+    ("llama7b_bf16_r32", (0, 4, 6, 223)),
+    ("dense32b_bf16_r64", (0, 1, 4, 6, 447)),
+]
+
+
+@pytest.mark.parametrize("name,sample", FULL, ids=[f[0] for f in FULL])
+def test_full_size_sampled_parity(lib, gpu, name, sample):
+    from paper_2608_15665_gb300 import workloads
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    wl = workloads.get(name)
+    weights = [workloads.init_weight(wl, i, gpu) for i in range(wl.n_mats)]
+    z = SubZeroPlus(weights, wl.r, wl.q, wl.seed)
+    z.init_subspace(0)
+    rs = np.random.default_rng(0)
+    rows = {i: np.sort(rs.choice(wl.shapes[i][0], size=min(192, wl.shapes[i][0]), replace=False))
+            for i in sample}
+
+    def grab(i):
+        idx = torch.from_numpy(rows[i]).to(gpu)
+        return to_f64(z.weights[i].index_select(0, idx))
+
+    torch.cuda.synchronize()
+    UV = {i: (to_f64(z.U[i]), to_f64(z.V[i])) for i in sample}
+    for i in sample:
+        m, n = wl.shapes[i]
+        U, V = haar.haar_proj(wl.seed, i, 0, m, n, wl.r)
+        assert np.max(np.abs(UV[i][0] - U)) <= UV_ABS, f"U of matrix {i}"
+        assert np.max(np.abs(UV[i][1] - V)) <= UV_ABS, f"V of matrix {i}"
+
+    # one fused perturbation pass (restore of query 0 + perturbation of query 1)
+    before = {i: grab(i) for i in sample}
+    z.perturb(0, 0, 1.0, 1, 1.0, wl.eps)
+    after = {i: grab(i) for i in sample}
+    for i in sample:
+        C = subzero.perturb_coeff(wl.seed, i, 0, wl.r, [(0, 1.0), (1, 1.0)], f32(wl.eps))
+        want = subzero.apply_pass(before[i], wl.dtype, UV[i][0], UV[i][1], C, rows=rows[i])
+        assert_weights(after[i], want, wl.dtype, f"{name} perturb, matrix {i}")
+
+    # the Adam step fused with the restore
+    losses = workloads.loss_table(wl, "central", steps=1)[0]
+    before = {i: grab(i) for i in sample}
+    z.step(0, 1, losses, "central", wl.eps, wl.lr, wl.beta1, wl.beta2, wl.eps_adam, wl.q - 1, 1.0)
+    after = {i: grab(i) for i in sample}
+    torch.cuda.synchronize()
+    for i in sample:
+        rho = subzero.rho_from_losses(losses, "central", f32(wl.eps), wl.q)
+        G = subzero.grad_G(wl.seed, i, 0, wl.r, rho)
+        M, Vm, D, _, _ = subzero.adam(np.zeros((wl.r, wl.r)), np.zeros((wl.r, wl.r)), G,
+                                      f32(wl.beta1), f32(wl.beta2), f32(wl.eps_adam), 1)
+        C = subzero.step_coeff(D, f32(wl.lr), f32(wl.eps), [(wl.q - 1, 1.0)], wl.seed, i, 0, wl.r)
+        want = subzero.apply_pass(before[i], wl.dtype, UV[i][0], UV[i][1], C, rows=rows[i])
+        assert_weights(after[i], want, wl.dtype, f"{name} step, matrix {i}")
+        assert_rel(to_f64(z.M[i]), M, f"M {i}")
+        assert_rel(to_f64(z.Vm[i]), Vm, f"Vm {i}")
+    z.sync()
+    z.close()
+    del weights, z
+    torch.cuda.empty_cache()
