@@ -242,10 +242,12 @@ def run_ours(args):
     from paper_2608_15665_gb300 import workloads
     from paper_2608_15665_gb300.schedule import SubZeroPlus, step_plan
 
-    wl0 = workloads.get(args.workload)
-    wl = workloads.scaled(wl0, seed=wl0.seed + 7919 * rank) if rank else wl0
-    weights = [workloads.init_weight(wl, i, dev) for i in range(wl.n_mats)]
-    z = SubZeroPlus(weights, wl.r, wl.q, wl.seed, matrix_index_base=rank * wl.n_mats)
+    wl0 = wl = workloads.get(args.workload)
+    part = workloads.partition(wl, rank, world)
+    weights = [workloads.init_weight(wl, i, dev, part["matrix_index_base"])
+               for i in range(wl.n_mats)]
+    z = SubZeroPlus(weights, wl.r, wl.q, part["seed"],
+                    matrix_index_base=part["matrix_index_base"])
     calls, (rq, rc) = step_plan(args.scheme, wl.q)
     passes = len(calls) + 1
     K, W = args.steps, args.warmup

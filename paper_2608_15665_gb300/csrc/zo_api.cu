@@ -11,6 +11,8 @@
 #include <string>
 #include <vector>
 
+#include <cudaTypedefs.h>
+
 #include "../../include/zo.h"
 #include "zo_kernels.h"
 
@@ -62,6 +64,17 @@ struct zo_ctx {
   int path_option = 0;
   int last_path = 0;
   int64_t launches = 0;          // kernels launched by this context
+  // tensor-core weight pass (all matrices bf16, r in {16, 32, 64})
+  bool tc_ok = false;
+  int sms = 0;
+  __nv_bfloat16* d_u_hl = nullptr;   // stacked [hi | lo] rows of every U_i, 128-row padded
+  __nv_bfloat16* d_p_hl = nullptr;   // stacked [hi | lo] rows of every P_i^T, 128-row padded
+  zo::TcMat* d_tc = nullptr;
+  int64_t tc_tiles = 0;
+  CUtensorMap* d_w_maps = nullptr;   // one TMA descriptor per W_i (device memory)
+  CUtensorMap tm_a{}, tm_b{};        // descriptors of the stacked operands (kernel parameters)
+  int2* d_u_units = nullptr;
+  int32_t n_u_units = 0;
   bool timing = false;
   std::vector<cudaEvent_t> ev_start, ev_stop;
   size_t ev_used = 0;
@@ -81,6 +94,11 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_qr_ws);
   cudaFree(c->d_qr_blocks);
   cudaFree(c->d_status);
+  cudaFree(c->d_u_hl);
+  cudaFree(c->d_p_hl);
+  cudaFree(c->d_tc);
+  cudaFree(c->d_w_maps);
+  cudaFree(c->d_u_units);
   for (auto e : c->ev_start) cudaEventDestroy(e);
   for (auto e : c->ev_stop) cudaEventDestroy(e);
   delete c;
@@ -172,16 +190,117 @@ zo_status record_stop(zo_ctx* c) {
 
 // Projection of C_i onto V_i and the weight pass, shared by zo_perturb and zo_step.
 zo_status run_weight_pass(zo_ctx* c) {
-  ZO_CUDA(zo::launch_project_fma(c->d_mats, c->d_proj_units, c->n_proj_units, c->r, c->stream),
-          "projection kernel");
+  const bool use_tc = c->tc_ok && c->path_option != 1;
+  if (use_tc) {
+    ZO_CUDA(zo::launch_project_split(c->d_mats, c->d_tc, c->d_proj_units, c->n_proj_units, c->r,
+                                     c->d_p_hl, c->stream),
+            "projection kernel");
+  } else {
+    ZO_CUDA(zo::launch_project_fma(c->d_mats, c->d_proj_units, c->n_proj_units, c->r, c->stream),
+            "projection kernel");
+  }
   ++c->launches;
   zo_status st = record_start(c);
   if (st != ZO_OK) return st;
-  ZO_CUDA(zo::launch_wpass_fma(c->d_mats, c->n_mats, c->d_tile_prefix, c->n_tiles, c->r, c->stream),
-          "weight-pass kernel");
+  if (use_tc) {
+    const int grid = (int)std::min<int64_t>(c->tc_tiles, c->sms);
+    ZO_CUDA(zo::launch_wpass_tc(c->tm_a, c->tm_b, c->d_w_maps, c->d_tc, c->n_mats, c->tc_tiles,
+                                grid, c->r, c->d_status, c->stream),
+            "tensor-core weight-pass kernel");
+    c->last_path = 2;
+  } else {
+    ZO_CUDA(zo::launch_wpass_fma(c->d_mats, c->n_mats, c->d_tile_prefix, c->n_tiles, c->r,
+                                 c->stream),
+            "weight-pass kernel");
+    c->last_path = 1;
+  }
   ++c->launches;
-  c->last_path = 1;
   return record_stop(c);
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor map: `cols` contiguous elements per row, `rows` rows `row_bytes` apart,
+// boxes of box_cols x box_rows with the 128-byte swizzle.
+bool encode_bf16_2d(CUtensorMap* tm, void* base, uint64_t cols, uint64_t rows, uint64_t row_bytes,
+                    uint32_t box_cols, uint32_t box_rows) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {row_bytes};
+  const cuuint32_t box[2] = {box_cols, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Buffers and descriptors of the tensor-core weight pass; leaves tc_ok false when
+// the context does not qualify (an fp32 matrix, or r outside {16, 32, 64}).
+zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
+  if (!zo::wpass_tc_supported(c->r)) return ZO_OK;
+  for (int32_t i = 0; i < c->n_mats; ++i)
+    if (mats[i].dtype != ZO_BF16) return ZO_OK;
+  const int64_t BM = zo::tc_tile_rows(), BN = zo::tc_tile_cols();
+  const int64_t HLW = zo::tc_hl_width(c->r);
+  std::vector<zo::TcMat> tc(c->n_mats);
+  std::vector<int2> uunits;
+  int64_t urows = 0, prows = 0, tiles = 0;
+  for (int32_t i = 0; i < c->n_mats; ++i) {
+    const int64_t m = mats[i].m, n = mats[i].n;
+    tc[i].m = m;
+    tc[i].n = n;
+    tc[i].tile0 = tiles;
+    tc[i].tiles_n = (int32_t)((n + BN - 1) / BN);
+    tc[i].u_row0 = (int32_t)urows;
+    tc[i].p_row0 = (int32_t)prows;
+    tc[i].pad = 0;
+    tiles += ((m + BM - 1) / BM) * tc[i].tiles_n;
+    urows += (m + BM - 1) / BM * BM;
+    prows += (n + BN - 1) / BN * BN;
+    for (int64_t r0 = 0; r0 < m; r0 += 128) uunits.push_back(make_int2(i, (int)r0));
+  }
+  if (urows >= (int64_t(1) << 31) || prows >= (int64_t(1) << 31)) return ZO_OK;
+  ZO_CUDA(cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, c->device), "SM count");
+  ZO_CUDA(cudaMalloc(&c->d_u_hl, sizeof(__nv_bfloat16) * urows * HLW), "cudaMalloc(U hi/lo)");
+  ZO_CUDA(cudaMalloc(&c->d_p_hl, sizeof(__nv_bfloat16) * prows * HLW), "cudaMalloc(P hi/lo)");
+  ZO_CUDA(cudaMemset(c->d_u_hl, 0, sizeof(__nv_bfloat16) * urows * HLW), "memset");
+  ZO_CUDA(cudaMemset(c->d_p_hl, 0, sizeof(__nv_bfloat16) * prows * HLW), "memset");
+  ZO_CUDA(cudaMalloc(&c->d_tc, sizeof(zo::TcMat) * c->n_mats), "cudaMalloc(tile table)");
+  ZO_CUDA(cudaMemcpy(c->d_tc, tc.data(), sizeof(zo::TcMat) * c->n_mats, cudaMemcpyHostToDevice),
+          "upload tile table");
+  ZO_CUDA(cudaMalloc(&c->d_u_units, sizeof(int2) * uunits.size()), "cudaMalloc(units)");
+  ZO_CUDA(cudaMemcpy(c->d_u_units, uunits.data(), sizeof(int2) * uunits.size(),
+                     cudaMemcpyHostToDevice),
+          "upload units");
+  c->n_u_units = (int32_t)uunits.size();
+  std::vector<CUtensorMap> wmaps(c->n_mats);
+  bool ok = encode_bf16_2d(&c->tm_a, c->d_u_hl, HLW, urows, HLW * 2, 64, 128) &&
+            encode_bf16_2d(&c->tm_b, c->d_p_hl, HLW, prows, HLW * 2, 64, 128);
+  for (int32_t i = 0; ok && i < c->n_mats; ++i)
+    ok = encode_bf16_2d(&wmaps[i], mats[i].W, mats[i].n, mats[i].m, mats[i].ldw * 2, 64, 32);
+  if (!ok) {
+    g_last_error = "cuTensorMapEncodeTiled unavailable or rejected a descriptor; using the FMA pass";
+    return ZO_OK;
+  }
+  ZO_CUDA(cudaMalloc(&c->d_w_maps, sizeof(CUtensorMap) * c->n_mats), "cudaMalloc(tensor maps)");
+  ZO_CUDA(cudaMemcpy(c->d_w_maps, wmaps.data(), sizeof(CUtensorMap) * c->n_mats,
+                     cudaMemcpyHostToDevice),
+          "upload tensor maps");
+  c->tc_tiles = tiles;
+  c->tc_ok = true;
+  return ZO_OK;
 }
 
 }  // namespace
@@ -354,6 +473,13 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
     cuda_fail(e, "zo_create upload");
     return fail(ZO_ERR_CUDA);
   }
+  zo_status st = setup_tc(c, mats);
+  if (st != ZO_OK) return fail(st);
+  e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    cuda_fail(e, "zo_create tensor-core setup");
+    return fail(ZO_ERR_CUDA);
+  }
   *out = c;
   return ZO_OK;
 }
@@ -385,6 +511,12 @@ zo_status zo_refresh(zo_ctx* c, uint32_t refresh_idx, int32_t reset_moments) {
   }
   if (reset_moments) {
     ZO_CUDA(zo::launch_zero_moments(c->d_mats, c->n_mats, c->r, c->stream), "zero moments");
+    ++c->launches;
+  }
+  if (c->tc_ok) {
+    ZO_CUDA(zo::launch_split_u(c->d_mats, c->d_tc, c->d_u_units, c->n_u_units, c->r, c->d_u_hl,
+                               c->stream),
+            "split U into hi/lo");
     ++c->launches;
   }
   return ZO_OK;
@@ -498,8 +630,8 @@ zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
   if (!c) return ZO_ERR_INVALID_ARG;
   if (option == ZO_OPTION_WPASS_PATH) {
     if (value < 0 || value > 2) return ZO_ERR_INVALID_ARG;
-    if (value == 2) {
-      g_last_error = "tcgen05 weight pass not available in this build";
+    if (value == 2 && !c->tc_ok) {
+      g_last_error = "the tensor-core weight pass needs every W in bf16 and r in {16, 32, 64}";
       return ZO_ERR_UNSUPPORTED;
     }
     c->path_option = (int)value;

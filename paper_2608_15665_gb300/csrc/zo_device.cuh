@@ -90,11 +90,17 @@ struct MatDesc {
   float* Vm;        // r x r second moment
   float* C;         // r x r coefficient of the current pass (workspace)
   float* P;         // FMA path: r x n, P = C V^T (workspace)
-  __nv_bfloat16* Pt_hi;  // tcgen05 path: n x r, hi/lo bf16 split of P^T (workspace)
-  __nv_bfloat16* Pt_lo;
-  __nv_bfloat16* U_hi;   // tcgen05 path: m x r, hi/lo bf16 split of U (workspace)
-  __nv_bfloat16* U_lo;
   int64_t tile0;    // first weight-pass tile of this matrix (FMA path)
+};
+
+// Per-matrix record of the tensor-core weight pass (128 x 128 tiles).
+struct TcMat {
+  int64_t m, n;
+  int64_t tile0;     // first tile of this matrix
+  int32_t tiles_n;   // column tiles
+  int32_t u_row0;    // first row of this matrix in the stacked hi/lo U operand
+  int32_t p_row0;    // first row of this matrix in the stacked hi/lo P^T operand
+  int32_t pad;
 };
 
 // One block of the batched TSQR used by the refresh (see zo_qr.cu).

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include "zo_device.cuh"
@@ -43,13 +44,6 @@ cudaError_t launch_coeff(const MatDesc* d_mats, int32_t n_mats, const CoeffParam
 cudaError_t launch_project_fma(const MatDesc* d_mats, const int2* d_units, int32_t n_units,
                                int32_t r, cudaStream_t s);
 
-// Pt_i = V_i C_i^T (n x r) split into bf16 hi + lo for the tensor-core pass.
-cudaError_t launch_project_split(const MatDesc* d_mats, const int2* d_units, int32_t n_units,
-                                 int32_t r, cudaStream_t s);
-
-// U_i split into bf16 hi + lo (after a refresh) for the tensor-core pass.
-cudaError_t launch_split_u(const MatDesc* d_mats, const int2* d_units, int32_t n_units, int32_t r,
-                           cudaStream_t s);
 
 // ---- weight pass, fp32 FMA path (zo_wpass_fma.cu) ---------------------------
 constexpr int kFmaTileRows = 32;
@@ -60,6 +54,19 @@ cudaError_t launch_wpass_fma(const MatDesc* d_mats, int32_t n_mats, const int64_
 
 // ---- weight pass, tcgen05 path (zo_wpass_tc.cu) --------------------------------
 bool wpass_tc_supported(int32_t r);
+int32_t tc_hl_width(int32_t r);   // bf16 elements per hi/lo operand row
+int32_t tc_tile_rows();
+int32_t tc_tile_cols();
+// U_HL rows of every matrix from U (after a refresh); units = (matrix, first row) x 128 rows
+cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                           int32_t n_units, int32_t r, __nv_bfloat16* u_hl, cudaStream_t s);
+// Pt_HL rows: hi/lo of (C V^T)^T; units = (matrix, first column) x 128 columns
+cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                                 int32_t n_units, int32_t r, __nv_bfloat16* p_hl, cudaStream_t s);
+cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
+                            const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
+                            int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
+                            cudaStream_t s);
 
 // ---- refresh: batched TSQR + sign correction (zo_qr.cu) ------------------------
 int32_t qr_block_rows(int32_t r);

@@ -1,0 +1,467 @@
+// Weight pass on the 5th-generation tensor cores: W_i <- rnd_bf16(W_i + U_i P_i)
+// for every bf16 matrix in one persistent launch (the fused form of Alg. 2's
+// "W_i <- W_i + eps U_i Z_i V_i^T", Eq. (4), and of the update of Eq. (10)).
+//
+// The contraction U (128 x r) . P (r x 128) of a 128 x 128 tile is r-deep, so it
+// costs 2r flops per weight against 4 bytes of HBM traffic; past r = 16 that is
+// more than the fp32 FMA pipes deliver at HBM speed, so it runs on tcgen05.mma.
+// To keep fp32-grade accuracy of the update with bf16 tensor-core inputs, both
+// operands are split x = hi + lo (hi = bf16(x), lo = bf16(x - hi)) and the tile
+// accumulates hi.hi + hi.lo + lo.hi in fp32 in Tensor Memory (relative error of
+// the product ~2^-16 instead of 2^-8).
+//
+// Roles of the 192 threads of a CTA (one CTA per SM, persistent over a
+// contiguous range of tiles ordered row block by row block):
+//   warp 0, lane 0: TMA producer -- W tile (8 boxes of 32 rows x 64 columns,
+//                   128-byte swizzle), the U operand tile when the row block
+//                   changes, the P operand tile of every column block.
+//   warp 1, lane 0: MMA issuer -- 3 * r/16 tcgen05.mma (M=128, N=128, K=16) per
+//                   tile into one of two TMEM accumulators; warp 1 also owns
+//                   the TMEM allocation.
+//   warps 2..5:     epilogue -- each warp owns 32 rows (its TMEM lane group):
+//                   tcgen05.ld the fp32 update, add it to the W rows in shared
+//                   memory, round to bf16 in place, TMA-store its rows.
+// Every mbarrier wait is bounded; on expiry the kernel records kDevTimeout in
+// the status word, lets the other roles stop, drains its copies and frees TMEM.
+#include <cuda.h>
+
+#include "zo_kernels.h"
+#include "zo_sm100.cuh"
+
+namespace zo {
+namespace {
+
+using namespace sm100;
+
+constexpr int kBM = 128;            // tile rows (TMEM lanes)
+constexpr int kBN = 128;            // tile columns (TMEM columns per accumulator)
+constexpr int kThreads = 192;
+constexpr int kWBoxBytes = 32 * 64 * 2;          // one TMA box of W: 32 rows x 64 bf16
+constexpr int kWStageBytes = kBM * kBN * 2;      // 32 KB
+constexpr int kPanelBytes = kBM * 64 * 2;        // 128 rows x 128 bytes = 16 KB
+constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz
+
+__host__ __device__ constexpr int hl_width(int r) { return 2 * r > 64 ? 2 * r : 64; }
+
+template <int R>
+struct TcCfg {
+  static constexpr int kHLW = hl_width(R);
+  static constexpr int kPanels = kHLW / 64;
+  static constexpr int kOpBytes = kPanels * kPanelBytes;        // one operand tile (hi + lo)
+  static constexpr int kWStages = R >= 64 ? 3 : 4;
+  static constexpr int kAStages = R >= 64 ? 1 : 2;
+  static constexpr int kBStages = 2;
+  static constexpr int kKC = R / 16;                            // K chunks of 16
+  static constexpr size_t kSmem = (size_t)kWStages * kWStageBytes + (size_t)kAStages * kOpBytes +
+                                  (size_t)kBStages * kOpBytes + 1024 /*barriers*/ + 1024 /*align*/;
+};
+
+struct Shared {
+  uint64_t w_full[4], w_empty[4];
+  uint64_t a_full[2], a_empty[2];
+  uint64_t b_full[2], b_empty[2];
+  uint64_t acc_full[2], acc_empty[2];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+// Walks the tiles [t, t_end) of this CTA in order: matrix, row block, column block.
+struct TileIter {
+  const TcMat* mats;
+  int64_t t, t_end;
+  int i;
+  int64_t rb, cb, tiles_m;
+  __device__ void init(const TcMat* m, int n_mats, int64_t t0, int64_t t1) {
+    mats = m;
+    t = t0;
+    t_end = t1;
+    int lo = 0, hi = n_mats - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (mats[mid].tile0 <= t0) lo = mid; else hi = mid - 1;
+    }
+    i = lo;
+    set_local();
+  }
+  __device__ void set_local() {
+    if (t >= t_end) return;
+    const int64_t local = t - mats[i].tile0;
+    rb = local / mats[i].tiles_n;
+    cb = local % mats[i].tiles_n;
+    tiles_m = (mats[i].m + kBM - 1) / kBM;
+  }
+  __device__ bool valid() const { return t < t_end; }
+  __device__ void next() {
+    ++t;
+    if (t >= t_end) return;
+    if (++cb == mats[i].tiles_n) {
+      cb = 0;
+      if (++rb == tiles_m) {
+        ++i;
+        rb = 0;
+        tiles_m = (mats[i].m + kBM - 1) / kBM;
+      }
+    }
+  }
+};
+
+// index of the last of n_issued ring entries that went into slot s (ring of S slots), or -1
+__device__ __forceinline__ int64_t last_in_slot(int64_t n_issued, int s, int S) {
+  if (n_issued <= s) return -1;
+  return s + (int64_t)S * ((n_issued - 1 - s) / S);
+}
+
+__device__ __forceinline__ void give_up(Shared& sh, uint32_t* status) {
+  atomicOr(status, (uint32_t)kDevTimeout);
+  *reinterpret_cast<volatile int*>(&sh.abort_flag) = 1;
+}
+
+template <int R>
+__global__ void __launch_bounds__(kThreads, 1)
+wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
+                const CUtensorMap* __restrict__ w_maps, const TcMat* __restrict__ mats, int n_mats,
+                int64_t n_tiles, uint32_t* __restrict__ status) {
+  using Cfg = TcCfg<R>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* w_smem = smem;
+  uint8_t* a_smem = w_smem + Cfg::kWStages * kWStageBytes;
+  uint8_t* b_smem = a_smem + Cfg::kAStages * Cfg::kOpBytes;
+  Shared& sh = *reinterpret_cast<Shared*>(b_smem + Cfg::kBStages * Cfg::kOpBytes);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t G = gridDim.x;
+  const int64_t t_begin = (int64_t)blockIdx.x * n_tiles / G;
+  const int64_t t_end = ((int64_t)blockIdx.x + 1) * n_tiles / G;
+  const volatile int* abort = &sh.abort_flag;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < Cfg::kWStages; ++s) {
+      mbar_init(&sh.w_full[s], 1);
+      mbar_init(&sh.w_empty[s], 4);
+    }
+    for (int s = 0; s < Cfg::kAStages; ++s) {
+      mbar_init(&sh.a_full[s], 1);
+      mbar_init(&sh.a_empty[s], 1);
+    }
+    for (int s = 0; s < Cfg::kBStages; ++s) {
+      mbar_init(&sh.b_full[s], 1);
+      mbar_init(&sh.b_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sh.acc_full[s], 1);
+      mbar_init(&sh.acc_empty[s], 4);
+    }
+    sh.abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tm_a);
+    prefetch_tmap(&tm_b);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sh.tmem_base, 2 * kBN);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sh.tmem_base;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------ TMA producer
+    int64_t n_w = 0, n_a = 0, n_b = 0;          // copies issued into each ring
+    int prev_i = -1;
+    int64_t prev_rb = -1;
+    bool ok = true;
+    TileIter ti;
+    ti.init(mats, n_mats, t_begin, t_end);
+    for (; ti.valid(); ti.next()) {
+      const TcMat& mt = mats[ti.i];
+      const CUtensorMap* wmap = w_maps + ti.i;
+      // W tile: 4 row groups x 2 column halves
+      {
+        const int s = (int)(n_w % Cfg::kWStages);
+        const uint32_t ph = (uint32_t)((n_w / Cfg::kWStages) & 1);
+        if (!mbar_wait_bounded(&sh.w_empty[s], ph ^ 1u, abort, kWaitCycles)) { ok = false; break; }
+        mbar_arrive_expect_tx(&sh.w_full[s], kWStageBytes);
+        uint8_t* dst = w_smem + s * kWStageBytes;
+        for (int g = 0; g < 4; ++g)
+          for (int h = 0; h < 2; ++h)
+            tma_load_2d(dst + (g * 2 + h) * kWBoxBytes, wmap, (int)(ti.cb * kBN + 64 * h),
+                        (int)(ti.rb * kBM + 32 * g), &sh.w_full[s]);
+        ++n_w;
+      }
+      // U operand tile, once per row block
+      if (ti.i != prev_i || ti.rb != prev_rb) {
+        const int s = (int)(n_a % Cfg::kAStages);
+        const uint32_t ph = (uint32_t)((n_a / Cfg::kAStages) & 1);
+        if (!mbar_wait_bounded(&sh.a_empty[s], ph ^ 1u, abort, kWaitCycles)) { ok = false; break; }
+        mbar_arrive_expect_tx(&sh.a_full[s], Cfg::kOpBytes);
+        for (int p = 0; p < Cfg::kPanels; ++p)
+          tma_load_2d(a_smem + s * Cfg::kOpBytes + p * kPanelBytes, &tm_a, 64 * p,
+                      (int)(mt.u_row0 + ti.rb * kBM), &sh.a_full[s]);
+        ++n_a;
+        prev_i = ti.i;
+        prev_rb = ti.rb;
+      }
+      // P operand tile of this column block
+      {
+        const int s = (int)(n_b % Cfg::kBStages);
+        const uint32_t ph = (uint32_t)((n_b / Cfg::kBStages) & 1);
+        if (!mbar_wait_bounded(&sh.b_empty[s], ph ^ 1u, abort, kWaitCycles)) { ok = false; break; }
+        mbar_arrive_expect_tx(&sh.b_full[s], Cfg::kOpBytes);
+        for (int p = 0; p < Cfg::kPanels; ++p)
+          tma_load_2d(b_smem + s * Cfg::kOpBytes + p * kPanelBytes, &tm_b, 64 * p,
+                      (int)(mt.p_row0 + ti.cb * kBN), &sh.b_full[s]);
+        ++n_b;
+      }
+    }
+    if (!ok) give_up(sh, status);
+    // drain: the last copy issued into every slot has landed before the CTA exits
+    for (int s = 0; s < Cfg::kWStages; ++s) {
+      const int64_t k = last_in_slot(n_w, s, Cfg::kWStages);
+      if (k >= 0) mbar_wait_bounded(&sh.w_full[s], (uint32_t)((k / Cfg::kWStages) & 1), nullptr, kWaitCycles);
+    }
+    for (int s = 0; s < Cfg::kAStages; ++s) {
+      const int64_t k = last_in_slot(n_a, s, Cfg::kAStages);
+      if (k >= 0) mbar_wait_bounded(&sh.a_full[s], (uint32_t)((k / Cfg::kAStages) & 1), nullptr, kWaitCycles);
+    }
+    for (int s = 0; s < Cfg::kBStages; ++s) {
+      const int64_t k = last_in_slot(n_b, s, Cfg::kBStages);
+      if (k >= 0) mbar_wait_bounded(&sh.b_full[s], (uint32_t)((k / Cfg::kBStages) & 1), nullptr, kWaitCycles);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------------------ MMA issuer
+    constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN);
+    int64_t it = 0, a_it = 0;
+    int prev_i = -1;
+    int64_t prev_rb = -1;
+    int sa = 0;
+    bool ok = true;
+    TileIter ti;
+    ti.init(mats, n_mats, t_begin, t_end);
+    for (; ti.valid(); ti.next(), ++it) {
+      if (ti.i != prev_i || ti.rb != prev_rb) {
+        if (a_it > 0) mma_commit(&sh.a_empty[(a_it - 1) % Cfg::kAStages]);
+        sa = (int)(a_it % Cfg::kAStages);
+        if (!mbar_wait_bounded(&sh.a_full[sa], (uint32_t)((a_it / Cfg::kAStages) & 1), abort,
+                               kWaitCycles)) { ok = false; break; }
+        ++a_it;
+        prev_i = ti.i;
+        prev_rb = ti.rb;
+      }
+      const int sb = (int)(it % Cfg::kBStages);
+      if (!mbar_wait_bounded(&sh.b_full[sb], (uint32_t)((it / Cfg::kBStages) & 1), abort,
+                             kWaitCycles)) { ok = false; break; }
+      const int acc = (int)(it & 1);
+      if (!mbar_wait_bounded(&sh.acc_empty[acc], (uint32_t)(((it >> 1) & 1) ^ 1), abort,
+                             kWaitCycles)) { ok = false; break; }
+      tc_fence_after();
+      const uint32_t d = tmem + (uint32_t)(acc * kBN);
+      const uint32_t a_base = smem_u32(a_smem + sa * Cfg::kOpBytes);
+      const uint32_t b_base = smem_u32(b_smem + sb * Cfg::kOpBytes);
+#pragma unroll
+      for (int kk = 0; kk < Cfg::kKC; ++kk) {
+        // hi chunk kk at element 16 kk of the operand row, lo chunk at R + 16 kk
+        const int e_hi = 16 * kk, e_lo = R + 16 * kk;
+        const uint32_t off_hi = (uint32_t)((e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
+        const uint32_t off_lo = (uint32_t)((e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
+        const uint64_t a_hi = sdesc_k_sw128(a_base + off_hi), a_lo = sdesc_k_sw128(a_base + off_lo);
+        const uint64_t b_hi = sdesc_k_sw128(b_base + off_hi), b_lo = sdesc_k_sw128(b_base + off_lo);
+        mma_bf16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
+        mma_bf16(d, a_hi, b_lo, idesc, 1u);
+        mma_bf16(d, a_lo, b_hi, idesc, 1u);
+      }
+      mma_commit(&sh.b_empty[sb]);
+      mma_commit(&sh.acc_full[acc]);
+    }
+    if (!ok) give_up(sh, status);
+    if (it > 0) {
+      // every MMA issued by this thread has completed before TMEM is released
+      const int64_t last = it - 1;
+      mbar_wait_bounded(&sh.acc_full[last & 1], (uint32_t)((last >> 1) & 1), nullptr, kWaitCycles);
+    }
+  } else if (warp >= 2) {
+    // ------------------------------------------------------------ epilogue
+    const int g = warp & 3;                      // TMEM lane group == tile row group
+    const uint32_t lane_base = (uint32_t)(g * 32) << 16;
+    int64_t it = 0;
+    bool ok = true;
+    TileIter ti;
+    ti.init(mats, n_mats, t_begin, t_end);
+    for (; ti.valid(); ti.next(), ++it) {
+      const TcMat& mt = mats[ti.i];
+      const int acc = (int)(it & 1);
+      if (!mbar_wait_bounded(&sh.acc_full[acc], (uint32_t)((it >> 1) & 1), abort, kWaitCycles)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const int s = (int)(it % Cfg::kWStages);
+      if (!mbar_wait_bounded(&sh.w_full[s], (uint32_t)((it / Cfg::kWStages) & 1), abort,
+                             kWaitCycles)) {
+        ok = false;
+        break;
+      }
+      uint8_t* stage = w_smem + s * kWStageBytes;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * kBN + c * 32), v);
+        tmem_ld_wait();
+        uint8_t* box = stage + (g * 2 + (c >> 1)) * kWBoxBytes + lane * 128;
+#pragma unroll
+        for (int j4 = 0; j4 < 4; ++j4) {
+          const int j = (c & 1) * 4 + j4;                       // logical 16-byte chunk
+          uint4* p = reinterpret_cast<uint4*>(box + ((j ^ (lane & 7)) << 4));
+          uint4 raw = *p;
+          uint32_t wv[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float lo = __uint_as_float(wv[e] << 16) + __uint_as_float(v[j4 * 8 + 2 * e]);
+            const float hi = __uint_as_float(wv[e] & 0xFFFF0000u) +
+                             __uint_as_float(v[j4 * 8 + 2 * e + 1]);
+            const __nv_bfloat162 h2 = __floats2bfloat162_rn(lo, hi);
+            wv[e] = *reinterpret_cast<const uint32_t*>(&h2);
+          }
+          *p = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sh.acc_empty[acc]);
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        const int64_t y = ti.rb * kBM + 32 * g;
+        if (y < mt.m) {
+          for (int h = 0; h < 2; ++h) {
+            const int64_t x = ti.cb * kBN + 64 * h;
+            if (x < mt.n)
+              tma_store_2d(w_maps + ti.i, (int)x, (int)y, stage + (g * 2 + h) * kWBoxBytes);
+          }
+        }
+        bulk_commit();
+        bulk_wait_read_all();
+        mbar_arrive(&sh.w_empty[s]);
+      }
+      __syncwarp();
+    }
+    if (!ok && lane == 0) give_up(sh, status);
+    if (lane == 0) bulk_wait_all();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 2 * kBN);
+  }
+}
+
+// U_HL[u_row0 + i] = [bf16 hi(U[i, :]) | bf16 lo(U[i, :]) | 0 ...]  (row width hl_width(R))
+template <int R>
+__global__ void split_u_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
+                               const int2* __restrict__ units, __nv_bfloat16* __restrict__ u_hl) {
+  const int2 u = units[blockIdx.x];
+  const MatDesc md = mats[u.x];
+  const int64_t row = (int64_t)u.y + threadIdx.x;
+  if (row >= md.m) return;
+  const float* src = md.U + row * R;
+  __nv_bfloat16* dst = u_hl + ((int64_t)tcm[u.x].u_row0 + row) * hl_width(R);
+#pragma unroll
+  for (int c = 0; c < R; ++c) {
+    const float x = src[c];
+    const __nv_bfloat16 h = __float2bfloat16_rn(x);
+    dst[c] = h;
+    dst[R + c] = __float2bfloat16_rn(x - __bfloat162float(h));
+  }
+}
+
+// Pt_HL[p_row0 + j] = [hi | lo] of P^T[j, :] = (C V^T)^T[j, :] = V[j, :] C^T
+template <int R>
+__global__ void __launch_bounds__(128)
+project_split_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
+                     const int2* __restrict__ units, __nv_bfloat16* __restrict__ p_hl) {
+  __shared__ float Cs[R * R];
+  const int2 u = units[blockIdx.x];
+  const MatDesc md = mats[u.x];
+  for (int e = threadIdx.x; e < R * R; e += blockDim.x) Cs[e] = md.C[e];
+  __syncthreads();
+  const int64_t j = (int64_t)u.y + threadIdx.x;
+  if (j >= md.n) return;
+  float v[R];
+  const float4* vrow = reinterpret_cast<const float4*>(md.V + j * R);
+#pragma unroll
+  for (int b = 0; b < R / 4; ++b) {
+    const float4 t = vrow[b];
+    v[4 * b] = t.x; v[4 * b + 1] = t.y; v[4 * b + 2] = t.z; v[4 * b + 3] = t.w;
+  }
+  __nv_bfloat16* dst = p_hl + ((int64_t)tcm[u.x].p_row0 + j) * hl_width(R);
+  for (int a = 0; a < R; ++a) {
+    float acc = 0.f;
+#pragma unroll
+    for (int b = 0; b < R; ++b) acc = fmaf(Cs[a * R + b], v[b], acc);
+    const __nv_bfloat16 h = __float2bfloat16_rn(acc);
+    dst[a] = h;
+    dst[R + a] = __float2bfloat16_rn(acc - __bfloat162float(h));
+  }
+}
+
+template <int R>
+cudaError_t launch_tc_r(const CUtensorMap& tm_a, const CUtensorMap& tm_b, const CUtensorMap* w_maps,
+                        const TcMat* mats, int n_mats, int64_t n_tiles, int grid, uint32_t* status,
+                        cudaStream_t s) {
+  const size_t smem = TcCfg<R>::kSmem;
+  cudaError_t e = cudaFuncSetAttribute(wpass_tc_kernel<R>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  wpass_tc_kernel<R><<<grid, kThreads, smem, s>>>(tm_a, tm_b, w_maps, mats, n_mats, n_tiles, status);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool wpass_tc_supported(int32_t r) { return r == 16 || r == 32 || r == 64; }
+int32_t tc_hl_width(int32_t r) { return hl_width(r); }
+int32_t tc_tile_rows() { return kBM; }
+int32_t tc_tile_cols() { return kBN; }
+
+cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                           int32_t n_units, int32_t r, __nv_bfloat16* u_hl, cudaStream_t s) {
+  if (n_units <= 0) return cudaSuccess;
+  switch (r) {
+    case 16: split_u_kernel<16><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, u_hl); break;
+    case 32: split_u_kernel<32><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, u_hl); break;
+    case 64: split_u_kernel<64><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, u_hl); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                                 int32_t n_units, int32_t r, __nv_bfloat16* p_hl, cudaStream_t s) {
+  if (n_units <= 0) return cudaSuccess;
+  switch (r) {
+    case 16: project_split_kernel<16><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, p_hl); break;
+    case 32: project_split_kernel<32><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, p_hl); break;
+    case 64: project_split_kernel<64><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, p_hl); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
+                            const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
+                            int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
+                            cudaStream_t s) {
+  if (n_tiles <= 0) return cudaSuccess;
+  switch (r) {
+    case 16: return launch_tc_r<16>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, s);
+    case 32: return launch_tc_r<32>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, s);
+    case 64: return launch_tc_r<64>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace zo

@@ -120,15 +120,28 @@ def loss_table(wl, scheme, steps=None, start=0):
     return np.stack(rows) if rows else np.zeros((0, n), np.float32)
 
 
-def init_weight(wl, i, device="cpu"):
-    """Initial W_i: N(0, 0.02^2) in the workload dtype (zero for LoRA B), via torch's generator."""
+def partition(wl, rank, world):
+    """Layer partition of a `world`-times larger parameter set: rank `rank` owns the
+    global matrix indices [rank * n_mats, (rank + 1) * n_mats) with this workload's
+    shapes.  Every rank uses the same Philox seed; the global index alone selects the
+    random streams, so the split changes no Z or Omega.  No data crosses ranks."""
+    if not 0 <= rank < world:
+        raise ValueError("rank out of range")
+    base = rank * wl.n_mats
+    return {"matrix_index_base": base, "global_indices": range(base, base + wl.n_mats),
+            "seed": wl.seed}
+
+
+def init_weight(wl, i, device="cpu", index_base=0):
+    """Initial W_i: N(0, 0.02^2) in the workload dtype (zero for LoRA B), via torch's
+    generator, seeded by the global matrix index index_base + i."""
     import torch
     m, n = wl.shapes[i]
     dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
     if i in wl.zero_init:
         return torch.zeros(m, n, dtype=dt, device=device)
     g = torch.Generator(device=device)
-    g.manual_seed(wl.seed * 100003 + i)
+    g.manual_seed(wl.seed * 100003 + index_base + i)
     w = torch.randn(m, n, generator=g, device=device, dtype=torch.float32)
     return w.mul_(0.02).to(dt)
 

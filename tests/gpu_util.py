@@ -4,7 +4,7 @@ import numpy as np
 import torch
 
 from oracle import subzero
-from parity import to_f64
+from parity import to_f64, update_terms
 
 
 def make_weight(m, n, dtype, seed, device, ldw=None, scale=0.02):
@@ -41,8 +41,11 @@ def f32(x):
 
 
 def oracle_perturb(before, i, dtype, seed, gidx, t, r, terms, eps):
+    """Expected W after a perturbation pass, and the (T, TZ) operand scale of the update."""
     C = subzero.perturb_coeff(seed, gidx, t, r, terms, f32(eps))
-    return subzero.apply_pass(before["W"][i], dtype, before["U"][i], before["V"][i], C)
+    W = subzero.apply_pass(before["W"][i], dtype, before["U"][i], before["V"][i], C)
+    zc = abs(f32(eps)) * sum(abs(c) for _, c in terms)
+    return W, update_terms(before["U"][i], C, before["V"][i], zc)
 
 
 def oracle_step(before, i, dtype, seed, gidx, t, r, q, losses, scheme, eps, lr, beta1, beta2,
@@ -56,4 +59,5 @@ def oracle_step(before, i, dtype, seed, gidx, t, r, q, losses, scheme, eps, lr, 
         M, Vm, D = before["M"][i], before["Vm"][i], subzero.sgd_direction(G)
     C = subzero.step_coeff(D, f32(lr), f32(eps), restore_terms, seed, gidx, t, r)
     W = subzero.apply_pass(before["W"][i], dtype, before["U"][i], before["V"][i], C)
-    return W, M, Vm, G
+    zc = abs(f32(eps)) * sum(abs(c) for _, c in restore_terms)
+    return W, M, Vm, G, update_terms(before["U"][i], C, before["V"][i], zc)

@@ -3,7 +3,7 @@
 Each test reads the library's state before a call (W, U, V, M, Vm), lets the
 oracle compute the call exactly in fp64 from that state, and compares:
 bf16 weights within 1 ulp of the oracle's rounded result, fp32 weights and the
-Adam moments within relative 1e-5 (floored at 1e-3 of the largest entry).
+Adam moments within relative 1e-5, both at the scale of the operands (tests/parity.py).
 """
 
 import numpy as np
@@ -11,7 +11,8 @@ import pytest
 import torch
 
 from gpu_util import dtype_of, f32, make_weight, oracle_perturb, oracle_step, snapshot
-from parity import assert_rel, assert_weights
+from oracle import rounding, subzero
+from parity import assert_moments, assert_weights, gabs, to_f64
 
 pytestmark = pytest.mark.gpu
 
@@ -46,8 +47,9 @@ def test_perturb_pass_matches_oracle(lib, gpu, case, eps):
         after = snapshot(z)
         terms = [(qa, ca)] + ([(qb, cb)] if qb >= 0 else [])
         for i, W in enumerate(z.weights):
-            want = oracle_perturb(before, i, dtype_of(W), z.seed, base + i, t, z.r, terms, eps)
-            assert_weights(after["W"][i], want, dtype_of(W), f"{case} matrix {i} t={t}")
+            want, T = oracle_perturb(before, i, dtype_of(W), z.seed, base + i, t, z.r, terms, eps)
+            assert_weights(after["W"][i], want, dtype_of(W), f"{case} matrix {i} t={t}",
+                           before=before["W"][i], terms=T)
     z.sync()
     z.close()
 
@@ -72,13 +74,16 @@ def test_step_matches_oracle(lib, gpu, case, scheme):
         after = snapshot(z)
         g = gamma.cpu().double().numpy()
         rterms = [restore] if restore[0] >= 0 else []
+        rho = subzero.rho_from_losses(losses, scheme, f32(eps), q)
         for i, W in enumerate(z.weights):
-            Wo, Mo, Vmo, G = oracle_step(before, i, dtype_of(W), z.seed, base + i, t, z.r, q,
-                                         losses, scheme, eps, lr, b1, b2, ea, step + 1, rterms)
-            assert_rel(after["M"][i], Mo, f"M {case} {i}")
-            assert_rel(after["Vm"][i], Vmo, f"Vm {case} {i}")
-            assert_weights(after["W"][i], Wo, dtype_of(W), f"W {case} {i} step {step}")
-            assert abs(g[i] - np.linalg.norm(G)) <= 1e-5 * np.linalg.norm(G)
+            Wo, Mo, Vmo, G, T = oracle_step(before, i, dtype_of(W), z.seed, base + i, t, z.r, q,
+                                            losses, scheme, eps, lr, b1, b2, ea, step + 1, rterms)
+            ga = gabs(z.seed, base + i, t, z.r, rho)
+            assert_moments(after["M"][i], after["Vm"][i], Mo, Vmo, before["M"][i],
+                           before["Vm"][i], ga, b1, b2, f"{case} {i}")
+            assert_weights(after["W"][i], Wo, dtype_of(W), f"W {case} {i} step {step}",
+                           before=before["W"][i], terms=T)
+            assert abs(g[i] - np.linalg.norm(G)) <= 1e-5 * np.linalg.norm(ga)
     z.close()
 
 
@@ -92,10 +97,11 @@ def test_sgd_step_matches_oracle_and_leaves_moments(lib, gpu):
            optimizer=zb.ZO_OPT_SGD)
     after = snapshot(z)
     for i, W in enumerate(z.weights):
-        Wo, _, _, _ = oracle_step(before, i, dtype_of(W), z.seed, base + i, 4, z.r, z.q, losses,
-                                  "central", 1e-3, 1e-4, 0.9, 0.95, 1e-8, 1, [(z.q - 1, 1.0)],
-                                  optimizer="sgd")
-        assert_weights(after["W"][i], Wo, dtype_of(W), f"sgd W {i}")
+        Wo, _, _, _, T = oracle_step(before, i, dtype_of(W), z.seed, base + i, 4, z.r, z.q, losses,
+                                     "central", 1e-3, 1e-4, 0.9, 0.95, 1e-8, 1, [(z.q - 1, 1.0)],
+                                     optimizer="sgd")
+        assert_weights(after["W"][i], Wo, dtype_of(W), f"sgd W {i}", before=before["W"][i],
+                       terms=T)
         assert np.array_equal(after["M"][i], before["M"][i])
     z.close()
 
@@ -107,10 +113,12 @@ def test_losses_from_device_memory(lib, gpu):
     z.step(0, 1, torch.from_numpy(losses).to(gpu), "central", 1e-3, 1e-3, 0.9, 0.95, 1e-8,
            z.q - 1, 1.0)
     after = snapshot(z)
-    Wo, Mo, _, _ = oracle_step(before, 0, "bf16", z.seed, base, 0, z.r, z.q, losses, "central",
-                               1e-3, 1e-3, 0.9, 0.95, 1e-8, 1, [(z.q - 1, 1.0)])
-    assert_rel(after["M"][0], Mo, "M")
-    assert_weights(after["W"][0], Wo, "bf16", "W")
+    Wo, Mo, Vmo, _, T = oracle_step(before, 0, "bf16", z.seed, base, 0, z.r, z.q, losses,
+                                    "central", 1e-3, 1e-3, 0.9, 0.95, 1e-8, 1, [(z.q - 1, 1.0)])
+    ga = gabs(z.seed, base, 0, z.r, subzero.rho_from_losses(losses, "central", f32(1e-3), z.q))
+    assert_moments(after["M"][0], after["Vm"][0], Mo, Vmo, before["M"][0], before["Vm"][0], ga,
+                   0.9, 0.95, "device losses")
+    assert_weights(after["W"][0], Wo, "bf16", "W", before=before["W"][0], terms=T)
     z.close()
 
 
@@ -160,3 +168,88 @@ def test_rejected_calls_launch_nothing(lib, gpu):
             assert np.array_equal(a, b)
     z.sync()
     z.close()
+
+
+# bf16-only contexts with r in {16, 32, 64} run the tensor-core weight pass:
+# tiles of 128 x 128 with ragged rows and columns, and a padded row stride.
+TC_CASES = {
+    "tc16": (16, [(300, 520, None), (130, 1000, 1008), (1030, 72, None), (128, 128, None)]),
+    "tc32": (32, [(300, 520, 528), (1030, 72, 80), (257, 2048, None)]),
+    "tc64": (64, [(300, 520, None), (130, 1000, None), (1030, 72, 72), (2048, 384, None)]),
+}
+
+
+def _build_tc(gpu, case, seed, base=11):
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    r, spec = TC_CASES[case]
+    weights = [make_weight(m, n, "bf16", 200 + k, gpu, ldw) for k, (m, n, ldw) in enumerate(spec)]
+    z = SubZeroPlus(weights, r, 4, seed, matrix_index_base=base)
+    z.init_subspace(0)
+    return z, base
+
+
+@pytest.mark.parametrize("case", list(TC_CASES))
+@pytest.mark.parametrize("eps", [1e-3, 1e-1])
+def test_tensor_core_pass_matches_oracle(lib, gpu, case, eps):
+    from paper_2608_15665_gb300 import binding as zb
+    z, base = _build_tc(gpu, case, seed=909)
+    calls = [(0, 1.0, -1, 0.0), (0, -2.0, -1, 0.0), (0, 1.0, 1, 1.0), (3, 1.0, 2, -1.0)]
+    for t, (qa, ca, qb, cb) in zip((0, 0, 7, 99), calls):
+        before = snapshot(z)
+        z.perturb(t, qa, ca, qb, cb, eps)
+        after = snapshot(z)
+        assert zb.zo_wpass_path(z.ctx) == 2
+        terms = [(qa, ca)] + ([(qb, cb)] if qb >= 0 else [])
+        for i in range(len(z.weights)):
+            want, T = oracle_perturb(before, i, "bf16", z.seed, base + i, t, z.r, terms, eps)
+            assert_weights(after["W"][i], want, "bf16", f"{case} matrix {i} t={t}",
+                           before=before["W"][i], terms=T)
+    z.sync()
+    z.close()
+
+
+@pytest.mark.parametrize("case", list(TC_CASES))
+def test_tensor_core_step_matches_oracle(lib, gpu, case):
+    z, base = _build_tc(gpu, case, seed=313)
+    q, eps, lr, b1, b2, ea = z.q, 1e-2, 1e-2, 0.9, 0.95, 1e-8
+    rs = np.random.default_rng(8)
+    for step in range(2):
+        losses = (2.0 + 0.01 * rs.standard_normal(2 * q)).astype(np.float32)
+        before = snapshot(z)
+        z.step(step, step + 1, losses, "central", eps, lr, b1, b2, ea, q - 1, 1.0)
+        after = snapshot(z)
+        rho = subzero.rho_from_losses(losses, "central", f32(eps), q)
+        for i in range(len(z.weights)):
+            Wo, Mo, Vmo, _, T = oracle_step(before, i, "bf16", z.seed, base + i, step, z.r, q,
+                                            losses, "central", eps, lr, b1, b2, ea, step + 1,
+                                            [(q - 1, 1.0)])
+            assert_moments(after["M"][i], after["Vm"][i], Mo, Vmo, before["M"][i],
+                           before["Vm"][i], gabs(z.seed, base + i, step, z.r, rho), b1, b2,
+                           f"{case} {i}")
+            assert_weights(after["W"][i], Wo, "bf16", f"W {case} {i} step {step}",
+                           before=before["W"][i], terms=T)
+    z.sync()
+    z.close()
+
+
+@pytest.mark.parametrize("case", list(TC_CASES))
+def test_tensor_core_and_fma_paths_agree(lib, gpu, case):
+    # one pass from the same state on both paths: each is within 1 ulp (at the operand
+    # scale) of the exact result, so they differ by at most 2 such ulps, and rarely at all
+    from paper_2608_15665_gb300 import binding as zb
+    out = {}
+    for path in (1, 2):
+        z, base = _build_tc(gpu, case, seed=4321)
+        before = snapshot(z)
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_WPASS_PATH, path)
+        z.perturb(0, 0, 1.0, 1, -1.0, 1e-1)
+        assert zb.zo_wpass_path(z.ctx) == path
+        out[path] = [to_f64(W) for W in z.weights]
+        z.close()
+    for i, (a, b) in enumerate(zip(out[1], out[2])):
+        _, (T, TZ) = oracle_perturb(before, i, "bf16", 4321, base + i, 0, TC_CASES[case][0],
+                                    [(0, 1.0), (1, -1.0)], 1e-1)
+        scale = np.maximum.reduce([np.abs(a), np.abs(b), np.abs(before["W"][i]), T])
+        d = np.abs(a - b)
+        assert np.all(d <= 2 * rounding.bf16_ulp(scale) + 2 * TZ)
+        assert (d > 0).mean() < 1e-2

@@ -23,7 +23,8 @@ CASES = [
 def test_refresh_matches_oracle(lib, gpu, r, shapes):
     from paper_2608_15665_gb300.schedule import SubZeroPlus
     seed, base = 4242 + r, 10
-    weights = [make_weight(m, n, "bf16", k, gpu) for k, (m, n) in enumerate(shapes)]
+    # W rows must start on 16-byte boundaries: pad the row stride, keep n ragged
+    weights = [make_weight(m, n, "bf16", k, gpu, ldw=(n + 7) // 8 * 8) for k, (m, n) in enumerate(shapes)]
     z = SubZeroPlus(weights, r, 2, seed, matrix_index_base=base)
     for j in (0, 3):
         z.refresh(j, reset_moments=True)
@@ -58,7 +59,7 @@ def test_refresh_resets_moments_only_when_asked(lib, gpu):
 
 def test_refresh_is_deterministic(lib, gpu):
     from paper_2608_15665_gb300.schedule import SubZeroPlus
-    z = SubZeroPlus([make_weight(3000, 700, "bf16", 2, gpu)], 32, 2, 77)
+    z = SubZeroPlus([make_weight(3000, 704, "bf16", 2, gpu)], 32, 2, 77)
     z.refresh(5)
     a = [z.U[0].clone(), z.V[0].clone()]
     z.refresh(6)

@@ -8,7 +8,8 @@ import torch
 
 from gpu_util import dtype_of, f32, snapshot
 from oracle import haar, subzero
-from parity import UV_ABS, assert_rel, assert_weights, to_f64
+from parity import (UV_ABS, assert_moments, assert_normwise, assert_weights, gabs, to_f64,
+                    update_terms)
 
 pytestmark = pytest.mark.gpu
 
@@ -41,9 +42,9 @@ def test_single256_trajectory(lib, gpu, scheme):
     table = _run_gpu_schedule(z, wl, scheme, wl.steps)
     s = snapshot(z)
     st = _oracle_trajectory(wl, to_f64(W0), 0, table, scheme, wl.steps)
-    assert_rel(s["W"][0], st.W, "W after 10 steps")
-    assert_rel(s["M"][0], st.M, "M after 10 steps")
-    assert_rel(s["Vm"][0], st.Vm, "Vm after 10 steps")
+    assert_normwise(s["W"][0], st.W, "W after 10 steps")
+    assert_normwise(s["M"][0], st.M, "M after 10 steps")
+    assert_normwise(s["Vm"][0], st.Vm, "Vm after 10 steps")
     assert np.max(np.abs(s["U"][0] - st.U)) <= UV_ABS
     assert np.max(np.abs(s["V"][0] - st.V)) <= UV_ABS
     # the weights did move: the update is not a no-op
@@ -61,9 +62,9 @@ def test_lora_trajectory_on_sampled_matrices(lib, gpu):
     s = snapshot(z)
     for i in (0, 1, 2, 3, 158, 159):
         st = _oracle_trajectory(wl, to_f64(W0[i]), i, table, "central", wl.steps)
-        assert_rel(s["W"][i], st.W, f"LoRA matrix {i} after 200 steps")
-        assert_rel(s["M"][i], st.M, f"M {i}")
-        assert_rel(s["Vm"][i], st.Vm, f"Vm {i}")
+        assert_normwise(s["W"][i], st.W, f"LoRA matrix {i} after 200 steps")
+        assert_normwise(s["M"][i], st.M, f"M {i}")
+        assert_normwise(s["Vm"][i], st.Vm, f"Vm {i}")
     z.close()
 
 
@@ -105,7 +106,9 @@ def test_full_size_sampled_parity(lib, gpu, name, sample):
     for i in sample:
         C = subzero.perturb_coeff(wl.seed, i, 0, wl.r, [(0, 1.0), (1, 1.0)], f32(wl.eps))
         want = subzero.apply_pass(before[i], wl.dtype, UV[i][0], UV[i][1], C, rows=rows[i])
-        assert_weights(after[i], want, wl.dtype, f"{name} perturb, matrix {i}")
+        T = update_terms(UV[i][0][rows[i]], C, UV[i][1], 2 * f32(wl.eps))
+        assert_weights(after[i], want, wl.dtype, f"{name} perturb, matrix {i}", before=before[i],
+                       terms=T)
 
     # the Adam step fused with the restore
     losses = workloads.loss_table(wl, "central", steps=1)[0]
@@ -120,9 +123,12 @@ def test_full_size_sampled_parity(lib, gpu, name, sample):
                                       f32(wl.beta1), f32(wl.beta2), f32(wl.eps_adam), 1)
         C = subzero.step_coeff(D, f32(wl.lr), f32(wl.eps), [(wl.q - 1, 1.0)], wl.seed, i, 0, wl.r)
         want = subzero.apply_pass(before[i], wl.dtype, UV[i][0], UV[i][1], C, rows=rows[i])
-        assert_weights(after[i], want, wl.dtype, f"{name} step, matrix {i}")
-        assert_rel(to_f64(z.M[i]), M, f"M {i}")
-        assert_rel(to_f64(z.Vm[i]), Vm, f"Vm {i}")
+        T = update_terms(UV[i][0][rows[i]], C, UV[i][1], f32(wl.eps))
+        assert_weights(after[i], want, wl.dtype, f"{name} step, matrix {i}", before=before[i],
+                       terms=T)
+        z0 = np.zeros((wl.r, wl.r))
+        assert_moments(to_f64(z.M[i]), to_f64(z.Vm[i]), M, Vm, z0, z0,
+                       gabs(wl.seed, i, 0, wl.r, rho), f32(wl.beta1), f32(wl.beta2), f"{name} {i}")
     z.sync()
     z.close()
     del weights, z
