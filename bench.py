@@ -48,6 +48,9 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="llama7b_bf16_r32")
     p.add_argument("--scheme", choices=["central", "forward"], default="central")
+    p.add_argument("--layers", type=int, default=0,
+                   help="use only the first N layers of the workload (shape-preserving subset, "
+                        "for profiling captures); 0 = all")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     return p.parse_args()
@@ -70,6 +73,18 @@ def kernel_source_hash():
         if os.path.exists(path):
             h.update(open(path, "rb").read())
     return h.hexdigest()[:16]
+
+
+def subset(wl, layers):
+    """The first `layers` layers of a workload (its matrices repeat per layer)."""
+    if not layers:
+        return wl
+    from paper_2608_15665_gb300 import workloads
+    per_layer = {"opt1.3b_bf16_r16": 6, "llama7b_bf16_r32": 7, "dense32b_bf16_r64": 7,
+                 "lora_opt13b_f32_r4": 4, "single256_f32_r8": 1}[wl.name]
+    k = min(len(wl.shapes), layers * per_layer)
+    return workloads.scaled(wl, name=f"{wl.name}[{layers} layers]", shapes=wl.shapes[:k],
+                            zero_init=[i for i in wl.zero_init if i < k])
 
 
 # --------------------------------------------------------------------------- clocks
@@ -242,7 +257,7 @@ def run_ours(args):
     from paper_2608_15665_gb300 import workloads
     from paper_2608_15665_gb300.schedule import SubZeroPlus, step_plan
 
-    wl0 = wl = workloads.get(args.workload)
+    wl0 = wl = subset(workloads.get(args.workload), args.layers)
     part = workloads.partition(wl, rank, world)
     weights = [workloads.init_weight(wl, i, dev, part["matrix_index_base"])
                for i in range(wl.n_mats)]
