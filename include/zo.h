@@ -202,6 +202,33 @@ ZO_API zo_status zo_philox_fill(uint64_t seed, uint32_t x1, uint32_t x2, uint32_
 ZO_API zo_status zo_normal_fill(uint64_t seed, uint32_t x1, uint32_t x2, uint32_t x3, float* out,
                          int64_t n, void* stream);
 
+/*
+ * zo_perturb_noalloc -- one perturbation pass on a single matrix that allocates no
+ * device memory.  The paper has no counterpart; it is for callers that cannot
+ * allocate: code whose GPU memory is already reserved by another allocator (a
+ * framework's caching pool), where a cudaMalloc would fail or fragment that pool,
+ * and loops that cannot afford the device synchronisation cudaMalloc/cudaFree may
+ * cause.  It computes what zo_perturb computes for one matrix on the fp32-FMA path:
+ *   W <- rnd(W + eps * U (ca Z^(qa) + cb Z^(qb)) V^T)   (qb = -1 drops the second term)
+ * with Z^(k) drawn for matrix index `matrix_index` at step t from `seed`
+ * (the counter contract above).  W (m x n, ldw, dtype), U (m x r) and V (n x r) are
+ * caller-owned device buffers; r in {4, 8, 16, 32, 64}.
+ * Scratch (the coefficient C, the projection C V^T and small work tables) lives in a
+ * fixed 8 MiB array inside the library (2^21 floats), which every GPU that loads the
+ * library holds until the process exits.  A request needing more -- about r * n + r * r
+ * floats -- is rejected with ZO_ERR_SHAPE before anything is launched.
+ * The first call on a device looks up that array's device address (cudaGetSymbolAddress)
+ * with the device current; make that first call before capturing any stream.
+ * All calls share the one array and rewrite everything they read from it before
+ * reading it, so nothing needs clearing between calls -- but two calls whose work
+ * overlaps on the GPU (different streams, or different host threads) race on it.
+ * Asynchronous on `stream` (void* cudaStream_t); errors as for zo_perturb.
+ */
+ZO_API zo_status zo_perturb_noalloc(void* W, int64_t m, int64_t n, int64_t ldw, int32_t dtype,
+                                    const float* U, const float* V, int32_t r, uint64_t seed,
+                                    uint32_t matrix_index, uint32_t t, int32_t qa, float ca,
+                                    int32_t qb, float cb, float eps, void* stream);
+
 /* zo_status_string -- static description of a status code. */
 ZO_API const char* zo_status_string(int32_t status);
 

@@ -80,6 +80,11 @@ _SIGNATURES = {
                                     _c.c_void_p, _c.c_int64, _c.c_void_p]),
     "zo_normal_fill": (_c.c_int32, [_c.c_uint64, _c.c_uint32, _c.c_uint32, _c.c_uint32,
                                     _c.c_void_p, _c.c_int64, _c.c_void_p]),
+    "zo_perturb_noalloc": (_c.c_int32, [_c.c_void_p, _c.c_int64, _c.c_int64, _c.c_int64,
+                                        _c.c_int32, _c.c_void_p, _c.c_void_p, _c.c_int32,
+                                        _c.c_uint64, _c.c_uint32, _c.c_uint32, _c.c_int32,
+                                        _c.c_float, _c.c_int32, _c.c_float, _c.c_float,
+                                        _c.c_void_p]),
     "zo_status_string": (_c.c_char_p, [_c.c_int32]),
     "zo_last_error": (_c.c_char_p, []),
 }
@@ -212,6 +217,16 @@ def zo_wpass_path(ctx):
 
 def zo_kernel_launches(ctx):
     return int(LIB.zo_kernel_launches(ctx))
+
+
+def zo_perturb_noalloc(W, U, V, r, seed, matrix_index, t, qa, ca, qb, cb, eps, stream=None):
+    """One perturbation pass on one matrix with no device allocation (see include/zo.h)."""
+    import torch
+    dt = ZO_BF16 if W.dtype == torch.bfloat16 else ZO_F32 if W.dtype == torch.float32 else -1
+    _check(LIB.zo_perturb_noalloc(_ptr(W), W.shape[0], W.shape[1], W.stride(0), dt, _ptr(U),
+                                  _ptr(V), int(r), int(seed) & (2**64 - 1), int(matrix_index),
+                                  int(t), int(qa), float(ca), int(qb), float(cb), float(eps),
+                                  _stream_handle(stream)), "zo_perturb_noalloc")
 
 
 def zo_philox_fill(seed, x1, x2, x3, out, stream=None):

@@ -2,12 +2,17 @@
 #pragma once
 
 #include <cstdint>
+#include <string>
 #include <cuda.h>
 #include <cuda_runtime.h>
 
 #include "zo_device.cuh"
 
 namespace zo {
+
+// Text returned by zo_last_error (zo_api.cu); thread-local.
+void set_last_error(const char* msg);
+inline void set_last_error(const std::string& msg) { set_last_error(msg.c_str()); }
 
 // ---- counter-based Gaussian contract (zo_rng.cu) ---------------------------
 cudaError_t launch_philox_fill(uint64_t seed, uint32_t x1, uint32_t x2, uint32_t x3, uint32_t* out,
