@@ -359,23 +359,63 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
   }
 }
 
+// Both split kernels below handle 128 consecutive rows of one matrix per CTA: each
+// thread splits one row into 16-byte chunks of hi and lo, staged in shared memory with
+// the chunk index XOR (row & 7) so a quarter-warp's stores hit distinct banks; the CTA
+// then writes its rows, which are contiguous in the stacked operand, with coalesced
+// 16-byte stores.  Padding columns of a row stay at the zero they were set to.
+template <int R>
+__device__ __forceinline__ void split8(const float (&x)[8], uint4& hi, uint4& lo) {
+  uint32_t hw[4], lw[4];
+#pragma unroll
+  for (int pr = 0; pr < 4; ++pr) {
+    const __nv_bfloat162 h2 = __floats2bfloat162_rn(x[2 * pr], x[2 * pr + 1]);
+    const __nv_bfloat162 l2 =
+        __floats2bfloat162_rn(x[2 * pr] - __low2float(h2), x[2 * pr + 1] - __high2float(h2));
+    hw[pr] = *reinterpret_cast<const uint32_t*>(&h2);
+    lw[pr] = *reinterpret_cast<const uint32_t*>(&l2);
+  }
+  hi = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+  lo = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+}
+
+template <int R>
+__device__ __forceinline__ void write_rows(const uint4* Os, __nv_bfloat16* dst_rows, int rows) {
+  constexpr int kVecPerRow = hl_width(R) * 2 / 16;   // 8 or 16 chunks per row
+  uint4* dst = reinterpret_cast<uint4*>(dst_rows);
+  for (int e = threadIdx.x; e < rows * kVecPerRow; e += blockDim.x) {
+    const int row = e / kVecPerRow, c = e % kVecPerRow;
+    if (c * 8 < 2 * R) dst[e] = Os[row * kVecPerRow + (c ^ (row & 7))];
+  }
+}
+
 // U_HL[u_row0 + i] = [bf16 hi(U[i, :]) | bf16 lo(U[i, :]) | 0 ...]  (row width hl_width(R))
 template <int R>
-__global__ void split_u_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
-                               const int2* __restrict__ units, __nv_bfloat16* __restrict__ u_hl) {
+__global__ void __launch_bounds__(128)
+split_u_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
+               const int2* __restrict__ units, __nv_bfloat16* __restrict__ u_hl) {
+  constexpr int kVecPerRow = hl_width(R) * 2 / 16;
+  __shared__ uint4 Os[128 * kVecPerRow];
   const int2 u = units[blockIdx.x];
   const MatDesc md = mats[u.x];
-  const int64_t row = (int64_t)u.y + threadIdx.x;
-  if (row >= md.m) return;
-  const float* src = md.U + row * R;
-  __nv_bfloat16* dst = u_hl + ((int64_t)tcm[u.x].u_row0 + row) * hl_width(R);
+  const int tid = threadIdx.x;
+  const int64_t i0 = u.y;
+  const int rows = (int)(md.m - i0 < 128 ? md.m - i0 : 128);
+  if (tid < rows) {
+    const float4* src = reinterpret_cast<const float4*>(md.U + (i0 + tid) * R);
+    uint4* orow = Os + tid * kVecPerRow;
 #pragma unroll
-  for (int c = 0; c < R; ++c) {
-    const float x = src[c];
-    const __nv_bfloat16 h = __float2bfloat16_rn(x);
-    dst[c] = h;
-    dst[R + c] = __float2bfloat16_rn(x - __bfloat162float(h));
+    for (int g = 0; g < R / 8; ++g) {
+      const float4 a = src[2 * g], b = src[2 * g + 1];
+      const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+      uint4 hi, lo;
+      split8<R>(x, hi, lo);
+      orow[g ^ (tid & 7)] = hi;
+      orow[(R / 8 + g) ^ (tid & 7)] = lo;
+    }
   }
+  __syncthreads();
+  write_rows<R>(Os, u_hl + ((int64_t)tcm[u.x].u_row0 + i0) * hl_width(R), rows);
 }
 
 // Pt_HL[p_row0 + j] = [hi | lo] of P^T[j, :] = (C V^T)^T[j, :] = V[j, :] C^T
@@ -383,29 +423,60 @@ template <int R>
 __global__ void __launch_bounds__(128)
 project_split_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
                      const int2* __restrict__ units, __nv_bfloat16* __restrict__ p_hl) {
-  __shared__ float Cs[R * R];
+  constexpr int kVecPerRow = hl_width(R) * 2 / 16;
+  extern __shared__ uint4 ps_smem[];
+  uint4* Os = ps_smem;                                                // 128 x kVecPerRow
+  float* Cs = reinterpret_cast<float*>(Os + 128 * kVecPerRow);        // R x R
   const int2 u = units[blockIdx.x];
   const MatDesc md = mats[u.x];
-  for (int e = threadIdx.x; e < R * R; e += blockDim.x) Cs[e] = md.C[e];
+  const int tid = threadIdx.x;
+  const int64_t j0 = u.y;
+  const int rows = (int)(md.n - j0 < 128 ? md.n - j0 : 128);
+  for (int e = tid; e < R * R; e += 128) Cs[e] = md.C[e];
   __syncthreads();
-  const int64_t j = (int64_t)u.y + threadIdx.x;
-  if (j >= md.n) return;
-  float v[R];
-  const float4* vrow = reinterpret_cast<const float4*>(md.V + j * R);
+  if (tid < rows) {
+    float v[R];
+    const float4* vrow = reinterpret_cast<const float4*>(md.V + (j0 + tid) * R);
 #pragma unroll
-  for (int b = 0; b < R / 4; ++b) {
-    const float4 t = vrow[b];
-    v[4 * b] = t.x; v[4 * b + 1] = t.y; v[4 * b + 2] = t.z; v[4 * b + 3] = t.w;
-  }
-  __nv_bfloat16* dst = p_hl + ((int64_t)tcm[u.x].p_row0 + j) * hl_width(R);
-  for (int a = 0; a < R; ++a) {
-    float acc = 0.f;
+    for (int b = 0; b < R / 4; ++b) {
+      const float4 t4 = vrow[b];
+      v[4 * b] = t4.x; v[4 * b + 1] = t4.y; v[4 * b + 2] = t4.z; v[4 * b + 3] = t4.w;
+    }
+    uint4* orow = Os + tid * kVecPerRow;
+    for (int g = 0; g < R / 8; ++g) {
+      float x[8];
 #pragma unroll
-    for (int b = 0; b < R; ++b) acc = fmaf(Cs[a * R + b], v[b], acc);
-    const __nv_bfloat16 h = __float2bfloat16_rn(acc);
-    dst[a] = h;
-    dst[R + a] = __float2bfloat16_rn(acc - __bfloat162float(h));
+      for (int k = 0; k < 8; ++k) {
+        const float* crow = Cs + (8 * g + k) * R;
+        float acc = 0.f;
+#pragma unroll
+        for (int b = 0; b < R; ++b) acc = fmaf(crow[b], v[b], acc);
+        x[k] = acc;
+      }
+      uint4 hi, lo;
+      split8<R>(x, hi, lo);
+      orow[g ^ (tid & 7)] = hi;
+      orow[(R / 8 + g) ^ (tid & 7)] = lo;
+    }
   }
+  __syncthreads();
+  write_rows<R>(Os, p_hl + ((int64_t)tcm[u.x].p_row0 + j0) * hl_width(R), rows);
+}
+
+template <int R>
+constexpr size_t project_split_smem() {
+  return 128 * (size_t)hl_width(R) * 2 + sizeof(float) * R * R;
+}
+
+template <int R>
+cudaError_t launch_project_split_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                                   int32_t n_units, __nv_bfloat16* p_hl, cudaStream_t s) {
+  const size_t smem = project_split_smem<R>();
+  cudaError_t e = cudaFuncSetAttribute(project_split_kernel<R>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  project_split_kernel<R><<<n_units, 128, smem, s>>>(d_mats, d_tc, d_units, p_hl);
+  return cudaGetLastError();
 }
 
 template <int R>
@@ -443,12 +514,11 @@ cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const
                                  int32_t n_units, int32_t r, __nv_bfloat16* p_hl, cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
-    case 16: project_split_kernel<16><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, p_hl); break;
-    case 32: project_split_kernel<32><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, p_hl); break;
-    case 64: project_split_kernel<64><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, p_hl); break;
+    case 16: return launch_project_split_r<16>(d_mats, d_tc, d_units, n_units, p_hl, s);
+    case 32: return launch_project_split_r<32>(d_mats, d_tc, d_units, n_units, p_hl, s);
+    case 64: return launch_project_split_r<64>(d_mats, d_tc, d_units, n_units, p_hl, s);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
