@@ -85,7 +85,12 @@ enum {
 /* Options for zo_set_option. */
 enum {
   ZO_OPTION_WPASS_PATH = 0, /* 0 = automatic, 1 = fp32-FMA path, 2 = tcgen05 path */
-  ZO_OPTION_TIMING = 1      /* 1 = record CUDA events around every weight-pass launch */
+  ZO_OPTION_TIMING = 1,     /* 1 = record CUDA events around every weight-pass launch */
+  ZO_OPTION_TEST_WAIT_TIMEOUT = 2 /* test hook: 1 = in the next tensor-core weight pass, one
+                                     CTA first waits on a barrier nothing arrives on, so its
+                                     bounded wait (~0.1 s) runs out; that pass then reports
+                                     ZO_ERR_TIMEOUT via zo_sync_status and leaves W partly
+                                     updated.  Nothing faults; the context stays usable. */
 };
 
 /* One trainable matrix W_i with its projection bases and Adam moments. */

@@ -35,6 +35,7 @@ ZO_OPT_SGD = 1
 
 ZO_OPTION_WPASS_PATH = 0
 ZO_OPTION_TIMING = 1
+ZO_OPTION_TEST_WAIT_TIMEOUT = 2
 
 
 class ZoError(RuntimeError):

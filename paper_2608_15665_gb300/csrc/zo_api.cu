@@ -65,6 +65,7 @@ struct zo_ctx {
   uint32_t* d_status = nullptr;
   int path_option = 0;
   int last_path = 0;
+  bool inject_wait = false;      // test hook armed for the next tensor-core pass
   int64_t launches = 0;          // kernels launched by this context
   // tensor-core weight pass (all matrices bf16, r in {16, 32, 64})
   bool tc_ok = false;
@@ -206,8 +207,10 @@ zo_status run_weight_pass(zo_ctx* c) {
   if (st != ZO_OK) return st;
   if (use_tc) {
     const int grid = (int)std::min<int64_t>(c->tc_tiles, c->sms);
+    const bool inject = c->inject_wait;
+    c->inject_wait = false;
     ZO_CUDA(zo::launch_wpass_tc(c->tm_a, c->tm_b, c->d_w_maps, c->d_tc, c->n_mats, c->tc_tiles,
-                                grid, c->r, c->d_status, c->stream),
+                                grid, c->r, c->d_status, inject, c->stream),
             "tensor-core weight-pass kernel");
     c->last_path = 2;
   } else {
@@ -637,6 +640,15 @@ zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
       return ZO_ERR_UNSUPPORTED;
     }
     c->path_option = (int)value;
+    return ZO_OK;
+  }
+  if (option == ZO_OPTION_TEST_WAIT_TIMEOUT) {
+    if (value != 0 && value != 1) return ZO_ERR_INVALID_ARG;
+    if (value == 1 && !c->tc_ok) {
+      g_last_error = "the wait-timeout test hook needs the tensor-core weight pass";
+      return ZO_ERR_UNSUPPORTED;
+    }
+    c->inject_wait = value != 0;
     return ZO_OK;
   }
   if (option == ZO_OPTION_TIMING) {

@@ -71,7 +71,7 @@ cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const
 cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
                             const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
                             int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
-                            cudaStream_t s);
+                            bool inject_wait, cudaStream_t s);
 
 // ---- refresh: batched TSQR + sign correction (zo_qr.cu) ------------------------
 int32_t qr_block_rows(int32_t r);
