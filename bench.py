@@ -37,7 +37,10 @@ FALLBACK_HBM_GBS = 6800.0
 # dram__bytes_read.sum + dram__bytes_write.sum per launch of the weight-pass kernel,
 # from the ncu capture summarised under profiles/, keyed by the sha256 of the kernel
 # source it was taken on (reported as null once the source differs).
-TRAFFIC_BY_SOURCE = {}
+TRAFFIC_BY_SOURCE = {
+    # profiles/wpass_tc_r32_llama7b_2layers.md: 1.577 GB on the 2-layer subset, x16.0 by weights
+    "64253833d2a89ac2": 25.24e9,
+}
 
 
 def parse_args():
@@ -67,8 +70,9 @@ def measured_peaks():
 
 
 def kernel_source_hash():
+    """sha256 (16 hex) of the sources of the tensor-core weight-pass kernel."""
     h = hashlib.sha256()
-    for name in ("zo_wpass_fma.cu", "zo_wpass_tc.cu"):
+    for name in ("zo_wpass_tc.cu", "zo_sm100.cuh", "zo_device.cuh"):
         path = os.path.join(ROOT, "paper_2608_15665_gb300", "csrc", name)
         if os.path.exists(path):
             h.update(open(path, "rb").read())
@@ -316,6 +320,16 @@ def run_ours(args):
     path = zb.zo_wpass_path(z.ctx)
     z.sync()
 
+    # ---- one subspace refresh (Alg. 1 for every matrix), timed on its own ----------
+    barrier()
+    r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    r0.record()
+    z.refresh((W + K) // wl.F)
+    r1.record()
+    barrier()
+    refresh_ms = max_over_ranks(r0.elapsed_time(r1))
+    z.sync()
+
     # ---- end to end through the public API with host buffers -------------------------
     e2e = None
     if not args.no_e2e:
@@ -352,6 +366,7 @@ def run_ours(args):
                    "l2": "inputs larger than L2 (%.1f GB of weights per pass)" % (bytes_pass / 2e9),
                    "parallelism": f"layer partition x{world}" if world > 1 else "single GPU"},
         "weight_pass_gbs": passes * bytes_pass * K / (elapsed_ms / 1e3) / 1e9,
+        "refresh_ms": refresh_ms,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "traffic": TRAFFIC_BY_SOURCE.get(src),
