@@ -172,6 +172,20 @@ ZO_API zo_status zo_step(zo_ctx* ctx, uint32_t t, int32_t adam_t, const float* l
                   float beta1, float beta2, float eps_adam, int32_t restore_query,
                   float restore_coef, float* gamma_out);
 
+/*
+ * zo_mezo_perturb -- the full-space SPSA perturbation of Sec. 3, Eq. (1) (MeZO, the
+ * paper's comparison baseline), for every matrix of the context:
+ *   W_i <- rnd(W_i + coef * Z_i),  Z_i[row, col] ~ N(0, 1) i.i.d., regenerated from the seed
+ * with counter = (row * ceil(n_i / 4) + col / 4, matrix index, t, 5 << 24), lane col % 4
+ * (each row starts on a fresh counter word).  coef = +eps, -2 eps, +eps give the two
+ * evaluations of Eq. (1) and the restore; coef = eps - lr * rho fuses the restore with
+ * MeZO's SGD update (rho = (L+ - L-) / (2 eps)).  U, V and the moments are not touched.
+ * Each weight costs one quarter of a Philox call plus half a Box-Muller transform, so
+ * this pass is bound by the ALU rather than HBM.  Timed like the weight passes when
+ * ZO_OPTION_TIMING is on.
+ */
+ZO_API zo_status zo_mezo_perturb(zo_ctx* ctx, uint32_t t, float coef);
+
 /* zo_sync_status -- synchronise the stream; return (and clear) the device status word. */
 ZO_API zo_status zo_sync_status(zo_ctx* ctx);
 

@@ -18,10 +18,12 @@ order (SubZero+, arXiv 2608.15665):
 * ``subzero``  -- Alg. 2 (PerturbParams) as a fused pass W <- rnd(W + U C V^T),
                   the multi-query estimator of Eq. (6), the subspace Adam of
                   Eqs. (7)-(10), and the Alg. 3 schedule driver.
+* ``mezo``     -- the full-space SPSA perturbation of Eq. (1) (MeZO's baseline):
+                  W <- rnd(W + coef Z) with Z i.i.d. N(0,1) per element.
 
 Pins (tests/test_oracle_*.py) tie each function to something other than
 itself: published known-answer vectors, closed forms, uniqueness of the
 positive-diagonal QR, brute-force Haar moments, a hand-computed 2x2 Adam step.
 """
 
-from . import rng, rounding, haar, subzero  # noqa: F401
+from . import rng, rounding, haar, subzero, mezo  # noqa: F401

@@ -72,6 +72,7 @@ _SIGNATURES = {
                              _c.c_int32, _c.c_int32, _c.c_int32, _c.c_float, _c.c_float,
                              _c.c_float, _c.c_float, _c.c_float, _c.c_int32, _c.c_float,
                              _c.c_void_p]),
+    "zo_mezo_perturb": (_c.c_int32, [_c.c_void_p, _c.c_uint32, _c.c_float]),
     "zo_sync_status": (_c.c_int32, [_c.c_void_p]),
     "zo_set_option": (_c.c_int32, [_c.c_void_p, _c.c_int32, _c.c_int64]),
     "zo_get_timing": (_c.c_int32, [_c.c_void_p, _c.POINTER(_c.c_double), _c.POINTER(_c.c_int64)]),
@@ -195,6 +196,10 @@ def zo_step(ctx, t, adam_t, losses, scheme, eps, lr, beta1, beta2, eps_adam, res
                        float(eps), float(lr), float(beta1), float(beta2), float(eps_adam),
                        int(restore_query), float(restore_coef), _ptr(gamma_out)), "zo_step")
     del keep
+
+
+def zo_mezo_perturb(ctx, t, coef):
+    _check(LIB.zo_mezo_perturb(ctx, int(t), float(coef)), "zo_mezo_perturb")
 
 
 def zo_sync_status(ctx):

@@ -618,6 +618,27 @@ zo_status zo_step(zo_ctx* c, uint32_t t, int32_t adam_t, const float* losses, in
   return run_weight_pass(c);
 }
 
+zo_status zo_mezo_perturb(zo_ctx* c, uint32_t t, float coef) {
+  if (!c) return ZO_ERR_INVALID_ARG;
+  if (!std::isfinite(coef)) {
+    g_last_error = "zo_mezo_perturb: non-finite coefficient";
+    return ZO_ERR_INVALID_ARG;
+  }
+  for (const auto& d : c->h_mats) {
+    if (d.m * ((d.n + 3) / 4) >= (int64_t(1) << 32)) {
+      g_last_error = "zo_mezo_perturb: matrix too large for the 32-bit counter word";
+      return ZO_ERR_SHAPE;
+    }
+  }
+  zo_status st = record_start(c);
+  if (st != ZO_OK) return st;
+  ZO_CUDA(zo::launch_mezo(c->d_mats, c->n_mats, c->d_tile_prefix, c->n_tiles, c->seed, t, coef,
+                          c->stream),
+          "full-space perturbation kernel");
+  ++c->launches;
+  return record_stop(c);
+}
+
 zo_status zo_sync_status(zo_ctx* c) {
   if (!c) return ZO_ERR_INVALID_ARG;
   ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");

@@ -57,6 +57,12 @@ __host__ __device__ constexpr int fma_tile_cols(int32_t dtype) { return dtype ==
 cudaError_t launch_wpass_fma(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_tile_prefix,
                              int64_t n_tiles, int32_t r, cudaStream_t s);
 
+// ---- full-space SPSA perturbation of Eq. (1) (zo_mezo.cu) -------------------------
+// W_i <- rnd(W_i + coef Z_i), Z_i per element from the counter contract (tag 5), on the
+// FMA pass's tiles (d_tile_prefix / MatDesc::tile0).
+cudaError_t launch_mezo(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_tile_prefix,
+                        int64_t n_tiles, uint64_t seed, uint32_t t, float coef, cudaStream_t s);
+
 // ---- weight pass, tcgen05 path (zo_wpass_tc.cu) --------------------------------
 bool wpass_tc_supported(int32_t r);
 int32_t tc_hl_width(int32_t r);   // bf16 elements per hi/lo operand row

@@ -65,6 +65,10 @@ class SubZeroPlus:
         zb.zo_step(self.ctx, t, adam_t, losses, SCHEMES[scheme], eps, lr, beta1, beta2, eps_adam,
                    restore_query, restore_coef, optimizer, gamma_out)
 
+    def mezo_perturb(self, t, coef):
+        """Full-space SPSA pass of Eq. (1): every W_i <- rnd(W_i + coef Z_i)."""
+        zb.zo_mezo_perturb(self.ctx, t, coef)
+
     def sync(self):
         zb.zo_sync_status(self.ctx)
 
