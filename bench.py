@@ -39,7 +39,12 @@ FALLBACK_HBM_GBS = 6800.0
 # source it was taken on (reported as null once the source differs).
 TRAFFIC_BY_SOURCE = {
     # profiles/wpass_tc_r32_llama7b_2layers.md: 1.577 GB on the 2-layer subset, x16.0 by weights
-    "64253833d2a89ac2": 25.24e9,
+    ("64253833d2a89ac2", "llama7b_bf16_r32"): 25.24e9,
+}
+# thread instructions per weight of the full-space SPSA kernel (ncu), keyed by source hash
+INSTR_PER_WEIGHT_BY_SOURCE = {
+    # profiles/mezo_kernel_llama7b_2layers.md: 762.5 M warp instructions x 32 / 404.75 M weights
+    "02f7804f216dbccd": 60.3,
 }
 
 
@@ -51,6 +56,9 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="llama7b_bf16_r32")
     p.add_argument("--scheme", choices=["central", "forward"], default="central")
+    p.add_argument("--method", choices=["subzero", "mezo"], default="subzero",
+                   help="subzero: the SubZero+ step (default); mezo: the full-space SPSA "
+                        "baseline of Eq. (1), 3 passes per step")
     p.add_argument("--layers", type=int, default=0,
                    help="use only the first N layers of the workload (shape-preserving subset, "
                         "for profiling captures); 0 = all")
@@ -89,6 +97,13 @@ def subset(wl, layers):
     k = min(len(wl.shapes), layers * per_layer)
     return workloads.scaled(wl, name=f"{wl.name}[{layers} layers]", shapes=wl.shapes[:k],
                             zero_init=[i for i in wl.zero_init if i < k])
+
+
+def mezo_source_hash():
+    h = hashlib.sha256()
+    for name in ("zo_mezo.cu", "zo_device.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2608_15665_gb300", "csrc", name), "rb").read())
+    return h.hexdigest()[:16]
 
 
 # --------------------------------------------------------------------------- clocks
@@ -273,7 +288,22 @@ def run_ours(args):
     table = workloads.loss_table(wl, args.scheme, steps=W + 2 * K)
     table_dev = torch.from_numpy(table).to(dev)
 
+    if args.method == "mezo":
+        passes = 3
+
+    def do_step_mezo(t, losses, gamma=None):
+        # Eq. (1): evaluate at W + eps Z and W - eps Z, then restore fused with the SGD
+        # update, W += (eps - lr rho) Z; rho from the step's first loss pair
+        lp, lm = (float(losses[0]), float(losses[1])) if not torch.is_tensor(losses) \
+            else (float(table[t][0]), float(table[t][1]))
+        rho = (lp - lm) / (2.0 * wl.eps)
+        z.mezo_perturb(t, wl.eps)
+        z.mezo_perturb(t, -2.0 * wl.eps)
+        z.mezo_perturb(t, wl.eps - wl.lr * rho)
+
     def do_step(t, losses, gamma=None):
+        if args.method == "mezo":
+            return do_step_mezo(t, losses, gamma)
         if t % wl.F == 0:
             z.refresh(t // wl.F, reset_moments=(t == 0))
         for (qa, ca), second in calls:
@@ -369,13 +399,29 @@ def run_ours(args):
         "refresh_ms": refresh_ms,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
-                     "traffic": TRAFFIC_BY_SOURCE.get(src),
+                     "traffic": TRAFFIC_BY_SOURCE.get((src, wl.name)),
                      "kernel": "wpass_fma" if path == 1 else "wpass_tc",
                      "algorithmic_bytes_per_launch": bytes_pass,
                      "avg_launch_ms": avg_launch_s * 1e3, "launches_timed": wpass_n},
         "clocks": clk,
         "gpu_launches": int(launches),
     }
+    if args.method == "mezo":
+        # bound by instruction issue: peak = SMs x 128 lanes x max SM clock (thread
+        # instructions per second); achieved = instructions per weight (ncu count of the
+        # kernel, profiles/mezo_kernel_llama7b_2layers.md) x weights / launch time
+        line["metric"] = "MeZO full-space SPSA (Eq. (1)) steps/s at 7B shape, 1 GB300"
+        ipw = INSTR_PER_WEIGHT_BY_SOURCE.get(mezo_source_hash())
+        issue_peak = 152 * 128 * 2.07e9 / 1e12
+        ach = ipw * wl.params / avg_launch_s / 1e12 if ipw else None
+        line["roofline"] = {"bound": "alu", "achieved": ach, "peak": issue_peak,
+                            "unit": "T thread-instructions/s", "frac": ach / issue_peak if ach else None,
+                            "peak_kind": "derived: 152 SMs x 128 lanes x 2.07 GHz",
+                            "instructions_per_weight": ipw, "kernel": "mezo_kernel",
+                            "weight_gbs": achieved, "weight_gbs_frac_of_hbm": achieved / peak,
+                            "avg_launch_ms": avg_launch_s * 1e3, "launches_timed": wpass_n}
+        line["config"]["method"] = "mezo"
+        line["config"].pop("r"); line["config"].pop("q")
     if e2e:
         line["e2e"] = e2e
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
