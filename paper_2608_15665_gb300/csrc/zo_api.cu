@@ -44,6 +44,7 @@ struct QrLevel {
 
 void zo::set_last_error(const char* msg) { g_last_error = msg; }
 
+
 struct zo_ctx {
   int device = 0;
   cudaStream_t stream = nullptr;
