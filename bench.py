@@ -93,6 +93,7 @@ def subset(wl, layers):
         return wl
     from paper_2608_15665_gb300 import workloads
     per_layer = {"opt1.3b_bf16_r16": 6, "llama7b_bf16_r32": 7, "dense32b_bf16_r64": 7,
+                 "llama7b_bf16_r128_q99": 7,
                  "lora_opt13b_f32_r4": 4, "single256_f32_r8": 1}[wl.name]
     k = min(len(wl.shapes), layers * per_layer)
     return workloads.scaled(wl, name=f"{wl.name}[{layers} layers]", shapes=wl.shapes[:k],

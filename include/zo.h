@@ -84,7 +84,8 @@ enum {
 
 /* Options for zo_set_option. */
 enum {
-  ZO_OPTION_WPASS_PATH = 0, /* 0 = automatic, 1 = fp32-FMA path, 2 = tcgen05 path */
+  ZO_OPTION_WPASS_PATH = 0, /* 0 = automatic (tcgen05 when every W is bf16 and r >= 16),
+                               1 = fp32-FMA path, 2 = tcgen05 path */
   ZO_OPTION_TIMING = 1,     /* 1 = record CUDA events around every weight-pass launch */
   ZO_OPTION_TEST_WAIT_TIMEOUT = 2 /* test hook: 1 = in the next tensor-core weight pass, one
                                      CTA first waits on a barrier nothing arrives on, so its
@@ -112,7 +113,7 @@ typedef struct zo_ctx zo_ctx;
 /*
  * zo_create -- bind the caller's matrices into a context (Alg. 3 "Require" line).
  *   mats[n_mats]: copied; the pointers inside must stay valid until zo_destroy.
- *   r: subspace rank, 1 <= r <= min(m_i, n_i); this build supports r in {4, 8, 16, 32, 64}.
+ *   r: subspace rank, 1 <= r <= min(m_i, n_i); this build supports r in {4, 8, 16, 32, 64, 128}.
  *   q: queries per step (K in the paper), 1 <= q <= 4096.
  *   seed: 64-bit base seed of the Philox key.
  *   matrix_index_base: matrix i of this table uses Philox matrix index base + i

@@ -33,7 +33,9 @@ zo_status cuda_fail(cudaError_t e, const char* what) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-bool supported_rank(int32_t r) { return r == 4 || r == 8 || r == 16 || r == 32 || r == 64; }
+bool supported_rank(int32_t r) {
+  return r == 4 || r == 8 || r == 16 || r == 32 || r == 64 || r == 128;
+}
 
 struct QrLevel {
   std::vector<zo::QrBlock> up;    // all blocks of this level (tops included)
@@ -339,7 +341,7 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
     return ZO_ERR_INVALID_ARG;
   }
   if (!supported_rank(r)) {
-    g_last_error = "rank r must be one of 4, 8, 16, 32, 64";
+    g_last_error = "rank r must be one of 4, 8, 16, 32, 64, 128";
     return ZO_ERR_SHAPE;
   }
   if (q < 1 || q > 4096) {
@@ -658,7 +660,7 @@ zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
   if (option == ZO_OPTION_WPASS_PATH) {
     if (value < 0 || value > 2) return ZO_ERR_INVALID_ARG;
     if (value == 2 && !c->tc_ok) {
-      g_last_error = "the tensor-core weight pass needs every W in bf16 and r in {16, 32, 64}";
+      g_last_error = "the tensor-core weight pass needs every W in bf16 and r in {16, 32, 64, 128}";
       return ZO_ERR_UNSUPPORTED;
     }
     c->path_option = (int)value;

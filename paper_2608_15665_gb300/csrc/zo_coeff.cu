@@ -117,7 +117,7 @@ __global__ void __launch_bounds__(256) coeff_kernel(const MatDesc* __restrict__ 
 template <int R>
 __global__ void __launch_bounds__(256) project_fma_kernel(const MatDesc* __restrict__ mats,
                                                           const int2* __restrict__ units) {
-  __shared__ float Cs[R * R];
+  extern __shared__ float Cs[];   // R x R
   const int2 u = units[blockIdx.x];
   const MatDesc md = mats[u.x];
   const int tid = threadIdx.x;
@@ -133,11 +133,31 @@ __global__ void __launch_bounds__(256) project_fma_kernel(const MatDesc* __restr
     v[4 * b] = t.x; v[4 * b + 1] = t.y; v[4 * b + 2] = t.z; v[4 * b + 3] = t.w;
   }
   for (int a = tid >> 7; a < R; a += 2) {
+    const float4* crow = reinterpret_cast<const float4*>(Cs + a * R);
     float acc = 0.f;
 #pragma unroll
-    for (int b = 0; b < R; ++b) acc = fmaf(Cs[a * R + b], v[b], acc);
+    for (int b4 = 0; b4 < R / 4; ++b4) {
+      const float4 c4 = crow[b4];
+      acc = fmaf(c4.x, v[4 * b4], acc);
+      acc = fmaf(c4.y, v[4 * b4 + 1], acc);
+      acc = fmaf(c4.z, v[4 * b4 + 2], acc);
+      acc = fmaf(c4.w, v[4 * b4 + 3], acc);
+    }
     md.P[(int64_t)a * md.n + j] = acc;
   }
+}
+
+template <int R>
+cudaError_t launch_project_fma_r(const MatDesc* d_mats, const int2* d_units, int32_t n_units,
+                                 cudaStream_t s) {
+  const size_t smem = sizeof(float) * R * R;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(project_fma_kernel<R>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  project_fma_kernel<R><<<n_units, 256, smem, s>>>(d_mats, d_units);
+  return cudaGetLastError();
 }
 
 }  // namespace
@@ -154,14 +174,14 @@ cudaError_t launch_project_fma(const MatDesc* d_mats, const int2* d_units, int32
                                int32_t r, cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
-    case 4: project_fma_kernel<4><<<n_units, 256, 0, s>>>(d_mats, d_units); break;
-    case 8: project_fma_kernel<8><<<n_units, 256, 0, s>>>(d_mats, d_units); break;
-    case 16: project_fma_kernel<16><<<n_units, 256, 0, s>>>(d_mats, d_units); break;
-    case 32: project_fma_kernel<32><<<n_units, 256, 0, s>>>(d_mats, d_units); break;
-    case 64: project_fma_kernel<64><<<n_units, 256, 0, s>>>(d_mats, d_units); break;
+    case 4: return launch_project_fma_r<4>(d_mats, d_units, n_units, s);
+    case 8: return launch_project_fma_r<8>(d_mats, d_units, n_units, s);
+    case 16: return launch_project_fma_r<16>(d_mats, d_units, n_units, s);
+    case 32: return launch_project_fma_r<32>(d_mats, d_units, n_units, s);
+    case 64: return launch_project_fma_r<64>(d_mats, d_units, n_units, s);
+    case 128: return launch_project_fma_r<128>(d_mats, d_units, n_units, s);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 }  // namespace zo

@@ -75,20 +75,31 @@ __device__ __forceinline__ void warp_reduce_scatter(float (&p)[R], int lane) {
   }
 }
 
-// Block-wide sum of R per-thread values into sm.red[buf][warp][c] (one partial per warp).
-template <int R>
-__device__ __forceinline__ void block_partials(float (&p)[R], QrSmem<R>& sm, int buf) {
+// Block-wide sum of H per-thread values (columns off .. off+H-1) into
+// red[warp][off + c] (one partial per warp).
+template <int H>
+__device__ __forceinline__ void block_partials(float (&p)[H], float* red_buf, int row_len,
+                                               int off) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  warp_reduce_scatter<R>(p, lane);
-  if (R >= 32) {
-    constexpr int kKeep = R >= 32 ? R / 32 : 1;
+  float* red = red_buf + warp * row_len + off;
+  warp_reduce_scatter<H>(p, lane);
+  if (H >= 32) {
+    constexpr int kKeep = H >= 32 ? H / 32 : 1;
 #pragma unroll
-    for (int k = 0; k < kKeep; ++k) sm.red[buf][warp][lane * kKeep + k] = p[k];
+    for (int k = 0; k < kKeep; ++k) red[lane * kKeep + k] = p[k];
   } else {
-    constexpr int kStride = R >= 32 ? 1 : 32 / R;
-    if (lane % kStride == 0) sm.red[buf][warp][lane / kStride] = p[0];
+    constexpr int kStride = H >= 32 ? 1 : 32 / H;
+    if (lane % kStride == 0) red[lane / kStride] = p[0];
   }
 }
+
+// Columns are reduced in groups of at most 64 so that R = 128 fits in registers.
+template <int R>
+struct QrHalves {
+  static constexpr int kH = R > 64 ? 64 : R;
+  static constexpr int kN = R / kH;
+  static constexpr int kC32 = (R + 31) / 32;       // 32-column groups handled by warp 0
+};
 
 // a[j] for a runtime j without indexing the register array dynamically.
 template <int R>
@@ -105,35 +116,47 @@ template <int R>
 __device__ void factor_block(float (&a)[QrShape<R>::kRPT][R], QrSmem<R>& sm) {
   constexpr int RPT = QrShape<R>::kRPT;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  using Hv = QrHalves<R>;
   for (int j = 0; j < R; ++j) {
     const int buf = j & 1;
-    float p[R];
 #pragma unroll
-    for (int c = 0; c < R; ++c) p[c] = 0.f;
+    for (int hh = 0; hh < Hv::kN; ++hh) {
+      float p[Hv::kH];
 #pragma unroll
-    for (int rho = 0; rho < RPT; ++rho) {
-      const int i = rho * kQrThreads + tid;
-      if (i > j) {
-        const float x = pick<R>(a[rho], j);
+      for (int c = 0; c < Hv::kH; ++c) p[c] = 0.f;
 #pragma unroll
-        for (int c = 0; c < R; ++c)
-          if (c >= j) p[c] = fmaf(x, a[rho][c], p[c]);
+      for (int rho = 0; rho < RPT; ++rho) {
+        const int i = rho * kQrThreads + tid;
+        if (i > j) {
+          const float x = pick<R>(a[rho], j);
+#pragma unroll
+          for (int c = 0; c < Hv::kH; ++c)
+            if (hh * Hv::kH + c >= j) p[c] = fmaf(x, a[rho][hh * Hv::kH + c], p[c]);
+        }
       }
+      block_partials<Hv::kH>(p, &sm.red[buf][0][0], R, hh * Hv::kH);
     }
     if (tid == j) {
 #pragma unroll
       for (int c = 0; c < R; ++c) sm.rowj[buf][c] = a[0][c];
     }
-    block_partials<R>(p, sm, buf);
     __syncthreads();
     if (warp == 0) {
-      float s_lo = 0.f, s_hi = 0.f;
+      float sk[Hv::kC32];
 #pragma unroll
-      for (int w = 0; w < kQrWarps; ++w) {
-        if (lane < R) s_lo += sm.red[buf][w][lane];
-        if (R > 32) s_hi += sm.red[buf][w][(lane + 32) % R];
+      for (int k = 0; k < Hv::kC32; ++k) {
+        const int c = lane + 32 * k;
+        sk[k] = 0.f;
+        if (c < R) {
+#pragma unroll
+          for (int w = 0; w < kQrWarps; ++w) sk[k] += sm.red[buf][w][c];
+        }
       }
-      const float s_j = __shfl_sync(0xffffffffu, j < 32 ? s_lo : s_hi, j & 31);
+      float sel = 0.f;
+#pragma unroll
+      for (int k = 0; k < Hv::kC32; ++k)
+        if (k == (j >> 5)) sel = sk[k];
+      const float s_j = __shfl_sync(0xffffffffu, sel, j & 31);
       const float alpha = sm.rowj[buf][j];
       float tau = 0.f, beta = alpha, scale = 0.f;
       if (s_j != 0.f) {
@@ -141,9 +164,11 @@ __device__ void factor_block(float (&a)[QrShape<R>::kRPT][R], QrSmem<R>& sm) {
         tau = (beta - alpha) / beta;
         scale = 1.0f / (alpha - beta);
       }
-      if (lane < R && lane > j) sm.wbuf[buf][lane] = fmaf(scale, s_lo, sm.rowj[buf][lane]);
-      if (R > 32 && lane + 32 > j)
-        sm.wbuf[buf][lane + 32] = fmaf(scale, s_hi, sm.rowj[buf][lane + 32]);
+#pragma unroll
+      for (int k = 0; k < Hv::kC32; ++k) {
+        const int c = lane + 32 * k;
+        if (c < R && c > j) sm.wbuf[buf][c] = fmaf(scale, sk[k], sm.rowj[buf][c]);
+      }
       if (lane == 0) {
         sm.scal[buf][0] = tau;
         sm.scal[buf][1] = scale;
@@ -183,21 +208,25 @@ __device__ void apply_reflectors_backward(float (&a)[QrShape<R>::kRPT][R], const
   constexpr int RPT = QrShape<R>::kRPT;
   constexpr int LD = QrShape<R>::kLd;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  using Hv = QrHalves<R>;
   for (int j = R - 1; j >= 0; --j) {
     const int buf = j & 1;
-    float p[R];
 #pragma unroll
-    for (int c = 0; c < R; ++c) p[c] = 0.f;
+    for (int hh = 0; hh < Hv::kN; ++hh) {
+      float p[Hv::kH];
 #pragma unroll
-    for (int rho = 0; rho < RPT; ++rho) {
-      const int i = rho * kQrThreads + tid;
-      if (i >= j) {
-        const float v = (i == j) ? 1.0f : refl[i * LD + j];
+      for (int c = 0; c < Hv::kH; ++c) p[c] = 0.f;
 #pragma unroll
-        for (int c = 0; c < R; ++c) p[c] = fmaf(v, a[rho][c], p[c]);
+      for (int rho = 0; rho < RPT; ++rho) {
+        const int i = rho * kQrThreads + tid;
+        if (i >= j) {
+          const float v = (i == j) ? 1.0f : refl[i * LD + j];
+#pragma unroll
+          for (int c = 0; c < Hv::kH; ++c) p[c] = fmaf(v, a[rho][hh * Hv::kH + c], p[c]);
+        }
       }
+      block_partials<Hv::kH>(p, &sm.red[buf][0][0], R, hh * Hv::kH);
     }
-    block_partials<R>(p, sm, buf);
     __syncthreads();
     if (warp == 0) {
 #pragma unroll
@@ -405,6 +434,7 @@ int32_t qr_block_rows(int32_t r) {
     case 16: return QrShape<16>::kB;
     case 32: return QrShape<32>::kB;
     case 64: return QrShape<64>::kB;
+    case 128: return QrShape<128>::kB;
     default: return 0;
   }
 }
@@ -418,6 +448,7 @@ cudaError_t launch_qr_up(const QrBlock* d_blocks, int32_t n_blocks, int32_t r, u
     case 16: return launch_up_r<16>(d_blocks, n_blocks, seed, refresh_idx, s);
     case 32: return launch_up_r<32>(d_blocks, n_blocks, seed, refresh_idx, s);
     case 64: return launch_up_r<64>(d_blocks, n_blocks, seed, refresh_idx, s);
+    case 128: return launch_up_r<128>(d_blocks, n_blocks, seed, refresh_idx, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -431,6 +462,7 @@ cudaError_t launch_qr_down(const QrBlock* d_blocks, int32_t n_blocks, int32_t r,
     case 16: return launch_down_r<16>(d_blocks, n_blocks, s);
     case 32: return launch_down_r<32>(d_blocks, n_blocks, s);
     case 64: return launch_down_r<64>(d_blocks, n_blocks, s);
+    case 128: return launch_down_r<128>(d_blocks, n_blocks, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -208,6 +208,7 @@ cudaError_t launch_wpass_fma(const MatDesc* d_mats, int32_t n_mats, const int64_
     case 16: return launch_r<16>(d_mats, n_mats, d_tile_prefix, n_tiles, s);
     case 32: return launch_r<32>(d_mats, n_mats, d_tile_prefix, n_tiles, s);
     case 64: return launch_r<64>(d_mats, n_mats, d_tile_prefix, n_tiles, s);
+    case 128: return launch_r<128>(d_mats, n_mats, d_tile_prefix, n_tiles, s);
     default: return cudaErrorInvalidValue;
   }
 }

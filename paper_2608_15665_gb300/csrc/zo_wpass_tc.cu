@@ -49,9 +49,10 @@ struct TcCfg {
   static constexpr int kHLW = hl_width(R);
   static constexpr int kPanels = kHLW / 64;
   static constexpr int kOpBytes = kPanels * kPanelBytes;        // one operand tile (hi + lo)
-  static constexpr int kWStages = R >= 64 ? 3 : 4;
-  static constexpr int kAStages = 2;
-  static constexpr int kBStages = 2;
+  // ring depths per rank: 32 KB W stages, operand tiles of 16 / 16 / 32 / 64 KB
+  static constexpr int kWStages = R >= 128 ? 2 : R >= 64 ? 3 : 4;
+  static constexpr int kAStages = R >= 128 ? 1 : 2;
+  static constexpr int kBStages = R >= 128 ? 1 : 2;
   static constexpr int kKC = R / 16;                            // K chunks of 16
   static constexpr size_t kSmem = (size_t)kWStages * kWStageBytes + (size_t)kAStages * kOpBytes +
                                   (size_t)kBStages * kOpBytes + 1024 /*barriers*/ + 1024 /*align*/;
@@ -437,7 +438,8 @@ __global__ void __launch_bounds__(128)
 split_u_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
                const int2* __restrict__ units, __nv_bfloat16* __restrict__ u_hl) {
   constexpr int kVecPerRow = hl_width(R) * 2 / 16;
-  __shared__ uint4 Os[128 * kVecPerRow];
+  extern __shared__ uint4 su_smem[];
+  uint4* Os = su_smem;                                     // 128 x kVecPerRow
   const int2 u = units[blockIdx.x];
   const MatDesc md = mats[u.x];
   const int tid = threadIdx.x;
@@ -489,10 +491,17 @@ project_split_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__
       float x[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
-        const float* crow = Cs + (8 * g + k) * R;
+        // C row read as 16-byte broadcasts: 4 FMAs per shared-memory load
+        const float4* crow = reinterpret_cast<const float4*>(Cs + (8 * g + k) * R);
         float acc = 0.f;
 #pragma unroll
-        for (int b = 0; b < R; ++b) acc = fmaf(crow[b], v[b], acc);
+        for (int b4 = 0; b4 < R / 4; ++b4) {
+          const float4 c4 = crow[b4];
+          acc = fmaf(c4.x, v[4 * b4], acc);
+          acc = fmaf(c4.y, v[4 * b4 + 1], acc);
+          acc = fmaf(c4.z, v[4 * b4 + 2], acc);
+          acc = fmaf(c4.w, v[4 * b4 + 3], acc);
+        }
         x[k] = acc;
       }
       uint4 hi, lo;
@@ -508,6 +517,19 @@ project_split_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__
 template <int R>
 constexpr size_t project_split_smem() {
   return 128 * (size_t)hl_width(R) * 2 + sizeof(float) * R * R;
+}
+
+template <int R>
+cudaError_t launch_split_u_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                             int32_t n_units, __nv_bfloat16* u_hl, cudaStream_t s) {
+  const size_t smem = 128 * (size_t)hl_width(R) * 2;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(split_u_kernel<R>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  split_u_kernel<R><<<n_units, 128, smem, s>>>(d_mats, d_tc, d_units, u_hl);
+  return cudaGetLastError();
 }
 
 template <int R>
@@ -538,7 +560,7 @@ cudaError_t launch_tc_r(const CUtensorMap& tm_a, const CUtensorMap& tm_b, const 
 
 }  // namespace
 
-bool wpass_tc_supported(int32_t r) { return r == 16 || r == 32 || r == 64; }
+bool wpass_tc_supported(int32_t r) { return r == 16 || r == 32 || r == 64 || r == 128; }
 int32_t tc_hl_width(int32_t r) { return hl_width(r); }
 int32_t tc_tile_rows() { return kBM; }
 int32_t tc_tile_cols() { return kBN; }
@@ -547,12 +569,12 @@ cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2*
                            int32_t n_units, int32_t r, __nv_bfloat16* u_hl, cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
-    case 16: split_u_kernel<16><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, u_hl); break;
-    case 32: split_u_kernel<32><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, u_hl); break;
-    case 64: split_u_kernel<64><<<n_units, 128, 0, s>>>(d_mats, d_tc, d_units, u_hl); break;
+    case 16: return launch_split_u_r<16>(d_mats, d_tc, d_units, n_units, u_hl, s);
+    case 32: return launch_split_u_r<32>(d_mats, d_tc, d_units, n_units, u_hl, s);
+    case 64: return launch_split_u_r<64>(d_mats, d_tc, d_units, n_units, u_hl, s);
+    case 128: return launch_split_u_r<128>(d_mats, d_tc, d_units, n_units, u_hl, s);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
@@ -562,6 +584,7 @@ cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const
     case 16: return launch_project_split_r<16>(d_mats, d_tc, d_units, n_units, p_hl, s);
     case 32: return launch_project_split_r<32>(d_mats, d_tc, d_units, n_units, p_hl, s);
     case 64: return launch_project_split_r<64>(d_mats, d_tc, d_units, n_units, p_hl, s);
+    case 128: return launch_project_split_r<128>(d_mats, d_tc, d_units, n_units, p_hl, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -575,6 +598,7 @@ cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
     case 16: return launch_tc_r<16>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
     case 32: return launch_tc_r<32>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
     case 64: return launch_tc_r<64>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
+    case 128: return launch_tc_r<128>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -87,6 +87,11 @@ def _build():
         "lora_opt13b_f32_r4", lora, "f32", r=4, q=8, eps=1e-3, lr=1e-2, beta1=0.9, beta2=0.95,
         eps_adam=1e-8, steps=200, F=50, seed=1004, zero_init=zero,
         note="OPT-13B LoRA on q,v: 40 x 2 x {A 8x5120, B 5120x8}, B zero at init")
+    wl["llama7b_bf16_r128_q99"] = Workload(
+        "llama7b_bf16_r128_q99", llama, "bf16", r=128, q=99, eps=1e-3, lr=1e-3, beta1=0.9,
+        beta2=0.95, eps_adam=1e-8, steps=400, F=50, seed=1006,
+        note="the paper's default scale (App. A.2, Table 7): r = 128, K = 99 queries, "
+             "F = 50, on the LLaMA-7B shapes")
     big = []
     for _ in range(64):
         big += [(8192, 5120), (1024, 5120), (1024, 5120), (5120, 8192),

@@ -24,6 +24,7 @@ CASES = {
     "r16": (16, [(300, 520, "bf16", 528), (130, 1000, "bf16", None), (100, 96, "f32", 100)]),
     "r32": (32, [(300, 520, "bf16", None), (1030, 72, "bf16", 80), (64, 2048, "f32", None)]),
     "r64": (64, [(300, 520, "bf16", None), (130, 1000, "bf16", None), (1030, 72, "f32", None)]),
+    "r128": (128, [(300, 520, "bf16", None), (130, 1000, "f32", None)]),
 }
 
 
@@ -54,7 +55,7 @@ def test_perturb_pass_matches_oracle(lib, gpu, case, eps):
     z.close()
 
 
-@pytest.mark.parametrize("case", ["r4", "r8", "r16", "r32", "r64"])
+@pytest.mark.parametrize("case", ["r4", "r8", "r16", "r32", "r64", "r128"])
 @pytest.mark.parametrize("scheme", ["central", "forward", "direct"])
 def test_step_matches_oracle(lib, gpu, case, scheme):
     z, base = _build(gpu, case, seed=777)
@@ -176,6 +177,7 @@ TC_CASES = {
     "tc16": (16, [(300, 520, None), (130, 1000, 1008), (1030, 72, None), (128, 128, None)]),
     "tc32": (32, [(300, 520, 528), (1030, 72, 80), (257, 2048, None)]),
     "tc64": (64, [(300, 520, None), (130, 1000, None), (1030, 72, 72), (2048, 384, None)]),
+    "tc128": (128, [(300, 520, None), (130, 1000, 1008), (1030, 136, None)]),
 }
 
 

@@ -16,6 +16,7 @@ CASES = [
     (16, [(2048, 8192), (1500, 40)]),
     (32, [(11008, 4096), (600, 33)]),                # three-level tree for 11008 rows
     (64, [(25600, 128), (300, 64), (64, 257)]),      # five levels for 25600 rows; m == r
+    (128, [(2048, 130), (300, 256)]),                 # four levels for 2048 rows; ragged tail
 ]
 
 
