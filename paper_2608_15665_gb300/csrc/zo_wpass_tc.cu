@@ -50,9 +50,14 @@ struct TcCfg {
   static constexpr int kPanels = kHLW / 64;
   static constexpr int kOpBytes = kPanels * kPanelBytes;        // one operand tile (hi + lo)
   // ring depths per rank: 32 KB W stages, operand tiles of 16 / 16 / 32 / 64 KB
-  static constexpr int kWStages = R >= 128 ? 2 : R >= 64 ? 3 : 4;
+  // (R = 128: 3 x 32 + 64 + 64 KB + barriers = 226 KB of the 227 KB a CTA may hold)
+  static constexpr int kWStages = R >= 64 ? 3 : 4;
   static constexpr int kAStages = R >= 128 ? 1 : 2;
   static constexpr int kBStages = R >= 128 ? 1 : 2;
+  // With one operand stage (R = 128) each operand tile is loaded and released in two
+  // K halves with barriers of their own -- half h = hi panel h + lo panel 2 + h -- so
+  // the next tile's first half loads while the MMAs still read the second.
+  static constexpr int kSplit = R >= 128 ? 2 : 1;
   static constexpr int kKC = R / 16;                            // K chunks of 16
   static constexpr size_t kSmem = (size_t)kWStages * kWStageBytes + (size_t)kAStages * kOpBytes +
                                   (size_t)kBStages * kOpBytes + 1024 /*barriers*/ + 1024 /*align*/;
@@ -146,6 +151,10 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
   static_assert(Cfg::kWStages >= 2 && Cfg::kWStages <= 4, "W ring must fit Shared::w_full");
   static_assert(Cfg::kAStages >= 1 && Cfg::kAStages <= 2, "A ring must fit Shared::a_full");
   static_assert(Cfg::kBStages >= 1 && Cfg::kBStages <= 2, "B ring must fit Shared::b_full");
+  static_assert(Cfg::kAStages * Cfg::kSplit <= 2 && Cfg::kBStages * Cfg::kSplit <= 2,
+                "operand barriers per stage and half must fit Shared::a_full / b_full");
+  static_assert(Cfg::kSplit == 1 || (Cfg::kPanels == 4 && Cfg::kKC == 8),
+                "the half split assumes hi = panels 0, 1 and lo = panels 2, 3");
   static_assert(sizeof(Shared) <= 1024, "barrier block");
   static_assert(Cfg::kSmem <= 227 * 1024, "shared memory per CTA");
   extern __shared__ uint8_t smem_raw[];
@@ -173,11 +182,11 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
       mbar_init(&sh.w_full[s], 1);
       mbar_init(&sh.w_empty[s], 4);
     }
-    for (int s = 0; s < Cfg::kAStages; ++s) {
+    for (int s = 0; s < Cfg::kAStages * Cfg::kSplit; ++s) {
       mbar_init(&sh.a_full[s], 1);
       mbar_init(&sh.a_empty[s], 1);
     }
-    for (int s = 0; s < Cfg::kBStages; ++s) {
+    for (int s = 0; s < Cfg::kBStages * Cfg::kSplit; ++s) {
       mbar_init(&sh.b_full[s], 1);
       mbar_init(&sh.b_empty[s], 1);
     }
@@ -225,30 +234,35 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
                         (int)(ti.rb * kBM + 32 * g), &sh.w_full[s]);
         ++n_w;
       }
-      // U operand tile, once per row block
-      if (ti.i != prev_i || ti.rb != prev_rb) {
-        const int s = (int)(n_a % Cfg::kAStages);
-        const uint32_t ph = (uint32_t)((n_a / Cfg::kAStages) & 1);
-        if (!mbar_wait_bounded(&sh.a_empty[s], ph ^ 1u, abort, wait_cycles)) { ok = false; break; }
-        mbar_arrive_expect_tx(&sh.a_full[s], Cfg::kOpBytes);
-        for (int p = 0; p < Cfg::kPanels; ++p)
-          tma_load_2d(a_smem + s * Cfg::kOpBytes + p * kPanelBytes, &tm_a, 64 * p,
-                      (int)(mt.u_row0 + ti.rb * kBM), &sh.a_full[s]);
+      // U operand tile once per row block, P operand tile of this column block; with the
+      // half split the order is U half 0, P half 0, U half 1, P half 1
+      const bool new_a = ti.i != prev_i || ti.rb != prev_rb;
+      const int sa = (int)(n_a % Cfg::kAStages), sb = (int)(n_b % Cfg::kBStages);
+      const uint32_t pa = (uint32_t)((n_a / Cfg::kAStages) & 1);
+      const uint32_t pb = (uint32_t)((n_b / Cfg::kBStages) & 1);
+      for (int h = 0; h < Cfg::kSplit && ok; ++h) {
+        if (new_a) {
+          const int bi = sa * Cfg::kSplit + h;
+          if (!mbar_wait_bounded(&sh.a_empty[bi], pa ^ 1u, abort, wait_cycles)) { ok = false; break; }
+          mbar_arrive_expect_tx(&sh.a_full[bi], Cfg::kOpBytes / Cfg::kSplit);
+          for (int p = h; p < Cfg::kPanels; p += Cfg::kSplit)
+            tma_load_2d(a_smem + sa * Cfg::kOpBytes + p * kPanelBytes, &tm_a, 64 * p,
+                        (int)(mt.u_row0 + ti.rb * kBM), &sh.a_full[bi]);
+        }
+        const int bi = sb * Cfg::kSplit + h;
+        if (!mbar_wait_bounded(&sh.b_empty[bi], pb ^ 1u, abort, wait_cycles)) { ok = false; break; }
+        mbar_arrive_expect_tx(&sh.b_full[bi], Cfg::kOpBytes / Cfg::kSplit);
+        for (int p = h; p < Cfg::kPanels; p += Cfg::kSplit)
+          tma_load_2d(b_smem + sb * Cfg::kOpBytes + p * kPanelBytes, &tm_b, 64 * p,
+                      (int)(mt.p_row0 + ti.cb * kBN), &sh.b_full[bi]);
+      }
+      if (!ok) break;
+      if (new_a) {
         ++n_a;
         prev_i = ti.i;
         prev_rb = ti.rb;
       }
-      // P operand tile of this column block
-      {
-        const int s = (int)(n_b % Cfg::kBStages);
-        const uint32_t ph = (uint32_t)((n_b / Cfg::kBStages) & 1);
-        if (!mbar_wait_bounded(&sh.b_empty[s], ph ^ 1u, abort, wait_cycles)) { ok = false; break; }
-        mbar_arrive_expect_tx(&sh.b_full[s], Cfg::kOpBytes);
-        for (int p = 0; p < Cfg::kPanels; ++p)
-          tma_load_2d(b_smem + s * Cfg::kOpBytes + p * kPanelBytes, &tm_b, 64 * p,
-                      (int)(mt.p_row0 + ti.cb * kBN), &sh.b_full[s]);
-        ++n_b;
-      }
+      ++n_b;
     }
     if (!ok) give_up(sh, status);
     // drain: the last copy issued into every slot has landed before the CTA exits
@@ -258,11 +272,15 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
     }
     for (int s = 0; s < Cfg::kAStages; ++s) {
       const int64_t k = last_in_slot(n_a, s, Cfg::kAStages);
-      if (k >= 0) mbar_wait_bounded(&sh.a_full[s], (uint32_t)((k / Cfg::kAStages) & 1), nullptr, wait_cycles);
+      for (int h = 0; h < Cfg::kSplit && k >= 0; ++h)
+        mbar_wait_bounded(&sh.a_full[s * Cfg::kSplit + h], (uint32_t)((k / Cfg::kAStages) & 1),
+                          nullptr, wait_cycles);
     }
     for (int s = 0; s < Cfg::kBStages; ++s) {
       const int64_t k = last_in_slot(n_b, s, Cfg::kBStages);
-      if (k >= 0) mbar_wait_bounded(&sh.b_full[s], (uint32_t)((k / Cfg::kBStages) & 1), nullptr, wait_cycles);
+      for (int h = 0; h < Cfg::kSplit && k >= 0; ++h)
+        mbar_wait_bounded(&sh.b_full[s * Cfg::kSplit + h], (uint32_t)((k / Cfg::kBStages) & 1),
+                          nullptr, wait_cycles);
     }
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA issuer
@@ -272,42 +290,59 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
     int64_t prev_rb = -1;
     int sa = 0;
     bool ok = true;
-    TileIter ti;
+    TileIter ti, nx;                            // nx runs one tile ahead of ti
     ti.init(mats, n_mats, t_begin, t_end, t_stride);
     ti.chunk = kTileChunk;
-    for (; ti.valid(); ti.next(), ++it) {
-      if (ti.i != prev_i || ti.rb != prev_rb) {
-        if (a_it > 0) mma_commit(&sh.a_empty[(a_it - 1) % Cfg::kAStages]);
+    nx = ti;
+    nx.next();
+    for (; ti.valid(); ti = nx, nx.next(), ++it) {
+      const bool new_a = ti.i != prev_i || ti.rb != prev_rb;
+      uint32_t pa = 0;
+      if (new_a) {
         sa = (int)(a_it % Cfg::kAStages);
-        if (!mbar_wait_bounded(&sh.a_full[sa], (uint32_t)((a_it / Cfg::kAStages) & 1), abort,
-                               wait_cycles)) { ok = false; break; }
+        pa = (uint32_t)((a_it / Cfg::kAStages) & 1);
         ++a_it;
         prev_i = ti.i;
         prev_rb = ti.rb;
       }
+      // the U tile is released after its last tile: the next tile starts another row
+      // block (or there is none)
+      const bool last_a = !nx.valid() || nx.i != ti.i || nx.rb != ti.rb;
       const int sb = (int)(it % Cfg::kBStages);
-      if (!mbar_wait_bounded(&sh.b_full[sb], (uint32_t)((it / Cfg::kBStages) & 1), abort,
-                             wait_cycles)) { ok = false; break; }
+      const uint32_t pb = (uint32_t)((it / Cfg::kBStages) & 1);
       const int acc = (int)(it & 1);
       if (!mbar_wait_bounded(&sh.acc_empty[acc], (uint32_t)(((it >> 1) & 1) ^ 1), abort,
                              wait_cycles)) { ok = false; break; }
-      tc_fence_after();
       const uint32_t d = tmem + (uint32_t)(acc * kBN);
       const uint32_t a_base = smem_u32(a_smem + sa * Cfg::kOpBytes);
       const uint32_t b_base = smem_u32(b_smem + sb * Cfg::kOpBytes);
+      for (int h = 0; h < Cfg::kSplit; ++h) {
+        if (new_a && !mbar_wait_bounded(&sh.a_full[sa * Cfg::kSplit + h], pa, abort, wait_cycles)) {
+          ok = false;
+          break;
+        }
+        if (!mbar_wait_bounded(&sh.b_full[sb * Cfg::kSplit + h], pb, abort, wait_cycles)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
 #pragma unroll
-      for (int kk = 0; kk < Cfg::kKC; ++kk) {
-        // hi chunk kk at element 16 kk of the operand row, lo chunk at R + 16 kk
-        const int e_hi = 16 * kk, e_lo = R + 16 * kk;
-        const uint32_t off_hi = (uint32_t)((e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
-        const uint32_t off_lo = (uint32_t)((e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
-        const uint64_t a_hi = sdesc_k_sw128(a_base + off_hi), a_lo = sdesc_k_sw128(a_base + off_lo);
-        const uint64_t b_hi = sdesc_k_sw128(b_base + off_hi), b_lo = sdesc_k_sw128(b_base + off_lo);
-        mma_bf16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
-        mma_bf16(d, a_hi, b_lo, idesc, 1u);
-        mma_bf16(d, a_lo, b_hi, idesc, 1u);
+        for (int k2 = 0; k2 < Cfg::kKC / Cfg::kSplit; ++k2) {
+          const int kk = h * (Cfg::kKC / Cfg::kSplit) + k2;
+          // hi chunk kk at element 16 kk of the operand row, lo chunk at R + 16 kk
+          const int e_hi = 16 * kk, e_lo = R + 16 * kk;
+          const uint32_t off_hi = (uint32_t)((e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
+          const uint32_t off_lo = (uint32_t)((e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
+          const uint64_t a_hi = sdesc_k_sw128(a_base + off_hi), a_lo = sdesc_k_sw128(a_base + off_lo);
+          const uint64_t b_hi = sdesc_k_sw128(b_base + off_hi), b_lo = sdesc_k_sw128(b_base + off_lo);
+          mma_bf16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
+          mma_bf16(d, a_hi, b_lo, idesc, 1u);
+          mma_bf16(d, a_lo, b_hi, idesc, 1u);
+        }
+        mma_commit(&sh.b_empty[sb * Cfg::kSplit + h]);
+        if (last_a) mma_commit(&sh.a_empty[sa * Cfg::kSplit + h]);
       }
-      mma_commit(&sh.b_empty[sb]);
+      if (!ok) break;
       mma_commit(&sh.acc_full[acc]);
     }
     if (!ok) give_up(sh, status);
