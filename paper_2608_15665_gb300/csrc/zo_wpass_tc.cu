@@ -10,11 +10,14 @@
 // accumulates hi.hi + hi.lo + lo.hi in fp32 in Tensor Memory (relative error of
 // the product ~2^-16 instead of 2^-8).
 //
-// Roles of the 192 threads of a CTA (one CTA per SM, persistent over every G-th
+// Roles of the 224 threads of a CTA (one CTA per SM, persistent over every G-th
 // tile, G = number of CTAs):
-//   warp 0, lane 0: TMA producer -- W tile (8 boxes of 32 rows x 64 columns,
-//                   128-byte swizzle), the U operand tile when the row block
-//                   changes, the P operand tile of every tile.
+//   warp 0, lane 0: TMA producer of W -- each tile as 8 boxes of 32 rows x 64
+//                   columns, 128-byte swizzle, as far ahead as the W ring allows.
+//   warp 6, lane 0: TMA producer of the operands -- the U tile when the row block
+//                   changes, the P tile of every tile.  Apart from the W producer,
+//                   so a W prefetch never queues behind an operand slot that the
+//                   MMAs of an earlier tile still hold.
 //   warp 1, lane 0: MMA issuer -- 3 * r/16 tcgen05.mma (M=128, N=128, K=16) per
 //                   tile into one of two TMEM accumulators; warp 1 also owns
 //                   the TMEM allocation.
@@ -35,7 +38,7 @@ using namespace sm100;
 
 constexpr int kBM = 128;            // tile rows (TMEM lanes)
 constexpr int kBN = 128;            // tile columns (TMEM columns per accumulator)
-constexpr int kThreads = 192;
+constexpr int kThreads = 224;
 constexpr int kWBoxBytes = 32 * 64 * 2;          // one TMA box of W: 32 rows x 64 bf16
 constexpr int kWStageBytes = kBM * kBN * 2;      // 32 KB
 constexpr int kPanelBytes = kBM * 64 * 2;        // 128 rows x 128 bytes = 16 KB
@@ -210,16 +213,13 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
   const uint32_t tmem = sh.tmem_base;
 
   if (warp == 0 && lane == 0) {
-    // ------------------------------------------------------------ TMA producer
-    int64_t n_w = 0, n_a = 0, n_b = 0;          // copies issued into each ring
-    int prev_i = -1;
-    int64_t prev_rb = -1;
+    // ------------------------------------------------------------ TMA producer: W tiles
+    int64_t n_w = 0;                              // copies issued into the W ring
     bool ok = true;
     TileIter ti;
     ti.init(mats, n_mats, t_begin, t_end, t_stride);
     ti.chunk = kTileChunk;
     for (; ti.valid(); ti.next()) {
-      const TcMat& mt = mats[ti.i];
       const CUtensorMap* wmap = w_maps + ti.i;
       // W tile: 4 row groups x 2 column halves
       {
@@ -234,6 +234,25 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
                         (int)(ti.rb * kBM + 32 * g), &sh.w_full[s]);
         ++n_w;
       }
+    }
+    if (!ok) give_up(sh, status);
+    // drain: the last copy issued into every slot has landed before the CTA exits
+    for (int s = 0; s < Cfg::kWStages; ++s) {
+      const int64_t k = last_in_slot(n_w, s, Cfg::kWStages);
+      if (k >= 0) mbar_wait_bounded(&sh.w_full[s], (uint32_t)((k / Cfg::kWStages) & 1), nullptr, wait_cycles);
+    }
+  } else if (warp == 6 && lane == 0) {
+    // ------------------------------------------------------------ TMA producer: operands
+    int64_t n_a = 0, n_b = 0;                     // operand tiles issued into each ring
+    int64_t a_iss[2] = {0, 0}, b_iss[2] = {0, 0};  // phases issued per barrier
+    int prev_i = -1;
+    int64_t prev_rb = -1;
+    bool ok = true;
+    TileIter ti;
+    ti.init(mats, n_mats, t_begin, t_end, t_stride);
+    ti.chunk = kTileChunk;
+    for (; ti.valid(); ti.next()) {
+      const TcMat& mt = mats[ti.i];
       // U operand tile once per row block, P operand tile of this column block; with the
       // half split the order is U half 0, P half 0, U half 1, P half 1
       const bool new_a = ti.i != prev_i || ti.rb != prev_rb;
@@ -245,6 +264,7 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
           const int bi = sa * Cfg::kSplit + h;
           if (!mbar_wait_bounded(&sh.a_empty[bi], pa ^ 1u, abort, wait_cycles)) { ok = false; break; }
           mbar_arrive_expect_tx(&sh.a_full[bi], Cfg::kOpBytes / Cfg::kSplit);
+          ++a_iss[bi];
           for (int p = h; p < Cfg::kPanels; p += Cfg::kSplit)
             tma_load_2d(a_smem + sa * Cfg::kOpBytes + p * kPanelBytes, &tm_a, 64 * p,
                         (int)(mt.u_row0 + ti.rb * kBM), &sh.a_full[bi]);
@@ -252,6 +272,7 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
         const int bi = sb * Cfg::kSplit + h;
         if (!mbar_wait_bounded(&sh.b_empty[bi], pb ^ 1u, abort, wait_cycles)) { ok = false; break; }
         mbar_arrive_expect_tx(&sh.b_full[bi], Cfg::kOpBytes / Cfg::kSplit);
+        ++b_iss[bi];
         for (int p = h; p < Cfg::kPanels; p += Cfg::kSplit)
           tma_load_2d(b_smem + sb * Cfg::kOpBytes + p * kPanelBytes, &tm_b, 64 * p,
                       (int)(mt.p_row0 + ti.cb * kBN), &sh.b_full[bi]);
@@ -265,23 +286,14 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
       ++n_b;
     }
     if (!ok) give_up(sh, status);
-    // drain: the last copy issued into every slot has landed before the CTA exits
-    for (int s = 0; s < Cfg::kWStages; ++s) {
-      const int64_t k = last_in_slot(n_w, s, Cfg::kWStages);
-      if (k >= 0) mbar_wait_bounded(&sh.w_full[s], (uint32_t)((k / Cfg::kWStages) & 1), nullptr, wait_cycles);
-    }
-    for (int s = 0; s < Cfg::kAStages; ++s) {
-      const int64_t k = last_in_slot(n_a, s, Cfg::kAStages);
-      for (int h = 0; h < Cfg::kSplit && k >= 0; ++h)
-        mbar_wait_bounded(&sh.a_full[s * Cfg::kSplit + h], (uint32_t)((k / Cfg::kAStages) & 1),
-                          nullptr, wait_cycles);
-    }
-    for (int s = 0; s < Cfg::kBStages; ++s) {
-      const int64_t k = last_in_slot(n_b, s, Cfg::kBStages);
-      for (int h = 0; h < Cfg::kSplit && k >= 0; ++h)
-        mbar_wait_bounded(&sh.b_full[s * Cfg::kSplit + h], (uint32_t)((k / Cfg::kBStages) & 1),
-                          nullptr, wait_cycles);
-    }
+    // drain: the last phase issued on every operand barrier (a partial tile included)
+    // has landed before the CTA exits
+    for (int bi = 0; bi < Cfg::kAStages * Cfg::kSplit; ++bi)
+      if (a_iss[bi] > 0)
+        mbar_wait_bounded(&sh.a_full[bi], (uint32_t)((a_iss[bi] - 1) & 1), nullptr, wait_cycles);
+    for (int bi = 0; bi < Cfg::kBStages * Cfg::kSplit; ++bi)
+      if (b_iss[bi] > 0)
+        mbar_wait_bounded(&sh.b_full[bi], (uint32_t)((b_iss[bi] - 1) & 1), nullptr, wait_cycles);
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA issuer
     constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN);
@@ -351,7 +363,7 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
       const int64_t last = it - 1;
       mbar_wait_bounded(&sh.acc_full[last & 1], (uint32_t)((last >> 1) & 1), nullptr, wait_cycles);
     }
-  } else if (warp >= 2) {
+  } else if (warp >= 2 && warp <= 5) {
     // ------------------------------------------------------------ epilogue
     const int g = warp & 3;                      // TMEM lane group == tile row group
     const uint32_t lane_base = (uint32_t)(g * 32) << 16;
