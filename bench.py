@@ -37,9 +37,12 @@ FALLBACK_HBM_GBS = 6800.0
 # dram__bytes_read.sum + dram__bytes_write.sum per launch of the weight-pass kernel,
 # from the ncu capture summarised under profiles/, keyed by the sha256 of the kernel
 # source it was taken on (reported as null once the source differs).
+L2_BYTES = 129e6          # GB300 L2 capacity
 TRAFFIC_BY_SOURCE = {
-    # profiles/wpass_tc_r32_llama7b_2layers.md: 1.577 GB on the 2-layer subset, x16.0 by weights
-    ("64253833d2a89ac2", "llama7b_bf16_r32"): 25.24e9,
+    # profiles/wpass_tc_r32_llama7b_2layers.md: 1.578 GB on the 2-layer subset, x16.0 by weights
+    ("606956737cbbef16", "llama7b_bf16_r32"): 25.25e9,
+    # profiles/wpass_tc_r128_llama7b_2layers.md: 1.639 GB on the 2-layer subset, x16.0 by weights
+    ("606956737cbbef16", "llama7b_bf16_r128_q99"): 26.22e9,
 }
 # thread instructions per weight of the full-space SPSA kernel (ncu), keyed by source hash
 INSTR_PER_WEIGHT_BY_SOURCE = {
@@ -93,7 +96,7 @@ def subset(wl, layers):
         return wl
     from paper_2608_15665_gb300 import workloads
     per_layer = {"opt1.3b_bf16_r16": 6, "llama7b_bf16_r32": 7, "dense32b_bf16_r64": 7,
-                 "llama7b_bf16_r128_q99": 7,
+                 "llama7b_bf16_r128_q99": 7, "llama13b_bf16_r128_q99": 7,
                  "lora_opt13b_f32_r4": 4, "single256_f32_r8": 1}[wl.name]
     k = min(len(wl.shapes), layers * per_layer)
     return workloads.scaled(wl, name=f"{wl.name}[{layers} layers]", shapes=wl.shapes[:k],
@@ -166,14 +169,16 @@ def oracle_sample_step_seconds(wl, scheme, sample=((0, 1024),), seed_shift=0):
     (matrix, n_rows) in ``sample``, the refresh of that matrix (Alg. 1 on its full m x r
     and n x r panels) and every weight pass of the step (perturbations, estimator,
     Adam, fused update) on n_rows of its rows (rows of W update independently).
-    Returns (step_seconds, refresh_seconds, sample_text) extrapolated to the workload:
-    passes by weight count, refresh by panel rows m + n."""
+    Returns (step_seconds, refresh_seconds, sample_text, cores) extrapolated to the
+    workload: passes by weight count, refresh by panel rows m + n; cores = process CPU
+    time / wall time over the timed work (the threads the oracle actually kept busy)."""
     import numpy as np
     import torch
     from oracle import subzero
     from paper_2608_15665_gb300 import workloads
     t_pass = t_ref = 0.0
     el_sample = uv_sample = 0
+    cpu_s = wall_s = 0.0
     seed = wl.seed + seed_shift
     for i, n_rows in sample:
         m, n = wl.shapes[i]
@@ -181,12 +186,13 @@ def oracle_sample_step_seconds(wl, scheme, sample=((0, 1024),), seed_shift=0):
         W0 = workloads.init_weight(wl, i, "cpu")[: rows.size].to(torch.float64).numpy()
         st = subzero.MatrixState(W0, wl.dtype, wl.r)
         st.m = m                                   # the panels keep the matrix's full shape
-        t0 = time.perf_counter()
+        t0, c0 = time.perf_counter(), time.process_time()
         subzero.refresh(st, seed, i, 0, reset_moments=True)
         t_ref += time.perf_counter() - t0
+        cpu_s += time.process_time() - c0
         losses = workloads.loss_table(wl, scheme, steps=1)[0]
         passes, restore = subzero.pass_plan(scheme, wl.q)
-        t0 = time.perf_counter()
+        t0, c0 = time.perf_counter(), time.process_time()
         for terms in passes:
             C = subzero.perturb_coeff(seed, i, 0, wl.r, terms, wl.eps)
             st.W = subzero.apply_pass(st.W, wl.dtype, st.U, st.V, C, rows=rows)
@@ -196,6 +202,7 @@ def oracle_sample_step_seconds(wl, scheme, sample=((0, 1024),), seed_shift=0):
         C = subzero.step_coeff(D, wl.lr, wl.eps, restore, seed, i, 0, wl.r)
         st.W = subzero.apply_pass(st.W, wl.dtype, st.U, st.V, C, rows=rows)
         t_pass += time.perf_counter() - t0
+        cpu_s += time.process_time() - c0
         el_sample += rows.size * n
         uv_sample += m + n
     step_s = t_pass * wl.params / el_sample
@@ -204,25 +211,16 @@ def oracle_sample_step_seconds(wl, scheme, sample=((0, 1024),), seed_shift=0):
             + ", ".join(f"{r} rows of matrix {i} {wl.shapes[i][0]}x{wl.shapes[i][1]}" for i, r in sample)
             + f" ({el_sample} of {wl.params} weights) and the refresh of those matrices; "
             f"extrapolated by weight count (refresh by m+n, amortized over F={wl.F})")
-    return step_s, refresh_s, text
-
-
-def oracle_threads():
-    try:
-        from threadpoolctl import threadpool_info
-        n = [d.get("num_threads", 1) for d in threadpool_info() if d.get("user_api") == "blas"]
-        if n:
-            return int(max(n))
-    except Exception:
-        pass
-    return os.cpu_count() or 1
+    cores = round(cpu_s / (t_pass + t_ref), 1) if t_pass + t_ref > 0 else 1.0
+    return step_s, refresh_s, text, cores
 
 
 def cpu_baseline(wl, scheme):
-    step_s, refresh_s, text = oracle_sample_step_seconds(wl, scheme, sample=((0, 1024), (4, 1024)))
+    step_s, refresh_s, text, cores = oracle_sample_step_seconds(wl, scheme,
+                                                                sample=((0, 1024), (4, 1024)))
     per_step = step_s + refresh_s / wl.F
-    return {"value": 1.0 / per_step, "unit": "ZO steps/s", "cores": oracle_threads(),
-            "kind": "oracle", "sample": text}
+    return {"value": 1.0 / per_step, "unit": "ZO steps/s", "cores": cores,
+            "host_cores": os.cpu_count(), "kind": "oracle", "sample": text}
 
 
 # --------------------------------------------------------------------------- reference arm
@@ -232,15 +230,16 @@ def run_reference(args):
         return
     from paper_2608_15665_gb300 import workloads
     wl = workloads.get(args.workload)
-    times = []
+    times, cores = [], []
     for s in range(args.warmup + args.steps):
-        step_s, refresh_s, text = oracle_sample_step_seconds(wl, args.scheme, sample=((0, 512),),
-                                                             seed_shift=s)
+        step_s, refresh_s, text, c = oracle_sample_step_seconds(wl, args.scheme, sample=((0, 512),),
+                                                                seed_shift=s)
         if s >= args.warmup:
             times.append(step_s + refresh_s / wl.F)
+            cores.append(c)
     per_step = sum(times) / len(times)
     value = 1.0 / per_step
-    passes = 2 * wl.q if args.scheme == "central" else wl.q + 1
+    passes = 2 * wl.q + 1 if args.scheme == "central" else wl.q + 1
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "ZO steps/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
@@ -249,8 +248,8 @@ def run_reference(args):
         "config": {"workload": wl.name, "matrices": wl.n_mats, "params": wl.params, "r": wl.r,
                    "q": wl.q, "scheme": args.scheme, "passes_per_step": passes,
                    "refresh_every": wl.F},
-        "cpu_baseline": {"value": value, "unit": "ZO steps/s", "cores": oracle_threads(),
-                         "kind": "oracle", "sample": text},
+        "cpu_baseline": {"value": value, "unit": "ZO steps/s", "cores": max(cores),
+                         "host_cores": os.cpu_count(), "kind": "oracle", "sample": text},
         "e2e": {"value": value, "unit": "ZO steps/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -385,6 +384,7 @@ def run_ours(args):
     avg_launch_s = (wpass_ms / wpass_n) / 1e3 if wpass_n else float("nan")
     achieved = bytes_pass / avg_launch_s / 1e9
     src = kernel_source_hash()
+    l2_resident = bytes_pass / 2 < L2_BYTES
     line = {
         "metric": METRIC, "value": value, "unit": "ZO steps/s", "n_gpus": world, "steps": K,
         "warmup": W, "ms_per_step": elapsed_ms / K, "higher_is_better": True, "scaling": "weak",
@@ -394,7 +394,9 @@ def run_ours(args):
                    "r": wl.r, "q": wl.q, "scheme": args.scheme, "passes_per_step": passes,
                    "refresh_every": wl.F, "refreshes_in_timed_region":
                        sum(1 for t in range(W, W + K) if t % wl.F == 0),
-                   "l2": "inputs larger than L2 (%.1f GB of weights per pass)" % (bytes_pass / 2e9),
+                   "l2": ("inputs larger than L2 (%.1f GB of weights per pass)" % (bytes_pass / 2e9)
+                          if not l2_resident else
+                          "weights fit in L2 (%.1f MB per pass): latency-bound" % (bytes_pass / 2e6)),
                    "parallelism": f"layer partition x{world}" if world > 1 else "single GPU"},
         "weight_pass_gbs": passes * bytes_pass * K / (elapsed_ms / 1e3) / 1e9,
         "refresh_ms": refresh_ms,
@@ -407,6 +409,13 @@ def run_ours(args):
         "clocks": clk,
         "gpu_launches": int(launches),
     }
+    if l2_resident:
+        # the whole set stays in the 129 MB L2 between passes: no HBM fraction, the pass
+        # is reported as its latency
+        line["roofline"] = {"bound": "latency", "achieved": None, "peak": None, "unit": "GB/s",
+                            "frac": None, "traffic": None,
+                            "kernel": line["roofline"]["kernel"],
+                            "us_per_pass": avg_launch_s * 1e6, "launches_timed": wpass_n}
     if args.method == "mezo":
         # bound by instruction issue: peak = SMs x 128 lanes x max SM clock (thread
         # instructions per second); achieved = instructions per weight (ncu count of the

@@ -2,7 +2,7 @@
 //
 // For each panel (Omega_U, m x r and Omega_V, n x r) we need the thin QR factor
 // with a positive diagonal of R (Eq. (11)).  Panels are tall and skinny (m up to
-// 25600, r <= 64) and there are up to ~900 of them, so the factorisation is a
+// 25600, r <= 128) and there are up to ~900 of them, so the factorisation is a
 // batched TSQR (communication-avoiding QR, Demmel et al. 2012):
 //
 //   up pass, level 0:  each block of B rows draws its Omega rows from the

@@ -92,6 +92,14 @@ def _build():
         beta2=0.95, eps_adam=1e-8, steps=400, F=50, seed=1006,
         note="the paper's default scale (App. A.2, Table 7): r = 128, K = 99 queries, "
              "F = 50, on the LLaMA-7B shapes")
+    llama13 = []
+    for _ in range(40):
+        llama13 += [(5120, 5120)] * 4 + [(13824, 5120), (13824, 5120), (5120, 13824)]
+    wl["llama13b_bf16_r128_q99"] = Workload(
+        "llama13b_bf16_r128_q99", llama13, "bf16", r=128, q=99, eps=1e-3, lr=1e-3, beta1=0.9,
+        beta2=0.95, eps_adam=1e-8, steps=400, F=100, seed=1007,
+        note="the paper's default scale on the LLaMA-13B shapes: 40 x {q,k,v,o 5120x5120, "
+             "gate,up 13824x5120, down 5120x13824}, r = 128, K = 99, F = 100")
     big = []
     for _ in range(64):
         big += [(8192, 5120), (1024, 5120), (1024, 5120), (5120, 8192),

@@ -13,6 +13,8 @@ from paper_2608_15665_gb300 import workloads
     ("llama7b_bf16_r32", 6_476_005_376, 224, 32, 4),
     ("lora_opt13b_f32_r4", 6_553_600, 160, 4, 8),
     ("dense32b_bf16_r64", 31_205_621_760, 448, 64, 8),
+    ("llama7b_bf16_r128_q99", 6_476_005_376, 224, 128, 99),
+    ("llama13b_bf16_r128_q99", 12_687_769_600, 280, 128, 99),
 ])
 def test_workload_shapes(name, params, n_mats, r, q):
     wl = workloads.get(name)
