@@ -81,9 +81,10 @@ def measured_peaks():
 
 
 def kernel_source_hash():
-    """sha256 (16 hex) of the sources of the tensor-core weight-pass kernel."""
+    """sha256 (16 hex) of the sources of the tensor-core weight-pass kernels."""
     h = hashlib.sha256()
-    for name in ("zo_wpass_tc.cu", "zo_sm100.cuh", "zo_device.cuh"):
+    for name in ("zo_wpass_tc.cu", "zo_wpass_tmem.cu", "zo_tc_common.cuh", "zo_sm100.cuh",
+                 "zo_device.cuh"):
         path = os.path.join(ROOT, "paper_2608_15665_gb300", "csrc", name)
         if os.path.exists(path):
             h.update(open(path, "rb").read())

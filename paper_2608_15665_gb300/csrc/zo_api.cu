@@ -73,7 +73,8 @@ struct zo_ctx {
   // tensor-core weight pass (all matrices bf16, r in {16, 32, 64})
   bool tc_ok = false;
   int sms = 0;
-  __nv_bfloat16* d_u_hl = nullptr;   // stacked [hi | lo] rows of every U_i, 128-row padded
+  void* d_u_op = nullptr;            // stacked U operand of every U_i, 128-row padded
+                                     // (rows [hi | lo | 0] for r <= 32, chunk-major for r >= 64)
   __nv_bfloat16* d_p_hl = nullptr;   // stacked [hi | lo] rows of every P_i^T, 128-row padded
   zo::TcMat* d_tc = nullptr;
   int64_t tc_tiles = 0;
@@ -100,7 +101,7 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_qr_ws);
   cudaFree(c->d_qr_blocks);
   cudaFree(c->d_status);
-  cudaFree(c->d_u_hl);
+  cudaFree(c->d_u_op);
   cudaFree(c->d_p_hl);
   cudaFree(c->d_tc);
   cudaFree(c->d_w_maps);
@@ -212,7 +213,7 @@ zo_status run_weight_pass(zo_ctx* c) {
     const int grid = (int)std::min<int64_t>(c->tc_tiles, c->sms);
     const bool inject = c->inject_wait;
     c->inject_wait = false;
-    ZO_CUDA(zo::launch_wpass_tc(c->tm_a, c->tm_b, c->d_w_maps, c->d_tc, c->n_mats, c->tc_tiles,
+    ZO_CUDA(zo::launch_wpass_tc(c->tm_a, c->d_u_op, c->tm_b, c->d_w_maps, c->d_tc, c->n_mats, c->tc_tiles,
                                 grid, c->r, c->d_status, inject, c->stream),
             "tensor-core weight-pass kernel");
     c->last_path = 2;
@@ -281,9 +282,10 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
   }
   if (urows >= (int64_t(1) << 31) || prows >= (int64_t(1) << 31)) return ZO_OK;
   ZO_CUDA(cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, c->device), "SM count");
-  ZO_CUDA(cudaMalloc(&c->d_u_hl, sizeof(__nv_bfloat16) * urows * HLW), "cudaMalloc(U hi/lo)");
+  const int64_t u_bytes = zo::tc_u_operand_bytes(c->r, urows);
+  ZO_CUDA(cudaMalloc(&c->d_u_op, u_bytes), "cudaMalloc(U hi/lo)");
   ZO_CUDA(cudaMalloc(&c->d_p_hl, sizeof(__nv_bfloat16) * prows * HLW), "cudaMalloc(P hi/lo)");
-  ZO_CUDA(cudaMemset(c->d_u_hl, 0, sizeof(__nv_bfloat16) * urows * HLW), "memset");
+  ZO_CUDA(cudaMemset(c->d_u_op, 0, u_bytes), "memset");
   ZO_CUDA(cudaMemset(c->d_p_hl, 0, sizeof(__nv_bfloat16) * prows * HLW), "memset");
   ZO_CUDA(cudaMalloc(&c->d_tc, sizeof(zo::TcMat) * c->n_mats), "cudaMalloc(tile table)");
   ZO_CUDA(cudaMemcpy(c->d_tc, tc.data(), sizeof(zo::TcMat) * c->n_mats, cudaMemcpyHostToDevice),
@@ -294,8 +296,9 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
           "upload units");
   c->n_u_units = (int32_t)uunits.size();
   std::vector<CUtensorMap> wmaps(c->n_mats);
-  bool ok = encode_bf16_2d(&c->tm_a, c->d_u_hl, HLW, urows, HLW * 2, 64, 128) &&
-            encode_bf16_2d(&c->tm_b, c->d_p_hl, HLW, prows, HLW * 2, 64, 128);
+  bool ok = encode_bf16_2d(&c->tm_b, c->d_p_hl, HLW, prows, HLW * 2, 64, 128);
+  if (ok && !zo::wpass_tc_u_in_tmem(c->r))   // r <= 32: U rows read by TMA
+    ok = encode_bf16_2d(&c->tm_a, c->d_u_op, HLW, urows, HLW * 2, 64, 128);
   for (int32_t i = 0; ok && i < c->n_mats; ++i)
     ok = encode_bf16_2d(&wmaps[i], mats[i].W, mats[i].n, mats[i].m, mats[i].ldw * 2, 64, 32);
   if (!ok) {
@@ -522,7 +525,7 @@ zo_status zo_refresh(zo_ctx* c, uint32_t refresh_idx, int32_t reset_moments) {
     ++c->launches;
   }
   if (c->tc_ok) {
-    ZO_CUDA(zo::launch_split_u(c->d_mats, c->d_tc, c->d_u_units, c->n_u_units, c->r, c->d_u_hl,
+    ZO_CUDA(zo::launch_split_u(c->d_mats, c->d_tc, c->d_u_units, c->n_u_units, c->r, c->d_u_op,
                                c->stream),
             "split U into hi/lo");
     ++c->launches;

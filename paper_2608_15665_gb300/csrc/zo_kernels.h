@@ -63,21 +63,34 @@ cudaError_t launch_wpass_fma(const MatDesc* d_mats, int32_t n_mats, const int64_
 cudaError_t launch_mezo(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_tile_prefix,
                         int64_t n_tiles, uint64_t seed, uint32_t t, float coef, cudaStream_t s);
 
-// ---- weight pass, tcgen05 path (zo_wpass_tc.cu) --------------------------------
+// ---- weight pass, tcgen05 path (zo_wpass_tc.cu: r <= 32, zo_wpass_tmem.cu: r >= 64) -----
 bool wpass_tc_supported(int32_t r);
-int32_t tc_hl_width(int32_t r);   // bf16 elements per hi/lo operand row
+bool wpass_tc_u_in_tmem(int32_t r);   // the U operand is read from Tensor Memory (r >= 64)
+int32_t tc_hl_width(int32_t r);       // bf16 elements per hi/lo operand row
 int32_t tc_tile_rows();
 int32_t tc_tile_cols();
-// U_HL rows of every matrix from U (after a refresh); units = (matrix, first row) x 128 rows
+// Bytes of the stacked U operand for `rows` rows (both layouts below fit).
+int64_t tc_u_operand_bytes(int32_t r, int64_t rows);
+// The U operand of every matrix from U (after a refresh); units = (matrix, first row) x
+// 128 rows.  r <= 32: rows [hi | lo | 0] of tc_hl_width(r) bf16, read by TMA (tm_a);
+// r >= 64: chunk-major per 128-row block, read into Tensor Memory (zo_wpass_tmem.cu).
 cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                           int32_t n_units, int32_t r, __nv_bfloat16* u_hl, cudaStream_t s);
+                           int32_t n_units, int32_t r, void* u_op, cudaStream_t s);
 // Pt_HL rows: hi/lo of (C V^T)^T; units = (matrix, first column) x 128 columns
 cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                                  int32_t n_units, int32_t r, __nv_bfloat16* p_hl, cudaStream_t s);
-cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
+// tm_a is used for r <= 32, u_op for r >= 64.
+cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const void* u_op, const CUtensorMap& tm_b,
                             const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
                             int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
                             bool inject_wait, cudaStream_t s);
+// r >= 64 (zo_wpass_tmem.cu)
+cudaError_t launch_split_u_chunks(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                                  int32_t n_units, int32_t r, uint4* u_t, cudaStream_t s);
+cudaError_t launch_wpass_tmem(const uint4* u_t, const CUtensorMap& tm_b,
+                              const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
+                              int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
+                              bool inject_wait, cudaStream_t s);
 
 // ---- refresh: batched TSQR + sign correction (zo_qr.cu) ------------------------
 int32_t qr_block_rows(int32_t r);

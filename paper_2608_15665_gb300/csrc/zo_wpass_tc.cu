@@ -1,6 +1,9 @@
 // Weight pass on the 5th-generation tensor cores: W_i <- rnd_bf16(W_i + U_i P_i)
 // for every bf16 matrix in one persistent launch (the fused form of Alg. 2's
 // "W_i <- W_i + eps U_i Z_i V_i^T", Eq. (4), and of the update of Eq. (10)).
+// This file holds the kernel for r <= 32 (both operands in shared memory), the operand
+// split kernels, the projection P = C V^T and the dispatch by rank; the r >= 64 kernel,
+// which reads U from Tensor Memory, is in zo_wpass_tmem.cu.
 //
 // The contraction U (128 x r) . P (r x 128) of a 128 x 128 tile is r-deep, so it
 // costs 2r flops per weight against 4 bytes of HBM traffic; past r = 16 that is
@@ -30,119 +33,30 @@
 
 #include "zo_kernels.h"
 #include "zo_sm100.cuh"
+#include "zo_tc_common.cuh"
 
 namespace zo {
 namespace {
 
 using namespace sm100;
+using namespace tc;
 
-constexpr int kBM = 128;            // tile rows (TMEM lanes)
-constexpr int kBN = 128;            // tile columns (TMEM columns per accumulator)
 constexpr int kThreads = 224;
-constexpr int kWBoxBytes = 32 * 64 * 2;          // one TMA box of W: 32 rows x 64 bf16
-constexpr int kWStageBytes = kBM * kBN * 2;      // 32 KB
-constexpr int kPanelBytes = kBM * 64 * 2;        // 128 rows x 128 bytes = 16 KB
-constexpr long long kWaitCycles = 4000000000LL;  // default wait limit, ~2 s at 2 GHz
-constexpr int kTileChunk = 4;                    // consecutive tiles per CTA visit (U reuse)
-
-__host__ __device__ constexpr int hl_width(int r) { return 2 * r > 64 ? 2 * r : 64; }
 
 template <int R>
 struct TcCfg {
+  static_assert(R == 16 || R == 32, "the shared-memory-operand kernel covers r = 16 and 32");
   static constexpr int kHLW = hl_width(R);
   static constexpr int kPanels = kHLW / 64;
   static constexpr int kOpBytes = kPanels * kPanelBytes;        // one operand tile (hi + lo)
-  // ring depths per rank: 32 KB W stages, operand tiles of 16 / 16 / 32 / 64 KB
-  // (R = 128: 3 x 32 + 64 + 64 KB + barriers = 226 KB of the 227 KB a CTA may hold)
-  static constexpr int kWStages = R >= 64 ? 3 : 4;
-  static constexpr int kAStages = R >= 128 ? 1 : 2;
-  static constexpr int kBStages = R >= 128 ? 1 : 2;
-  // With one operand stage (R = 128) each operand tile is loaded and released in two
-  // K halves with barriers of their own -- half h = hi panel h + lo panel 2 + h -- so
-  // the next tile's first half loads while the MMAs still read the second.
-  static constexpr int kSplit = R >= 128 ? 2 : 1;
+  // 4 W stages of 32 KB, 2 + 2 operand stages of 16 KB: 192 KB
+  static constexpr int kWStages = 4;
+  static constexpr int kAStages = 2;
+  static constexpr int kBStages = 2;
   static constexpr int kKC = R / 16;                            // K chunks of 16
   static constexpr size_t kSmem = (size_t)kWStages * kWStageBytes + (size_t)kAStages * kOpBytes +
                                   (size_t)kBStages * kOpBytes + 1024 /*barriers*/ + 1024 /*align*/;
 };
-
-struct Shared {
-  uint64_t w_full[4], w_empty[4];
-  uint64_t a_full[2], a_empty[2];
-  uint64_t b_full[2], b_empty[2];
-  uint64_t acc_full[2], acc_empty[2];
-  uint64_t never;          // test hook: a barrier no thread ever arrives on
-  uint32_t tmem_base;
-  int abort_flag;
-};
-
-// Walks this CTA's tiles t0, t0 + stride, ... (< t_end), each decoded into (matrix, row
-// block, column block); tiles are numbered matrix by matrix, row block by row block.
-struct TileIter {
-  const TcMat* mats;
-  int n_mats;
-  int64_t t, t_end, stride;
-  int i;
-  int64_t rb, cb, tiles_m;
-  __device__ void init(const TcMat* m, int nm, int64_t t0, int64_t t1, int64_t step) {
-    mats = m;
-    n_mats = nm;
-    t = t0;
-    t_end = t1;
-    stride = step;
-    int lo = 0, hi = nm - 1;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (mats[mid].tile0 <= t0) lo = mid; else hi = mid - 1;
-    }
-    i = lo;
-    set_local();
-  }
-  __device__ void set_local() {
-    if (t >= t_end) return;
-    const int64_t local = t - mats[i].tile0;
-    rb = local / mats[i].tiles_n;
-    cb = local % mats[i].tiles_n;
-    tiles_m = (mats[i].m + kBM - 1) / kBM;
-  }
-  int64_t chunk = 1, in_chunk = 0;   // take `chunk` consecutive tiles, then jump
-  __device__ bool valid() const { return t < t_end; }
-  __device__ void next() {
-    if (stride != 1) {
-      if (++in_chunk < chunk) {
-        t += 1;
-      } else {
-        in_chunk = 0;
-        t += stride - (chunk - 1);
-      }
-      if (t >= t_end) return;
-      while (i + 1 < n_mats && mats[i + 1].tile0 <= t) ++i;
-      set_local();
-      return;
-    }
-    ++t;
-    if (t >= t_end) return;
-    if (++cb == mats[i].tiles_n) {
-      cb = 0;
-      if (++rb == tiles_m) {
-        ++i;
-        rb = 0;
-        tiles_m = (mats[i].m + kBM - 1) / kBM;
-      }
-    }
-  }
-};
-
-// index of the last of n_issued ring entries that went into slot s (ring of S slots), or -1
-__device__ __forceinline__ int64_t last_in_slot(int64_t n_issued, int s, int S) {
-  if (n_issued <= s) return -1;
-  return s + (int64_t)S * ((n_issued - 1 - s) / S);
-}
-
-__device__ __forceinline__ void give_up(Shared& sh, uint32_t* status) {
-  atomicOr(status, (uint32_t)kDevTimeout);
-  *reinterpret_cast<volatile int*>(&sh.abort_flag) = 1;
-}
 
 template <int R>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -154,10 +68,6 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
   static_assert(Cfg::kWStages >= 2 && Cfg::kWStages <= 4, "W ring must fit Shared::w_full");
   static_assert(Cfg::kAStages >= 1 && Cfg::kAStages <= 2, "A ring must fit Shared::a_full");
   static_assert(Cfg::kBStages >= 1 && Cfg::kBStages <= 2, "B ring must fit Shared::b_full");
-  static_assert(Cfg::kAStages * Cfg::kSplit <= 2 && Cfg::kBStages * Cfg::kSplit <= 2,
-                "operand barriers per stage and half must fit Shared::a_full / b_full");
-  static_assert(Cfg::kSplit == 1 || (Cfg::kPanels == 4 && Cfg::kKC == 8),
-                "the half split assumes hi = panels 0, 1 and lo = panels 2, 3");
   static_assert(sizeof(Shared) <= 1024, "barrier block");
   static_assert(Cfg::kSmem <= 227 * 1024, "shared memory per CTA");
   extern __shared__ uint8_t smem_raw[];
@@ -185,11 +95,11 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
       mbar_init(&sh.w_full[s], 1);
       mbar_init(&sh.w_empty[s], 4);
     }
-    for (int s = 0; s < Cfg::kAStages * Cfg::kSplit; ++s) {
+    for (int s = 0; s < Cfg::kAStages; ++s) {
       mbar_init(&sh.a_full[s], 1);
       mbar_init(&sh.a_empty[s], 1);
     }
-    for (int s = 0; s < Cfg::kBStages * Cfg::kSplit; ++s) {
+    for (int s = 0; s < Cfg::kBStages; ++s) {
       mbar_init(&sh.b_full[s], 1);
       mbar_init(&sh.b_empty[s], 1);
     }
@@ -253,45 +163,36 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
     ti.chunk = kTileChunk;
     for (; ti.valid(); ti.next()) {
       const TcMat& mt = mats[ti.i];
-      // U operand tile once per row block, P operand tile of this column block; with the
-      // half split the order is U half 0, P half 0, U half 1, P half 1
-      const bool new_a = ti.i != prev_i || ti.rb != prev_rb;
-      const int sa = (int)(n_a % Cfg::kAStages), sb = (int)(n_b % Cfg::kBStages);
-      const uint32_t pa = (uint32_t)((n_a / Cfg::kAStages) & 1);
-      const uint32_t pb = (uint32_t)((n_b / Cfg::kBStages) & 1);
-      for (int h = 0; h < Cfg::kSplit && ok; ++h) {
-        if (new_a) {
-          const int bi = sa * Cfg::kSplit + h;
-          if (!mbar_wait_bounded(&sh.a_empty[bi], pa ^ 1u, abort, wait_cycles)) { ok = false; break; }
-          mbar_arrive_expect_tx(&sh.a_full[bi], Cfg::kOpBytes / Cfg::kSplit);
-          ++a_iss[bi];
-          for (int p = h; p < Cfg::kPanels; p += Cfg::kSplit)
-            tma_load_2d(a_smem + sa * Cfg::kOpBytes + p * kPanelBytes, &tm_a, 64 * p,
-                        (int)(mt.u_row0 + ti.rb * kBM), &sh.a_full[bi]);
-        }
-        const int bi = sb * Cfg::kSplit + h;
-        if (!mbar_wait_bounded(&sh.b_empty[bi], pb ^ 1u, abort, wait_cycles)) { ok = false; break; }
-        mbar_arrive_expect_tx(&sh.b_full[bi], Cfg::kOpBytes / Cfg::kSplit);
-        ++b_iss[bi];
-        for (int p = h; p < Cfg::kPanels; p += Cfg::kSplit)
-          tma_load_2d(b_smem + sb * Cfg::kOpBytes + p * kPanelBytes, &tm_b, 64 * p,
-                      (int)(mt.p_row0 + ti.cb * kBN), &sh.b_full[bi]);
-      }
-      if (!ok) break;
-      if (new_a) {
+      // U operand tile once per row block, P operand tile of this column block
+      if (ti.i != prev_i || ti.rb != prev_rb) {
+        const int sa = (int)(n_a % Cfg::kAStages);
+        const uint32_t pa = (uint32_t)((n_a / Cfg::kAStages) & 1);
+        if (!mbar_wait_bounded(&sh.a_empty[sa], pa ^ 1u, abort, wait_cycles)) { ok = false; break; }
+        mbar_arrive_expect_tx(&sh.a_full[sa], Cfg::kOpBytes);
+        ++a_iss[sa];
+        for (int p = 0; p < Cfg::kPanels; ++p)
+          tma_load_2d(a_smem + sa * Cfg::kOpBytes + p * kPanelBytes, &tm_a, 64 * p,
+                      (int)(mt.u_row0 + ti.rb * kBM), &sh.a_full[sa]);
         ++n_a;
         prev_i = ti.i;
         prev_rb = ti.rb;
       }
+      const int sb = (int)(n_b % Cfg::kBStages);
+      const uint32_t pb = (uint32_t)((n_b / Cfg::kBStages) & 1);
+      if (!mbar_wait_bounded(&sh.b_empty[sb], pb ^ 1u, abort, wait_cycles)) { ok = false; break; }
+      mbar_arrive_expect_tx(&sh.b_full[sb], Cfg::kOpBytes);
+      ++b_iss[sb];
+      for (int p = 0; p < Cfg::kPanels; ++p)
+        tma_load_2d(b_smem + sb * Cfg::kOpBytes + p * kPanelBytes, &tm_b, 64 * p,
+                    (int)(mt.p_row0 + ti.cb * kBN), &sh.b_full[sb]);
       ++n_b;
     }
     if (!ok) give_up(sh, status);
-    // drain: the last phase issued on every operand barrier (a partial tile included)
-    // has landed before the CTA exits
-    for (int bi = 0; bi < Cfg::kAStages * Cfg::kSplit; ++bi)
+    // drain: the last phase issued on every operand barrier has landed before the CTA exits
+    for (int bi = 0; bi < Cfg::kAStages; ++bi)
       if (a_iss[bi] > 0)
         mbar_wait_bounded(&sh.a_full[bi], (uint32_t)((a_iss[bi] - 1) & 1), nullptr, wait_cycles);
-    for (int bi = 0; bi < Cfg::kBStages * Cfg::kSplit; ++bi)
+    for (int bi = 0; bi < Cfg::kBStages; ++bi)
       if (b_iss[bi] > 0)
         mbar_wait_bounded(&sh.b_full[bi], (uint32_t)((b_iss[bi] - 1) & 1), nullptr, wait_cycles);
   } else if (warp == 1 && lane == 0) {
@@ -328,33 +229,29 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
       const uint32_t d = tmem + (uint32_t)(acc * kBN);
       const uint32_t a_base = smem_u32(a_smem + sa * Cfg::kOpBytes);
       const uint32_t b_base = smem_u32(b_smem + sb * Cfg::kOpBytes);
-      for (int h = 0; h < Cfg::kSplit; ++h) {
-        if (new_a && !mbar_wait_bounded(&sh.a_full[sa * Cfg::kSplit + h], pa, abort, wait_cycles)) {
-          ok = false;
-          break;
-        }
-        if (!mbar_wait_bounded(&sh.b_full[sb * Cfg::kSplit + h], pb, abort, wait_cycles)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-#pragma unroll
-        for (int k2 = 0; k2 < Cfg::kKC / Cfg::kSplit; ++k2) {
-          const int kk = h * (Cfg::kKC / Cfg::kSplit) + k2;
-          // hi chunk kk at element 16 kk of the operand row, lo chunk at R + 16 kk
-          const int e_hi = 16 * kk, e_lo = R + 16 * kk;
-          const uint32_t off_hi = (uint32_t)((e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
-          const uint32_t off_lo = (uint32_t)((e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
-          const uint64_t a_hi = sdesc_k_sw128(a_base + off_hi), a_lo = sdesc_k_sw128(a_base + off_lo);
-          const uint64_t b_hi = sdesc_k_sw128(b_base + off_hi), b_lo = sdesc_k_sw128(b_base + off_lo);
-          mma_bf16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
-          mma_bf16(d, a_hi, b_lo, idesc, 1u);
-          mma_bf16(d, a_lo, b_hi, idesc, 1u);
-        }
-        mma_commit(&sh.b_empty[sb * Cfg::kSplit + h]);
-        if (last_a) mma_commit(&sh.a_empty[sa * Cfg::kSplit + h]);
+      if (new_a && !mbar_wait_bounded(&sh.a_full[sa], pa, abort, wait_cycles)) {
+        ok = false;
+        break;
       }
-      if (!ok) break;
+      if (!mbar_wait_bounded(&sh.b_full[sb], pb, abort, wait_cycles)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+#pragma unroll
+      for (int kk = 0; kk < Cfg::kKC; ++kk) {
+        // hi chunk kk at element 16 kk of the operand row, lo chunk at R + 16 kk
+        const int e_hi = 16 * kk, e_lo = R + 16 * kk;
+        const uint32_t off_hi = (uint32_t)((e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
+        const uint32_t off_lo = (uint32_t)((e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
+        const uint64_t a_hi = sdesc_k_sw128(a_base + off_hi), a_lo = sdesc_k_sw128(a_base + off_lo);
+        const uint64_t b_hi = sdesc_k_sw128(b_base + off_hi), b_lo = sdesc_k_sw128(b_base + off_lo);
+        mma_bf16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
+        mma_bf16(d, a_hi, b_lo, idesc, 1u);
+        mma_bf16(d, a_lo, b_hi, idesc, 1u);
+      }
+      mma_commit(&sh.b_empty[sb]);
+      if (last_a) mma_commit(&sh.a_empty[sa]);
       mma_commit(&sh.acc_full[acc]);
     }
     if (!ok) give_up(sh, status);
@@ -449,26 +346,12 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
   }
 }
 
-// Both split kernels below handle 128 consecutive rows of one matrix per CTA: each
+// Both split kernels below (U rows for r <= 32, P rows for every r) handle 128
+// consecutive rows of one matrix per CTA: each
 // thread splits one row into 16-byte chunks of hi and lo, staged in shared memory with
 // the chunk index XOR (row & 7) so a quarter-warp's stores hit distinct banks; the CTA
 // then writes its rows, which are contiguous in the stacked operand, with coalesced
 // 16-byte stores.  Padding columns of a row stay at the zero they were set to.
-template <int R>
-__device__ __forceinline__ void split8(const float (&x)[8], uint4& hi, uint4& lo) {
-  uint32_t hw[4], lw[4];
-#pragma unroll
-  for (int pr = 0; pr < 4; ++pr) {
-    const __nv_bfloat162 h2 = __floats2bfloat162_rn(x[2 * pr], x[2 * pr + 1]);
-    const __nv_bfloat162 l2 =
-        __floats2bfloat162_rn(x[2 * pr] - __low2float(h2), x[2 * pr + 1] - __high2float(h2));
-    hw[pr] = *reinterpret_cast<const uint32_t*>(&h2);
-    lw[pr] = *reinterpret_cast<const uint32_t*>(&l2);
-  }
-  hi = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-  lo = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-}
-
 template <int R>
 __device__ __forceinline__ void write_rows(const uint4* Os, __nv_bfloat16* dst_rows, int rows) {
   constexpr int kVecPerRow = hl_width(R) * 2 / 16;   // 8 or 16 chunks per row
@@ -500,7 +383,7 @@ split_u_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
       const float4 a = src[2 * g], b = src[2 * g + 1];
       const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
       uint4 hi, lo;
-      split8<R>(x, hi, lo);
+      split8(x, hi, lo);
       orow[g ^ (tid & 7)] = hi;
       orow[(R / 8 + g) ^ (tid & 7)] = lo;
     }
@@ -552,7 +435,7 @@ project_split_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__
         x[k] = acc;
       }
       uint4 hi, lo;
-      split8<R>(x, hi, lo);
+      split8(x, hi, lo);
       orow[g ^ (tid & 7)] = hi;
       orow[(R / 8 + g) ^ (tid & 7)] = lo;
     }
@@ -704,7 +587,7 @@ cudaError_t launch_tc_r(const CUtensorMap& tm_a, const CUtensorMap& tm_b, const 
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   // with the test hook armed the wait limit is ~0.1 s so the test ends quickly
-  const long long wait = inject_wait ? 200000000LL : kWaitCycles;
+  const long long wait = inject_wait ? kTestWaitCycles : kWaitCycles;
   wpass_tc_kernel<R><<<grid, kThreads, smem, s>>>(tm_a, tm_b, w_maps, mats, n_mats, n_tiles, status,
                                                   wait, inject_wait ? 1 : 0);
   return cudaGetLastError();
@@ -713,18 +596,24 @@ cudaError_t launch_tc_r(const CUtensorMap& tm_a, const CUtensorMap& tm_b, const 
 }  // namespace
 
 bool wpass_tc_supported(int32_t r) { return r == 16 || r == 32 || r == 64 || r == 128; }
+bool wpass_tc_u_in_tmem(int32_t r) { return r >= 64; }
 int32_t tc_hl_width(int32_t r) { return hl_width(r); }
 int32_t tc_tile_rows() { return kBM; }
 int32_t tc_tile_cols() { return kBN; }
+int64_t tc_u_operand_bytes(int32_t r, int64_t rows) {
+  const int64_t row_layout = rows * hl_width(r) * 2;        // bf16 [hi | lo | 0] rows
+  const int64_t chunk_layout = rows * r * 4;                // R 32-bit words per row
+  return row_layout > chunk_layout ? row_layout : chunk_layout;
+}
 
 cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                           int32_t n_units, int32_t r, __nv_bfloat16* u_hl, cudaStream_t s) {
+                           int32_t n_units, int32_t r, void* u_op, cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
-    case 16: return launch_split_u_r<16>(d_mats, d_tc, d_units, n_units, u_hl, s);
-    case 32: return launch_split_u_r<32>(d_mats, d_tc, d_units, n_units, u_hl, s);
-    case 64: return launch_split_u_r<64>(d_mats, d_tc, d_units, n_units, u_hl, s);
-    case 128: return launch_split_u_r<128>(d_mats, d_tc, d_units, n_units, u_hl, s);
+    case 16: return launch_split_u_r<16>(d_mats, d_tc, d_units, n_units, static_cast<__nv_bfloat16*>(u_op), s);
+    case 32: return launch_split_u_r<32>(d_mats, d_tc, d_units, n_units, static_cast<__nv_bfloat16*>(u_op), s);
+    case 64:
+    case 128: return launch_split_u_chunks(d_mats, d_tc, d_units, n_units, r, static_cast<uint4*>(u_op), s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -741,7 +630,7 @@ cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const
   }
 }
 
-cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
+cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const void* u_op, const CUtensorMap& tm_b,
                             const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
                             int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
                             bool inject_wait, cudaStream_t s) {
@@ -749,8 +638,10 @@ cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
   switch (r) {
     case 16: return launch_tc_r<16>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
     case 32: return launch_tc_r<32>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
-    case 64: return launch_tc_r<64>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
-    case 128: return launch_tc_r<128>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
+    case 64:
+    case 128:
+      return launch_wpass_tmem(static_cast<const uint4*>(u_op), tm_b, d_w_maps, d_tc, n_mats, n_tiles,
+                               grid, r, d_status, inject_wait, s);
     default: return cudaErrorInvalidValue;
   }
 }
