@@ -40,9 +40,11 @@ FALLBACK_HBM_GBS = 6800.0
 L2_BYTES = 129e6          # GB300 L2 capacity
 TRAFFIC_BY_SOURCE = {
     # profiles/wpass_tc_r32_llama7b_2layers.md: 1.578 GB on the 2-layer subset, x16.0 by weights
-    ("606956737cbbef16", "llama7b_bf16_r32"): 25.25e9,
-    # profiles/wpass_tc_r128_llama7b_2layers.md: 1.639 GB on the 2-layer subset, x16.0 by weights
-    ("606956737cbbef16", "llama7b_bf16_r128_q99"): 26.22e9,
+    ("3509e1472d06a465", "llama7b_bf16_r32"): 25.24e9,
+    # profiles/wpass_tmem_r128_llama7b_2layers.md: 1.638 GB on the 2-layer subset, x16.0 by weights
+    ("3509e1472d06a465", "llama7b_bf16_r128_q99"): 26.21e9,
+    # profiles/wpass_tmem_r64_dense32b_1layer.md: 1.925 GB on the 1-layer subset, x64.0 by weights
+    ("3509e1472d06a465", "dense32b_bf16_r64"): 123.22e9,
 }
 # thread instructions per weight of the full-space SPSA kernel (ncu), keyed by source hash
 INSTR_PER_WEIGHT_BY_SOURCE = {
