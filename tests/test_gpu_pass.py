@@ -234,6 +234,40 @@ def test_tensor_core_step_matches_oracle(lib, gpu, case):
     z.close()
 
 
+@pytest.mark.parametrize("r", [16, 32, 64, 128])
+def test_tensor_core_rings_wrap(lib, gpu, r):
+    # 1280 + 15 tiles over 152 CTAs in chunks of 4: some CTAs take 3 chunks, so their U
+    # operand ring (two stages / two TMEM buffers) is reused and every barrier phase
+    # wraps; checked element by element for one pass and one step.
+    from paper_2608_15665_gb300 import binding as zb
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    base = 40
+    weights = [make_weight(m, n, "bf16", 600 + k, gpu, None)
+               for k, (m, n) in enumerate([(4096, 5120), (300, 520)])]
+    z = SubZeroPlus(weights, r, 2, 2024, matrix_index_base=base)
+    z.init_subspace(0)
+    before = snapshot(z)
+    z.perturb(0, 0, 1.0, 1, -1.0, 1e-1)
+    after = snapshot(z)
+    assert zb.zo_wpass_path(z.ctx) == 2
+    for i in range(2):
+        want, T = oracle_perturb(before, i, "bf16", z.seed, base + i, 0, r, [(0, 1.0), (1, -1.0)],
+                                 1e-1)
+        assert_weights(after["W"][i], want, "bf16", f"r{r} matrix {i} pass", before=before["W"][i],
+                       terms=T)
+    losses = np.array([2.01, 1.99, 2.0, 2.02], np.float32)
+    before = after
+    z.step(0, 1, losses, "central", 1e-1, 1e-2, 0.9, 0.95, 1e-8, 1, 1.0)
+    after = snapshot(z)
+    for i in range(2):
+        Wo, _, _, _, T = oracle_step(before, i, "bf16", z.seed, base + i, 0, r, 2, losses, "central",
+                                     1e-1, 1e-2, 0.9, 0.95, 1e-8, 1, [(1, 1.0)])
+        assert_weights(after["W"][i], Wo, "bf16", f"r{r} matrix {i} step", before=before["W"][i],
+                       terms=T)
+    z.sync()
+    z.close()
+
+
 @pytest.mark.parametrize("case", list(TC_CASES))
 def test_tensor_core_and_fma_paths_agree(lib, gpu, case):
     # one pass from the same state on both paths: each is within 1 ulp (at the operand

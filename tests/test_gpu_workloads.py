@@ -72,6 +72,7 @@ FULL = [
     ("opt1.3b_bf16_r16", (0, 4, 5, 143)),
     ("llama7b_bf16_r32", (0, 4, 6, 223)),
     ("dense32b_bf16_r64", (0, 1, 4, 6, 447)),
+    ("llama7b_bf16_r128_q99", (0, 4, 6, 223)),
 ]
 
 
