@@ -70,8 +70,9 @@ struct zo_ctx {
   int last_path = 0;
   bool inject_wait = false;      // test hook armed for the next tensor-core pass
   int64_t launches = 0;          // kernels launched by this context
-  // tensor-core weight pass (all matrices bf16, r in {16, 32, 64})
+  // tensor-core weight pass (all matrices bf16, r in {16, 32, 64, 128})
   bool tc_ok = false;
+  bool proj_tc = false;              // projection on the tensor cores too (r >= 64)
   int sms = 0;
   void* d_u_op = nullptr;            // stacked U operand of every U_i, 128-row padded
                                      // (rows [hi | lo | 0] for r <= 32, chunk-major for r >= 64)
@@ -82,6 +83,9 @@ struct zo_ctx {
   CUtensorMap tm_a{}, tm_b{};        // descriptors of the stacked operands (kernel parameters)
   int2* d_u_units = nullptr;
   int32_t n_u_units = 0;
+  __nv_bfloat16* d_v_hl = nullptr;   // [hi | lo] rows of every V_i (r >= 64), rows as P_HL
+  __nv_bfloat16* d_c_hl = nullptr;   // [hi | lo] rows of every C_i (r >= 64), r rows each
+  CUtensorMap tm_v{}, tm_c{}, tm_p{};  // V_HL, C_HL, and P_HL in 32-row boxes
   bool timing = false;
   std::vector<cudaEvent_t> ev_start, ev_stop;
   size_t ev_used = 0;
@@ -106,6 +110,8 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_tc);
   cudaFree(c->d_w_maps);
   cudaFree(c->d_u_units);
+  cudaFree(c->d_v_hl);
+  cudaFree(c->d_c_hl);
   for (auto e : c->ev_start) cudaEventDestroy(e);
   for (auto e : c->ev_stop) cudaEventDestroy(e);
   delete c;
@@ -198,7 +204,14 @@ zo_status record_stop(zo_ctx* c) {
 // Projection of C_i onto V_i and the weight pass, shared by zo_perturb and zo_step.
 zo_status run_weight_pass(zo_ctx* c) {
   const bool use_tc = c->tc_ok && c->path_option != 1;
-  if (use_tc) {
+  if (use_tc && c->proj_tc) {
+    ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, c->r, c->d_c_hl, c->stream), "split C");
+    ++c->launches;
+    const int grid = std::min<int>(c->n_proj_units, c->sms);
+    ZO_CUDA(zo::launch_project_tc(c->tm_v, c->tm_c, c->tm_p, c->d_tc, c->d_proj_units,
+                                  c->n_proj_units, grid, c->r, c->d_status, c->stream),
+            "tensor-core projection kernel");
+  } else if (use_tc) {
     ZO_CUDA(zo::launch_project_split(c->d_mats, c->d_tc, c->d_proj_units, c->n_proj_units, c->r,
                                      c->d_p_hl, c->stream),
             "projection kernel");
@@ -311,6 +324,16 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
           "upload tensor maps");
   c->tc_tiles = tiles;
   c->tc_ok = true;
+  if (zo::project_tc_supported(c->r)) {
+    const int64_t crows = (int64_t)c->n_mats * c->r;
+    ZO_CUDA(cudaMalloc(&c->d_v_hl, sizeof(__nv_bfloat16) * prows * HLW), "cudaMalloc(V hi/lo)");
+    ZO_CUDA(cudaMemset(c->d_v_hl, 0, sizeof(__nv_bfloat16) * prows * HLW), "memset");
+    ZO_CUDA(cudaMalloc(&c->d_c_hl, sizeof(__nv_bfloat16) * crows * HLW), "cudaMalloc(C hi/lo)");
+    ZO_CUDA(cudaMemset(c->d_c_hl, 0, sizeof(__nv_bfloat16) * crows * HLW), "memset");
+    c->proj_tc = encode_bf16_2d(&c->tm_v, c->d_v_hl, HLW, prows, HLW * 2, 64, 128) &&
+                 encode_bf16_2d(&c->tm_c, c->d_c_hl, HLW, crows, HLW * 2, 64, (uint32_t)c->r) &&
+                 encode_bf16_2d(&c->tm_p, c->d_p_hl, HLW, prows, HLW * 2, 64, 32);
+  }
   return ZO_OK;
 }
 
@@ -529,6 +552,12 @@ zo_status zo_refresh(zo_ctx* c, uint32_t refresh_idx, int32_t reset_moments) {
                                c->stream),
             "split U into hi/lo");
     ++c->launches;
+    if (c->proj_tc) {
+      ZO_CUDA(zo::launch_split_v(c->d_mats, c->d_tc, c->d_proj_units, c->n_proj_units, c->r,
+                                 c->d_v_hl, c->stream),
+              "split V into hi/lo");
+      ++c->launches;
+    }
   }
   return ZO_OK;
 }

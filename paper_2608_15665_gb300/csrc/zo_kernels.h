@@ -92,6 +92,21 @@ cudaError_t launch_wpass_tmem(const uint4* u_t, const CUtensorMap& tm_b,
                               int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
                               bool inject_wait, cudaStream_t s);
 
+// ---- projection P = C V^T on the tensor cores, r >= 64 (zo_project_tc.cu) ---------
+bool project_tc_supported(int32_t r);
+// V_HL rows [hi | lo] of V (after a refresh); units = the projection units (matrix, first row)
+cudaError_t launch_split_v(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                           int32_t n_units, int32_t r, __nv_bfloat16* v_hl, cudaStream_t s);
+// C_HL rows [hi | lo] of C (every pass), r rows per matrix at matrix * r
+cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, __nv_bfloat16* c_hl,
+                           cudaStream_t s);
+// P_HL = [hi | lo] of V C^T: tm_v over V_HL (box 64 x 128), tm_c over C_HL (box 64 x r),
+// tm_p over P_HL (box 64 x 32)
+cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
+                              const CUtensorMap& tm_p, const TcMat* d_tc, const int2* d_units,
+                              int32_t n_units, int32_t grid, int32_t r, uint32_t* d_status,
+                              cudaStream_t s);
+
 // ---- refresh: batched TSQR + sign correction (zo_qr.cu) ------------------------
 int32_t qr_block_rows(int32_t r);
 cudaError_t launch_qr_up(const QrBlock* d_blocks, int32_t n_blocks, int32_t r, uint64_t seed,

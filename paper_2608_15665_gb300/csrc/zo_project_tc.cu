@@ -1,0 +1,368 @@
+// Projection P_i^T = V_i C_i^T on the 5th-generation tensor cores, r >= 64: the
+// prologue of every weight pass (Eq. (4) and Eq. (10) need U_i C_i V_i^T; the weight
+// pass takes P_i = C_i V_i^T as its second operand).
+//
+// At r = 128 the projection is an r^2-deep contraction per column of P -- 2 r^2 flops
+// per row of V, 37 GFLOP per pass on the LLaMA-7B set -- so it runs as a GEMM on
+// tcgen05.mma: D (128 rows of V x r columns) = V_tile . C^T with M = 128, N = K = r.
+// Both operands are split x = hi + lo in bf16 like the weight pass's operands and the
+// products hi.hi + hi.lo + lo.hi accumulate in fp32 in Tensor Memory (relative error
+// ~2^-16 against the summed terms); the epilogue splits D into the bf16 hi/lo rows of
+// P_HL.  V_HL ([hi | lo] rows of V) is formed once per refresh, C_HL once per pass.
+//
+// Roles of the 192 threads of a CTA (one CTA per SM, each over a contiguous range of
+// 128-row units, so C_HL is reloaded only when the matrix changes):
+//   warp 0, lane 0: TMA producer -- the C_HL tile of a new matrix (r rows), the V_HL
+//                   tile of every unit (128 rows).
+//   warp 1, lane 0: MMA issuer -- 3 * r/16 tcgen05.mma (M=128, N=r, K=16) per unit into
+//                   one of two TMEM accumulators; warp 1 also owns the TMEM allocation.
+//   warps 2..5:     epilogue -- warp w owns 32 rows (its TMEM lane group): tcgen05.ld
+//                   the fp32 row of D, split it into bf16 hi/lo, write the 32 x 64 boxes
+//                   of P_HL into shared memory (128-byte swizzle), TMA-store them.
+// Every mbarrier wait is bounded; on expiry the kernel records kDevTimeout in the
+// status word, lets the other roles stop, drains its copies and frees TMEM.
+#include <cuda.h>
+
+#include "zo_kernels.h"
+#include "zo_sm100.cuh"
+#include "zo_tc_common.cuh"
+
+namespace zo {
+namespace {
+
+using namespace sm100;
+using namespace tc;
+
+constexpr int kProjThreads = 192;
+
+template <int R>
+struct ProjCfg {
+  static_assert(R == 64 || R == 128, "the tensor-core projection covers r = 64 and r = 128");
+  static constexpr int kHLW = hl_width(R);                 // 2R bf16 per operand row
+  static constexpr int kPanels = kHLW / 64;                // 128-byte panels per row
+  static constexpr int kVBytes = kPanels * kPanelBytes;    // V tile: 128 rows
+  static constexpr int kCPanelBytes = R * 128;             // C panel: R rows x 128 bytes
+  static constexpr int kCBytes = kPanels * kCPanelBytes;
+  static constexpr int kOutBoxBytes = 32 * 128;            // 32 rows x 64 bf16
+  static constexpr int kOutBytes = 4 * kPanels * kOutBoxBytes;
+  static constexpr int kKC = R / 16;                       // K chunks of 16
+  static constexpr int kTmemCols = 2 * R;                  // two accumulators
+  // R = 128: 64 + 64 + 64 KB; R = 64: 32 + 16 + 32 KB
+  static constexpr size_t kSmem = (size_t)kVBytes + kCBytes + kOutBytes + 1024 + 1024;
+};
+
+struct ProjShared {
+  uint64_t v_full, v_empty, c_full, c_empty;
+  uint64_t acc_full[2], acc_empty[2];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+__device__ __forceinline__ void proj_give_up(ProjShared& sh, uint32_t* status) {
+  atomicOr(status, (uint32_t)kDevTimeout);
+  *reinterpret_cast<volatile int*>(&sh.abort_flag) = 1;
+}
+
+template <int R>
+__global__ void __launch_bounds__(kProjThreads, 1)
+project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_c,
+                  const __grid_constant__ CUtensorMap tm_p, const TcMat* __restrict__ mats,
+                  const int2* __restrict__ units, int n_units, uint32_t* __restrict__ status,
+                  long long wait_cycles) {
+  using Cfg = ProjCfg<R>;
+  static_assert(sizeof(ProjShared) <= 1024, "barrier block");
+  static_assert(Cfg::kSmem <= 227 * 1024, "shared memory per CTA");
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* v_smem = smem;
+  uint8_t* c_smem = v_smem + Cfg::kVBytes;
+  uint8_t* o_smem = c_smem + Cfg::kCBytes;
+  ProjShared& sh = *reinterpret_cast<ProjShared*>(o_smem + Cfg::kOutBytes);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int u_begin = (int)((int64_t)n_units * blockIdx.x / gridDim.x);
+  const int u_end = (int)((int64_t)n_units * (blockIdx.x + 1) / gridDim.x);
+  const volatile int* abort = &sh.abort_flag;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&sh.v_full, 1);
+    mbar_init(&sh.v_empty, 1);
+    mbar_init(&sh.c_full, 1);
+    mbar_init(&sh.c_empty, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sh.acc_full[s], 1);
+      mbar_init(&sh.acc_empty[s], 4);
+    }
+    sh.abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tm_v);
+    prefetch_tmap(&tm_c);
+    prefetch_tmap(&tm_p);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sh.tmem_base, Cfg::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sh.tmem_base;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------ TMA producer
+    int64_t n_v = 0, n_c = 0;                     // tiles issued into each single-slot ring
+    int prev_i = -1;
+    bool ok = true;
+    for (int u = u_begin; u < u_end; ++u) {
+      const int2 un = units[u];
+      if (un.x != prev_i) {
+        if (!mbar_wait_bounded(&sh.c_empty, (uint32_t)((n_c & 1) ^ 1), abort, wait_cycles)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(&sh.c_full, Cfg::kCBytes);
+        for (int p = 0; p < Cfg::kPanels; ++p)
+          tma_load_2d(c_smem + p * Cfg::kCPanelBytes, &tm_c, 64 * p, un.x * R, &sh.c_full);
+        ++n_c;
+        prev_i = un.x;
+      }
+      if (!mbar_wait_bounded(&sh.v_empty, (uint32_t)((n_v & 1) ^ 1), abort, wait_cycles)) {
+        ok = false;
+        break;
+      }
+      mbar_arrive_expect_tx(&sh.v_full, Cfg::kVBytes);
+      for (int p = 0; p < Cfg::kPanels; ++p)
+        tma_load_2d(v_smem + p * kPanelBytes, &tm_v, 64 * p, mats[un.x].p_row0 + un.y, &sh.v_full);
+      ++n_v;
+    }
+    if (!ok) proj_give_up(sh, status);
+    // drain: the last copy issued into each slot has landed before the CTA exits
+    if (n_c > 0) mbar_wait_bounded(&sh.c_full, (uint32_t)((n_c - 1) & 1), nullptr, wait_cycles);
+    if (n_v > 0) mbar_wait_bounded(&sh.v_full, (uint32_t)((n_v - 1) & 1), nullptr, wait_cycles);
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------------------ MMA issuer
+    constexpr uint32_t idesc = idesc_bf16_f32(kBM, R);
+    int64_t it = 0, n_c = 0;
+    int prev_i = -1;
+    bool ok = true;
+    for (int u = u_begin; u < u_end; ++u, ++it) {
+      const int2 un = units[u];
+      const bool new_c = un.x != prev_i;
+      const bool last_c = u + 1 >= u_end || units[u + 1].x != un.x;
+      const int acc = (int)(it & 1);
+      if (!mbar_wait_bounded(&sh.acc_empty[acc], (uint32_t)(((it >> 1) & 1) ^ 1), abort,
+                             wait_cycles)) { ok = false; break; }
+      if (new_c) {
+        if (!mbar_wait_bounded(&sh.c_full, (uint32_t)(n_c & 1), abort, wait_cycles)) {
+          ok = false;
+          break;
+        }
+        ++n_c;
+        prev_i = un.x;
+      }
+      if (!mbar_wait_bounded(&sh.v_full, (uint32_t)(it & 1), abort, wait_cycles)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t d = tmem + (uint32_t)(acc * R);
+      const uint32_t a_base = smem_u32(v_smem), b_base = smem_u32(c_smem);
+#pragma unroll
+      for (int kk = 0; kk < Cfg::kKC; ++kk) {
+        // hi chunk kk at element 16 kk of an operand row, lo chunk at R + 16 kk
+        const int e_hi = 16 * kk, e_lo = R + 16 * kk;
+        const uint64_t a_hi = sdesc_k_sw128(a_base + (e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
+        const uint64_t a_lo = sdesc_k_sw128(a_base + (e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
+        const uint64_t b_hi =
+            sdesc_k_sw128(b_base + (e_hi / 64) * Cfg::kCPanelBytes + (e_hi % 64) * 2);
+        const uint64_t b_lo =
+            sdesc_k_sw128(b_base + (e_lo / 64) * Cfg::kCPanelBytes + (e_lo % 64) * 2);
+        mma_bf16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
+        mma_bf16(d, a_hi, b_lo, idesc, 1u);
+        mma_bf16(d, a_lo, b_hi, idesc, 1u);
+      }
+      mma_commit(&sh.v_empty);
+      if (last_c) mma_commit(&sh.c_empty);
+      mma_commit(&sh.acc_full[acc]);
+    }
+    if (!ok) proj_give_up(sh, status);
+    if (it > 0) {
+      // every MMA issued by this thread has completed before TMEM is released
+      const int64_t last = it - 1;
+      mbar_wait_bounded(&sh.acc_full[last & 1], (uint32_t)((last >> 1) & 1), nullptr, wait_cycles);
+    }
+  } else if (warp >= 2 && warp <= 5) {
+    // ------------------------------------------------------------ epilogue
+    const int g = warp & 3;                      // TMEM lane group == rows 32 g .. + 31
+    const uint32_t lane_base = (uint32_t)(g * 32) << 16;
+    uint8_t* obox = o_smem + g * Cfg::kPanels * Cfg::kOutBoxBytes;   // this warp's boxes
+    int64_t it = 0;
+    bool ok = true;
+    for (int u = u_begin; u < u_end; ++u, ++it) {
+      const int2 un = units[u];
+      const int acc = (int)(it & 1);
+      if (!mbar_wait_bounded(&sh.acc_full[acc], (uint32_t)((it >> 1) & 1), abort, wait_cycles)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      // the previous unit's stores have finished reading this warp's boxes
+      if (lane == 0) bulk_wait_read_all();
+      __syncwarp();
+#pragma unroll
+      for (int h = 0; h < R / 64; ++h) {         // 64 columns of D at a time
+        uint32_t v[2][32];
+        tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R + 64 * h), v[0]);
+        tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R + 64 * h + 32), v[1]);
+        tmem_ld_wait();
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {            // columns 64 h + 8 j .. + 7
+          float x[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) x[e] = __uint_as_float(v[j >> 2][(j & 3) * 8 + e]);
+          uint4 hi, lo;
+          split8(x, hi, lo);
+          // hi at P_HL column 64 h + 8 j (box h), lo at column R + 64 h + 8 j (box R/64 + h)
+          const int sw = (j ^ (lane & 7)) << 4;
+          *reinterpret_cast<uint4*>(obox + h * Cfg::kOutBoxBytes + lane * 128 + sw) = hi;
+          *reinterpret_cast<uint4*>(obox + (R / 64 + h) * Cfg::kOutBoxBytes + lane * 128 + sw) = lo;
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sh.acc_empty[acc]);
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        const int y = mats[un.x].p_row0 + un.y + 32 * g;
+        for (int p = 0; p < Cfg::kPanels; ++p)
+          tma_store_2d(&tm_p, 64 * p, y, obox + p * Cfg::kOutBoxBytes);
+        bulk_commit();
+      }
+      __syncwarp();
+    }
+    if (!ok && lane == 0) proj_give_up(sh, status);
+    if (lane == 0) bulk_wait_all();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, Cfg::kTmemCols);
+  }
+}
+
+// Rows [bf16 hi(x) | bf16 lo(x)] of V (units = (matrix, first row) x 128 rows, into V_HL at
+// p_row0) or of C (one CTA per matrix, r rows into C_HL at matrix * r).  Each thread
+// splits one row; the rows are staged in shared memory with the 16-byte chunk index XOR
+// (row & 7) and written with coalesced 16-byte stores.
+template <int R, bool kC>
+__global__ void __launch_bounds__(128)
+split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
+                  const int2* __restrict__ units, __nv_bfloat16* __restrict__ dst) {
+  constexpr int kVecPerRow = 2 * R * 2 / 16;
+  extern __shared__ uint4 Os[];                  // 128 x kVecPerRow
+  const int tid = threadIdx.x;
+  int i, rows;
+  int64_t row0, dst_row0;
+  const float* src;
+  if constexpr (kC) {
+    i = blockIdx.x;
+    row0 = 0;
+    rows = R;
+    src = mats[i].C;
+    dst_row0 = (int64_t)i * R;
+  } else {
+    const int2 u = units[blockIdx.x];
+    i = u.x;
+    row0 = u.y;
+    rows = (int)(mats[i].n - row0 < 128 ? mats[i].n - row0 : 128);
+    src = mats[i].V;
+    dst_row0 = (int64_t)tcm[i].p_row0 + row0;
+  }
+  if (tid < rows) {
+    const float4* s4 = reinterpret_cast<const float4*>(src + (row0 + tid) * R);
+    uint4* orow = Os + tid * kVecPerRow;
+#pragma unroll
+    for (int g = 0; g < R / 8; ++g) {
+      const float4 a = s4[2 * g], b = s4[2 * g + 1];
+      const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+      uint4 hi, lo;
+      split8(x, hi, lo);
+      orow[g ^ (tid & 7)] = hi;
+      orow[(R / 8 + g) ^ (tid & 7)] = lo;
+    }
+  }
+  __syncthreads();
+  uint4* d4 = reinterpret_cast<uint4*>(dst + dst_row0 * (2 * R));
+  for (int e = tid; e < rows * kVecPerRow; e += 128) {
+    const int row = e / kVecPerRow, c = e % kVecPerRow;
+    d4[e] = Os[row * kVecPerRow + (c ^ (row & 7))];
+  }
+}
+
+template <int R>
+cudaError_t launch_project_tc_r(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
+                                const CUtensorMap& tm_p, const TcMat* d_tc, const int2* d_units,
+                                int32_t n_units, int32_t grid, uint32_t* d_status, cudaStream_t s) {
+  const size_t smem = ProjCfg<R>::kSmem;
+  cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<R>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  project_tc_kernel<R><<<grid, kProjThreads, smem, s>>>(tm_v, tm_c, tm_p, d_tc, d_units, n_units,
+                                                        d_status, kWaitCycles);
+  return cudaGetLastError();
+}
+
+template <int R, bool kC>
+cudaError_t launch_split_rows_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                                int32_t n_blocks, __nv_bfloat16* dst, cudaStream_t s) {
+  constexpr size_t smem = 128 * (size_t)(2 * R * 2);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(split_rows_kernel<R, kC>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  split_rows_kernel<R, kC><<<n_blocks, 128, smem, s>>>(d_mats, d_tc, d_units, dst);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool project_tc_supported(int32_t r) { return r == 64 || r == 128; }
+
+cudaError_t launch_split_v(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                           int32_t n_units, int32_t r, __nv_bfloat16* v_hl, cudaStream_t s) {
+  if (n_units <= 0) return cudaSuccess;
+  switch (r) {
+    case 64: return launch_split_rows_r<64, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
+    case 128: return launch_split_rows_r<128, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, __nv_bfloat16* c_hl,
+                           cudaStream_t s) {
+  if (n_mats <= 0) return cudaSuccess;
+  switch (r) {
+    case 64: return launch_split_rows_r<64, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
+    case 128: return launch_split_rows_r<128, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
+                              const CUtensorMap& tm_p, const TcMat* d_tc, const int2* d_units,
+                              int32_t n_units, int32_t grid, int32_t r, uint32_t* d_status,
+                              cudaStream_t s) {
+  if (n_units <= 0) return cudaSuccess;
+  switch (r) {
+    case 64: return launch_project_tc_r<64>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
+    case 128: return launch_project_tc_r<128>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace zo
