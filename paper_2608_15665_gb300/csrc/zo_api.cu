@@ -333,6 +333,10 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
     c->proj_tc = encode_bf16_2d(&c->tm_v, c->d_v_hl, HLW, prows, HLW * 2, 64, 128) &&
                  encode_bf16_2d(&c->tm_c, c->d_c_hl, HLW, crows, HLW * 2, 64, (uint32_t)c->r) &&
                  encode_bf16_2d(&c->tm_p, c->d_p_hl, HLW, prows, HLW * 2, 64, 32);
+    if (!c->proj_tc) {
+      g_last_error = "cuTensorMapEncodeTiled rejected a projection descriptor; using the FMA pass";
+      c->tc_ok = false;
+    }
   }
   return ZO_OK;
 }

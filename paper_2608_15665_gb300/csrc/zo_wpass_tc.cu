@@ -346,7 +346,7 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
   }
 }
 
-// Both split kernels below (U rows for r <= 32, P rows for every r) handle 128
+// Both split kernels below (U rows and P rows, r <= 32) handle 128
 // consecutive rows of one matrix per CTA: each
 // thread splits one row into 16-byte chunks of hi and lo, staged in shared memory with
 // the chunk index XOR (row & 7) so a quarter-warp's stores hit distinct banks; the CTA
@@ -444,105 +444,6 @@ project_split_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__
   write_rows<R>(Os, p_hl + ((int64_t)tcm[u.x].p_row0 + j0) * hl_width(R), rows);
 }
 
-// The same product for R >= 64, where it is a real contraction (R^2 FMAs per row of V):
-// a register-tiled SIMT GEMM.  256 threads own the CTA's 128 rows x R outputs as 16 x 16
-// thread blocks of 8 rows (ty*4 + {0..3}, 64 + ty*4 + {0..3}) x 4 R/64 columns
-// (64 p + tx*4 + {0..3}); V and C stream through shared memory in chunks of 32 values of
-// the contraction index b, both stored b-major so one 16-byte load feeds 4 rows or 4
-// columns.  Each output still sums b = 0..R-1 in order with one fmaf per term, so the
-// result equals the per-row kernel's above bit for bit.  Outputs are split and stored
-// straight from registers: 16 threads write one row's 64-byte run of hi (or lo).
-constexpr int kPjChunk = 32;
-
-__device__ __forceinline__ uint2 split4_store(const float (&x)[4], uint2& lo) {
-  const __nv_bfloat162 h0 = __floats2bfloat162_rn(x[0], x[1]);
-  const __nv_bfloat162 h1 = __floats2bfloat162_rn(x[2], x[3]);
-  const __nv_bfloat162 l0 = __floats2bfloat162_rn(x[0] - __low2float(h0), x[1] - __high2float(h0));
-  const __nv_bfloat162 l1 = __floats2bfloat162_rn(x[2] - __low2float(h1), x[3] - __high2float(h1));
-  lo = make_uint2(*reinterpret_cast<const uint32_t*>(&l0), *reinterpret_cast<const uint32_t*>(&l1));
-  return make_uint2(*reinterpret_cast<const uint32_t*>(&h0), *reinterpret_cast<const uint32_t*>(&h1));
-}
-
-template <int R>
-__global__ void __launch_bounds__(256, 2)
-project_split_gemm_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
-                          const int2* __restrict__ units, __nv_bfloat16* __restrict__ p_hl) {
-  static_assert(R == 64 || R == 128, "register tiling covers R = 64 and R = 128");
-  constexpr int kP = R / 64;                    // 4-column pieces per thread
-  constexpr int kLdV = 128 + 4, kLdC = R + 4;   // row pitch in floats (16-byte multiples)
-  __shared__ __align__(16) float Vs[kPjChunk * kLdV];   // Vs[b][row] = V[j0 + row, b0 + b]
-  __shared__ __align__(16) float Cs[kPjChunk * kLdC];   // Cs[b][a]   = C[a, b0 + b]
-  const int2 u = units[blockIdx.x];
-  const MatDesc md = mats[u.x];
-  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
-  const int64_t j0 = u.y;
-  const int rows = (int)(md.n - j0 < 128 ? md.n - j0 : 128);
-  const float* __restrict__ vsrc = md.V + j0 * R;
-  float acc[8][4 * kP];
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
-#pragma unroll
-    for (int c = 0; c < 4 * kP; ++c) acc[i][c] = 0.f;
-
-  for (int b0 = 0; b0 < R; b0 += kPjChunk) {
-    // a warp loads one 16-byte column group of 32 consecutive rows: conflict-free stores
-#pragma unroll
-    for (int it = 0; it < 4; ++it) {
-      const int e = tid + 256 * it, row = e & 127, c4 = e >> 7;
-      float4 t4 = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (row < rows) t4 = *reinterpret_cast<const float4*>(vsrc + (int64_t)row * R + b0 + 4 * c4);
-      Vs[(4 * c4 + 0) * kLdV + row] = t4.x;
-      Vs[(4 * c4 + 1) * kLdV + row] = t4.y;
-      Vs[(4 * c4 + 2) * kLdV + row] = t4.z;
-      Vs[(4 * c4 + 3) * kLdV + row] = t4.w;
-    }
-#pragma unroll
-    for (int it = 0; it < R * (kPjChunk / 4) / 256; ++it) {
-      const int e = tid + 256 * it, a = e % R, c4 = e / R;
-      const float4 t4 = *reinterpret_cast<const float4*>(md.C + a * R + b0 + 4 * c4);
-      Cs[(4 * c4 + 0) * kLdC + a] = t4.x;
-      Cs[(4 * c4 + 1) * kLdC + a] = t4.y;
-      Cs[(4 * c4 + 2) * kLdC + a] = t4.z;
-      Cs[(4 * c4 + 3) * kLdC + a] = t4.w;
-    }
-    __syncthreads();
-#pragma unroll 8
-    for (int b = 0; b < kPjChunk; ++b) {
-      const float4 v0 = *reinterpret_cast<const float4*>(Vs + b * kLdV + ty * 4);
-      const float4 v1 = *reinterpret_cast<const float4*>(Vs + b * kLdV + 64 + ty * 4);
-      const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-      float c[4 * kP];
-#pragma unroll
-      for (int p = 0; p < kP; ++p) {
-        const float4 c4 = *reinterpret_cast<const float4*>(Cs + b * kLdC + 64 * p + tx * 4);
-        c[4 * p] = c4.x; c[4 * p + 1] = c4.y; c[4 * p + 2] = c4.z; c[4 * p + 3] = c4.w;
-      }
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-#pragma unroll
-        for (int cc = 0; cc < 4 * kP; ++cc) acc[i][cc] = fmaf(c[cc], v[i], acc[i][cc]);
-    }
-    __syncthreads();
-  }
-
-  __nv_bfloat16* dst = p_hl + ((int64_t)tcm[u.x].p_row0 + j0) * hl_width(R);
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int row = (i < 4 ? 0 : 64) + ty * 4 + (i & 3);
-    if (row >= rows) continue;
-    __nv_bfloat16* drow = dst + (int64_t)row * hl_width(R);
-#pragma unroll
-    for (int p = 0; p < kP; ++p) {
-      const float x[4] = {acc[i][4 * p], acc[i][4 * p + 1], acc[i][4 * p + 2], acc[i][4 * p + 3]};
-      uint2 lo;
-      const uint2 hi = split4_store(x, lo);
-      const int col = 64 * p + tx * 4;
-      *reinterpret_cast<uint2*>(drow + col) = hi;
-      *reinterpret_cast<uint2*>(drow + R + col) = lo;
-    }
-  }
-}
-
 template <int R>
 constexpr size_t project_split_smem() {
   return 128 * (size_t)hl_width(R) * 2 + sizeof(float) * R * R;
@@ -564,17 +465,13 @@ cudaError_t launch_split_u_r(const MatDesc* d_mats, const TcMat* d_tc, const int
 template <int R>
 cudaError_t launch_project_split_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                                    int32_t n_units, __nv_bfloat16* p_hl, cudaStream_t s) {
-  if constexpr (R >= 64) {
-    project_split_gemm_kernel<R><<<n_units, 256, 0, s>>>(d_mats, d_tc, d_units, p_hl);
-  } else {
-    const size_t smem = project_split_smem<R>();
-    if (smem > 48 * 1024) {
-      cudaError_t e = cudaFuncSetAttribute(project_split_kernel<R>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      if (e != cudaSuccess) return e;
-    }
-    project_split_kernel<R><<<n_units, 128, smem, s>>>(d_mats, d_tc, d_units, p_hl);
+  const size_t smem = project_split_smem<R>();
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(project_split_kernel<R>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
   }
+  project_split_kernel<R><<<n_units, 128, smem, s>>>(d_mats, d_tc, d_units, p_hl);
   return cudaGetLastError();
 }
 
@@ -624,8 +521,6 @@ cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const
   switch (r) {
     case 16: return launch_project_split_r<16>(d_mats, d_tc, d_units, n_units, p_hl, s);
     case 32: return launch_project_split_r<32>(d_mats, d_tc, d_units, n_units, p_hl, s);
-    case 64: return launch_project_split_r<64>(d_mats, d_tc, d_units, n_units, p_hl, s);
-    case 128: return launch_project_split_r<128>(d_mats, d_tc, d_units, n_units, p_hl, s);
     default: return cudaErrorInvalidValue;
   }
 }
