@@ -64,6 +64,12 @@ struct zo_ctx {
   int32_t max_losses = 0;
   float* d_qr_ws = nullptr;      // TSQR stacks and tau
   zo::QrBlock* d_qr_blocks = nullptr;
+  // tall panels at r = 64, 128 are refreshed by CholeskyQR2 instead of the TSQR
+  zo::CqPanel* d_cq_panels = nullptr;
+  zo::CqChunk* d_cq_chunks = nullptr;
+  float* d_cq_partial = nullptr;
+  float* d_cq_linv = nullptr;
+  int32_t n_cq_panels = 0, n_cq_chunks = 0;
   std::vector<int64_t> up_off, up_cnt, down_off, down_cnt;   // per level, into d_qr_blocks
   uint32_t* d_status = nullptr;
   int path_option = 0;
@@ -104,6 +110,10 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_losses);
   cudaFree(c->d_qr_ws);
   cudaFree(c->d_qr_blocks);
+  cudaFree(c->d_cq_panels);
+  cudaFree(c->d_cq_chunks);
+  cudaFree(c->d_cq_partial);
+  cudaFree(c->d_cq_linv);
   cudaFree(c->d_status);
   cudaFree(c->d_u_op);
   cudaFree(c->d_p_hl);
@@ -456,11 +466,13 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
   // refresh plan (dry run for sizes, then the real pass with pointers)
   const int32_t B = zo::qr_block_rows(r);
   int64_t qr_floats = 0;
+  // a panel with rows >= 4r has kappa(Omega) <= ~3, well inside CholeskyQR2's range
+  auto use_cholqr = [&](int64_t rows) { return zo::cholqr_supported(r) && rows >= 4 * (int64_t)r; };
   {
     std::vector<QrLevel> dry;
     for (int32_t i = 0; i < n_mats; ++i) {
-      plan_panel(nullptr, mats[i].m, r, 0, zo::kTagOmegaU, B, dry, nullptr, &qr_floats);
-      plan_panel(nullptr, mats[i].n, r, 0, zo::kTagOmegaV, B, dry, nullptr, &qr_floats);
+      if (!use_cholqr(mats[i].m)) plan_panel(nullptr, mats[i].m, r, 0, zo::kTagOmegaU, B, dry, nullptr, &qr_floats);
+      if (!use_cholqr(mats[i].n)) plan_panel(nullptr, mats[i].n, r, 0, zo::kTagOmegaV, B, dry, nullptr, &qr_floats);
     }
   }
   e = cudaMalloc(&c->d_qr_ws, sizeof(float) * std::max<int64_t>(qr_floats, 4));
@@ -470,12 +482,26 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
   }
   std::vector<QrLevel> levels;
   int64_t off = 0;
+  std::vector<zo::CqPanel> cq_panels;
+  std::vector<zo::CqChunk> cq_chunks;
+  auto add_cholqr = [&](float* out, int64_t rows, uint32_t gidx, uint32_t tag) {
+    zo::CqPanel p{out, rows, gidx, tag, (int32_t)cq_chunks.size(), 0};
+    for (int64_t r0 = 0; r0 < rows; r0 += zo::kCqChunkRows) {
+      cq_chunks.push_back({r0, (int32_t)cq_panels.size(),
+                           (int32_t)std::min<int64_t>(zo::kCqChunkRows, rows - r0)});
+      ++p.n_chunks;
+    }
+    cq_panels.push_back(p);
+  };
   for (int32_t i = 0; i < n_mats; ++i) {
-    plan_panel(mats[i].U, mats[i].m, r, matrix_index_base + (uint32_t)i, zo::kTagOmegaU, B, levels,
-               c->d_qr_ws, &off);
-    plan_panel(mats[i].V, mats[i].n, r, matrix_index_base + (uint32_t)i, zo::kTagOmegaV, B, levels,
-               c->d_qr_ws, &off);
+    const uint32_t gidx = matrix_index_base + (uint32_t)i;
+    if (use_cholqr(mats[i].m)) add_cholqr(mats[i].U, mats[i].m, gidx, zo::kTagOmegaU);
+    else plan_panel(mats[i].U, mats[i].m, r, gidx, zo::kTagOmegaU, B, levels, c->d_qr_ws, &off);
+    if (use_cholqr(mats[i].n)) add_cholqr(mats[i].V, mats[i].n, gidx, zo::kTagOmegaV);
+    else plan_panel(mats[i].V, mats[i].n, r, gidx, zo::kTagOmegaV, B, levels, c->d_qr_ws, &off);
   }
+  c->n_cq_panels = (int32_t)cq_panels.size();
+  c->n_cq_chunks = (int32_t)cq_chunks.size();
   std::vector<zo::QrBlock> all_blocks;
   for (auto& lv : levels) {
     c->up_off.push_back((int64_t)all_blocks.size());
@@ -493,6 +519,14 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
   if (e == cudaSuccess) e = cudaMalloc(&c->d_proj_units, sizeof(int2) * std::max<size_t>(units.size(), 1));
   if (e == cudaSuccess) e = cudaMalloc(&c->d_qr_blocks, sizeof(zo::QrBlock) * std::max<size_t>(all_blocks.size(), 1));
   if (e == cudaSuccess) e = cudaMalloc(&c->d_status, sizeof(uint32_t));
+  if (e == cudaSuccess && c->n_cq_panels > 0) {
+    e = cudaMalloc(&c->d_cq_panels, sizeof(zo::CqPanel) * cq_panels.size());
+    if (e == cudaSuccess) e = cudaMalloc(&c->d_cq_chunks, sizeof(zo::CqChunk) * cq_chunks.size());
+    if (e == cudaSuccess)
+      e = cudaMalloc(&c->d_cq_partial, sizeof(float) * (size_t)cq_chunks.size() * r * r);
+    if (e == cudaSuccess)
+      e = cudaMalloc(&c->d_cq_linv, sizeof(float) * (size_t)cq_panels.size() * r * r);
+  }
   if (e != cudaSuccess) {
     cuda_fail(e, "cudaMalloc(context tables)");
     return fail(ZO_ERR_NOMEM);
@@ -504,6 +538,12 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
     e = cudaMemcpy(c->d_proj_units, units.data(), sizeof(int2) * units.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess && !all_blocks.empty())
     e = cudaMemcpy(c->d_qr_blocks, all_blocks.data(), sizeof(zo::QrBlock) * all_blocks.size(),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && c->n_cq_panels > 0)
+    e = cudaMemcpy(c->d_cq_panels, cq_panels.data(), sizeof(zo::CqPanel) * cq_panels.size(),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && c->n_cq_panels > 0)
+    e = cudaMemcpy(c->d_cq_chunks, cq_chunks.data(), sizeof(zo::CqChunk) * cq_chunks.size(),
                    cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemset(c->d_status, 0, sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
@@ -546,6 +586,13 @@ zo_status zo_refresh(zo_ctx* c, uint32_t refresh_idx, int32_t reset_moments) {
                                c->d_status, c->stream),
             "refresh down-pass kernel");
     ++c->launches;
+  }
+  if (c->n_cq_panels > 0) {
+    ZO_CUDA(zo::launch_cholqr(c->d_cq_panels, c->n_cq_panels, c->d_cq_chunks, c->n_cq_chunks,
+                              c->d_cq_partial, c->d_cq_linv, c->r, c->seed, refresh_idx,
+                              c->d_status, c->stream),
+            "refresh CholeskyQR2 kernels");
+    c->launches += 6;
   }
   if (reset_moments) {
     ZO_CUDA(zo::launch_zero_moments(c->d_mats, c->n_mats, c->r, c->stream), "zero moments");
@@ -685,8 +732,14 @@ zo_status zo_sync_status(zo_ctx* c) {
   ZO_CUDA(cudaMemcpy(&s, c->d_status, sizeof(s), cudaMemcpyDeviceToHost), "read status");
   if (s != 0) {
     ZO_CUDA(cudaMemset(c->d_status, 0, sizeof(uint32_t)), "clear status");
-    g_last_error = s == zo::kDevTimeout ? "a device-side wait ran out" : "a device-side bound check failed";
-    return s == zo::kDevTimeout ? ZO_ERR_TIMEOUT : ZO_ERR_CUDA;
+    if (s & zo::kDevTimeout) {
+      g_last_error = "a device-side wait ran out";
+      return ZO_ERR_TIMEOUT;
+    }
+    g_last_error = (s & zo::kDevNotPosDef)
+                       ? "refresh: a Gram matrix of a panel was not positive definite"
+                       : "a device-side bound check failed";
+    return ZO_ERR_CUDA;
   }
   return ZO_OK;
 }

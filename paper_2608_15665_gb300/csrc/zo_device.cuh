@@ -19,6 +19,7 @@ enum DeviceStatus : uint32_t {
   kDevOk = 0,
   kDevTimeout = 1,   // a bounded mbarrier / flag wait gave up
   kDevBounds = 2,    // an internal bound check failed; the access was skipped
+  kDevNotPosDef = 4, // refresh: a Gram matrix had a non-positive Cholesky pivot
 };
 
 // ---------------------------------------------------------------------------

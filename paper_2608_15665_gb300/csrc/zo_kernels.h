@@ -107,6 +107,28 @@ cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
                               int32_t n_units, int32_t grid, int32_t r, uint32_t* d_status,
                               cudaStream_t s);
 
+// ---- refresh of tall panels at r = 64, 128: CholeskyQR2 (zo_cholqr.cu) ------------
+constexpr int32_t kCqChunkRows = 1024;   // rows per partial Gram matrix
+struct CqPanel {
+  float* out;          // U_i or V_i: rows x r, row-major; receives Q
+  int64_t rows;
+  uint32_t gidx;       // matrix index for Omega
+  uint32_t tag;        // kTagOmegaU or kTagOmegaV
+  int32_t chunk0;      // first chunk of this panel
+  int32_t n_chunks;
+};
+struct CqChunk {
+  int64_t row0;        // first panel row of the chunk
+  int32_t panel;
+  int32_t nrows;       // <= kCqChunkRows
+};
+bool cholqr_supported(int32_t r);
+// Six launches: Gram, Cholesky + inverse, apply; twice.  d_partial: n_chunks x r x r
+// floats, d_linv: n_panels x r x r floats.
+cudaError_t launch_cholqr(const CqPanel* d_panels, int32_t n_panels, const CqChunk* d_chunks,
+                          int32_t n_chunks, float* d_partial, float* d_linv, int32_t r,
+                          uint64_t seed, uint32_t refresh_idx, uint32_t* d_status, cudaStream_t s);
+
 // ---- refresh: batched TSQR + sign correction (zo_qr.cu) ------------------------
 int32_t qr_block_rows(int32_t r);
 cudaError_t launch_qr_up(const QrBlock* d_blocks, int32_t n_blocks, int32_t r, uint64_t seed,
