@@ -64,7 +64,7 @@ struct zo_ctx {
   int32_t max_losses = 0;
   float* d_qr_ws = nullptr;      // TSQR stacks and tau
   zo::QrBlock* d_qr_blocks = nullptr;
-  // tall panels at r = 64, 128 are refreshed by CholeskyQR2 instead of the TSQR
+  // tall panels at r = 16 ... 128 are refreshed by CholeskyQR2 instead of the TSQR
   zo::CqPanel* d_cq_panels = nullptr;
   zo::CqChunk* d_cq_chunks = nullptr;
   float* d_cq_partial = nullptr;

@@ -1,4 +1,4 @@
-// Subspace refresh for tall panels at r = 64 and r = 128: Alg. 1's Haar factor by
+// Subspace refresh for tall panels at r = 16 ... 128: Alg. 1's Haar factor by
 // CholeskyQR2 (Fukaya, Nakatsukasa, Yanagisawa and Yamamoto, 2014).
 //
 // Alg. 1 wants Q of the QR factorisation of a Gaussian panel Omega (rows x r) with the
@@ -15,7 +15,7 @@
 // of r dependent Householder steps per block.  Omega is drawn in the kernels from the
 // counter contract (tags 2 / 3, element e = row * r + col at counter e / 4, lane e % 4),
 // exactly as the TSQR of zo_qr.cu draws it; panels shorter than 4r, and every panel at
-// other ranks, keep the TSQR.
+// r = 4 and 8, keep the TSQR.
 //
 // Launches per refresh: gram(Omega), chol, apply(Omega -> Q1), gram(Q1), chol,
 // apply(Q1 -> Q).  Sums over rows are fixed-order (per 1024-row chunk, then chunk by
@@ -48,6 +48,35 @@ __device__ __forceinline__ void stage_rows(const CqPanel& pn, int64_t r0, int n,
   }
 }
 
+// T consecutive floats (T = 1, 2, 4 or 8) from shared memory, and the same to global memory.
+template <int T>
+__device__ __forceinline__ void load_t(const float* p, float (&v)[T]) {
+  if constexpr (T >= 4) {
+#pragma unroll
+    for (int q = 0; q < T / 4; ++q) {
+      const float4 a = reinterpret_cast<const float4*>(p)[q];
+      v[4 * q] = a.x; v[4 * q + 1] = a.y; v[4 * q + 2] = a.z; v[4 * q + 3] = a.w;
+    }
+  } else if constexpr (T == 2) {
+    const float2 a = *reinterpret_cast<const float2*>(p);
+    v[0] = a.x; v[1] = a.y;
+  } else {
+    v[0] = p[0];
+  }
+}
+template <int T>
+__device__ __forceinline__ void store_t(float* p, const float (&v)[T]) {
+  if constexpr (T >= 4) {
+#pragma unroll
+    for (int q = 0; q < T / 4; ++q)
+      reinterpret_cast<float4*>(p)[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+  } else if constexpr (T == 2) {
+    *reinterpret_cast<float2*>(p) = make_float2(v[0], v[1]);
+  } else {
+    p[0] = v[0];
+  }
+}
+
 // Partial Gram matrix X^T X of one chunk (<= kCqChunkRows rows of one panel).  Thread
 // (ty, tx) of a 16 x 16 grid accumulates the T x T block rows ty*T.., columns tx*T..,
 // T = R / 16, over the chunk's rows.
@@ -73,13 +102,8 @@ cq_gram_kernel(const CqPanel* __restrict__ panels, const CqChunk* __restrict__ c
     __syncthreads();
     for (int k = 0; k < n; ++k) {
       float xa[T], xb[T];
-#pragma unroll
-      for (int q = 0; q < T / 4; ++q) {
-        const float4 a4 = *reinterpret_cast<const float4*>(X + k * kLd + ty * T + 4 * q);
-        const float4 b4 = *reinterpret_cast<const float4*>(X + k * kLd + tx * T + 4 * q);
-        xa[4 * q] = a4.x; xa[4 * q + 1] = a4.y; xa[4 * q + 2] = a4.z; xa[4 * q + 3] = a4.w;
-        xb[4 * q] = b4.x; xb[4 * q + 1] = b4.y; xb[4 * q + 2] = b4.z; xb[4 * q + 3] = b4.w;
-      }
+      load_t<T>(X + k * kLd + ty * T, xa);
+      load_t<T>(X + k * kLd + tx * T, xb);
 #pragma unroll
       for (int a = 0; a < T; ++a)
 #pragma unroll
@@ -191,11 +215,7 @@ cq_apply_kernel(const CqPanel* __restrict__ panels, const CqChunk* __restrict__ 
       const float4 x4 = *reinterpret_cast<const float4*>(XT + b * kLdX + 4 * ty);
       const float x[4] = {x4.x, x4.y, x4.z, x4.w};
       float l[T];
-#pragma unroll
-      for (int q = 0; q < T / 4; ++q) {
-        const float4 l4 = *reinterpret_cast<const float4*>(LT + b * kLdL + tx * T + 4 * q);
-        l[4 * q] = l4.x; l[4 * q + 1] = l4.y; l[4 * q + 2] = l4.z; l[4 * q + 3] = l4.w;
-      }
+      load_t<T>(LT + b * kLdL + tx * T, l);
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -205,10 +225,7 @@ cq_apply_kernel(const CqPanel* __restrict__ panels, const CqChunk* __restrict__ 
     for (int i = 0; i < 4; ++i) {
       const int j = 4 * ty + i;
       if (j >= n) continue;
-      float4* dst = reinterpret_cast<float4*>(pn.out + (ch.row0 + s0 + j) * R + tx * T);
-#pragma unroll
-      for (int q = 0; q < T / 4; ++q)
-        dst[q] = make_float4(acc[i][4 * q], acc[i][4 * q + 1], acc[i][4 * q + 2], acc[i][4 * q + 3]);
+      store_t<T>(pn.out + (ch.row0 + s0 + j) * R + tx * T, acc[i]);
     }
   }
 }
@@ -248,13 +265,15 @@ cudaError_t run_cholqr_r(const CqPanel* d_panels, int32_t n_panels, const CqChun
 
 }  // namespace
 
-bool cholqr_supported(int32_t r) { return r == 64 || r == 128; }
+bool cholqr_supported(int32_t r) { return r == 16 || r == 32 || r == 64 || r == 128; }
 
 cudaError_t launch_cholqr(const CqPanel* d_panels, int32_t n_panels, const CqChunk* d_chunks,
                           int32_t n_chunks, float* d_partial, float* d_linv, int32_t r,
                           uint64_t seed, uint32_t refresh_idx, uint32_t* d_status, cudaStream_t s) {
   if (n_panels <= 0) return cudaSuccess;
   switch (r) {
+    case 16: return run_cholqr_r<16>(d_panels, n_panels, d_chunks, n_chunks, d_partial, d_linv, seed, refresh_idx, d_status, s);
+    case 32: return run_cholqr_r<32>(d_panels, n_panels, d_chunks, n_chunks, d_partial, d_linv, seed, refresh_idx, d_status, s);
     case 64: return run_cholqr_r<64>(d_panels, n_panels, d_chunks, n_chunks, d_partial, d_linv, seed, refresh_idx, d_status, s);
     case 128: return run_cholqr_r<128>(d_panels, n_panels, d_chunks, n_chunks, d_partial, d_linv, seed, refresh_idx, d_status, s);
     default: return cudaErrorInvalidValue;

@@ -107,7 +107,7 @@ cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
                               int32_t n_units, int32_t grid, int32_t r, uint32_t* d_status,
                               cudaStream_t s);
 
-// ---- refresh of tall panels at r = 64, 128: CholeskyQR2 (zo_cholqr.cu) ------------
+// ---- refresh of tall panels at r = 16 ... 128: CholeskyQR2 (zo_cholqr.cu) ----------
 constexpr int32_t kCqChunkRows = 1024;   // rows per partial Gram matrix
 struct CqPanel {
   float* out;          // U_i or V_i: rows x r, row-major; receives Q
