@@ -49,7 +49,7 @@ TRAFFIC_BY_SOURCE = {
 # thread instructions per weight of the full-space SPSA kernel (ncu), keyed by source hash
 INSTR_PER_WEIGHT_BY_SOURCE = {
     # profiles/mezo_kernel_llama7b_2layers.md: 762.5 M warp instructions x 32 / 404.75 M weights
-    "02f7804f216dbccd": 60.3,
+    "bb20a98787164398": 60.3,
 }
 
 

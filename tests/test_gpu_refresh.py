@@ -1,4 +1,6 @@
-"""GPU parity of the refresh (Alg. 1 / Eq. (11)): batched TSQR + sign correction."""
+"""GPU parity of the refresh (Alg. 1 / Eq. (11)): CholeskyQR2 for panels with >= 4r rows at
+r >= 16, batched TSQR + sign correction for the others -- both must give the unique
+positive-diagonal factor of the oracle."""
 
 import numpy as np
 import pytest
@@ -17,10 +19,12 @@ CASES = [
     (32, [(11008, 4096), (600, 33)]),                # three-level tree for 11008 rows
     (64, [(25600, 128), (300, 64), (64, 257)]),      # five levels for 25600 rows; m == r
     (128, [(2048, 130), (300, 256)]),                 # four levels for 2048 rows; ragged tail
+    (16, [(64, 63), (1025, 64)]),                    # rows = 4r (CholeskyQR2) next to 4r - 1 (TSQR)
+    (32, [(128, 127), (2049, 128)]),                 # the same at r = 32; a 1-row last chunk
 ]
 
 
-@pytest.mark.parametrize("r,shapes", CASES, ids=[f"r{c[0]}" for c in CASES])
+@pytest.mark.parametrize("r,shapes", CASES, ids=[f"r{c[0]}-{k}" for k, c in enumerate(CASES)])
 def test_refresh_matches_oracle(lib, gpu, r, shapes):
     from paper_2608_15665_gb300.schedule import SubZeroPlus
     seed, base = 4242 + r, 10
