@@ -131,9 +131,14 @@ ZO_API zo_status zo_destroy(zo_ctx* ctx);
 /*
  * zo_refresh -- Alg. 1 (HaarProjMatrix) for every matrix at refresh index j
  * (Alg. 3 calls it when t mod F == 0; j = t / F).  Draws Omega_U (m x r, tag 2)
- * and Omega_V (n x r, tag 3) from the counter contract, takes their thin
- * Householder QR and multiplies column c of Q by sgn(R_cc) (Eq. (11), sgn(0) = +1),
- * writing U_i and V_i in place.  reset_moments != 0 also zeroes M_i and Vm_i.
+ * and Omega_V (n x r, tag 3) from the counter contract and writes into U_i and V_i
+ * the Q of their thin QR factorisation with diag(R) > 0, i.e. Q with column c
+ * multiplied by sgn(R_cc) (Eq. (11), sgn(0) = +1).  That factor is unique; panels
+ * with at least 4r rows at r >= 16 reach it by CholeskyQR2 (two rounds of Cholesky
+ * of the Gram matrix and a triangular solve), the others by a batched Householder
+ * TSQR with the sign fix.  A Gram matrix without a positive pivot (not expected for
+ * such panels) makes the next zo_sync_status return ZO_ERR_CUDA.  reset_moments != 0
+ * also zeroes M_i and Vm_i.
  */
 ZO_API zo_status zo_refresh(zo_ctx* ctx, uint32_t refresh_idx, int32_t reset_moments);
 
