@@ -20,6 +20,7 @@ barrier and the max over ranks of the timed region.
 
 import argparse
 import hashlib
+import re
 import json
 import os
 import statistics
@@ -39,17 +40,19 @@ FALLBACK_HBM_GBS = 6800.0
 # source it was taken on (reported as null once the source differs).
 L2_BYTES = 129e6          # GB300 L2 capacity
 TRAFFIC_BY_SOURCE = {
-    # profiles/wpass_tc_r32_llama7b_2layers.md: 1.578 GB on the 2-layer subset, x16.0 by weights
-    ("3509e1472d06a465", "llama7b_bf16_r32"): 25.24e9,
-    # profiles/wpass_tmem_r128_llama7b_2layers.md: 1.638 GB on the 2-layer subset, x16.0 by weights
-    ("3509e1472d06a465", "llama7b_bf16_r128_q99"): 26.21e9,
-    # profiles/wpass_tmem_r64_dense32b_1layer.md: 1.925 GB on the 1-layer subset, x64.0 by weights
-    ("3509e1472d06a465", "dense32b_bf16_r64"): 123.22e9,
+    # code hash (comments ignored) -> dram read + write bytes of one launch, from ncu
+    # --metrics dram__bytes_read.sum,dram__bytes_write.sum on a small case, scaled by weights
+    # profiles/wpass_tc_r32_llama7b_2layers.md: 1.5775 GB on the 2-layer subset, x16.0
+    ("4db8c342d3045808", "llama7b_bf16_r32"): 25.24e9,
+    # profiles/wpass_tmem_r128_llama7b_2layers.md: 1.6377 GB on the 2-layer subset, x16.0
+    ("4db8c342d3045808", "llama7b_bf16_r128_q99"): 26.20e9,
+    # profiles/wpass_tmem_r64_dense32b_1layer.md: 1.9266 GB on the 1-layer subset, x64.0
+    ("4db8c342d3045808", "dense32b_bf16_r64"): 123.30e9,
 }
 # thread instructions per weight of the full-space SPSA kernel (ncu), keyed by source hash
 INSTR_PER_WEIGHT_BY_SOURCE = {
     # profiles/mezo_kernel_llama7b_2layers.md: 762.5 M warp instructions x 32 / 404.75 M weights
-    "bb20a98787164398": 60.3,
+    "58c22d72c437f0a4": 60.3,
 }
 
 
@@ -82,15 +85,25 @@ def measured_peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_hash():
-    """sha256 (16 hex) of the sources of the tensor-core weight-pass kernels."""
+def _code_hash(names):
+    """sha256 (16 hex) of CUDA sources with comments and blank space removed, so that a
+    comment edit keeps the hash of the code the ncu counters were taken on."""
     h = hashlib.sha256()
-    for name in ("zo_wpass_tc.cu", "zo_wpass_tmem.cu", "zo_tc_common.cuh", "zo_sm100.cuh",
-                 "zo_device.cuh"):
+    for name in names:
         path = os.path.join(ROOT, "paper_2608_15665_gb300", "csrc", name)
-        if os.path.exists(path):
-            h.update(open(path, "rb").read())
+        if not os.path.exists(path):
+            continue
+        text = open(path, encoding="utf-8").read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        h.update(" ".join(text.split()).encode())
     return h.hexdigest()[:16]
+
+
+def kernel_source_hash():
+    """Code hash of the tensor-core weight-pass kernels and the headers they include."""
+    return _code_hash(("zo_wpass_tc.cu", "zo_wpass_tmem.cu", "zo_tc_common.cuh", "zo_sm100.cuh",
+                       "zo_device.cuh"))
 
 
 def subset(wl, layers):
@@ -107,10 +120,7 @@ def subset(wl, layers):
 
 
 def mezo_source_hash():
-    h = hashlib.sha256()
-    for name in ("zo_mezo.cu", "zo_device.cuh"):
-        h.update(open(os.path.join(ROOT, "paper_2608_15665_gb300", "csrc", name), "rb").read())
-    return h.hexdigest()[:16]
+    return _code_hash(("zo_mezo.cu", "zo_device.cuh"))
 
 
 # --------------------------------------------------------------------------- clocks

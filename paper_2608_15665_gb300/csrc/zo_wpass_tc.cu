@@ -1,9 +1,10 @@
 // Weight pass on the 5th-generation tensor cores: W_i <- rnd_bf16(W_i + U_i P_i)
 // for every bf16 matrix in one persistent launch (the fused form of Alg. 2's
 // "W_i <- W_i + eps U_i Z_i V_i^T", Eq. (4), and of the update of Eq. (10)).
-// This file holds the kernel for r <= 32 (both operands in shared memory), the operand
-// split kernels, the projection P = C V^T and the dispatch by rank; the r >= 64 kernel,
-// which reads U from Tensor Memory, is in zo_wpass_tmem.cu.
+// This file holds the kernel for r <= 32 (both operands in shared memory), its operand
+// split kernels, the projection P = C V^T for r <= 32 and the dispatch by rank; the
+// r >= 64 kernel, which reads U from Tensor Memory, is in zo_wpass_tmem.cu, its
+// projection in zo_project_tc.cu.
 //
 // The contraction U (128 x r) . P (r x 128) of a 128 x 128 tile is r-deep, so it
 // costs 2r flops per weight against 4 bytes of HBM traffic; past r = 16 that is
@@ -13,8 +14,8 @@
 // accumulates hi.hi + hi.lo + lo.hi in fp32 in Tensor Memory (relative error of
 // the product ~2^-16 instead of 2^-8).
 //
-// Roles of the 224 threads of a CTA (one CTA per SM, persistent over every G-th
-// tile, G = number of CTAs):
+// Roles of the 224 threads of a CTA (one CTA per SM, persistent over the chunks of 4
+// tiles b, b + G, b + 2G, ... of the interleaved walk, G = number of CTAs):
 //   warp 0, lane 0: TMA producer of W -- each tile as 8 boxes of 32 rows x 64
 //                   columns, 128-byte swizzle, as far ahead as the W ring allows.
 //   warp 6, lane 0: TMA producer of the operands -- the U tile when the row block
