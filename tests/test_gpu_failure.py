@@ -1,6 +1,7 @@
 """Failure detection on the GPU without a GPU fault.
 
-Every mbarrier wait of the tensor-core weight pass is bounded.  The test hook
+Every mbarrier wait of the tensor-core weight passes is bounded (both kernels: r <= 32
+with the operands in shared memory, r >= 64 with U in Tensor Memory).  The test hook
 ZO_OPTION_TEST_WAIT_TIMEOUT makes one CTA of the next pass wait on a barrier that
 nothing arrives on (a flag nothing sets); its wait runs out after ~0.1 s, the kernel
 records a timeout in the context's status word, the other roles of that CTA stop
@@ -15,12 +16,13 @@ from parity import assert_weights
 pytestmark = pytest.mark.gpu
 
 
-def test_expired_wait_reports_timeout_and_the_context_recovers(lib, gpu):
+@pytest.mark.parametrize("r", [32, 64, 128])
+def test_expired_wait_reports_timeout_and_the_context_recovers(lib, gpu, r):
     from paper_2608_15665_gb300 import binding as zb
     from paper_2608_15665_gb300.schedule import SubZeroPlus
     base, seed = 40, 6060
     z = SubZeroPlus([make_weight(300, 520, "bf16", 1, gpu), make_weight(1030, 264, "bf16", 2, gpu)],
-                    32, 2, seed, matrix_index_base=base)
+                    r, 2, seed, matrix_index_base=base)
     z.init_subspace(0)
     z.perturb(0, 0, 1.0, -1, 0.0, 1e-3)
     z.sync()
@@ -37,7 +39,7 @@ def test_expired_wait_reports_timeout_and_the_context_recovers(lib, gpu):
     after = snapshot(z)
     z.sync()
     for i in range(2):
-        want, T = oracle_perturb(before, i, "bf16", seed, base + i, 1, 32, [(1, 1.0)], 1e-1)
+        want, T = oracle_perturb(before, i, "bf16", seed, base + i, 1, r, [(1, 1.0)], 1e-1)
         assert_weights(after["W"][i], want, "bf16", f"after recovery, matrix {i}",
                        before=before["W"][i], terms=T)
     z.close()
