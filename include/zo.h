@@ -129,7 +129,7 @@ ZO_API zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, 
 ZO_API zo_status zo_destroy(zo_ctx* ctx);
 
 /*
- * zo_refresh -- Alg. 1 (HaarProjMatrix) for every matrix at refresh index j
+ * zo_refresh -- Alg. 1 (Haar-distributed bases) for every matrix at refresh index j
  * (Alg. 3 calls it when t mod F == 0; j = t / F).  Draws Omega_U (m x r, tag 2)
  * and Omega_V (n x r, tag 3) from the counter contract and writes into U_i and V_i
  * the Q of their thin QR factorisation with diag(R) > 0, i.e. Q with column c
@@ -147,7 +147,7 @@ ZO_API zo_status zo_refresh(zo_ctx* ctx, uint32_t refresh_idx, int32_t reset_mom
 ZO_API zo_status zo_init_subspace(zo_ctx* ctx, uint32_t refresh_idx);
 
 /*
- * zo_perturb -- one fused weight pass of Alg. 2 (PerturbParams) over all matrices:
+ * zo_perturb -- one fused weight pass of Alg. 2 (the in-place perturbation) over all matrices:
  *   W_i <- rnd(W_i + eps * U_i (ca Z_i^(qa) + cb Z_i^(qb)) V_i^T)
  * with Z_i^(k) the step-t Gaussian of query k (tag 1).  qb = -1 drops the second
  * term.  Two terms fuse the restore of one query with the perturbation of the

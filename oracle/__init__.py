@@ -13,9 +13,9 @@ order (SubZero+, arXiv 2608.15665):
                   al., SC'11) and Box-Muller; the seeds of Alg. 2 / Alg. 3.
 * ``rounding`` -- rounding of an exact fp64 value to the weight storage dtype
                   (bf16 / fp32, round-to-nearest-even, one rounding per pass).
-* ``haar``     -- Alg. 1 (HaarProjMatrix): thin Householder QR of a Gaussian
+* ``haar``     -- Alg. 1 (Haar-distributed bases): thin Householder QR of a Gaussian
                   matrix followed by the sign correction of Eq. (11).
-* ``subzero``  -- Alg. 2 (PerturbParams) as a fused pass W <- rnd(W + U C V^T),
+* ``subzero``  -- Alg. 2 (the in-place perturbation) as a fused pass W <- rnd(W + U C V^T),
                   the multi-query estimator of Eq. (6), the subspace Adam of
                   Eqs. (7)-(10), and the Alg. 3 schedule driver.
 * ``mezo``     -- the full-space SPSA perturbation of Eq. (1) (MeZO's baseline):

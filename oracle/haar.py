@@ -1,4 +1,4 @@
-"""Alg. 1 (HaarProjMatrix) of the oracle (test infrastructure only).
+"""Alg. 1 (Haar-distributed projection bases) of the oracle (test infrastructure only).
 
 Sec. 4.3 / Eq. (11): draw a Gaussian Omega (rows x r), take its thin QR
 Omega = Q~ R~, and multiply column j of Q~ by sgn(R~_jj).  The result is the
@@ -76,7 +76,7 @@ def haar_from_gaussian(omega):
 
 
 def haar_proj(seed, i, j, m, n, r):
-    """Alg. 1 HaarProjMatrix(r, m_i, n_i) at refresh j for matrix i.
+    """Alg. 1 for matrix i (m_i x r and n_i x r bases) at refresh j.
 
     Omega_U (m x r) and Omega_V (n x r) come from the counter contract of
     ``oracle.rng`` (tags 2 and 3).  Returns (U, V), both fp64.

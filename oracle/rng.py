@@ -1,9 +1,9 @@
 """Counter-based Gaussian contract of the oracle (test infrastructure only).
 
-The paper draws every random matrix from a seed: Alg. 2 "reset RNG with seed
-s" then i.i.d. N(0,1) entries for Z_i; Alg. 3 "sample a random seed s_k^t";
-App. A.1 keeps only the seeds and regenerates each Z when needed; Alg. 1 draws
-the Gaussian Omega_U, Omega_V.  The paper does not say which generator.  The
+The paper draws every random matrix from a seed: Alg. 2 reseeds the generator
+and then draws i.i.d. N(0,1) entries for Z_i; Alg. 3 takes a fresh seed for each
+query of each step; App. A.1 keeps only the seeds and regenerates each Z when
+needed; Alg. 1 draws the Gaussian Omega_U, Omega_V.  The paper does not say which generator.  The
 contract fixed here (and implemented independently by the CUDA library) is:
 
 * generator: Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random

@@ -2,7 +2,7 @@
 
 Plain fp64 restatement of Sec. 4 of the paper:
 
-* ``perturb_coeff`` / ``apply_pass`` -- Alg. 2 (PerturbParams) and Eq. (4):
+* ``perturb_coeff`` / ``apply_pass`` -- Alg. 2 (the in-place perturbation) and Eq. (4):
   W_i <- W_i + eps U_i Z_i V_i^T.  Consecutive updates that touch W with no
   loss evaluation in between (restore of query k, perturbation of query k+1,
   the Adam update) are summed into one r x r coefficient C and applied as ONE
@@ -122,7 +122,7 @@ def sgd_direction(G):
 
 def step_coeff(D, lr, eps, restore_terms, seed, i, t, r):
     """C = -lr D + eps * sum_(k, c) c Z_i^(k): the Adam update of Eq. (10) fused
-    with the restore of the last query (Alg. 3, second PerturbParams call)."""
+    with the restore of the last query (Alg. 3, its second perturbation call)."""
     C = -float(lr) * np.asarray(D, np.float64)
     for k, c in restore_terms:
         C = C + float(eps) * float(c) * rng.gen_Z(seed, i, t, k, r)
@@ -142,7 +142,7 @@ def pass_plan(scheme, q, fused=True):
 
     central (Eq. (3), loss pairs): +Z0 | -2Z0 | +Z0+Z1 | -2Z1 | ... | -2Z_(q-1); restore +Z_(q-1)
     forward (Alg. 3):              +Z0 | Z1-Z0 | ... | Z_(q-1)-Z_(q-2);         restore -Z_(q-1)
-    With fused=False every PerturbParams call of Alg. 3 is its own rounded pass
+    With fused=False every perturbation call of Alg. 3 is its own rounded pass
     (restores become separate passes with no loss evaluation after them).
     """
     passes = []
@@ -182,7 +182,7 @@ class MatrixState:
 
 
 def refresh(state, seed, i, j, reset_moments=False):
-    """Alg. 3 lines 'if t mod F == 0: U, V <- HaarProjMatrix'."""
+    """Alg. 3's refresh: new bases U, V from Alg. 1 every F steps."""
     state.U, state.V = haar.haar_proj(seed, i, j, state.m, state.n, state.r)
     if reset_moments:
         state.M[:] = 0.0

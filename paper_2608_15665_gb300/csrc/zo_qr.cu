@@ -1,4 +1,4 @@
-// Subspace refresh: Alg. 1 (HaarProjMatrix) for every matrix in a few launches.
+// Subspace refresh: Alg. 1 (the Haar-distributed bases U, V) for every matrix in a few launches.
 //
 // For each panel (Omega_U, m x r and Omega_V, n x r) we need the thin QR factor
 // with a positive diagonal of R (Eq. (11)).  Panels are tall and skinny (m up to
