@@ -43,11 +43,11 @@ TRAFFIC_BY_SOURCE = {
     # code hash (comments ignored) -> dram read + write bytes of one launch, from ncu
     # --metrics dram__bytes_read.sum,dram__bytes_write.sum on a small case, scaled by weights
     # profiles/wpass_tc_r32_llama7b_2layers.md: 1.5775 GB on the 2-layer subset, x16.0
-    ("4db8c342d3045808", "llama7b_bf16_r32"): 25.24e9,
+    ("d85d2a44b97e1c78", "llama7b_bf16_r32"): 25.25e9,
     # profiles/wpass_tmem_r128_llama7b_2layers.md: 1.6377 GB on the 2-layer subset, x16.0
-    ("4db8c342d3045808", "llama7b_bf16_r128_q99"): 26.20e9,
+    ("d85d2a44b97e1c78", "llama7b_bf16_r128_q99"): 26.20e9,
     # profiles/wpass_tmem_r64_dense32b_1layer.md: 1.9266 GB on the 1-layer subset, x64.0
-    ("4db8c342d3045808", "dense32b_bf16_r64"): 123.30e9,
+    ("d85d2a44b97e1c78", "dense32b_bf16_r64"): 123.30e9,
 }
 # thread instructions per weight of the full-space SPSA kernel (ncu), keyed by source hash
 INSTR_PER_WEIGHT_BY_SOURCE = {

@@ -1,10 +1,10 @@
 // Weight pass on the 5th-generation tensor cores: W_i <- rnd_bf16(W_i + U_i P_i)
 // for every bf16 matrix in one persistent launch (the fused form of Alg. 2's
 // "W_i <- W_i + eps U_i Z_i V_i^T", Eq. (4), and of the update of Eq. (10)).
-// This file holds the kernel for r <= 32 (both operands in shared memory), its operand
-// split kernels, the projection P = C V^T for r <= 32 and the dispatch by rank; the
-// r >= 64 kernel, which reads U from Tensor Memory, is in zo_wpass_tmem.cu, its
-// projection in zo_project_tc.cu.
+// This file holds the kernel for r <= 32 (both operands in shared memory) and the
+// dispatch by rank; the r >= 64 kernel, which reads U from Tensor Memory, is in
+// zo_wpass_tmem.cu; the operands are prepared in zo_operands.cu (r <= 32) and
+// zo_project_tc.cu / zo_wpass_tmem.cu (r >= 64).
 //
 // The contraction U (128 x r) . P (r x 128) of a 128 x 128 tile is r-deep, so it
 // costs 2r flops per weight against 4 bytes of HBM traffic; past r = 16 that is
@@ -347,135 +347,6 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
   }
 }
 
-// Both split kernels below (U rows and P rows, r <= 32) handle 128
-// consecutive rows of one matrix per CTA: each
-// thread splits one row into 16-byte chunks of hi and lo, staged in shared memory with
-// the chunk index XOR (row & 7) so a quarter-warp's stores hit distinct banks; the CTA
-// then writes its rows, which are contiguous in the stacked operand, with coalesced
-// 16-byte stores.  Padding columns of a row stay at the zero they were set to.
-template <int R>
-__device__ __forceinline__ void write_rows(const uint4* Os, __nv_bfloat16* dst_rows, int rows) {
-  constexpr int kVecPerRow = hl_width(R) * 2 / 16;   // 8 or 16 chunks per row
-  uint4* dst = reinterpret_cast<uint4*>(dst_rows);
-  for (int e = threadIdx.x; e < rows * kVecPerRow; e += blockDim.x) {
-    const int row = e / kVecPerRow, c = e % kVecPerRow;
-    if (c * 8 < 2 * R) dst[e] = Os[row * kVecPerRow + (c ^ (row & 7))];
-  }
-}
-
-// U_HL[u_row0 + i] = [bf16 hi(U[i, :]) | bf16 lo(U[i, :]) | 0 ...]  (row width hl_width(R))
-template <int R>
-__global__ void __launch_bounds__(128)
-split_u_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
-               const int2* __restrict__ units, __nv_bfloat16* __restrict__ u_hl) {
-  constexpr int kVecPerRow = hl_width(R) * 2 / 16;
-  extern __shared__ uint4 su_smem[];
-  uint4* Os = su_smem;                                     // 128 x kVecPerRow
-  const int2 u = units[blockIdx.x];
-  const MatDesc md = mats[u.x];
-  const int tid = threadIdx.x;
-  const int64_t i0 = u.y;
-  const int rows = (int)(md.m - i0 < 128 ? md.m - i0 : 128);
-  if (tid < rows) {
-    const float4* src = reinterpret_cast<const float4*>(md.U + (i0 + tid) * R);
-    uint4* orow = Os + tid * kVecPerRow;
-#pragma unroll
-    for (int g = 0; g < R / 8; ++g) {
-      const float4 a = src[2 * g], b = src[2 * g + 1];
-      const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-      uint4 hi, lo;
-      split8(x, hi, lo);
-      orow[g ^ (tid & 7)] = hi;
-      orow[(R / 8 + g) ^ (tid & 7)] = lo;
-    }
-  }
-  __syncthreads();
-  write_rows<R>(Os, u_hl + ((int64_t)tcm[u.x].u_row0 + i0) * hl_width(R), rows);
-}
-
-// Pt_HL[p_row0 + j] = [hi | lo] of P^T[j, :] = (C V^T)^T[j, :] = V[j, :] C^T
-template <int R>
-__global__ void __launch_bounds__(128)
-project_split_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
-                     const int2* __restrict__ units, __nv_bfloat16* __restrict__ p_hl) {
-  constexpr int kVecPerRow = hl_width(R) * 2 / 16;
-  extern __shared__ uint4 ps_smem[];
-  uint4* Os = ps_smem;                                                // 128 x kVecPerRow
-  float* Cs = reinterpret_cast<float*>(Os + 128 * kVecPerRow);        // R x R
-  const int2 u = units[blockIdx.x];
-  const MatDesc md = mats[u.x];
-  const int tid = threadIdx.x;
-  const int64_t j0 = u.y;
-  const int rows = (int)(md.n - j0 < 128 ? md.n - j0 : 128);
-  for (int e = tid; e < R * R; e += 128) Cs[e] = md.C[e];
-  __syncthreads();
-  if (tid < rows) {
-    float v[R];
-    const float4* vrow = reinterpret_cast<const float4*>(md.V + (j0 + tid) * R);
-#pragma unroll
-    for (int b = 0; b < R / 4; ++b) {
-      const float4 t4 = vrow[b];
-      v[4 * b] = t4.x; v[4 * b + 1] = t4.y; v[4 * b + 2] = t4.z; v[4 * b + 3] = t4.w;
-    }
-    uint4* orow = Os + tid * kVecPerRow;
-    for (int g = 0; g < R / 8; ++g) {
-      float x[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        // C row read as 16-byte broadcasts: 4 FMAs per shared-memory load
-        const float4* crow = reinterpret_cast<const float4*>(Cs + (8 * g + k) * R);
-        float acc = 0.f;
-#pragma unroll
-        for (int b4 = 0; b4 < R / 4; ++b4) {
-          const float4 c4 = crow[b4];
-          acc = fmaf(c4.x, v[4 * b4], acc);
-          acc = fmaf(c4.y, v[4 * b4 + 1], acc);
-          acc = fmaf(c4.z, v[4 * b4 + 2], acc);
-          acc = fmaf(c4.w, v[4 * b4 + 3], acc);
-        }
-        x[k] = acc;
-      }
-      uint4 hi, lo;
-      split8(x, hi, lo);
-      orow[g ^ (tid & 7)] = hi;
-      orow[(R / 8 + g) ^ (tid & 7)] = lo;
-    }
-  }
-  __syncthreads();
-  write_rows<R>(Os, p_hl + ((int64_t)tcm[u.x].p_row0 + j0) * hl_width(R), rows);
-}
-
-template <int R>
-constexpr size_t project_split_smem() {
-  return 128 * (size_t)hl_width(R) * 2 + sizeof(float) * R * R;
-}
-
-template <int R>
-cudaError_t launch_split_u_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                             int32_t n_units, __nv_bfloat16* u_hl, cudaStream_t s) {
-  const size_t smem = 128 * (size_t)hl_width(R) * 2;
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(split_u_kernel<R>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-  }
-  split_u_kernel<R><<<n_units, 128, smem, s>>>(d_mats, d_tc, d_units, u_hl);
-  return cudaGetLastError();
-}
-
-template <int R>
-cudaError_t launch_project_split_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                                   int32_t n_units, __nv_bfloat16* p_hl, cudaStream_t s) {
-  const size_t smem = project_split_smem<R>();
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(project_split_kernel<R>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-  }
-  project_split_kernel<R><<<n_units, 128, smem, s>>>(d_mats, d_tc, d_units, p_hl);
-  return cudaGetLastError();
-}
-
 template <int R>
 cudaError_t launch_tc_r(const CUtensorMap& tm_a, const CUtensorMap& tm_b, const CUtensorMap* w_maps,
                         const TcMat* mats, int n_mats, int64_t n_tiles, int grid, uint32_t* status,
@@ -502,28 +373,6 @@ int64_t tc_u_operand_bytes(int32_t r, int64_t rows) {
   const int64_t row_layout = rows * hl_width(r) * 2;        // bf16 [hi | lo | 0] rows
   const int64_t chunk_layout = rows * r * 4;                // R 32-bit words per row
   return row_layout > chunk_layout ? row_layout : chunk_layout;
-}
-
-cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                           int32_t n_units, int32_t r, void* u_op, cudaStream_t s) {
-  if (n_units <= 0) return cudaSuccess;
-  switch (r) {
-    case 16: return launch_split_u_r<16>(d_mats, d_tc, d_units, n_units, static_cast<__nv_bfloat16*>(u_op), s);
-    case 32: return launch_split_u_r<32>(d_mats, d_tc, d_units, n_units, static_cast<__nv_bfloat16*>(u_op), s);
-    case 64:
-    case 128: return launch_split_u_chunks(d_mats, d_tc, d_units, n_units, r, static_cast<uint4*>(u_op), s);
-    default: return cudaErrorInvalidValue;
-  }
-}
-
-cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                                 int32_t n_units, int32_t r, __nv_bfloat16* p_hl, cudaStream_t s) {
-  if (n_units <= 0) return cudaSuccess;
-  switch (r) {
-    case 16: return launch_project_split_r<16>(d_mats, d_tc, d_units, n_units, p_hl, s);
-    case 32: return launch_project_split_r<32>(d_mats, d_tc, d_units, n_units, p_hl, s);
-    default: return cudaErrorInvalidValue;
-  }
 }
 
 cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const void* u_op, const CUtensorMap& tm_b,
