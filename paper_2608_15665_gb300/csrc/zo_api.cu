@@ -404,6 +404,7 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
 
   zo_ctx* c = new zo_ctx();
   c->device = dev;
+  c->sms = prop.multiProcessorCount;
   c->stream = reinterpret_cast<cudaStream_t>(stream);
   c->n_mats = n_mats;
   c->r = r;
@@ -635,6 +636,20 @@ zo_status zo_perturb(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t qb, fl
   p.ca = ca;
   p.cb = cb;
   p.eps = eps;
+  const bool use_tc = c->tc_ok && c->path_option != 1;
+  if (!use_tc && zo::wpass_fma_fused_supported(c->r) && c->n_tiles <= 4 * (int64_t)c->sms) {
+    // small r on the FMA path and a pass of a few waves at most (launch-bound, as for
+    // sets that fit in L2): C, P and the weight update in one launch.  On larger passes
+    // every CTA drawing C again costs more than the two launches it saves.
+    zo_status st = record_start(c);
+    if (st != ZO_OK) return st;
+    ZO_CUDA(zo::launch_wpass_fma_fused(c->d_mats, c->n_mats, c->d_tile_prefix, c->n_tiles, p,
+                                       c->stream),
+            "fused weight-pass kernel");
+    c->last_path = 1;
+    ++c->launches;
+    return record_stop(c);
+  }
   ZO_CUDA(zo::launch_coeff(c->d_mats, c->n_mats, p, c->stream), "coefficient kernel");
   ++c->launches;
   return run_weight_pass(c);

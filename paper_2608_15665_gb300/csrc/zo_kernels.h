@@ -57,6 +57,13 @@ __host__ __device__ constexpr int fma_tile_cols(int32_t dtype) { return dtype ==
 cudaError_t launch_wpass_fma(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_tile_prefix,
                              int64_t n_tiles, int32_t r, cudaStream_t s);
 
+// One-launch perturbation pass of the FMA path at r in {4, 8}: each CTA forms C from p
+// (mode kCoeffPerturb) and its tile's P columns itself (zo_wpass_fma.cu).
+bool wpass_fma_fused_supported(int32_t r);
+cudaError_t launch_wpass_fma_fused(const MatDesc* d_mats, int32_t n_mats,
+                                   const int64_t* d_tile_prefix, int64_t n_tiles,
+                                   const CoeffParams& p, cudaStream_t s);
+
 // ---- full-space SPSA perturbation of Eq. (1) (zo_mezo.cu) -------------------------
 // W_i <- rnd(W_i + coef Z_i), Z_i per element from the counter contract (tag 5), on the
 // FMA pass's tiles (d_tile_prefix / MatDesc::tile0).

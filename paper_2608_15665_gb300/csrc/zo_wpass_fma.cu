@@ -72,8 +72,12 @@ __device__ __forceinline__ int find_matrix(const int64_t* __restrict__ prefix, i
   return lo;
 }
 
-template <int R, typename T>
-__device__ __forceinline__ void wpass_tile(const MatDesc& md, int64_t local, float* Us, float* Ps) {
+// With kFused, P's columns of this tile are formed here from C (already in shared memory,
+// Cs) and V, in the projection kernel's order (sum over b ascending, one fmaf per term),
+// instead of being read from md.P.
+template <int R, typename T, bool kFused>
+__device__ __forceinline__ void wpass_tile(const MatDesc& md, int64_t local, float* Us, float* Ps,
+                                           const float* Cs) {
   constexpr int VEC = Vec<T>::N;
   constexpr int TN = 32 * VEC;
   const int tid = threadIdx.x;
@@ -103,13 +107,30 @@ __device__ __forceinline__ void wpass_tile(const MatDesc& md, int64_t local, flo
       const int64_t row = row0 + idx / (R / 4);
       Us4[idx] = row < md.m ? U4[row0 * (R / 4) + idx] : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    for (int idx = tid; idx < R * TN; idx += blockDim.x) {
-      const int k = idx / TN, c = idx % TN;
-      const int64_t gc = col0 + c;
-      const float pv = gc < md.n ? md.P[(int64_t)k * md.n + gc] : 0.f;
-      // layout [k][c % VEC / 4][c / VEC][c % 4]: a thread's 16-B chunks are contiguous across lanes
-      const int lane = c / VEC, part = (c % VEC) / 4, l4 = c % 4;
-      Ps[k * TN + part * 128 + lane * 4 + l4] = pv;
+    // layout [k][c % VEC / 4][c / VEC][c % 4]: a thread's 16-B chunks are contiguous across lanes
+    if constexpr (kFused) {
+      for (int c = tid; c < TN; c += blockDim.x) {
+        const int64_t gc = col0 + c;
+        const int lane = c / VEC, part = (c % VEC) / 4, l4 = c % 4;
+        float v[R];
+#pragma unroll
+        for (int b = 0; b < R; ++b) v[b] = gc < md.n ? md.V[gc * R + b] : 0.f;
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+          float acc = 0.f;
+#pragma unroll
+          for (int b = 0; b < R; ++b) acc = fmaf(Cs[k * R + b], v[b], acc);
+          Ps[k * TN + part * 128 + lane * 4 + l4] = gc < md.n ? acc : 0.f;
+        }
+      }
+    } else {
+      for (int idx = tid; idx < R * TN; idx += blockDim.x) {
+        const int k = idx / TN, c = idx % TN;
+        const int64_t gc = col0 + c;
+        const float pv = gc < md.n ? md.P[(int64_t)k * md.n + gc] : 0.f;
+        const int lane = c / VEC, part = (c % VEC) / 4, l4 = c % 4;
+        Ps[k * TN + part * 128 + lane * 4 + l4] = pv;
+      }
     }
   }
   __syncthreads();
@@ -176,9 +197,43 @@ wpass_fma_kernel(const MatDesc* __restrict__ mats, int n_mats, const int64_t* __
   const MatDesc md = mats[i];
   const int64_t local = tile - md.tile0;
   if (md.dtype == 1)
-    wpass_tile<R, __nv_bfloat16>(md, local, Us, Ps);
+    wpass_tile<R, __nv_bfloat16, false>(md, local, Us, Ps, nullptr);
   else
-    wpass_tile<R, float>(md, local, Us, Ps);
+    wpass_tile<R, float, false>(md, local, Us, Ps, nullptr);
+}
+
+// One launch per perturbation pass at small r: every CTA forms its matrix's C = eps (ca
+// Z_qa + cb Z_qb) in shared memory -- r^2 Gaussians, the coefficient kernel's arithmetic --
+// and the P columns of its tile, then updates the tile.  For the L2-resident sets the pass
+// is launch-bound, and one launch replaces three.
+template <int R>
+__global__ void __launch_bounds__(256, 2)
+wpass_fma_fused_kernel(const MatDesc* __restrict__ mats, int n_mats,
+                       const int64_t* __restrict__ prefix, CoeffParams p) {
+  extern __shared__ float4 smem4[];
+  float* Us = reinterpret_cast<float*>(smem4);
+  float* Ps = Us + kRows * R;
+  float* Cs = Ps + R * 256;
+  const int64_t tile = blockIdx.x;
+  const int i = find_matrix(prefix, n_mats, tile);
+  const MatDesc md = mats[i];
+  for (int c = threadIdx.x; c < R * R / 4; c += blockDim.x) {
+    const float4 za = normal4(p.seed, (uint32_t)c, md.gidx, p.t, query_word(kTagZ, (uint32_t)p.qa));
+    float4 acc = make_float4(p.ca * za.x, p.ca * za.y, p.ca * za.z, p.ca * za.w);
+    if (p.qb >= 0) {
+      const float4 zb = normal4(p.seed, (uint32_t)c, md.gidx, p.t, query_word(kTagZ, (uint32_t)p.qb));
+      acc = make_float4(fmaf(p.cb, zb.x, acc.x), fmaf(p.cb, zb.y, acc.y), fmaf(p.cb, zb.z, acc.z),
+                        fmaf(p.cb, zb.w, acc.w));
+    }
+    reinterpret_cast<float4*>(Cs)[c] =
+        make_float4(p.eps * acc.x, p.eps * acc.y, p.eps * acc.z, p.eps * acc.w);
+  }
+  __syncthreads();
+  const int64_t local = tile - md.tile0;
+  if (md.dtype == 1)
+    wpass_tile<R, __nv_bfloat16, true>(md, local, Us, Ps, Cs);
+  else
+    wpass_tile<R, float, true>(md, local, Us, Ps, Cs);
 }
 
 template <int R>
@@ -196,7 +251,29 @@ cudaError_t launch_r(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_pre
   return cudaGetLastError();
 }
 
+template <int R>
+cudaError_t launch_fused_r(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_prefix,
+                           int64_t n_tiles, const CoeffParams& p, cudaStream_t s) {
+  const size_t smem = sizeof(float) * (size_t)(kRows * R + R * 256 + R * R);
+  wpass_fma_fused_kernel<R><<<(unsigned)n_tiles, 256, smem, s>>>(d_mats, n_mats, d_prefix, p);
+  return cudaGetLastError();
+}
+
 }  // namespace
+
+bool wpass_fma_fused_supported(int32_t r) { return r == 4 || r == 8; }
+
+cudaError_t launch_wpass_fma_fused(const MatDesc* d_mats, int32_t n_mats,
+                                   const int64_t* d_tile_prefix, int64_t n_tiles,
+                                   const CoeffParams& p, cudaStream_t s) {
+  if (n_tiles <= 0) return cudaSuccess;
+  if (n_tiles > 0x7FFFFFFF) return cudaErrorInvalidValue;
+  switch (p.r) {
+    case 4: return launch_fused_r<4>(d_mats, n_mats, d_tile_prefix, n_tiles, p, s);
+    case 8: return launch_fused_r<8>(d_mats, n_mats, d_tile_prefix, n_tiles, p, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
 
 cudaError_t launch_wpass_fma(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_tile_prefix,
                              int64_t n_tiles, int32_t r, cudaStream_t s) {
