@@ -84,8 +84,13 @@ enum {
 
 /* Options for zo_set_option. */
 enum {
-  ZO_OPTION_WPASS_PATH = 0, /* 0 = automatic (tcgen05 when every W is bf16 and r >= 16),
-                               1 = fp32-FMA path, 2 = tcgen05 path */
+  ZO_OPTION_WPASS_PATH = 0, /* 0 = automatic: tcgen05 when every W is bf16 and r >= 16;
+                                   else, at r in {4, 8}, the narrow-tile FMA pass when its
+                                   tiles number at most half of the 32-row tiles (sets of
+                                   thin matrices such as LoRA factors); else the FMA pass,
+                               1 = FMA path on 32-row tiles, 2 = tcgen05 path,
+                               3 = FMA path on narrow tiles (r in {4, 8}).  All FMA
+                               tilings give bit-identical weights. */
   ZO_OPTION_TIMING = 1,     /* 1 = record CUDA events around every weight-pass launch */
   ZO_OPTION_TEST_WAIT_TIMEOUT = 2 /* test hook: 1 = in the next tensor-core weight pass, one
                                      CTA first waits on a barrier nothing arrives on, so its
@@ -204,7 +209,8 @@ ZO_API zo_status zo_set_option(zo_ctx* ctx, int32_t option, int64_t value);
  */
 ZO_API zo_status zo_get_timing(zo_ctx* ctx, double* total_ms, int64_t* launches);
 
-/* zo_wpass_path -- the weight-pass path the last zo_perturb / zo_step launched (1 = FMA, 2 = tcgen05). */
+/* zo_wpass_path -- the weight-pass path the last zo_perturb / zo_step launched
+   (1 = FMA on 32-row tiles, 2 = tcgen05, 3 = FMA on narrow tiles). */
 ZO_API int32_t zo_wpass_path(const zo_ctx* ctx);
 
 /* zo_kernel_launches -- number of kernels this context has launched since zo_create. */

@@ -57,6 +57,12 @@ struct zo_ctx {
   zo::MatDesc* d_mats = nullptr;
   int64_t* d_tile_prefix = nullptr;
   int64_t n_tiles = 0;
+  // narrow tiles of the FMA path (r in {4, 8}); chosen automatically when they need at
+  // most half the CTAs of the 32-row tiles
+  zo::NarrowMat* d_narrow = nullptr;
+  int32_t* d_narrow_tile_mat = nullptr;   // matrix of each narrow tile
+  int64_t n_narrow_tiles = 0, narrow_p = 0, narrow_u = 0;
+  bool narrow_ok = false, narrow_auto = false;
   int2* d_proj_units = nullptr;
   int32_t n_proj_units = 0;
   float* d_coeff_ws = nullptr;   // C_i and P_i
@@ -105,6 +111,8 @@ void free_ctx(zo_ctx* c) {
   if (!c) return;
   cudaFree(c->d_mats);
   cudaFree(c->d_tile_prefix);
+  cudaFree(c->d_narrow);
+  cudaFree(c->d_narrow_tile_mat);
   cudaFree(c->d_proj_units);
   cudaFree(c->d_coeff_ws);
   cudaFree(c->d_losses);
@@ -211,9 +219,28 @@ zo_status record_stop(zo_ctx* c) {
   return ZO_OK;
 }
 
+bool tc_path(const zo_ctx* c) { return c->tc_ok && (c->path_option == 0 || c->path_option == 2); }
+bool narrow_path(const zo_ctx* c) {
+  return c->narrow_ok && (c->path_option == 3 || (c->path_option == 0 && c->narrow_auto));
+}
+
 // Projection of C_i onto V_i and the weight pass, shared by zo_perturb and zo_step.
 zo_status run_weight_pass(zo_ctx* c) {
-  const bool use_tc = c->tc_ok && c->path_option != 1;
+  const bool use_tc = tc_path(c);
+  if (!use_tc && narrow_path(c)) {
+    // C_i is the coefficient kernel's output; P columns are formed in the pass
+    zo::CoeffParams p{};
+    p.mode = zo::kCoeffStep;
+    p.r = c->r;
+    zo_status st = record_start(c);
+    if (st != ZO_OK) return st;
+    ZO_CUDA(zo::launch_wpass_narrow(c->d_mats, c->d_narrow, c->d_narrow_tile_mat,
+                                    c->n_narrow_tiles, p, c->narrow_p, c->narrow_u, c->stream),
+            "narrow-tile weight-pass kernel");
+    c->last_path = 3;
+    ++c->launches;
+    return record_stop(c);
+  }
   if (use_tc && c->proj_tc) {
     ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, c->r, c->d_c_hl, c->stream), "split C");
     ++c->launches;
@@ -276,6 +303,45 @@ bool encode_bf16_2d(CUtensorMap* tm, void* base, uint64_t cols, uint64_t rows, u
   return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Tile table of the narrow-tile FMA pass (r in {4, 8}).
+zo_status setup_narrow(zo_ctx* c, const zo_matrix* mats) {
+  if (!zo::wpass_narrow_supported(c->r)) return ZO_OK;
+  std::vector<zo::NarrowMat> nm(c->n_mats);
+  int64_t tiles = 0;
+  for (int32_t i = 0; i < c->n_mats; ++i) {
+    int32_t rows = 1, chunks = 1;
+    zo::narrow_tile_shape(mats[i].m, mats[i].n, mats[i].dtype, &rows, &chunks);
+    const int64_t vec = mats[i].dtype == ZO_BF16 ? 8 : 4;
+    const int64_t cpr = (mats[i].n + vec - 1) / vec;
+    nm[i] = {tiles, rows, chunks};
+    tiles += ((mats[i].m + rows - 1) / rows) * ((cpr + chunks - 1) / chunks);
+    c->narrow_p = std::max(c->narrow_p, zo::narrow_p_floats(c->r, chunks, mats[i].dtype));
+    c->narrow_u = std::max(c->narrow_u, zo::narrow_u_floats(c->r, rows));
+  }
+  c->n_narrow_tiles = tiles;
+  if (tiles > 0x7FFFFFFF) return ZO_OK;   // beyond one grid: the 32-row tiles only
+  std::vector<int32_t> tile_mat((size_t)tiles);
+  for (int32_t i = 0; i < c->n_mats; ++i) {
+    const int64_t end = i + 1 < c->n_mats ? nm[i + 1].tile0 : tiles;
+    for (int64_t t = nm[i].tile0; t < end; ++t) tile_mat[(size_t)t] = i;
+  }
+  cudaError_t e = cudaMalloc(&c->d_narrow, sizeof(zo::NarrowMat) * c->n_mats);
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_narrow_tile_mat, sizeof(int32_t) * std::max<int64_t>(tiles, 1));
+  if (e == cudaSuccess)
+    e = cudaMemcpy(c->d_narrow, nm.data(), sizeof(zo::NarrowMat) * c->n_mats, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && tiles > 0)
+    e = cudaMemcpy(c->d_narrow_tile_mat, tile_mat.data(), sizeof(int32_t) * tiles,
+                   cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    cuda_fail(e, "narrow-tile table");
+    return e == cudaErrorMemoryAllocation ? ZO_ERR_NOMEM : ZO_ERR_CUDA;
+  }
+  c->narrow_ok = true;
+  // chosen automatically for sets that need at most half the CTAs of the 32-row tiles
+  c->narrow_auto = 2 * tiles <= c->n_tiles;
+  return ZO_OK;
 }
 
 // Buffers and descriptors of the tensor-core weight pass; leaves tc_ok false when
@@ -554,6 +620,8 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
   }
   zo_status st = setup_tc(c, mats);
   if (st != ZO_OK) return fail(st);
+  st = setup_narrow(c, mats);
+  if (st != ZO_OK) return fail(st);
   e = cudaDeviceSynchronize();
   if (e != cudaSuccess) {
     cuda_fail(e, "zo_create tensor-core setup");
@@ -636,7 +704,17 @@ zo_status zo_perturb(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t qb, fl
   p.ca = ca;
   p.cb = cb;
   p.eps = eps;
-  const bool use_tc = c->tc_ok && c->path_option != 1;
+  const bool use_tc = tc_path(c);
+  if (!use_tc && narrow_path(c)) {
+    zo_status st = record_start(c);
+    if (st != ZO_OK) return st;
+    ZO_CUDA(zo::launch_wpass_narrow(c->d_mats, c->d_narrow, c->d_narrow_tile_mat,
+                                    c->n_narrow_tiles, p, c->narrow_p, c->narrow_u, c->stream),
+            "narrow-tile weight-pass kernel");
+    c->last_path = 3;
+    ++c->launches;
+    return record_stop(c);
+  }
   if (!use_tc && zo::wpass_fma_fused_supported(c->r) && c->n_tiles <= 4 * (int64_t)c->sms) {
     // small r on the FMA path and a pass of a few waves at most (launch-bound, as for
     // sets that fit in L2): C, P and the weight update in one launch.  On larger passes
@@ -762,9 +840,13 @@ zo_status zo_sync_status(zo_ctx* c) {
 zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
   if (!c) return ZO_ERR_INVALID_ARG;
   if (option == ZO_OPTION_WPASS_PATH) {
-    if (value < 0 || value > 2) return ZO_ERR_INVALID_ARG;
+    if (value < 0 || value > 3) return ZO_ERR_INVALID_ARG;
     if (value == 2 && !c->tc_ok) {
       g_last_error = "the tensor-core weight pass needs every W in bf16 and r in {16, 32, 64, 128}";
+      return ZO_ERR_UNSUPPORTED;
+    }
+    if (value == 3 && !c->narrow_ok) {
+      g_last_error = "the narrow-tile weight pass needs r in {4, 8}";
       return ZO_ERR_UNSUPPORTED;
     }
     c->path_option = (int)value;

@@ -64,6 +64,30 @@ cudaError_t launch_wpass_fma_fused(const MatDesc* d_mats, int32_t n_mats,
                                    const int64_t* d_tile_prefix, int64_t n_tiles,
                                    const CoeffParams& p, cudaStream_t s);
 
+// Narrow-tile FMA pass at r in {4, 8} for thin matrices (LoRA factors and the like):
+// matrix i is cut into tiles of `rows` rows x `chunks` 16-byte column chunks
+// (rows x chunks <= kNarrowChunks, chunks x elements-per-chunk <= kNarrowMaxCols), numbered
+// from tile0 on.  Each CTA forms C (drawn from p.mode == kCoeffPerturb, or read from
+// MatDesc::C with kCoeffStep) and its tile's P columns itself (zo_wpass_fma.cu).
+struct NarrowMat {
+  int64_t tile0;
+  int32_t rows;
+  int32_t chunks;
+};
+constexpr int kNarrowChunks = 1024;
+constexpr int kNarrowMaxCols = 512;
+bool wpass_narrow_supported(int32_t r);
+// Tile shape of an m x n matrix of the given dtype (0 = fp32, 1 = bf16).
+void narrow_tile_shape(int64_t m, int64_t n, int32_t dtype, int32_t* rows, int32_t* chunks);
+// Shared-memory floats of the P and U parts of one tile of this shape.
+int64_t narrow_p_floats(int32_t r, int32_t chunks, int32_t dtype);
+int64_t narrow_u_floats(int32_t r, int32_t rows);
+// d_tile_mat[t]: the matrix of tile t; p_floats / u_floats: the largest P and U parts over
+// the set's tiles.
+cudaError_t launch_wpass_narrow(const MatDesc* d_mats, const NarrowMat* d_narrow,
+                                const int32_t* d_tile_mat, int64_t n_tiles, const CoeffParams& p,
+                                int64_t p_floats, int64_t u_floats, cudaStream_t s);
+
 // ---- full-space SPSA perturbation of Eq. (1) (zo_mezo.cu) -------------------------
 // W_i <- rnd(W_i + coef Z_i), Z_i per element from the counter contract (tag 5), on the
 // FMA pass's tiles (d_tile_prefix / MatDesc::tile0).

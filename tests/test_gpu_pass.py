@@ -289,3 +289,97 @@ def test_tensor_core_and_fma_paths_agree(lib, gpu, case):
         d = np.abs(a - b)
         assert np.all(d <= 2 * rounding.bf16_ulp(scale) + 2 * TZ)
         assert (d > 0).mean() < 1e-2
+
+
+# Sets of thin matrices at r in {4, 8}: LoRA-like factors in both orientations, ragged
+# widths, padded rows, a tall matrix of a single 16-byte chunk per row.
+NARROW_CASES = {
+    "lora4": (4, [(8, 1000, "f32", 1004), (1000, 8, "f32", None), (8, 520, "bf16", None),
+                  (520, 8, "bf16", 16), (5, 77, "f32", 80), (3000, 4, "f32", None)]),
+    "lora8": (8, [(8, 5120, "f32", None), (5120, 8, "f32", None), (16, 1030, "bf16", 1032),
+                  (1030, 12, "bf16", 16)]),
+    "r4": CASES["r4"],
+    "r8": CASES["r8"],
+}
+
+
+def _build_narrow(gpu, case, seed, base=21):
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    r, spec = NARROW_CASES[case]
+    weights = [make_weight(m, n, dt, 300 + k, gpu, ldw) for k, (m, n, dt, ldw) in enumerate(spec)]
+    z = SubZeroPlus(weights, r, 4, seed, matrix_index_base=base)
+    z.init_subspace(0)
+    return z, base
+
+
+@pytest.mark.parametrize("case", list(NARROW_CASES))
+def test_narrow_tile_pass_and_step_match_oracle(lib, gpu, case):
+    from paper_2608_15665_gb300 import binding as zb
+    z, base = _build_narrow(gpu, case, seed=2468)
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_WPASS_PATH, 3)
+    calls = [(0, 1.0, -1, 0.0), (0, -2.0, 1, 1.0), (3, 1.0, 2, -1.0)]
+    for t, (qa, ca, qb, cb) in zip((0, 0, 5), calls):
+        before = snapshot(z)
+        z.perturb(t, qa, ca, qb, cb, 1e-1)
+        after = snapshot(z)
+        assert zb.zo_wpass_path(z.ctx) == 3
+        terms = [(qa, ca)] + ([(qb, cb)] if qb >= 0 else [])
+        for i, W in enumerate(z.weights):
+            want, T = oracle_perturb(before, i, dtype_of(W), z.seed, base + i, t, z.r, terms, 1e-1)
+            assert_weights(after["W"][i], want, dtype_of(W), f"{case} matrix {i} t={t}",
+                           before=before["W"][i], terms=T)
+    q, eps, lr, b1, b2, ea = z.q, 1e-2, 1e-2, 0.9, 0.95, 1e-8
+    losses = np.array([2.01, 1.99, 2.0, 2.02, 1.97, 2.0, 2.03, 1.98], np.float32)
+    before = snapshot(z)
+    z.step(5, 1, losses, "central", eps, lr, b1, b2, ea, q - 1, 1.0)
+    after = snapshot(z)
+    assert zb.zo_wpass_path(z.ctx) == 3
+    rho = subzero.rho_from_losses(losses, "central", f32(eps), q)
+    for i, W in enumerate(z.weights):
+        Wo, Mo, Vmo, _, T = oracle_step(before, i, dtype_of(W), z.seed, base + i, 5, z.r, q, losses,
+                                        "central", eps, lr, b1, b2, ea, 1, [(q - 1, 1.0)])
+        assert_moments(after["M"][i], after["Vm"][i], Mo, Vmo, before["M"][i], before["Vm"][i],
+                       gabs(z.seed, base + i, 5, z.r, rho), b1, b2, f"{case} {i}")
+        assert_weights(after["W"][i], Wo, dtype_of(W), f"W {case} {i} step",
+                       before=before["W"][i], terms=T)
+    z.sync()
+    z.close()
+
+
+@pytest.mark.parametrize("case", list(NARROW_CASES))
+def test_narrow_and_32_row_tiles_are_bit_identical(lib, gpu, case):
+    # the two FMA tilings share C, the order of P's sum and of the update's sum, and the one
+    # rounding: every weight must come out bit for bit the same, pass after pass
+    from paper_2608_15665_gb300 import binding as zb
+    out = {}
+    losses = np.array([2.01, 1.99, 2.0, 2.02, 1.97, 2.0, 2.03, 1.98], np.float32)
+    for path in (1, 3):
+        z, _ = _build_narrow(gpu, case, seed=1357)
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_WPASS_PATH, path)
+        z.perturb(0, 0, 1.0, -1, 0.0, 1e-1)
+        z.perturb(0, 0, -2.0, 1, 1.0, 1e-1)
+        z.step(0, 1, losses, "central", 1e-1, 1e-2, 0.9, 0.95, 1e-8, z.q - 1, 1.0)
+        assert zb.zo_wpass_path(z.ctx) == path
+        z.sync()
+        out[path] = [W.detach().cpu().contiguous() for W in z.weights]
+        z.close()
+    for i, (a, b) in enumerate(zip(out[1], out[3])):
+        assert torch.equal(a.view(torch.int16) if a.dtype == torch.bfloat16 else a.view(torch.int32),
+                           b.view(torch.int16) if b.dtype == torch.bfloat16 else b.view(torch.int32)), \
+            f"{case} matrix {i}"
+
+
+def test_narrow_tiles_are_chosen_for_thin_sets(lib, gpu):
+    from paper_2608_15665_gb300 import binding as zb
+    z, _ = _build_narrow(gpu, "lora4", seed=11)
+    z.perturb(0, 0, 1.0, -1, 0.0, 1e-3)
+    assert zb.zo_wpass_path(z.ctx) == 3           # automatic: thin set -> narrow tiles
+    z.close()
+    z, _ = _build(gpu, "r8", seed=11)
+    z.perturb(0, 0, 1.0, -1, 0.0, 1e-3)
+    assert zb.zo_wpass_path(z.ctx) == 1           # 256 x 256 etc.: the 32-row tiles
+    z.close()
+    z, _ = _build_tc(gpu, "tc32", seed=11)
+    with pytest.raises(RuntimeError):
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_WPASS_PATH, 3)   # r = 32: no narrow tiles
+    z.close()
