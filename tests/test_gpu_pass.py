@@ -178,6 +178,9 @@ TC_CASES = {
     "tc32": (32, [(300, 520, 528), (1030, 72, 80), (257, 2048, None)]),
     "tc64": (64, [(300, 520, None), (130, 1000, None), (1030, 72, 72), (2048, 384, None)]),
     "tc128": (128, [(300, 520, None), (130, 1000, 1008), (1030, 136, None)]),
+    # widths that end inside a 16-byte chunk (the r = 128 epilogue stores W itself)
+    "tc128r": (128, [(300, 517, 520), (259, 133, 136), (131, 1001, 1008)]),
+    "tc64r": (64, [(300, 517, 520), (131, 1001, 1008)]),
 }
 
 
