@@ -51,8 +51,8 @@ TRAFFIC_BY_SOURCE = {
 }
 # thread instructions per weight of the full-space SPSA kernel (ncu), keyed by source hash
 INSTR_PER_WEIGHT_BY_SOURCE = {
-    # profiles/mezo_kernel_llama7b_2layers.md: 762.5 M warp instructions x 32 / 404.75 M weights
-    "58c22d72c437f0a4": 60.3,
+    # profiles/mezo_kernel_llama7b_2layers.md: 751.9 M warp instructions x 32 / 404.75 M weights
+    "a1a0ede2c35a3971": 59.4,
 }
 
 

@@ -16,6 +16,43 @@ namespace {
 
 constexpr uint32_t kTagMezo = 5;
 
+// The Philox round keys of one seed: (k0, k1) = (seed_lo, seed_hi) advanced by the Weyl
+// constants (0x9E3779B9, 0xBB67AE85) once per round -- the key schedule of zo_device.cuh's
+// philox4x32_10, formed once on the host.  Passed as a kernel parameter, each key is read
+// from the constant bank by the round's XOR: the eight Philox calls of a thread spend no
+// instructions and no registers on it.
+struct RoundKeys {
+  uint32_t k0[10], k1[10];
+};
+
+RoundKeys round_keys(uint64_t seed) {
+  RoundKeys k;
+  k.k0[0] = (uint32_t)seed;
+  k.k1[0] = (uint32_t)(seed >> 32);
+  for (int r = 1; r < 10; ++r) {
+    k.k0[r] = k.k0[r - 1] + 0x9E3779B9u;
+    k.k1[r] = k.k1[r - 1] + 0xBB67AE85u;
+  }
+  return k;
+}
+
+// philox4x32_10 and normal4 of zo_device.cuh with the round keys given.
+__device__ __forceinline__ float4 normal4_keyed(const RoundKeys& k, uint32_t c4, uint32_t x1,
+                                                uint32_t x2, uint32_t x3) {
+  uint4 c = make_uint4(c4, x1, x2, x3);
+#pragma unroll
+  for (int rnd = 0; rnd < 10; ++rnd) {
+    const uint32_t hi_a = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo_a = 0xD2511F53u * c.x;
+    const uint32_t hi_b = __umulhi(0xCD9E8D57u, c.z);
+    const uint32_t lo_b = 0xCD9E8D57u * c.z;
+    c = make_uint4(hi_b ^ c.y ^ k.k0[rnd], lo_b, hi_a ^ c.w ^ k.k1[rnd], lo_a);
+  }
+  const float2 a = box_muller(c.x, c.y);
+  const float2 b = box_muller(c.z, c.w);
+  return make_float4(a.x, a.y, b.x, b.y);
+}
+
 __device__ __forceinline__ int find_matrix_tile(const int64_t* __restrict__ prefix, int n_mats,
                                                 int64_t tile) {
   int lo = 0, hi = n_mats - 1;
@@ -33,7 +70,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 
 __global__ void __launch_bounds__(256)
 mezo_kernel(const MatDesc* __restrict__ mats, int n_mats, const int64_t* __restrict__ prefix,
-            uint64_t seed, uint32_t t, float coef) {
+            const __grid_constant__ RoundKeys keys, uint32_t t, float coef) {
   const int64_t tile = blockIdx.x;
   const MatDesc md = mats[find_matrix_tile(prefix, n_mats, tile)];
   const int bf16 = md.dtype == 1;
@@ -52,10 +89,10 @@ mezo_kernel(const MatDesc* __restrict__ mats, int n_mats, const int64_t* __restr
     if (row >= md.m) break;
     const uint32_t c0 = (uint32_t)(row * n4 + col / 4);
     float z[8];
-    const float4 za = normal4(seed, c0, md.gidx, t, x3);
+    const float4 za = normal4_keyed(keys, c0, md.gidx, t, x3);
     z[0] = za.x; z[1] = za.y; z[2] = za.z; z[3] = za.w;
     if (bf16) {
-      const float4 zb = normal4(seed, c0 + 1, md.gidx, t, x3);
+      const float4 zb = normal4_keyed(keys, c0 + 1, md.gidx, t, x3);
       z[4] = zb.x; z[5] = zb.y; z[6] = zb.z; z[7] = zb.w;
     }
     if (bf16) {
@@ -95,7 +132,8 @@ cudaError_t launch_mezo(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_
                         int64_t n_tiles, uint64_t seed, uint32_t t, float coef, cudaStream_t s) {
   if (n_tiles <= 0) return cudaSuccess;
   if (n_tiles > 0x7FFFFFFF) return cudaErrorInvalidValue;
-  mezo_kernel<<<(unsigned)n_tiles, 256, 0, s>>>(d_mats, n_mats, d_tile_prefix, seed, t, coef);
+  mezo_kernel<<<(unsigned)n_tiles, 256, 0, s>>>(d_mats, n_mats, d_tile_prefix, round_keys(seed), t,
+                                                coef);
   return cudaGetLastError();
 }
 
