@@ -84,7 +84,7 @@ struct zo_ctx {
   int64_t launches = 0;          // kernels launched by this context
   // tensor-core weight pass (all matrices bf16, r in {16, 32, 64, 128})
   bool tc_ok = false;
-  bool proj_tc = false;              // projection on the tensor cores too (r >= 64)
+  bool proj_tc = false;              // projection on the tensor cores too (r >= 32)
   int sms = 0;
   void* d_u_op = nullptr;            // stacked U operand of every U_i, 128-row padded
                                      // (rows [hi | lo | 0] for r <= 32, chunk-major for r >= 64)
@@ -95,8 +95,8 @@ struct zo_ctx {
   CUtensorMap tm_a{}, tm_b{};        // descriptors of the stacked operands (kernel parameters)
   int2* d_u_units = nullptr;
   int32_t n_u_units = 0;
-  __nv_bfloat16* d_v_hl = nullptr;   // [hi | lo] rows of every V_i (r >= 64), rows as P_HL
-  __nv_bfloat16* d_c_hl = nullptr;   // [hi | lo] rows of every C_i (r >= 64), r rows each
+  __nv_bfloat16* d_v_hl = nullptr;   // [hi | lo] rows of every V_i (r >= 32), rows as P_HL
+  __nv_bfloat16* d_c_hl = nullptr;   // [hi | lo] rows of every C_i (r >= 32), r rows each
   CUtensorMap tm_v{}, tm_c{}, tm_p{};  // V_HL, C_HL, and P_HL in 32-row boxes
   bool timing = false;
   std::vector<cudaEvent_t> ev_start, ev_stop;

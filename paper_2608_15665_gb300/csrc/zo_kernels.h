@@ -123,7 +123,7 @@ cudaError_t launch_wpass_tmem(const uint4* u_t, const CUtensorMap& tm_b,
                               int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
                               bool inject_wait, cudaStream_t s);
 
-// ---- projection P = C V^T on the tensor cores, r >= 64 (zo_project_tc.cu) ---------
+// ---- projection P = C V^T on the tensor cores, r >= 32 (zo_project_tc.cu) ---------
 bool project_tc_supported(int32_t r);
 // V_HL rows [hi | lo] of V (after a refresh); units = the projection units (matrix, first row)
 cudaError_t launch_split_v(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,

@@ -1,4 +1,4 @@
-// Projection P_i^T = V_i C_i^T on the 5th-generation tensor cores, r >= 64: the
+// Projection P_i^T = V_i C_i^T on the 5th-generation tensor cores, r >= 32: the
 // prologue of every weight pass (Eq. (4) and Eq. (10) need U_i C_i V_i^T; the weight
 // pass takes P_i = C_i V_i^T as its second operand).
 //
@@ -13,12 +13,14 @@
 // Roles of the 192 threads of a CTA (one CTA per SM, each over a contiguous range of
 // 128-row units, so C_HL is reloaded only when the matrix changes):
 //   warp 0, lane 0: TMA producer -- the C_HL tile of a new matrix (r rows), the V_HL
-//                   tile of every unit (128 rows).
+//                   tile of every unit (128 rows) into a ring of 2-4 stages, so the
+//                   loads of later units overlap the MMAs and the epilogue.
 //   warp 1, lane 0: MMA issuer -- 3 * r/16 tcgen05.mma (M=128, N=r, K=16) per unit into
 //                   one of two TMEM accumulators; warp 1 also owns the TMEM allocation.
 //   warps 2..5:     epilogue -- warp w owns 32 rows (its TMEM lane group): tcgen05.ld
-//                   the fp32 row of D, split it into bf16 hi/lo, write the 32 x 64 boxes
-//                   of P_HL into shared memory (128-byte swizzle), TMA-store them.
+//                   the fp32 row of D, split it into bf16 hi/lo, write them as 32 x 64
+//                   boxes of P_HL into shared memory (128-byte swizzle) and TMA-store
+//                   them, 64 columns of D at a time (one hi and one lo box staged).
 // Every mbarrier wait is bounded; on expiry the kernel records kDevTimeout in the
 // status word, lets the other roles stop, drains its copies and frees TMEM.
 #include <cuda.h>
@@ -37,22 +39,29 @@ constexpr int kProjThreads = 192;
 
 template <int R>
 struct ProjCfg {
-  static_assert(R == 64 || R == 128, "the tensor-core projection covers r = 64 and r = 128");
+  static_assert(R == 32 || R == 64 || R == 128,
+                "the tensor-core projection covers r = 32, 64 and 128");
   static constexpr int kHLW = hl_width(R);                 // 2R bf16 per operand row
   static constexpr int kPanels = kHLW / 64;                // 128-byte panels per row
   static constexpr int kVBytes = kPanels * kPanelBytes;    // V tile: 128 rows
   static constexpr int kCPanelBytes = R * 128;             // C panel: R rows x 128 bytes
   static constexpr int kCBytes = kPanels * kCPanelBytes;
   static constexpr int kOutBoxBytes = 32 * 128;            // 32 rows x 64 bf16
-  static constexpr int kOutBytes = 4 * kPanels * kOutBoxBytes;
+  // each epilogue warp stages one hi and one lo box (R = 32: one box holds both) and
+  // stores them 64 columns of D at a time
+  static constexpr int kWarpOutBytes = (R == 32 ? 1 : 2) * kOutBoxBytes;
+  static constexpr int kOutBytes = 4 * kWarpOutBytes;
   static constexpr int kKC = R / 16;                       // K chunks of 16
   static constexpr int kTmemCols = 2 * R;                  // two accumulators
-  // R = 128: 64 + 64 + 64 KB; R = 64: 32 + 16 + 32 KB
-  static constexpr size_t kSmem = (size_t)kVBytes + kCBytes + kOutBytes + 1024 + 1024;
+  // V ring: a unit's V tile is loaded while earlier units are multiplied
+  static constexpr int kVStages = R == 128 ? 2 : R == 64 ? 3 : 4;
+  // R = 128: 2 x 64 + 64 + 32 KB; R = 64: 3 x 32 + 16 + 32 KB; R = 32: 4 x 16 + 4 + 16 KB
+  static constexpr size_t kSmem =
+      (size_t)kVStages * kVBytes + kCBytes + kOutBytes + 1024 + 1024;
 };
 
 struct ProjShared {
-  uint64_t v_full, v_empty, c_full, c_empty;
+  uint64_t v_full[4], v_empty[4], c_full, c_empty;
   uint64_t acc_full[2], acc_empty[2];
   uint32_t tmem_base;
   int abort_flag;
@@ -76,7 +85,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint8_t* v_smem = smem;
-  uint8_t* c_smem = v_smem + Cfg::kVBytes;
+  uint8_t* c_smem = v_smem + Cfg::kVStages * Cfg::kVBytes;
   uint8_t* o_smem = c_smem + Cfg::kCBytes;
   ProjShared& sh = *reinterpret_cast<ProjShared*>(o_smem + Cfg::kOutBytes);
 
@@ -86,8 +95,10 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
   const volatile int* abort = &sh.abort_flag;
 
   if (threadIdx.x == 0) {
-    mbar_init(&sh.v_full, 1);
-    mbar_init(&sh.v_empty, 1);
+    for (int s = 0; s < Cfg::kVStages; ++s) {
+      mbar_init(&sh.v_full[s], 1);
+      mbar_init(&sh.v_empty[s], 1);
+    }
     mbar_init(&sh.c_full, 1);
     mbar_init(&sh.c_empty, 1);
     for (int s = 0; s < 2; ++s) {
@@ -111,7 +122,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
 
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------ TMA producer
-    int64_t n_v = 0, n_c = 0;                     // tiles issued into each single-slot ring
+    int64_t n_v = 0, n_c = 0;                     // tiles issued into the V ring and C slot
     int prev_i = -1;
     bool ok = true;
     for (int u = u_begin; u < u_end; ++u) {
@@ -127,19 +138,26 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
         ++n_c;
         prev_i = un.x;
       }
-      if (!mbar_wait_bounded(&sh.v_empty, (uint32_t)((n_v & 1) ^ 1), abort, wait_cycles)) {
+      const int vs = (int)(n_v % Cfg::kVStages);
+      if (!mbar_wait_bounded(&sh.v_empty[vs], (uint32_t)(((n_v / Cfg::kVStages) & 1) ^ 1), abort,
+                             wait_cycles)) {
         ok = false;
         break;
       }
-      mbar_arrive_expect_tx(&sh.v_full, Cfg::kVBytes);
+      mbar_arrive_expect_tx(&sh.v_full[vs], Cfg::kVBytes);
       for (int p = 0; p < Cfg::kPanels; ++p)
-        tma_load_2d(v_smem + p * kPanelBytes, &tm_v, 64 * p, mats[un.x].p_row0 + un.y, &sh.v_full);
+        tma_load_2d(v_smem + vs * Cfg::kVBytes + p * kPanelBytes, &tm_v, 64 * p,
+                    mats[un.x].p_row0 + un.y, &sh.v_full[vs]);
       ++n_v;
     }
     if (!ok) proj_give_up(sh, status);
     // drain: the last copy issued into each slot has landed before the CTA exits
     if (n_c > 0) mbar_wait_bounded(&sh.c_full, (uint32_t)((n_c - 1) & 1), nullptr, wait_cycles);
-    if (n_v > 0) mbar_wait_bounded(&sh.v_full, (uint32_t)((n_v - 1) & 1), nullptr, wait_cycles);
+    for (int vs = 0; vs < Cfg::kVStages; ++vs) {
+      const int64_t k = last_in_slot(n_v, vs, Cfg::kVStages);
+      if (k >= 0)
+        mbar_wait_bounded(&sh.v_full[vs], (uint32_t)((k / Cfg::kVStages) & 1), nullptr, wait_cycles);
+    }
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA issuer
     constexpr uint32_t idesc = idesc_bf16_f32(kBM, R);
@@ -161,13 +179,15 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
         ++n_c;
         prev_i = un.x;
       }
-      if (!mbar_wait_bounded(&sh.v_full, (uint32_t)(it & 1), abort, wait_cycles)) {
+      const int vs = (int)(it % Cfg::kVStages);
+      if (!mbar_wait_bounded(&sh.v_full[vs], (uint32_t)((it / Cfg::kVStages) & 1), abort,
+                             wait_cycles)) {
         ok = false;
         break;
       }
       tc_fence_after();
       const uint32_t d = tmem + (uint32_t)(acc * R);
-      const uint32_t a_base = smem_u32(v_smem), b_base = smem_u32(c_smem);
+      const uint32_t a_base = smem_u32(v_smem + vs * Cfg::kVBytes), b_base = smem_u32(c_smem);
 #pragma unroll
       for (int kk = 0; kk < Cfg::kKC; ++kk) {
         // hi chunk kk at element 16 kk of an operand row, lo chunk at R + 16 kk
@@ -182,7 +202,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
         mma_bf16(d, a_hi, b_lo, idesc, 1u);
         mma_bf16(d, a_lo, b_hi, idesc, 1u);
       }
-      mma_commit(&sh.v_empty);
+      mma_commit(&sh.v_empty[vs]);
       if (last_c) mma_commit(&sh.c_empty);
       mma_commit(&sh.acc_full[acc]);
     }
@@ -196,7 +216,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
     // ------------------------------------------------------------ epilogue
     const int g = warp & 3;                      // TMEM lane group == rows 32 g .. + 31
     const uint32_t lane_base = (uint32_t)(g * 32) << 16;
-    uint8_t* obox = o_smem + g * Cfg::kPanels * Cfg::kOutBoxBytes;   // this warp's boxes
+    uint8_t* obox = o_smem + g * Cfg::kWarpOutBytes;   // this warp's boxes
     int64_t it = 0;
     bool ok = true;
     for (int u = u_begin; u < u_end; ++u, ++it) {
@@ -207,39 +227,68 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
         break;
       }
       tc_fence_after();
+      const int y = mats[un.x].p_row0 + un.y + 32 * g;
       // the previous unit's stores have finished reading this warp's boxes
       if (lane == 0) bulk_wait_read_all();
       __syncwarp();
-#pragma unroll
-      for (int h = 0; h < R / 64; ++h) {         // 64 columns of D at a time
-        uint32_t v[2][32];
-        tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R + 64 * h), v[0]);
-        tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R + 64 * h + 32), v[1]);
+      if constexpr (R == 32) {
+        // one 64-wide box per row: hi at columns 8 j, lo at 32 + 8 j
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R), v);
         tmem_ld_wait();
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {            // columns 64 h + 8 j .. + 7
+        for (int j = 0; j < 4; ++j) {
           float x[8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) x[e] = __uint_as_float(v[j >> 2][(j & 3) * 8 + e]);
+          for (int e = 0; e < 8; ++e) x[e] = __uint_as_float(v[8 * j + e]);
           uint4 hi, lo;
           split8(x, hi, lo);
-          // hi at P_HL column 64 h + 8 j (box h), lo at column R + 64 h + 8 j (box R/64 + h)
-          const int sw = (j ^ (lane & 7)) << 4;
-          *reinterpret_cast<uint4*>(obox + h * Cfg::kOutBoxBytes + lane * 128 + sw) = hi;
-          *reinterpret_cast<uint4*>(obox + (R / 64 + h) * Cfg::kOutBoxBytes + lane * 128 + sw) = lo;
+          *reinterpret_cast<uint4*>(obox + lane * 128 + ((j ^ (lane & 7)) << 4)) = hi;
+          *reinterpret_cast<uint4*>(obox + lane * 128 + (((4 + j) ^ (lane & 7)) << 4)) = lo;
+        }
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_2d(&tm_p, 0, y, obox);
+          bulk_commit();
+        }
+      } else {
+#pragma unroll
+        for (int h = 0; h < R / 64; ++h) {       // 64 columns of D: one hi and one lo box
+          if (h > 0) {
+            // the stores of the previous 64 columns have read the two boxes
+            if (lane == 0) bulk_wait_read_all();
+            __syncwarp();
+          }
+          uint32_t v[2][32];
+          tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R + 64 * h), v[0]);
+          tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R + 64 * h + 32), v[1]);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {          // columns 64 h + 8 j .. + 7
+            float x[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[e] = __uint_as_float(v[j >> 2][(j & 3) * 8 + e]);
+            uint4 hi, lo;
+            split8(x, hi, lo);
+            const int sw = (j ^ (lane & 7)) << 4;
+            *reinterpret_cast<uint4*>(obox + lane * 128 + sw) = hi;
+            *reinterpret_cast<uint4*>(obox + Cfg::kOutBoxBytes + lane * 128 + sw) = lo;
+          }
+          fence_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            // hi to P_HL columns 64 h .. + 63, lo to R + 64 h .. + 63
+            tma_store_2d(&tm_p, 64 * h, y, obox);
+            tma_store_2d(&tm_p, R + 64 * h, y, obox + Cfg::kOutBoxBytes);
+            bulk_commit();
+          }
+          __syncwarp();
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sh.acc_empty[acc]);
-      fence_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        const int y = mats[un.x].p_row0 + un.y + 32 * g;
-        for (int p = 0; p < Cfg::kPanels; ++p)
-          tma_store_2d(&tm_p, 64 * p, y, obox + p * Cfg::kOutBoxBytes);
-        bulk_commit();
-      }
       __syncwarp();
     }
     if (!ok && lane == 0) proj_give_up(sh, status);
@@ -331,12 +380,13 @@ cudaError_t launch_split_rows_r(const MatDesc* d_mats, const TcMat* d_tc, const 
 
 }  // namespace
 
-bool project_tc_supported(int32_t r) { return r == 64 || r == 128; }
+bool project_tc_supported(int32_t r) { return r == 32 || r == 64 || r == 128; }
 
 cudaError_t launch_split_v(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                            int32_t n_units, int32_t r, __nv_bfloat16* v_hl, cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
+    case 32: return launch_split_rows_r<32, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
     case 64: return launch_split_rows_r<64, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
     case 128: return launch_split_rows_r<128, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
     default: return cudaErrorInvalidValue;
@@ -347,6 +397,7 @@ cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, __n
                            cudaStream_t s) {
   if (n_mats <= 0) return cudaSuccess;
   switch (r) {
+    case 32: return launch_split_rows_r<32, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
     case 64: return launch_split_rows_r<64, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
     case 128: return launch_split_rows_r<128, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
     default: return cudaErrorInvalidValue;
@@ -359,6 +410,7 @@ cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
                               cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
+    case 32: return launch_project_tc_r<32>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
     case 64: return launch_project_tc_r<64>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
     case 128: return launch_project_tc_r<128>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
     default: return cudaErrorInvalidValue;
