@@ -143,8 +143,8 @@ def test_full_size_sampled_parity(lib, gpu, name, sample):
 # add or remove one).  The ulp is taken at max(|W_gpu|, |W_oracle|, rms(W_0)) so that
 # weights passing through zero are measured at the scale of the weights.  Bounds are set
 # with a margin over measured GB300 histograms (r = 8 FMA, r = 32 / 64 tensor cores):
-#   eps = 1e-3 (the paper's): 0.014% / 0.020% / 0.042% of elements differ, max 1 / 1 / 2 ulp;
-#   eps = 1e-1 (stress, the update is ~40% of |W| per pass): 0.03% / 1.2% / 2.7%, max 2 / 6 / 8.
+#   eps = 1e-3 (the paper's): 0.014% / 0.022% / 0.042% of elements differ, max 1 / 1 / 2 ulp;
+#   eps = 1e-1 (stress, the update is ~40% of |W| per pass): 0.03% / 1.7% / 2.7% differ.
 TRAJ = [(8, [(256, 320), (130, 72)]), (32, [(512, 384), (300, 136)]),
         (64, [(512, 264), (1030, 136)])]
 TRAJ_BOUNDS = {  # eps -> (FMA or tensor cores) -> (max fraction differing, max ulps)
@@ -164,7 +164,7 @@ def test_bf16_trajectory_rounding_flips(lib, gpu, r, shapes, eps):
     z = SubZeroPlus([W.clone().to(gpu) for W in W0], wl.r, wl.q, wl.seed)
     table = _run_gpu_schedule(z, wl, "central", wl.steps)
     s = snapshot(z)
-    hist, total = np.zeros(4, np.int64), 0
+    hist, total, worst = np.zeros(4, np.int64), 0, 0
     for i in range(wl.n_mats):
         st = _oracle_trajectory(wl, to_f64(W0[i]), i, table, "central", wl.steps)
         w_rms = float(np.sqrt(np.mean(to_f64(W0[i]) ** 2)))
@@ -175,8 +175,9 @@ def test_bf16_trajectory_rounding_flips(lib, gpu, r, shapes, eps):
         dmax = int(d.max())
         frac_max, ulp_max = TRAJ_BOUNDS[eps]["fma" if r < 16 else "tc"]
         assert dmax <= ulp_max, f"matrix {i}: {dmax} ulps"
+        worst = max(worst, dmax)
     frac = 1.0 - hist[0] / total
     print(f"\nbf16 trajectory r={r} eps={eps}: elements at 0/1/2/3+ ulps {hist.tolist()}, "
-          f"{frac:.2e} differ")
+          f"{frac:.2e} differ, max {worst} ulps")
     assert frac <= frac_max
     z.close()
