@@ -84,7 +84,7 @@ struct zo_ctx {
   int64_t launches = 0;          // kernels launched by this context
   // tensor-core weight pass (all matrices bf16, r in {16, 32, 64, 128})
   bool tc_ok = false;
-  bool proj_tc = false;              // projection on the tensor cores too (r >= 32)
+  bool proj_tc = false;              // the projection's descriptors are in place
   int sms = 0;
   void* d_u_op = nullptr;            // stacked U operand of every U_i, 128-row padded
                                      // (rows [hi | lo | 0] for r <= 32, chunk-major for r >= 64)
@@ -95,8 +95,8 @@ struct zo_ctx {
   CUtensorMap tm_a{}, tm_b{};        // descriptors of the stacked operands (kernel parameters)
   int2* d_u_units = nullptr;
   int32_t n_u_units = 0;
-  __nv_bfloat16* d_v_hl = nullptr;   // [hi | lo] rows of every V_i (r >= 32), rows as P_HL
-  __nv_bfloat16* d_c_hl = nullptr;   // [hi | lo] rows of every C_i (r >= 32), r rows each
+  __nv_bfloat16* d_v_hl = nullptr;   // [hi | lo] rows of every V_i, rows as P_HL
+  __nv_bfloat16* d_c_hl = nullptr;   // [hi | lo] rows of every C_i, r rows each
   CUtensorMap tm_v{}, tm_c{}, tm_p{};  // V_HL, C_HL, and P_HL in 32-row boxes
   bool timing = false;
   std::vector<cudaEvent_t> ev_start, ev_stop;
@@ -241,17 +241,14 @@ zo_status run_weight_pass(zo_ctx* c) {
     ++c->launches;
     return record_stop(c);
   }
-  if (use_tc && c->proj_tc) {
+  if (use_tc) {
+    // setup_tc keeps tc_ok only with the projection's descriptors in place (proj_tc)
     ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, c->r, c->d_c_hl, c->stream), "split C");
     ++c->launches;
     const int grid = std::min<int>(c->n_proj_units, c->sms);
     ZO_CUDA(zo::launch_project_tc(c->tm_v, c->tm_c, c->tm_p, c->d_tc, c->d_proj_units,
                                   c->n_proj_units, grid, c->r, c->d_status, c->stream),
             "tensor-core projection kernel");
-  } else if (use_tc) {
-    ZO_CUDA(zo::launch_project_split(c->d_mats, c->d_tc, c->d_proj_units, c->n_proj_units, c->r,
-                                     c->d_p_hl, c->stream),
-            "projection kernel");
   } else {
     ZO_CUDA(zo::launch_project_fma(c->d_mats, c->d_proj_units, c->n_proj_units, c->r, c->stream),
             "projection kernel");
@@ -400,19 +397,19 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
           "upload tensor maps");
   c->tc_tiles = tiles;
   c->tc_ok = true;
-  if (zo::project_tc_supported(c->r)) {
-    const int64_t crows = (int64_t)c->n_mats * c->r;
-    ZO_CUDA(cudaMalloc(&c->d_v_hl, sizeof(__nv_bfloat16) * prows * HLW), "cudaMalloc(V hi/lo)");
-    ZO_CUDA(cudaMemset(c->d_v_hl, 0, sizeof(__nv_bfloat16) * prows * HLW), "memset");
-    ZO_CUDA(cudaMalloc(&c->d_c_hl, sizeof(__nv_bfloat16) * crows * HLW), "cudaMalloc(C hi/lo)");
-    ZO_CUDA(cudaMemset(c->d_c_hl, 0, sizeof(__nv_bfloat16) * crows * HLW), "memset");
-    c->proj_tc = encode_bf16_2d(&c->tm_v, c->d_v_hl, HLW, prows, HLW * 2, 64, 128) &&
-                 encode_bf16_2d(&c->tm_c, c->d_c_hl, HLW, crows, HLW * 2, 64, (uint32_t)c->r) &&
-                 encode_bf16_2d(&c->tm_p, c->d_p_hl, HLW, prows, HLW * 2, 64, 32);
-    if (!c->proj_tc) {
-      g_last_error = "cuTensorMapEncodeTiled rejected a projection descriptor; using the FMA pass";
-      c->tc_ok = false;
-    }
+  // the projection P = C V^T on the tensor cores (every tensor-core rank): V_HL, C_HL
+  const int64_t crows = (int64_t)c->n_mats * c->r;
+  ZO_CUDA(cudaMalloc(&c->d_v_hl, sizeof(__nv_bfloat16) * prows * HLW), "cudaMalloc(V hi/lo)");
+  ZO_CUDA(cudaMemset(c->d_v_hl, 0, sizeof(__nv_bfloat16) * prows * HLW), "memset");
+  ZO_CUDA(cudaMalloc(&c->d_c_hl, sizeof(__nv_bfloat16) * crows * HLW), "cudaMalloc(C hi/lo)");
+  ZO_CUDA(cudaMemset(c->d_c_hl, 0, sizeof(__nv_bfloat16) * crows * HLW), "memset");
+  c->proj_tc = zo::project_tc_supported(c->r) &&
+               encode_bf16_2d(&c->tm_v, c->d_v_hl, HLW, prows, HLW * 2, 64, 128) &&
+               encode_bf16_2d(&c->tm_c, c->d_c_hl, HLW, crows, HLW * 2, 64, (uint32_t)c->r) &&
+               encode_bf16_2d(&c->tm_p, c->d_p_hl, HLW, prows, HLW * 2, 64, 32);
+  if (!c->proj_tc) {
+    g_last_error = "cuTensorMapEncodeTiled rejected a projection descriptor; using the FMA pass";
+    c->tc_ok = false;
   }
   return ZO_OK;
 }

@@ -107,9 +107,6 @@ int64_t tc_u_operand_bytes(int32_t r, int64_t rows);
 // r >= 64: chunk-major per 128-row block, read into Tensor Memory (zo_wpass_tmem.cu).
 cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                            int32_t n_units, int32_t r, void* u_op, cudaStream_t s);
-// Pt_HL rows: hi/lo of (C V^T)^T; units = (matrix, first column) x 128 columns
-cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                                 int32_t n_units, int32_t r, __nv_bfloat16* p_hl, cudaStream_t s);
 // tm_a is used for r <= 32, u_op for r >= 64.
 cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const void* u_op, const CUtensorMap& tm_b,
                             const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
@@ -123,7 +120,7 @@ cudaError_t launch_wpass_tmem(const uint4* u_t, const CUtensorMap& tm_b,
                               int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
                               bool inject_wait, cudaStream_t s);
 
-// ---- projection P = C V^T on the tensor cores, r >= 32 (zo_project_tc.cu) ---------
+// ---- projection P = C V^T on the tensor cores, r >= 16 (zo_project_tc.cu) ---------
 bool project_tc_supported(int32_t r);
 // V_HL rows [hi | lo] of V (after a refresh); units = the projection units (matrix, first row)
 cudaError_t launch_split_v(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,

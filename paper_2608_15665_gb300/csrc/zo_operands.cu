@@ -1,8 +1,8 @@
-// Operands of the r <= 32 tensor-core weight pass (zo_wpass_tc.cu): the rows
-// [bf16 hi(x) | bf16 lo(x) | 0 ...] of U (once per refresh) and of P^T = V C^T (every pass),
-// stacked per matrix in 128-row blocks and read by TMA.  x = hi + lo with hi = bf16(x),
-// lo = bf16(x - hi).  Also the dispatch of both splits by rank (r >= 64: the chunk-major U
-// of zo_wpass_tmem.cu; the projection of zo_project_tc.cu).
+// The U operand of the r <= 32 tensor-core weight pass (zo_wpass_tc.cu): rows
+// [bf16 hi(U) | bf16 lo(U) | 0 ...], formed once per refresh, stacked per matrix in 128-row
+// blocks and read by TMA.  x = hi + lo with hi = bf16(x), lo = bf16(x - hi).  Also the
+// dispatch of the split by rank (r >= 64: the chunk-major U of zo_wpass_tmem.cu).  P^T =
+// V C^T, the other operand, comes from the tensor-core projection (zo_project_tc.cu).
 #include "zo_kernels.h"
 #include "zo_tc_common.cuh"
 
@@ -11,8 +11,8 @@ namespace {
 
 using namespace tc;
 
-// Both split kernels below (U rows and P rows, r <= 32) handle 128 consecutive rows of
-// one matrix per CTA: each thread splits one row into 16-byte chunks of hi and lo, staged
+// The split kernel below (U rows, r <= 32) handles 128 consecutive rows of one matrix
+// per CTA: each thread splits one row into 16-byte chunks of hi and lo, staged
 // in shared memory with the chunk index XOR (row & 7) so a quarter-warp's stores hit
 // distinct banks; the CTA then writes its rows, which are contiguous in the stacked
 // operand, with coalesced 16-byte stores.  Padding columns of a row stay at the zero they
@@ -57,66 +57,6 @@ split_u_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
   write_rows<R>(Os, u_hl + ((int64_t)tcm[u.x].u_row0 + i0) * hl_width(R), rows);
 }
 
-// Pt_HL[p_row0 + j] = [hi | lo] of P^T[j, :] = (C V^T)^T[j, :] = V[j, :] C^T
-template <int R>
-__global__ void __launch_bounds__(128)
-project_split_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
-                     const int2* __restrict__ units, __nv_bfloat16* __restrict__ p_hl) {
-  constexpr int kVecPerRow = hl_width(R) * 2 / 16;
-  extern __shared__ uint4 ps_smem[];
-  uint4* Os = ps_smem;                                                // 128 x kVecPerRow
-  float* Cs = reinterpret_cast<float*>(Os + 128 * kVecPerRow);        // R x R
-  const int2 u = units[blockIdx.x];
-  const MatDesc md = mats[u.x];
-  const int tid = threadIdx.x;
-  const int64_t j0 = u.y;
-  const int rows = (int)(md.n - j0 < 128 ? md.n - j0 : 128);
-  // the thread's row of V is requested before C, so both global latencies overlap
-  float v[R];
-  if (tid < rows) {
-    const float4* vrow = reinterpret_cast<const float4*>(md.V + (j0 + tid) * R);
-#pragma unroll
-    for (int b = 0; b < R / 4; ++b) {
-      const float4 t4 = vrow[b];
-      v[4 * b] = t4.x; v[4 * b + 1] = t4.y; v[4 * b + 2] = t4.z; v[4 * b + 3] = t4.w;
-    }
-  }
-  for (int e = tid; e < R * R; e += 128) Cs[e] = md.C[e];
-  __syncthreads();
-  if (tid < rows) {
-    uint4* orow = Os + tid * kVecPerRow;
-    for (int g = 0; g < R / 8; ++g) {
-      float x[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        // C row read as 16-byte broadcasts: 4 FMAs per shared-memory load
-        const float4* crow = reinterpret_cast<const float4*>(Cs + (8 * g + k) * R);
-        float acc = 0.f;
-#pragma unroll
-        for (int b4 = 0; b4 < R / 4; ++b4) {
-          const float4 c4 = crow[b4];
-          acc = fmaf(c4.x, v[4 * b4], acc);
-          acc = fmaf(c4.y, v[4 * b4 + 1], acc);
-          acc = fmaf(c4.z, v[4 * b4 + 2], acc);
-          acc = fmaf(c4.w, v[4 * b4 + 3], acc);
-        }
-        x[k] = acc;
-      }
-      uint4 hi, lo;
-      split8(x, hi, lo);
-      orow[g ^ (tid & 7)] = hi;
-      orow[(R / 8 + g) ^ (tid & 7)] = lo;
-    }
-  }
-  __syncthreads();
-  write_rows<R>(Os, p_hl + ((int64_t)tcm[u.x].p_row0 + j0) * hl_width(R), rows);
-}
-
-template <int R>
-constexpr size_t project_split_smem() {
-  return 128 * (size_t)hl_width(R) * 2 + sizeof(float) * R * R;
-}
-
 template <int R>
 cudaError_t launch_split_u_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                              int32_t n_units, __nv_bfloat16* u_hl, cudaStream_t s) {
@@ -130,19 +70,6 @@ cudaError_t launch_split_u_r(const MatDesc* d_mats, const TcMat* d_tc, const int
   return cudaGetLastError();
 }
 
-template <int R>
-cudaError_t launch_project_split_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                                   int32_t n_units, __nv_bfloat16* p_hl, cudaStream_t s) {
-  const size_t smem = project_split_smem<R>();
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(project_split_kernel<R>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-  }
-  project_split_kernel<R><<<n_units, 128, smem, s>>>(d_mats, d_tc, d_units, p_hl);
-  return cudaGetLastError();
-}
-
 }  // namespace
 
 cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
@@ -153,16 +80,6 @@ cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2*
     case 32: return launch_split_u_r<32>(d_mats, d_tc, d_units, n_units, static_cast<__nv_bfloat16*>(u_op), s);
     case 64:
     case 128: return launch_split_u_chunks(d_mats, d_tc, d_units, n_units, r, static_cast<uint4*>(u_op), s);
-    default: return cudaErrorInvalidValue;
-  }
-}
-
-cudaError_t launch_project_split(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                                 int32_t n_units, int32_t r, __nv_bfloat16* p_hl, cudaStream_t s) {
-  if (n_units <= 0) return cudaSuccess;
-  switch (r) {
-    case 16: return launch_project_split_r<16>(d_mats, d_tc, d_units, n_units, p_hl, s);
-    case 32: return launch_project_split_r<32>(d_mats, d_tc, d_units, n_units, p_hl, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -1,4 +1,4 @@
-// Projection P_i^T = V_i C_i^T on the 5th-generation tensor cores, r >= 32: the
+// Projection P_i^T = V_i C_i^T on the 5th-generation tensor cores, r >= 16: the
 // prologue of every weight pass (Eq. (4) and Eq. (10) need U_i C_i V_i^T; the weight
 // pass takes P_i = C_i V_i^T as its second operand).
 //
@@ -37,25 +37,38 @@ using namespace tc;
 
 constexpr int kProjThreads = 192;
 
+// 32 lanes x 16 consecutive 32-bit columns of Tensor Memory (the R = 16 accumulator).
+__device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&v)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+        "=r"(v[14]), "=r"(v[15])
+      : "r"(taddr));
+}
+
 template <int R>
 struct ProjCfg {
-  static_assert(R == 32 || R == 64 || R == 128,
-                "the tensor-core projection covers r = 32, 64 and 128");
-  static constexpr int kHLW = hl_width(R);                 // 2R bf16 per operand row
+  static_assert(R == 16 || R == 32 || R == 64 || R == 128,
+                "the tensor-core projection covers r = 16 ... 128");
+  static constexpr int kHLW = hl_width(R);                 // bf16 per operand row (2R, or
+                                                           // 64 with zeros past 2R at R = 16)
   static constexpr int kPanels = kHLW / 64;                // 128-byte panels per row
   static constexpr int kVBytes = kPanels * kPanelBytes;    // V tile: 128 rows
   static constexpr int kCPanelBytes = R * 128;             // C panel: R rows x 128 bytes
   static constexpr int kCBytes = kPanels * kCPanelBytes;
   static constexpr int kOutBoxBytes = 32 * 128;            // 32 rows x 64 bf16
-  // each epilogue warp stages one hi and one lo box (R = 32: one box holds both) and
+  // each epilogue warp stages one hi and one lo box (R <= 32: one box holds both) and
   // stores them 64 columns of D at a time
-  static constexpr int kWarpOutBytes = (R == 32 ? 1 : 2) * kOutBoxBytes;
+  static constexpr int kWarpOutBytes = (R <= 32 ? 1 : 2) * kOutBoxBytes;
   static constexpr int kOutBytes = 4 * kWarpOutBytes;
   static constexpr int kKC = R / 16;                       // K chunks of 16
   static constexpr int kTmemCols = 2 * R;                  // two accumulators
   // V ring: a unit's V tile is loaded while earlier units are multiplied
   static constexpr int kVStages = R == 128 ? 2 : R == 64 ? 3 : 4;
-  // R = 128: 2 x 64 + 64 + 32 KB; R = 64: 3 x 32 + 16 + 32 KB; R = 32: 4 x 16 + 4 + 16 KB
+  // R = 128: 2 x 64 + 64 + 32 KB; R = 64: 3 x 32 + 16 + 32 KB; R = 32: 4 x 16 + 4 + 16 KB;
+  // R = 16: 4 x 16 + 2 + 16 KB
   static constexpr size_t kSmem =
       (size_t)kVStages * kVBytes + kCBytes + kOutBytes + 1024 + 1024;
 };
@@ -231,21 +244,28 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
       // the previous unit's stores have finished reading this warp's boxes
       if (lane == 0) bulk_wait_read_all();
       __syncwarp();
-      if constexpr (R == 32) {
-        // one 64-wide box per row: hi at columns 8 j, lo at 32 + 8 j
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R), v);
+      if constexpr (R <= 32) {
+        // one 64-wide box per row: hi at columns 8 j, lo at R + 8 j, zeros past 2R
+        uint32_t v[R];
+        if constexpr (R == 32)
+          tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R), v);
+        else
+          tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)(acc * R), v);
         tmem_ld_wait();
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
+        for (int j = 0; j < R / 8; ++j) {
           float x[8];
 #pragma unroll
           for (int e = 0; e < 8; ++e) x[e] = __uint_as_float(v[8 * j + e]);
           uint4 hi, lo;
           split8(x, hi, lo);
           *reinterpret_cast<uint4*>(obox + lane * 128 + ((j ^ (lane & 7)) << 4)) = hi;
-          *reinterpret_cast<uint4*>(obox + lane * 128 + (((4 + j) ^ (lane & 7)) << 4)) = lo;
+          *reinterpret_cast<uint4*>(obox + lane * 128 + (((R / 8 + j) ^ (lane & 7)) << 4)) = lo;
         }
+#pragma unroll
+        for (int j = 2 * R / 8; j < 8; ++j)
+          *reinterpret_cast<uint4*>(obox + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+              make_uint4(0u, 0u, 0u, 0u);
         fence_async_smem();
         __syncwarp();
         if (lane == 0) {
@@ -311,7 +331,9 @@ template <int R, bool kC>
 __global__ void __launch_bounds__(128)
 split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
                   const int2* __restrict__ units, __nv_bfloat16* __restrict__ dst) {
-  constexpr int kVecPerRow = 2 * R * 2 / 16;
+  constexpr int kVecPerRow = 2 * R * 2 / 16;     // 16-byte chunks of [hi | lo]
+  constexpr int kSw = kVecPerRow >= 8 ? 7 : kVecPerRow - 1;   // chunk swizzle within a row
+  constexpr int kStride = hl_width(R) / 8;       // chunks per row of V_HL / C_HL
   extern __shared__ uint4 Os[];                  // 128 x kVecPerRow
   const int tid = threadIdx.x;
   int i, rows;
@@ -340,15 +362,16 @@ split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tc
       const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
       uint4 hi, lo;
       split8(x, hi, lo);
-      orow[g ^ (tid & 7)] = hi;
-      orow[(R / 8 + g) ^ (tid & 7)] = lo;
+      orow[g ^ (tid & kSw)] = hi;
+      orow[(R / 8 + g) ^ (tid & kSw)] = lo;
     }
   }
   __syncthreads();
-  uint4* d4 = reinterpret_cast<uint4*>(dst + dst_row0 * (2 * R));
+  // rows are hl_width(R) wide; at R = 16 the chunks past [hi | lo] keep their zeros
+  uint4* d4 = reinterpret_cast<uint4*>(dst + dst_row0 * hl_width(R));
   for (int e = tid; e < rows * kVecPerRow; e += 128) {
     const int row = e / kVecPerRow, c = e % kVecPerRow;
-    d4[e] = Os[row * kVecPerRow + (c ^ (row & 7))];
+    d4[row * kStride + c] = Os[row * kVecPerRow + (c ^ (row & kSw))];
   }
 }
 
@@ -380,12 +403,13 @@ cudaError_t launch_split_rows_r(const MatDesc* d_mats, const TcMat* d_tc, const 
 
 }  // namespace
 
-bool project_tc_supported(int32_t r) { return r == 32 || r == 64 || r == 128; }
+bool project_tc_supported(int32_t r) { return r == 16 || r == 32 || r == 64 || r == 128; }
 
 cudaError_t launch_split_v(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                            int32_t n_units, int32_t r, __nv_bfloat16* v_hl, cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
+    case 16: return launch_split_rows_r<16, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
     case 32: return launch_split_rows_r<32, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
     case 64: return launch_split_rows_r<64, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
     case 128: return launch_split_rows_r<128, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
@@ -397,6 +421,7 @@ cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, __n
                            cudaStream_t s) {
   if (n_mats <= 0) return cudaSuccess;
   switch (r) {
+    case 16: return launch_split_rows_r<16, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
     case 32: return launch_split_rows_r<32, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
     case 64: return launch_split_rows_r<64, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
     case 128: return launch_split_rows_r<128, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
@@ -410,6 +435,7 @@ cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
                               cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
+    case 16: return launch_project_tc_r<16>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
     case 32: return launch_project_tc_r<32>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
     case 64: return launch_project_tc_r<64>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
     case 128: return launch_project_tc_r<128>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
