@@ -73,6 +73,7 @@ FULL = [
     ("llama7b_bf16_r32", (0, 4, 6, 223)),
     ("dense32b_bf16_r64", (0, 1, 4, 6, 447)),
     ("llama7b_bf16_r128_q99", (0, 4, 6, 223)),
+    ("llama13b_bf16_r128_q99", (0, 4, 6, 279)),
 ]
 
 
@@ -144,7 +145,7 @@ def test_full_size_sampled_parity(lib, gpu, name, sample):
 # weights passing through zero are measured at the scale of the weights.  Bounds are set
 # with a margin over measured GB300 histograms (r = 8 FMA, r = 32 / 64 tensor cores):
 #   eps = 1e-3 (the paper's): 0.014% / 0.022% / 0.042% of elements differ, max 1 / 1 / 2 ulp;
-#   eps = 1e-1 (stress, the update is ~40% of |W| per pass): 0.03% / 1.7% / 2.7% differ.
+#   eps = 1e-1 (stress, the update is ~40% of |W| per pass): 0.03% / 1.7% / 2.7%, max 2 / 6 / 8.
 TRAJ = [(8, [(256, 320), (130, 72)]), (32, [(512, 384), (300, 136)]),
         (64, [(512, 264), (1030, 136)])]
 TRAJ_BOUNDS = {  # eps -> (FMA or tensor cores) -> (max fraction differing, max ulps)
