@@ -416,7 +416,8 @@ def run_ours(args):
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "traffic": TRAFFIC_BY_SOURCE.get((src, wl.name)),
-                     "kernel": {1: "wpass_fma", 2: "wpass_tc", 3: "wpass_narrow"}.get(path, "?"),
+                     "kernel": {1: "wpass_fma", 2: "wpass_tmem" if wl.r >= 64 else "wpass_tc",
+                                3: "wpass_narrow"}.get(path, "?"),
                      "algorithmic_bytes_per_launch": bytes_pass,
                      "avg_launch_ms": avg_launch_s * 1e3, "launches_timed": wpass_n},
         "clocks": clk,
