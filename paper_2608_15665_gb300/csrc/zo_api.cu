@@ -60,7 +60,7 @@ struct zo_ctx {
   // narrow tiles of the FMA path (r in {4, 8}); chosen automatically when they need at
   // most half the CTAs of the 32-row tiles
   zo::NarrowMat* d_narrow = nullptr;
-  int32_t* d_narrow_tile_mat = nullptr;   // matrix of each narrow tile
+  int4* d_narrow_tiles = nullptr;          // (matrix, first row, first chunk) of each tile
   int64_t n_narrow_tiles = 0, narrow_p = 0, narrow_u = 0;
   bool narrow_ok = false, narrow_auto = false;
   int2* d_proj_units = nullptr;
@@ -112,7 +112,7 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_mats);
   cudaFree(c->d_tile_prefix);
   cudaFree(c->d_narrow);
-  cudaFree(c->d_narrow_tile_mat);
+  cudaFree(c->d_narrow_tiles);
   cudaFree(c->d_proj_units);
   cudaFree(c->d_coeff_ws);
   cudaFree(c->d_losses);
@@ -234,7 +234,7 @@ zo_status run_weight_pass(zo_ctx* c) {
     p.r = c->r;
     zo_status st = record_start(c);
     if (st != ZO_OK) return st;
-    ZO_CUDA(zo::launch_wpass_narrow(c->d_mats, c->d_narrow, c->d_narrow_tile_mat,
+    ZO_CUDA(zo::launch_wpass_narrow(c->d_mats, c->d_narrow, c->d_narrow_tiles,
                                     c->n_narrow_tiles, p, c->narrow_p, c->narrow_u, c->stream),
             "narrow-tile weight-pass kernel");
     c->last_path = 3;
@@ -319,18 +319,25 @@ zo_status setup_narrow(zo_ctx* c, const zo_matrix* mats) {
   }
   c->n_narrow_tiles = tiles;
   if (tiles > 0x7FFFFFFF) return ZO_OK;   // beyond one grid: the 32-row tiles only
-  std::vector<int32_t> tile_mat((size_t)tiles);
+  std::vector<int4> tab((size_t)tiles);
   for (int32_t i = 0; i < c->n_mats; ++i) {
+    const int64_t vec = mats[i].dtype == ZO_BF16 ? 8 : 4;
+    const int64_t cpr = (mats[i].n + vec - 1) / vec;
+    if (mats[i].m > 0x7FFFFFFF || cpr > 0x7FFFFFFF) return ZO_OK;   // rows, chunks as int
+    const int64_t tiles_c = (cpr + nm[i].chunks - 1) / nm[i].chunks;
     const int64_t end = i + 1 < c->n_mats ? nm[i + 1].tile0 : tiles;
-    for (int64_t t = nm[i].tile0; t < end; ++t) tile_mat[(size_t)t] = i;
+    for (int64_t t = nm[i].tile0; t < end; ++t) {
+      const int64_t local = t - nm[i].tile0;
+      tab[(size_t)t] = make_int4(i, (int)((local / tiles_c) * nm[i].rows),
+                                 (int)((local % tiles_c) * nm[i].chunks), 0);
+    }
   }
   cudaError_t e = cudaMalloc(&c->d_narrow, sizeof(zo::NarrowMat) * c->n_mats);
-  if (e == cudaSuccess) e = cudaMalloc(&c->d_narrow_tile_mat, sizeof(int32_t) * std::max<int64_t>(tiles, 1));
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_narrow_tiles, sizeof(int4) * std::max<int64_t>(tiles, 1));
   if (e == cudaSuccess)
     e = cudaMemcpy(c->d_narrow, nm.data(), sizeof(zo::NarrowMat) * c->n_mats, cudaMemcpyHostToDevice);
   if (e == cudaSuccess && tiles > 0)
-    e = cudaMemcpy(c->d_narrow_tile_mat, tile_mat.data(), sizeof(int32_t) * tiles,
-                   cudaMemcpyHostToDevice);
+    e = cudaMemcpy(c->d_narrow_tiles, tab.data(), sizeof(int4) * tiles, cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     cuda_fail(e, "narrow-tile table");
     return e == cudaErrorMemoryAllocation ? ZO_ERR_NOMEM : ZO_ERR_CUDA;
@@ -705,7 +712,7 @@ zo_status zo_perturb(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t qb, fl
   if (!use_tc && narrow_path(c)) {
     zo_status st = record_start(c);
     if (st != ZO_OK) return st;
-    ZO_CUDA(zo::launch_wpass_narrow(c->d_mats, c->d_narrow, c->d_narrow_tile_mat,
+    ZO_CUDA(zo::launch_wpass_narrow(c->d_mats, c->d_narrow, c->d_narrow_tiles,
                                     c->n_narrow_tiles, p, c->narrow_p, c->narrow_u, c->stream),
             "narrow-tile weight-pass kernel");
     c->last_path = 3;

@@ -82,10 +82,10 @@ void narrow_tile_shape(int64_t m, int64_t n, int32_t dtype, int32_t* rows, int32
 // Shared-memory floats of the P and U parts of one tile of this shape.
 int64_t narrow_p_floats(int32_t r, int32_t chunks, int32_t dtype);
 int64_t narrow_u_floats(int32_t r, int32_t rows);
-// d_tile_mat[t]: the matrix of tile t; p_floats / u_floats: the largest P and U parts over
-// the set's tiles.
+// d_tiles[t] = (matrix, first row, first 16-byte chunk, 0) of tile t; p_floats / u_floats:
+// the largest P and U parts over the set's tiles.
 cudaError_t launch_wpass_narrow(const MatDesc* d_mats, const NarrowMat* d_narrow,
-                                const int32_t* d_tile_mat, int64_t n_tiles, const CoeffParams& p,
+                                const int4* d_tiles, int64_t n_tiles, const CoeffParams& p,
                                 int64_t p_floats, int64_t u_floats, cudaStream_t s);
 
 // ---- full-space SPSA perturbation of Eq. (1) (zo_mezo.cu) -------------------------

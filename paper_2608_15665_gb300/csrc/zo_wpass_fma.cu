@@ -298,17 +298,14 @@ __device__ __forceinline__ void split_cell(int f, int chunks, float inv, int& rl
 }
 
 template <int R, typename T, bool kDraw>
-__device__ __forceinline__ void narrow_tile(const MatDesc& md, const NarrowMat& g, int64_t local,
-                                            const CoeffParams& p, float* Cs, float* Ps,
-                                            float* Us) {
+__device__ __forceinline__ void narrow_tile(const MatDesc& md, const NarrowMat& g, int64_t row0,
+                                            int64_t ch0, const CoeffParams& p, float* Cs,
+                                            float* Ps, float* Us) {
   constexpr int VEC = Vec<T>::N;
   const int tid = threadIdx.x;
   const int rows = g.rows, chunks = g.chunks, cols = chunks * VEC, cells = rows * chunks;
   const float inv = __frcp_rn((float)chunks);
   const int64_t cpr = (md.n + VEC - 1) / VEC;   // chunks per row of W
-  const int64_t tiles_c = (cpr + chunks - 1) / chunks;
-  const int64_t row0 = (local / tiles_c) * rows;
-  const int64_t ch0 = (local % tiles_c) * chunks;
   const int64_t col0 = ch0 * VEC;
   const int row_end = (int)min64(rows, md.m - row0);     // live rows of the tile
   const int ch_end = (int)min64(chunks, cpr - ch0);       // live chunks of the tile
@@ -427,24 +424,24 @@ __device__ __forceinline__ void narrow_tile(const MatDesc& md, const NarrowMat& 
 template <int R, bool kDraw>
 __global__ void __launch_bounds__(kNarrowThreads, R <= 4 ? 4 : 3)
 wpass_narrow_kernel(const MatDesc* __restrict__ mats, const NarrowMat* __restrict__ narrow,
-                    const int32_t* __restrict__ tile_mat, CoeffParams p, int32_t p_floats) {
+                    const int4* __restrict__ tiles, CoeffParams p, int32_t p_floats) {
   extern __shared__ float4 smem4[];
   float* Cs = reinterpret_cast<float*>(smem4);
   float* Ps = Cs + R * R;
   float* Us = Ps + p_floats;
-  const int i = __ldg(tile_mat + blockIdx.x);
-  const MatDesc md = mats[i];
-  const NarrowMat g = narrow[i];
-  const int64_t local = (int64_t)blockIdx.x - g.tile0;
+  // (matrix, first row, first chunk) of this tile, laid out by the host
+  const int4 td = __ldg(tiles + blockIdx.x);
+  const MatDesc md = mats[td.x];
+  const NarrowMat g = narrow[td.x];
   if (md.dtype == 1)
-    narrow_tile<R, __nv_bfloat16, kDraw>(md, g, local, p, Cs, Ps, Us);
+    narrow_tile<R, __nv_bfloat16, kDraw>(md, g, td.y, td.z, p, Cs, Ps, Us);
   else
-    narrow_tile<R, float, kDraw>(md, g, local, p, Cs, Ps, Us);
+    narrow_tile<R, float, kDraw>(md, g, td.y, td.z, p, Cs, Ps, Us);
 }
 
 template <int R, bool kDraw>
 cudaError_t launch_narrow_r(const MatDesc* d_mats, const NarrowMat* d_narrow,
-                            const int32_t* d_tile_mat, int64_t n_tiles, const CoeffParams& p,
+                            const int4* d_tiles, int64_t n_tiles, const CoeffParams& p,
                             int64_t p_floats, int64_t u_floats, cudaStream_t s) {
   const size_t smem = sizeof(float) * (size_t)(R * R + p_floats + u_floats);
   static bool configured = false;
@@ -458,7 +455,7 @@ cudaError_t launch_narrow_r(const MatDesc* d_mats, const NarrowMat* d_narrow,
     configured = true;
   }
   wpass_narrow_kernel<R, kDraw><<<(unsigned)n_tiles, kNarrowThreads, smem, s>>>(
-      d_mats, d_narrow, d_tile_mat, p, (int32_t)p_floats);
+      d_mats, d_narrow, d_tiles, p, (int32_t)p_floats);
   return cudaGetLastError();
 }
 }  // namespace
@@ -497,7 +494,7 @@ int64_t narrow_p_floats(int32_t r, int32_t chunks, int32_t dtype) {
 int64_t narrow_u_floats(int32_t r, int32_t rows) { return (int64_t)r * rows; }
 
 cudaError_t launch_wpass_narrow(const MatDesc* d_mats, const NarrowMat* d_narrow,
-                                const int32_t* d_tile_mat, int64_t n_tiles, const CoeffParams& p,
+                                const int4* d_tiles, int64_t n_tiles, const CoeffParams& p,
                                 int64_t p_floats, int64_t u_floats, cudaStream_t s) {
   if (n_tiles <= 0) return cudaSuccess;
   if (n_tiles > 0x7FFFFFFF || p_floats < 0 || u_floats < 0 ||
@@ -506,11 +503,11 @@ cudaError_t launch_wpass_narrow(const MatDesc* d_mats, const NarrowMat* d_narrow
   const bool draw = p.mode == kCoeffPerturb;
   switch (p.r) {
     case 4:
-      return draw ? launch_narrow_r<4, true>(d_mats, d_narrow, d_tile_mat, n_tiles, p, p_floats, u_floats, s)
-                  : launch_narrow_r<4, false>(d_mats, d_narrow, d_tile_mat, n_tiles, p, p_floats, u_floats, s);
+      return draw ? launch_narrow_r<4, true>(d_mats, d_narrow, d_tiles, n_tiles, p, p_floats, u_floats, s)
+                  : launch_narrow_r<4, false>(d_mats, d_narrow, d_tiles, n_tiles, p, p_floats, u_floats, s);
     case 8:
-      return draw ? launch_narrow_r<8, true>(d_mats, d_narrow, d_tile_mat, n_tiles, p, p_floats, u_floats, s)
-                  : launch_narrow_r<8, false>(d_mats, d_narrow, d_tile_mat, n_tiles, p, p_floats, u_floats, s);
+      return draw ? launch_narrow_r<8, true>(d_mats, d_narrow, d_tiles, n_tiles, p, p_floats, u_floats, s)
+                  : launch_narrow_r<8, false>(d_mats, d_narrow, d_tiles, n_tiles, p, p_floats, u_floats, s);
     default: return cudaErrorInvalidValue;
   }
 }
