@@ -9,6 +9,7 @@
 // a row), U and P tiles are staged through shared memory.  HBM traffic per
 // element is one read and one write of W; U and P tiles come from L2.
 #include <algorithm>
+#include <atomic>
 
 #include "zo_kernels.h"
 
@@ -245,17 +246,27 @@ wpass_fma_fused_kernel(const MatDesc* __restrict__ mats, int n_mats,
     wpass_tile<R, float, true>(md, local, Us, Ps, Cs);
 }
 
+// The dynamic shared-memory limit of a kernel belongs to each device's context: raise it
+// once per device (bit d of `done`), before the kernel's first launch there.
+template <typename Kernel>
+cudaError_t allow_smem(Kernel kernel, int bytes, std::atomic<uint64_t>& done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = dev < 64 ? (uint64_t)1 << dev : 0;
+  if (bit && (done.load(std::memory_order_relaxed) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) done.fetch_or(bit, std::memory_order_relaxed);
+  return e;
+}
+
 template <int R>
 cudaError_t launch_r(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_prefix,
                      int64_t n_tiles, cudaStream_t s) {
   const size_t smem = sizeof(float) * (size_t)(kRows * R + R * 256);
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(wpass_fma_kernel<R>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static std::atomic<uint64_t> done{0};
+  cudaError_t e = allow_smem(wpass_fma_kernel<R>, (int)smem, done);
+  if (e != cudaSuccess) return e;
   wpass_fma_kernel<R><<<(unsigned)n_tiles, 256, smem, s>>>(d_mats, n_mats, d_prefix);
   return cudaGetLastError();
 }
@@ -444,16 +455,12 @@ cudaError_t launch_narrow_r(const MatDesc* d_mats, const NarrowMat* d_narrow,
                             const int4* d_tiles, int64_t n_tiles, const CoeffParams& p,
                             int64_t p_floats, int64_t u_floats, cudaStream_t s) {
   const size_t smem = sizeof(float) * (size_t)(R * R + p_floats + u_floats);
-  static bool configured = false;
-  if (!configured) {
-    // the largest shape narrow_tile_shape can give: kNarrowMaxCols P columns, or
-    // kNarrowChunks rows of U
-    const int most = (int)(sizeof(float) * (R * R + R * kNarrowMaxCols + R * kNarrowChunks));
-    cudaError_t e = cudaFuncSetAttribute(wpass_narrow_kernel<R, kDraw>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, most);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  // the largest shape narrow_tile_shape can give: kNarrowMaxCols P columns, or
+  // kNarrowChunks rows of U
+  static std::atomic<uint64_t> done{0};
+  const int most = (int)(sizeof(float) * (R * R + R * kNarrowMaxCols + R * kNarrowChunks));
+  cudaError_t e = allow_smem(wpass_narrow_kernel<R, kDraw>, most, done);
+  if (e != cudaSuccess) return e;
   wpass_narrow_kernel<R, kDraw><<<(unsigned)n_tiles, kNarrowThreads, smem, s>>>(
       d_mats, d_narrow, d_tiles, p, (int32_t)p_floats);
   return cudaGetLastError();
