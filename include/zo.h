@@ -24,6 +24,8 @@
  *   passed as void*; NULL = legacy default stream).  Arguments are validated on the
  *   host before anything is launched; a rejected call launches nothing and
  *   leaves all buffers untouched.
+ * - A context belongs to the device that was current at zo_create; each call on it
+ *   makes that device current for its duration and restores the caller's device.
  * - Kernels that detect a problem at run time (an mbarrier wait that ran out of
  *   iterations, an internal bound check) write a code to a device status word;
  *   zo_sync_status() synchronises the stream and returns and clears it.

@@ -46,6 +46,25 @@ struct QrLevel {
 
 void zo::set_last_error(const char* msg) { g_last_error = msg; }
 
+namespace {
+
+// Makes a context's device current for the length of a call and gives the caller's back:
+// every kernel of a context runs on the device it was created on, whatever device the
+// calling thread has selected since.
+struct DeviceGuard {
+  int prev = -1;
+  bool switched = false;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev && cudaSetDevice(dev) == cudaSuccess)
+      switched = true;
+  }
+  ~DeviceGuard() {
+    if (switched) cudaSetDevice(prev);
+  }
+};
+
+}  // namespace
+
 
 struct zo_ctx {
   int device = 0;
@@ -637,6 +656,7 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
 
 zo_status zo_destroy(zo_ctx* c) {
   if (!c) return ZO_OK;
+  DeviceGuard guard(c->device);
   cudaError_t e = cudaStreamSynchronize(c->stream);
   free_ctx(c);
   if (e != cudaSuccess) return cuda_fail(e, "zo_destroy");
@@ -645,6 +665,7 @@ zo_status zo_destroy(zo_ctx* c) {
 
 zo_status zo_refresh(zo_ctx* c, uint32_t refresh_idx, int32_t reset_moments) {
   if (!c) return ZO_ERR_INVALID_ARG;
+  DeviceGuard guard(c->device);
   const int n_levels = (int)c->up_off.size();
   for (int lv = 0; lv < n_levels; ++lv) {
     if (c->up_cnt[lv] == 0) continue;
@@ -692,6 +713,7 @@ zo_status zo_init_subspace(zo_ctx* c, uint32_t refresh_idx) {
 
 zo_status zo_perturb(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t qb, float cb, float eps) {
   if (!c) return ZO_ERR_INVALID_ARG;
+  DeviceGuard guard(c->device);
   if (qa < 0 || qa >= c->q || qb < -1 || qb >= c->q || !std::isfinite(ca) || !std::isfinite(cb) ||
       !std::isfinite(eps)) {
     g_last_error = "zo_perturb: query index out of range or non-finite scalar";
@@ -742,6 +764,7 @@ zo_status zo_step(zo_ctx* c, uint32_t t, int32_t adam_t, const float* losses, in
                   float beta1, float beta2, float eps_adam, int32_t restore_query,
                   float restore_coef, float* gamma_out) {
   if (!c || !losses) return ZO_ERR_INVALID_ARG;
+  DeviceGuard guard(c->device);
   int32_t want = -1;
   if (scheme == ZO_SCHEME_CENTRAL) want = 2 * c->q;
   else if (scheme == ZO_SCHEME_FORWARD) want = c->q + 1;
@@ -803,6 +826,7 @@ zo_status zo_step(zo_ctx* c, uint32_t t, int32_t adam_t, const float* losses, in
 
 zo_status zo_mezo_perturb(zo_ctx* c, uint32_t t, float coef) {
   if (!c) return ZO_ERR_INVALID_ARG;
+  DeviceGuard guard(c->device);
   if (!std::isfinite(coef)) {
     g_last_error = "zo_mezo_perturb: non-finite coefficient";
     return ZO_ERR_INVALID_ARG;
@@ -824,6 +848,7 @@ zo_status zo_mezo_perturb(zo_ctx* c, uint32_t t, float coef) {
 
 zo_status zo_sync_status(zo_ctx* c) {
   if (!c) return ZO_ERR_INVALID_ARG;
+  DeviceGuard guard(c->device);
   ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
   uint32_t s = 0;
   ZO_CUDA(cudaMemcpy(&s, c->d_status, sizeof(s), cudaMemcpyDeviceToHost), "read status");
@@ -843,6 +868,7 @@ zo_status zo_sync_status(zo_ctx* c) {
 
 zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
   if (!c) return ZO_ERR_INVALID_ARG;
+  DeviceGuard guard(c->device);
   if (option == ZO_OPTION_WPASS_PATH) {
     if (value < 0 || value > 3) return ZO_ERR_INVALID_ARG;
     if (value == 2 && !c->tc_ok) {
@@ -879,6 +905,7 @@ zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
 
 zo_status zo_get_timing(zo_ctx* c, double* total_ms, int64_t* launches) {
   if (!c || !total_ms || !launches) return ZO_ERR_INVALID_ARG;
+  DeviceGuard guard(c->device);
   ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
   for (size_t k = 0; k < c->ev_used; ++k) {
     float ms = 0.f;
