@@ -3,8 +3,8 @@
 // "W_i <- W_i + eps U_i Z_i V_i^T", Eq. (4), and of the update of Eq. (10)).
 // This file holds the kernel for r <= 32 (both operands in shared memory) and the
 // dispatch by rank; the r >= 64 kernel, which reads U from Tensor Memory, is in
-// zo_wpass_tmem.cu; the operands are prepared in zo_operands.cu (r <= 32) and
-// zo_project_tc.cu / zo_wpass_tmem.cu (r >= 64).
+// zo_wpass_tmem.cu; the U operand is prepared in zo_operands.cu (r <= 32) or
+// zo_wpass_tmem.cu (r >= 64), the P operand by zo_project_tc.cu.
 //
 // The contraction U (128 x r) . P (r x 128) of a 128 x 128 tile is r-deep, so it
 // costs 2r flops per weight against 4 bytes of HBM traffic; past r = 16 that is
