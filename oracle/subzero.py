@@ -2,6 +2,8 @@
 
 Plain fp64 restatement of Sec. 4 of the paper:
 
+* ``perturbed_linear`` -- one linear layer of the loss evaluation of Alg. 3 at the
+  perturbed weights, Y = X (W + U C V^T)^T, with W left as it is.
 * ``perturb_coeff`` / ``apply_pass`` -- Alg. 2 (the in-place perturbation) and Eq. (4):
   W_i <- W_i + eps U_i Z_i V_i^T.  Consecutive updates that touch W with no
   loss evaluation in between (restore of query k, perturbation of query k+1,
@@ -60,6 +62,17 @@ def apply_pass(W, dtype, U, V, C, rows=None):
     W = np.asarray(W, np.float64)
     Uu = np.asarray(U, np.float64) if rows is None else np.asarray(U, np.float64)[rows]
     return rounding.round_to(W + delta(Uu, V, C), dtype)
+
+
+def perturbed_linear(X, W, U, V, C, dtype="bf16"):
+    """Y = X (W + U C V^T)^T: a linear layer y = W' x (nn.Linear's W, out x in) applied to
+    the rows of X at the perturbed weights W' = W + U C V^T at which Alg. 3 evaluates the
+    loss, without W' being written anywhere.  Exact in fp64, rounded once to ``dtype``.
+    (The weight-pass form evaluates the same layer at rnd(W + U C V^T), a weight already
+    rounded to W's storage type.)"""
+    X = np.asarray(X, np.float64)
+    Wp = np.asarray(W, np.float64) + delta(U, V, C)
+    return rounding.round_to(X @ Wp.T, dtype)
 
 
 # ----------------------------------------------------------------------------
