@@ -86,7 +86,9 @@ enum {
 
 /* Options for zo_set_option. */
 enum {
-  ZO_OPTION_WPASS_PATH = 0, /* 0 = automatic: tcgen05 when every W is bf16 and r >= 16;
+  ZO_OPTION_WPASS_PATH = 0, /* 0 = automatic: tcgen05 when every W is bf16 with n a
+                                   multiple of 8 (its TMA stores write 16-byte chunks) and
+                                   r >= 16;
                                    else, at r in {4, 8}, the narrow-tile FMA pass when its
                                    tiles number at most half of the 32-row tiles (sets of
                                    thin matrices such as LoRA factors); else the FMA pass,
@@ -198,6 +200,25 @@ ZO_API zo_status zo_step(zo_ctx* ctx, uint32_t t, int32_t adam_t, const float* l
  * ZO_OPTION_TIMING is on.
  */
 ZO_API zo_status zo_mezo_perturb(zo_ctx* ctx, uint32_t t, float coef);
+
+/*
+ * zo_linear_perturbed -- one linear layer of a loss evaluation at the perturbed weights
+ * (Alg. 3's forward at W_i' = W_i + U_i C V_i^T, Eq. (4) form) WITHOUT a weight pass:
+ *   Y = X (W_i + U_i C V_i^T)^T = X W_i^T + (X V_i C^T) U_i^T,
+ *   C = eps (ca Z_i^(qa) + cb Z_i^(qb)) at step t (qb = -1: one term) -- the coefficient
+ *   that zo_perturb(ctx, t, qa, ca, qb, cb, eps) would add to W_i.
+ * W_i is read, never written.  X: T x n_i bf16, row stride ldx elements; Y: T x m_i bf16,
+ * row stride ldy (both device, caller-owned, 16-byte aligned, strides multiples of 8;
+ * m_i a multiple of 8, else ZO_ERR_SHAPE).
+ * The dense product is exact in bf16 with fp32 accumulation; the rank-r term carries
+ * the bf16 hi/lo split's ~2^-16 relative error; Y is rounded to bf16 once.  Needs the
+ * tensor-core path (every W bf16) with r in {16, 32}; otherwise ZO_ERR_UNSUPPORTED.
+ * Overwrites the context's C_i / P_i workspace of matrix i (the next zo_perturb or
+ * zo_step forms its own).  Asynchronous; device errors go to the status word.
+ */
+ZO_API zo_status zo_linear_perturbed(zo_ctx* ctx, int32_t i, const void* X, int64_t T,
+                                     int64_t ldx, void* Y, int64_t ldy, uint32_t t,
+                                     int32_t qa, float ca, int32_t qb, float cb, float eps);
 
 /* zo_sync_status -- synchronise the stream; return (and clear) the device status word. */
 ZO_API zo_status zo_sync_status(zo_ctx* ctx);

@@ -109,6 +109,13 @@ struct zo_ctx {
                                      // (rows [hi | lo | 0] for r <= 32, chunk-major for r >= 64)
   __nv_bfloat16* d_p_hl = nullptr;   // stacked [hi | lo] rows of every P_i^T, 128-row padded
   zo::TcMat* d_tc = nullptr;
+  std::vector<zo::TcMat> h_tc;       // host copy (operand rows of each matrix)
+  std::vector<int32_t> h_unit0;      // first projection unit of each matrix
+  // zo_linear_perturbed's workspace: P_K ([P_hi ; P_lo] rows, K-major) and S_HL
+  __nv_bfloat16* d_pk = nullptr;
+  int64_t pk_ld = 0;
+  __nv_bfloat16* d_s_hl = nullptr;
+  int64_t s_cap = 0;
   int64_t tc_tiles = 0;
   CUtensorMap* d_w_maps = nullptr;   // one TMA descriptor per W_i (device memory)
   CUtensorMap tm_a{}, tm_b{};        // descriptors of the stacked operands (kernel parameters)
@@ -145,6 +152,8 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_u_op);
   cudaFree(c->d_p_hl);
   cudaFree(c->d_tc);
+  cudaFree(c->d_pk);
+  cudaFree(c->d_s_hl);
   cudaFree(c->d_w_maps);
   cudaFree(c->d_u_units);
   cudaFree(c->d_v_hl);
@@ -368,11 +377,13 @@ zo_status setup_narrow(zo_ctx* c, const zo_matrix* mats) {
 }
 
 // Buffers and descriptors of the tensor-core weight pass; leaves tc_ok false when
-// the context does not qualify (an fp32 matrix, or r outside {16, 32, 64}).
+// the context does not qualify: an fp32 matrix, r outside {16, 32, 64, 128}, or a
+// width n not a multiple of 8 -- TMA stores write whole 16-byte chunks, and the chunk
+// that holds a row's last element would also overwrite the caller's elements past n.
 zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
   if (!zo::wpass_tc_supported(c->r)) return ZO_OK;
   for (int32_t i = 0; i < c->n_mats; ++i)
-    if (mats[i].dtype != ZO_BF16) return ZO_OK;
+    if (mats[i].dtype != ZO_BF16 || mats[i].n % 8 != 0) return ZO_OK;
   const int64_t BM = zo::tc_tile_rows(), BN = zo::tc_tile_cols();
   const int64_t HLW = zo::tc_hl_width(c->r);
   std::vector<zo::TcMat> tc(c->n_mats);
@@ -393,6 +404,7 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
     for (int64_t r0 = 0; r0 < m; r0 += 128) uunits.push_back(make_int2(i, (int)r0));
   }
   if (urows >= (int64_t(1) << 31) || prows >= (int64_t(1) << 31)) return ZO_OK;
+  c->h_tc = tc;
   ZO_CUDA(cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, c->device), "SM count");
   const int64_t u_bytes = zo::tc_u_operand_bytes(c->r, urows);
   ZO_CUDA(cudaMalloc(&c->d_u_op, u_bytes), "cudaMalloc(U hi/lo)");
@@ -543,6 +555,7 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
     const int64_t tiles = ((mt.m + zo::kFmaTileRows - 1) / zo::kFmaTileRows) * ((mt.n + tn - 1) / tn);
     d.tile0 = prefix[i];
     prefix[i + 1] = prefix[i] + tiles;
+    c->h_unit0.push_back((int32_t)units.size());
     for (int64_t j0 = 0; j0 < mt.n; j0 += 128) units.push_back(make_int2(i, (int)j0));
     c->h_mats[i] = d;
   }
@@ -824,6 +837,95 @@ zo_status zo_step(zo_ctx* c, uint32_t t, int32_t adam_t, const float* losses, in
   return run_weight_pass(c);
 }
 
+zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, int64_t ldx,
+                              void* Y, int64_t ldy, uint32_t t, int32_t qa, float ca,
+                              int32_t qb, float cb, float eps) {
+  if (!c || !X || !Y) return ZO_ERR_INVALID_ARG;
+  DeviceGuard guard(c->device);
+  if (!c->tc_ok || !zo::linear_supported(c->r)) {
+    g_last_error = "zo_linear_perturbed needs the tensor-core path with r in {16, 32}";
+    return ZO_ERR_UNSUPPORTED;
+  }
+  if (mat < 0 || mat >= c->n_mats || qa < 0 || qa >= c->q || qb < -1 || qb >= c->q ||
+      !std::isfinite(ca) || !std::isfinite(cb) || !std::isfinite(eps)) {
+    g_last_error = "zo_linear_perturbed: matrix or query index out of range, or non-finite scalar";
+    return ZO_ERR_INVALID_ARG;
+  }
+  const zo::MatDesc& md = c->h_mats[mat];
+  const int64_t m = md.m, n = md.n;
+  if (T < 1 || T >= (int64_t(1) << 31) || ldx < n || ldy < m || m % 8 != 0) {
+    // (Y's rows are written by TMA in 16-byte chunks: m % 8 keeps them inside Y's columns)
+    g_last_error = "zo_linear_perturbed: need 1 <= T < 2^31, ldx >= n, ldy >= m, m % 8 == 0";
+    return ZO_ERR_SHAPE;
+  }
+  if (!aligned16(X) || !aligned16(Y) || (ldx * 2) % 16 != 0 || (ldy * 2) % 16 != 0) {
+    g_last_error = "zo_linear_perturbed: X, Y and their row strides must be 16-byte aligned";
+    return ZO_ERR_ALIGN;
+  }
+  const int32_t r = c->r;
+  const int64_t HLW = zo::tc_hl_width(r);
+  // workspace: P_K (2r x pk_ld) for the widest matrix, S_HL (T rows of 64)
+  if (!c->d_pk) {
+    int64_t nmax = 0;
+    for (const auto& d : c->h_mats) nmax = std::max(nmax, d.n);
+    c->pk_ld = (nmax + 63) / 64 * 64;
+    ZO_CUDA(cudaMalloc(&c->d_pk, sizeof(__nv_bfloat16) * 2 * r * c->pk_ld), "cudaMalloc(P_K)");
+  }
+  if (T > c->s_cap) {
+    ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
+    cudaFree(c->d_s_hl);
+    c->d_s_hl = nullptr;
+    c->s_cap = 0;
+    const int64_t cap = (T + 127) / 128 * 128;
+    ZO_CUDA(cudaMalloc(&c->d_s_hl, sizeof(__nv_bfloat16) * cap * HLW), "cudaMalloc(S_HL)");
+    c->s_cap = cap;
+  }
+  CUtensorMap tm_x{}, tm_pk{}, tm_s_st{}, tm_s_ld{}, tm_y{};
+  const bool enc =
+      encode_bf16_2d(&tm_x, const_cast<void*>(X), n, T, ldx * 2, 64, 128) &&
+      encode_bf16_2d(&tm_pk, c->d_pk, n, 2 * r, c->pk_ld * 2, 64, (uint32_t)(2 * r)) &&
+      encode_bf16_2d(&tm_s_st, c->d_s_hl, HLW, T, HLW * 2, 64, 32) &&
+      encode_bf16_2d(&tm_s_ld, c->d_s_hl, HLW, T, HLW * 2, 64, 128) &&
+      encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 64, 32);
+  if (!enc) {
+    g_last_error = "zo_linear_perturbed: cuTensorMapEncodeTiled rejected a descriptor";
+    return ZO_ERR_CUDA;
+  }
+  // C_i = eps (ca Z_qa + cb Z_qb), the coefficient zo_perturb would apply; P_i = C_i V_i^T
+  zo::CoeffParams p{};
+  p.mode = zo::kCoeffPerturb;
+  p.seed = c->seed;
+  p.t = t;
+  p.r = r;
+  p.q = c->q;
+  p.qa = qa;
+  p.qb = qb;
+  p.ca = ca;
+  p.cb = cb;
+  p.eps = eps;
+  ZO_CUDA(zo::launch_coeff(c->d_mats + mat, 1, p, c->stream), "coefficient kernel");
+  ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, r, c->d_c_hl, c->stream), "split C");
+  const int32_t unit0 = c->h_unit0[mat];
+  const int32_t n_units = (int32_t)((n + 127) / 128);
+  ZO_CUDA(zo::launch_project_tc(c->tm_v, c->tm_c, c->tm_p, c->d_tc, c->d_proj_units + unit0,
+                                n_units, std::min<int32_t>(n_units, c->sms), r, c->d_status,
+                                c->stream),
+          "tensor-core projection kernel");
+  ZO_CUDA(zo::launch_transpose_p(c->d_p_hl, c->h_tc[mat].p_row0, (int32_t)HLW, n, r, c->d_pk,
+                                 c->pk_ld, c->stream),
+          "P transpose");
+  // S = X P^T, then Y = X W^T + S U^T
+  const int32_t gs = std::min<int32_t>(zo::linear_tiles(T, 2 * r, true, r), c->sms);
+  ZO_CUDA(zo::launch_linear_s(tm_x, tm_pk, tm_s_st, T, n, r, gs, c->d_status, c->stream),
+          "S = X P^T kernel");
+  const int32_t gy = std::min<int32_t>(zo::linear_tiles(T, m, false, r), c->sms);
+  ZO_CUDA(zo::launch_linear_y(tm_x, c->d_w_maps + mat, tm_s_ld, c->tm_a, tm_y, T, m, n,
+                              c->h_tc[mat].u_row0, r, gy, c->d_status, c->stream),
+          "perturbed linear kernel");
+  c->launches += 6;
+  return ZO_OK;
+}
+
 zo_status zo_mezo_perturb(zo_ctx* c, uint32_t t, float coef) {
   if (!c) return ZO_ERR_INVALID_ARG;
   DeviceGuard guard(c->device);
@@ -872,7 +974,8 @@ zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
   if (option == ZO_OPTION_WPASS_PATH) {
     if (value < 0 || value > 3) return ZO_ERR_INVALID_ARG;
     if (value == 2 && !c->tc_ok) {
-      g_last_error = "the tensor-core weight pass needs every W in bf16 and r in {16, 32, 64, 128}";
+      g_last_error = "the tensor-core weight pass needs every W in bf16 with n a multiple of 8, "
+                     "and r in {16, 32, 64, 128}";
       return ZO_ERR_UNSUPPORTED;
     }
     if (value == 3 && !c->narrow_ok) {

@@ -1,0 +1,137 @@
+"""A linear layer at the perturbed weights without a weight pass (zo_linear_perturbed)
+against the oracle: Y = X (W + U C V^T)^T with C = eps (ca Z_qa + cb Z_qb), W untouched.
+
+The GPU sums X W^T in fp32 from exact bf16 products, adds the rank-r term S U^T with the
+bf16 hi/lo split, and rounds Y to bf16 once; the oracle rounds the fp64 value once.  The
+two differ by at most one bf16 ulp of the output plus the fp32 accumulation bound
+(n 2^-24 sum |X||W|), the split's 2^-14 of sum |X||V||C||U| and the fp32 Gaussians'
+allowance (tests/parity.py NORMAL_ABS) carried through |X||V| and |U|.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from gpu_util import f32, make_weight, snapshot
+from oracle import rounding, subzero
+from parity import NORMAL_ABS, to_f64
+
+pytestmark = pytest.mark.gpu
+
+# (r, [(m, n, ldw)], token counts)
+LINEAR_CASES = {
+    "r32": (32, [(304, 520, None), (264, 2048, None), (1032, 72, 80)], (1, 130, 300)),
+    "r16": (16, [(304, 520, 528), (136, 1000, 1008), (64, 136, None)], (7, 257)),
+}
+
+
+def _context(gpu, case, seed, base=31):
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    r, spec, _ = LINEAR_CASES[case]
+    weights = [make_weight(m, n, "bf16", 700 + k, gpu, ldw) for k, (m, n, ldw) in enumerate(spec)]
+    z = SubZeroPlus(weights, r, 4, seed, matrix_index_base=base)
+    z.init_subspace(0)
+    return z, base
+
+
+def _tokens(T, n, seed, gpu):
+    g = torch.Generator().manual_seed(seed)
+    return torch.randn(T, n, generator=g).to(torch.bfloat16).to(gpu)
+
+
+def _check(Y, X, W, U, V, C, zc, what):
+    Xd, Wd = to_f64(X), np.asarray(W, np.float64)
+    want = subzero.perturbed_linear(Xd, Wd, U, V, C, "bf16")
+    got = to_f64(Y)
+    aX = np.abs(Xd)
+    a_w = aX @ np.abs(Wd).T
+    a_s = aX @ (np.abs(V) @ np.abs(C).T) @ np.abs(U).T
+    a_z = zc * NORMAL_ABS * np.outer(aX @ np.abs(V).sum(axis=1), np.abs(U).sum(axis=1))
+    n = Wd.shape[1]
+    tol = (rounding.bf16_ulp(np.maximum(np.abs(want), np.abs(got)))
+           + 2.0 * (n * 2.0 ** -24 * a_w + 2.0 ** -14 * a_s + a_z))
+    d = np.abs(got - want)
+    bad = d > tol
+    assert not bad.any(), (f"{what}: {int(bad.sum())} of {d.size} outside the bound, worst "
+                           f"{float((d - tol).max()):.3g} over")
+    return want
+
+
+@pytest.mark.parametrize("case", list(LINEAR_CASES))
+@pytest.mark.parametrize("eps", [1e-3, 1e-1])
+def test_perturbed_linear_matches_oracle_and_leaves_W(lib, gpu, case, eps):
+    from paper_2608_15665_gb300 import binding as zb
+    z, base = _context(gpu, case, seed=4242)
+    r, spec, tokens = LINEAR_CASES[case]
+    before = snapshot(z)
+    W_bits = [W.detach().clone() for W in z.weights]
+    terms = [(1, 1.0), (2, -1.0)]
+    for i, (m, n, _) in enumerate(spec):
+        for T in tokens:
+            X = _tokens(T, n, 17 * T + i, gpu)
+            ldy = (m + 7) // 8 * 8
+            Ybuf = torch.full((T, ldy), float("nan"), dtype=torch.bfloat16, device=gpu)
+            Y = Ybuf[:, :m]
+            zb.zo_linear_perturbed(z.ctx, i, X, Y, 5, 1, 1.0, 2, -1.0, eps)
+            z.sync()
+            C = subzero.perturb_coeff(z.seed, base + i, 5, r, terms, f32(eps))
+            zc = abs(f32(eps)) * 2.0
+            want = _check(Y, X, before["W"][i], before["U"][i], before["V"][i], C, zc,
+                          f"{case} matrix {i} T={T} eps={eps}")
+            # the padding columns of Y's rows are not written
+            assert torch.isnan(Ybuf[:, m:].float()).all()
+            if eps == 1e-1:
+                # the perturbation is visible: most outputs differ from the plain layer's
+                plain = rounding.round_to_bf16(to_f64(X) @ before["W"][i].T)
+                assert (plain != want).mean() > 0.5
+    for W, Wb in zip(z.weights, W_bits):
+        assert torch.equal(W.view(torch.int16), Wb.view(torch.int16))
+    z.close()
+
+
+def test_perturbed_linear_single_query_and_repeat(lib, gpu):
+    from paper_2608_15665_gb300 import binding as zb
+    z, base = _context(gpu, "r32", seed=99)
+    r, spec, _ = LINEAR_CASES["r32"]
+    before = snapshot(z)
+    m, n, _ = spec[1]
+    X = _tokens(64, n, 3, gpu)
+    Y1 = torch.empty((64, m), dtype=torch.bfloat16, device=gpu)
+    Y2 = torch.empty_like(Y1)
+    zb.zo_linear_perturbed(z.ctx, 1, X, Y1, 0, 3, -2.0, -1, 0.0, 1e-2)
+    zb.zo_linear_perturbed(z.ctx, 1, X, Y2, 0, 3, -2.0, -1, 0.0, 1e-2)
+    z.sync()
+    assert torch.equal(Y1.view(torch.int16), Y2.view(torch.int16))   # deterministic
+    C = subzero.perturb_coeff(z.seed, base + 1, 0, r, [(3, -2.0)], f32(1e-2))
+    _check(Y1, X, before["W"][1], before["U"][1], before["V"][1], C, 2.0 * f32(1e-2),
+           "single query")
+    z.close()
+
+
+def test_perturbed_linear_rejections(lib, gpu):
+    from paper_2608_15665_gb300 import binding as zb
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    z, _ = _context(gpu, "r32", seed=5)
+    X = _tokens(8, 520, 1, gpu)
+    Y = torch.empty((8, 304), dtype=torch.bfloat16, device=gpu)
+    with pytest.raises(RuntimeError):
+        zb.zo_linear_perturbed(z.ctx, 3, X, Y, 0, 0, 1.0, -1, 0.0, 1e-3)            # no matrix 3
+    with pytest.raises(RuntimeError):
+        zb.zo_linear_perturbed(z.ctx, 0, X, Y, 0, 4, 1.0, -1, 0.0, 1e-3)            # query 4 of 4
+    Ybad = torch.empty((8, 312), dtype=torch.bfloat16, device=gpu)[:, 1:305]       # misaligned
+    with pytest.raises(RuntimeError):
+        zb.zo_linear_perturbed(z.ctx, 0, X, Ybad, 0, 0, 1.0, -1, 0.0, 1e-3)
+    z.close()
+    # an output width that is not a multiple of 8 (TMA stores write 16-byte chunks)
+    w = [make_weight(300, 520, "bf16", 2, gpu)]
+    zo = SubZeroPlus(w, 32, 4, 1)
+    zo.init_subspace(0)
+    with pytest.raises(RuntimeError):
+        zb.zo_linear_perturbed(zo.ctx, 0, X, Y[:, :300], 0, 0, 1.0, -1, 0.0, 1e-3)
+    zo.close()
+    w = [make_weight(304, 520, "f32", 1, gpu)]
+    zf = SubZeroPlus(w, 32, 4, 1)
+    zf.init_subspace(0)
+    with pytest.raises(RuntimeError):                                             # FMA path
+        zb.zo_linear_perturbed(zf.ctx, 0, X, Y, 0, 0, 1.0, -1, 0.0, 1e-3)
+    zf.close()

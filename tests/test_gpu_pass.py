@@ -178,9 +178,6 @@ TC_CASES = {
     "tc32": (32, [(300, 520, 528), (1030, 72, 80), (257, 2048, None)]),
     "tc64": (64, [(300, 520, None), (130, 1000, None), (1030, 72, 72), (2048, 384, None)]),
     "tc128": (128, [(300, 520, None), (130, 1000, 1008), (1030, 136, None)]),
-    # widths that end inside a 16-byte chunk (the r = 128 epilogue stores W itself)
-    "tc128r": (128, [(300, 517, 520), (259, 133, 136), (131, 1001, 1008)]),
-    "tc64r": (64, [(300, 517, 520), (131, 1001, 1008)]),
 }
 
 
@@ -385,4 +382,40 @@ def test_narrow_tiles_are_chosen_for_thin_sets(lib, gpu):
     z, _ = _build_tc(gpu, "tc32", seed=11)
     with pytest.raises(RuntimeError):
         zb.zo_set_option(z.ctx, zb.ZO_OPTION_WPASS_PATH, 3)   # r = 32: no narrow tiles
+    z.close()
+
+
+@pytest.mark.parametrize("r", [16, 32, 64, 128])
+@pytest.mark.parametrize("widths,path", [((512, 136), 2), ((517, 133), 1)], ids=["n%8=0", "odd-n"])
+def test_row_padding_past_n_is_untouched(lib, gpu, r, widths, path):
+    # W is a column slice of a wider buffer (ldw > n): the elements past n in each row
+    # belong to the caller and keep their (NaN) contents.  TMA stores write whole 16-byte
+    # chunks, so a set with a width that is not a multiple of 8 takes the FMA path.
+    from paper_2608_15665_gb300 import binding as zb
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    shapes = [(300, widths[0], 528), (259, widths[1], 144)]
+    bufs, weights = [], []
+    for k, (m, n, ldw) in enumerate(shapes):
+        g = torch.Generator().manual_seed(900 + k)
+        buf = torch.full((m, ldw), float("nan"), dtype=torch.bfloat16)
+        buf[:, :n] = (torch.randn(m, n, generator=g) * 0.02).to(torch.bfloat16)
+        buf = buf.to(gpu)
+        bufs.append(buf)
+        weights.append(buf[:, :n])
+    z = SubZeroPlus(weights, r, 2, 77)
+    z.init_subspace(0)
+    before = snapshot(z)
+    z.perturb(0, 0, 1.0, 1, -1.0, 1e-1)
+    assert zb.zo_wpass_path(z.ctx) == path
+    after = snapshot(z)
+    for i in range(2):
+        want, T = oracle_perturb(before, i, "bf16", z.seed, i, 0, r, [(0, 1.0), (1, -1.0)], 1e-1)
+        assert_weights(after["W"][i], want, "bf16", f"r{r} matrix {i}", before=before["W"][i],
+                       terms=T)
+    z.step(0, 1, np.array([2.01, 1.99, 2.0, 2.02], np.float32), "central", 1e-1, 1e-2, 0.9, 0.95,
+           1e-8, 1, 1.0)
+    z.sync()
+    for (m, n, ldw), buf in zip(shapes, bufs):
+        assert torch.isnan(buf[:, n:].float()).all(), f"row padding of a {m}x{n} matrix written"
+        assert not torch.isnan(buf[:, :n].float()).any()
     z.close()
