@@ -64,9 +64,13 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="llama7b_bf16_r32")
     p.add_argument("--scheme", choices=["central", "forward"], default="central")
-    p.add_argument("--method", choices=["subzero", "mezo"], default="subzero",
+    p.add_argument("--method", choices=["subzero", "mezo", "linear"], default="subzero",
                    help="subzero: the SubZero+ step (default); mezo: the full-space SPSA "
-                        "baseline of Eq. (1), 3 passes per step")
+                        "baseline of Eq. (1), 3 passes per step; linear: the linear layers of "
+                        "one layer evaluated at the perturbed weights without a weight pass "
+                        "(zo_linear_perturbed), --tokens rows of activations")
+    p.add_argument("--tokens", type=int, default=4096,
+                   help="--method linear: activation rows T per linear layer")
     p.add_argument("--layers", type=int, default=0,
                    help="use only the first N layers of the workload (shape-preserving subset, "
                         "for profiling captures); 0 = all")
@@ -458,10 +462,128 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def run_linear(args):
+    """The linear layers of the first `--layers` (default 1) layers of the workload at the
+    perturbed weights, Y_i = X_i (W_i + U_i C V_i^T)^T with no weight pass (the forward
+    route of one loss evaluation: C_i and P_i once, then S = X P^T and X W^T + S U^T per
+    layer).
+    X_i: --tokens x n_i bf16 activations, N(0, 1), resident.  A step is one
+    zo_linear_prepare and the layer's zo_linear_perturbed calls.  value = TFLOP/s of the
+    exact-arithmetic work 2 T (m n + r (m + n)) per layer; roofline against the measured
+    bf16 tensor peak.  For context, the same GEMMs without the perturbation (torch, i.e.
+    cuBLAS) and the weight-pass route (one zo_perturb pass over the layer, then those
+    GEMMs) are timed too."""
+    import torch
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    from paper_2608_15665_gb300 import build
+    build.build()
+    from paper_2608_15665_gb300 import binding as zb
+    from paper_2608_15665_gb300 import workloads
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+
+    wl = subset(workloads.get(args.workload), args.layers or 1)
+    T = args.tokens
+    weights = [workloads.init_weight(wl, i, dev) for i in range(wl.n_mats)]
+    z = SubZeroPlus(weights, wl.r, wl.q, wl.seed)
+    z.init_subspace(0)
+    g = torch.Generator(device=dev).manual_seed(wl.seed)
+    X = {n: torch.randn(T, n, generator=g, device=dev).to(torch.bfloat16)
+         for n in sorted({n for _, n in wl.shapes})}
+    Y = [torch.empty(T, m, dtype=torch.bfloat16, device=dev) for m, _ in wl.shapes]
+    flops = sum(2.0 * T * (m * n + wl.r * (m + n)) for m, n in wl.shapes)
+
+    def fused(t):
+        zb.zo_linear_prepare(z.ctx, t, 0, 1.0, -1, 0.0, wl.eps)
+        for i, (m, n) in enumerate(wl.shapes):
+            zb.zo_linear_perturbed(z.ctx, i, X[n], Y[i])
+
+    def plain():
+        for i, (m, n) in enumerate(wl.shapes):
+            torch.matmul(X[n], z.weights[i].t(), out=Y[i])
+
+    def timed(fn, K):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record()
+        for k in range(K):
+            fn(k)
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / K
+
+    K, W = args.steps, args.warmup
+    for k in range(W):
+        fused(k)
+        plain()
+    z.sync()
+    launches0 = zb.zo_kernel_launches(z.ctx)
+    clocks = ClockSampler(0)
+    clocks.start()
+    fused_ms = timed(fused, K)
+    clk = clocks.stop()
+    launches = zb.zo_kernel_launches(z.ctx) - launches0
+    z.sync()
+    plain_ms = timed(lambda k: plain(), K)
+    wpass_ms = timed(lambda k: (z.perturb(k, 0, 1.0, -1, 0.0, wl.eps), plain()), K)
+    z.sync()
+
+    # end to end: the activations copied from pinned host memory every step, one output row
+    # read back
+    host = {n: x.cpu().pin_memory() for n, x in X.items()}
+    out_row = torch.empty(wl.shapes[-1][0], dtype=torch.bfloat16).pin_memory()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for k in range(K):
+        for n, h in host.items():
+            X[n].copy_(h, non_blocking=True)
+        fused(k)
+        out_row.copy_(Y[-1][0])
+    torch.cuda.synchronize()
+    e2e_s = (time.perf_counter() - t0) / K
+    h2d = sum(h.numel() * 2 for h in host.values())
+
+    peak = None
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            mp = json.load(f)
+        # the layer's GEMMs run back to back for tens of ms: the sustained figure
+        peak = float(mp.get("bf16_tflops_sustained") or 0.0) or None
+        peak_kind = "measured (cuBLAS bf16, sustained)"
+    except Exception:
+        peak_kind = "unavailable"
+    if peak is None:
+        peak, peak_kind = 1700.0, "fallback (sustained)"
+    achieved = flops / (fused_ms / 1e3) / 1e12
+    line = {
+        "metric": "perturbed linear forward TFLOP/s (zo_linear_perturbed, LLaMA-7B layer shapes, 1 GB300)",
+        "value": achieved, "unit": "TFLOP/s", "n_gpus": 1, "steps": K, "warmup": W,
+        "ms_per_step": fused_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "matrices": wl.n_mats, "tokens": T, "r": wl.r,
+                   "method": "linear",
+                   "l2": "inputs larger than L2 (%.0f MB of weights)" % (sum(m * n for m, n in wl.shapes) * 2 / 1e6),
+                   "parallelism": "single GPU"},
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "peak_kind": peak_kind, "traffic": None,
+                     "kernel": "linear_kernel", "algorithmic_flops_per_step": flops},
+        "plain_gemm_ms": plain_ms,
+        "weight_pass_route_ms": wpass_ms,
+        "e2e": {"value": flops / e2e_s / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(out_row.numel() * 2)},
+        "clocks": clk,
+        "gpu_launches": int(launches),
+    }
+    z.close()
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         run_reference(args)
+    elif args.method == "linear":
+        run_linear(args)
     else:
         run_ours(args)
 

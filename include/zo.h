@@ -202,23 +202,27 @@ ZO_API zo_status zo_step(zo_ctx* ctx, uint32_t t, int32_t adam_t, const float* l
 ZO_API zo_status zo_mezo_perturb(zo_ctx* ctx, uint32_t t, float coef);
 
 /*
- * zo_linear_perturbed -- one linear layer of a loss evaluation at the perturbed weights
- * (Alg. 3's forward at W_i' = W_i + U_i C V_i^T, Eq. (4) form) WITHOUT a weight pass:
- *   Y = X (W_i + U_i C V_i^T)^T = X W_i^T + (X V_i C^T) U_i^T,
- *   C = eps (ca Z_i^(qa) + cb Z_i^(qb)) at step t (qb = -1: one term) -- the coefficient
- *   that zo_perturb(ctx, t, qa, ca, qb, cb, eps) would add to W_i.
- * W_i is read, never written.  X: T x n_i bf16, row stride ldx elements; Y: T x m_i bf16,
- * row stride ldy (both device, caller-owned, 16-byte aligned, strides multiples of 8;
- * m_i a multiple of 8, else ZO_ERR_SHAPE).
- * The dense product is exact in bf16 with fp32 accumulation; the rank-r term carries
- * the bf16 hi/lo split's ~2^-16 relative error; Y is rounded to bf16 once.  Needs the
- * tensor-core path (every W bf16) with r in {16, 32}; otherwise ZO_ERR_UNSUPPORTED.
- * Overwrites the context's C_i / P_i workspace of matrix i (the next zo_perturb or
- * zo_step forms its own).  Asynchronous; device errors go to the status word.
+ * Linear layers at the perturbed weights WITHOUT a weight pass: the forward of a loss
+ * evaluation of Alg. 3 at W_i' = W_i + U_i C_i V_i^T (Eq. (4) form) with every W_i left as
+ * it is, for contexts on the tensor-core path (every W bf16, n a multiple of 8) with r in
+ * {16, 32}; otherwise ZO_ERR_UNSUPPORTED.
+ *
+ * zo_linear_prepare -- once per loss evaluation: C_i = eps (ca Z_i^(qa) + cb Z_i^(qb)) at
+ *   step t (qb = -1: one term) for every matrix -- the coefficient zo_perturb(ctx, t, qa,
+ *   ca, qb, cb, eps) would add to W_i -- and P_i = C_i V_i^T, kept for the calls below
+ *   until the next zo_linear_prepare.
+ * zo_linear_perturbed -- one layer: Y = X (W_i + U_i C_i V_i^T)^T = X W_i^T +
+ *   (X V_i C_i^T) U_i^T.  X: T x n_i bf16, row stride ldx elements; Y: T x m_i bf16, row
+ *   stride ldy (device, caller-owned, 16-byte aligned, strides multiples of 8; m_i a
+ *   multiple of 8, else ZO_ERR_SHAPE).  The dense product is exact in bf16 with fp32
+ *   accumulation; the rank-r term carries the bf16 hi/lo split's ~2^-16 relative error;
+ *   Y is rounded to bf16 once.  W_i is read, never written.  Asynchronous; device errors
+ *   go to the status word.
  */
+ZO_API zo_status zo_linear_prepare(zo_ctx* ctx, uint32_t t, int32_t qa, float ca, int32_t qb,
+                                   float cb, float eps);
 ZO_API zo_status zo_linear_perturbed(zo_ctx* ctx, int32_t i, const void* X, int64_t T,
-                                     int64_t ldx, void* Y, int64_t ldy, uint32_t t,
-                                     int32_t qa, float ca, int32_t qb, float cb, float eps);
+                                     int64_t ldx, void* Y, int64_t ldy);
 
 /* zo_sync_status -- synchronise the stream; return (and clear) the device status word. */
 ZO_API zo_status zo_sync_status(zo_ctx* ctx);

@@ -73,10 +73,10 @@ _SIGNATURES = {
                              _c.c_float, _c.c_float, _c.c_float, _c.c_int32, _c.c_float,
                              _c.c_void_p]),
     "zo_mezo_perturb": (_c.c_int32, [_c.c_void_p, _c.c_uint32, _c.c_float]),
+    "zo_linear_prepare": (_c.c_int32, [_c.c_void_p, _c.c_uint32, _c.c_int32, _c.c_float,
+                                       _c.c_int32, _c.c_float, _c.c_float]),
     "zo_linear_perturbed": (_c.c_int32, [_c.c_void_p, _c.c_int32, _c.c_void_p, _c.c_int64,
-                                         _c.c_int64, _c.c_void_p, _c.c_int64, _c.c_uint32,
-                                         _c.c_int32, _c.c_float, _c.c_int32, _c.c_float,
-                                         _c.c_float]),
+                                         _c.c_int64, _c.c_void_p, _c.c_int64]),
     "zo_sync_status": (_c.c_int32, [_c.c_void_p]),
     "zo_set_option": (_c.c_int32, [_c.c_void_p, _c.c_int32, _c.c_int64]),
     "zo_get_timing": (_c.c_int32, [_c.c_void_p, _c.POINTER(_c.c_double), _c.POINTER(_c.c_int64)]),
@@ -206,14 +206,20 @@ def zo_mezo_perturb(ctx, t, coef):
     _check(LIB.zo_mezo_perturb(ctx, int(t), float(coef)), "zo_mezo_perturb")
 
 
-def zo_linear_perturbed(ctx, i, X, Y, t, qa, ca, qb, cb, eps):
-    """Y = X (W_i + U_i C V_i^T)^T with C = eps (ca Z_qa + cb Z_qb) at step t; X (T x n) and
-    Y (T x m) bf16 CUDA tensors with unit column stride."""
+def zo_linear_prepare(ctx, t, qa, ca, qb, cb, eps):
+    """C_i = eps (ca Z_qa + cb Z_qb) at step t and P_i = C_i V_i^T for every matrix, for the
+    zo_linear_perturbed calls of one loss evaluation."""
+    _check(LIB.zo_linear_prepare(ctx, int(t), int(qa), float(ca), int(qb), float(cb),
+                                 float(eps)), "zo_linear_prepare")
+
+
+def zo_linear_perturbed(ctx, i, X, Y):
+    """Y = X (W_i + U_i C_i V_i^T)^T with the prepared C_i; X (T x n) and Y (T x m) bf16
+    CUDA tensors with unit column stride."""
     if X.dim() != 2 or Y.dim() != 2 or X.stride(1) != 1 or Y.stride(1) != 1 or X.shape[0] != Y.shape[0]:
         raise ValueError("X and Y must be 2-D, row-major (unit column stride), with the same rows")
     _check(LIB.zo_linear_perturbed(ctx, int(i), _ptr(X), int(X.shape[0]), int(X.stride(0)),
-                                   _ptr(Y), int(Y.stride(0)), int(t), int(qa), float(ca),
-                                   int(qb), float(cb), float(eps)), "zo_linear_perturbed")
+                                   _ptr(Y), int(Y.stride(0))), "zo_linear_perturbed")
 
 
 def zo_sync_status(ctx):

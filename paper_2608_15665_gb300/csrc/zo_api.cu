@@ -110,12 +110,15 @@ struct zo_ctx {
   __nv_bfloat16* d_p_hl = nullptr;   // stacked [hi | lo] rows of every P_i^T, 128-row padded
   zo::TcMat* d_tc = nullptr;
   std::vector<zo::TcMat> h_tc;       // host copy (operand rows of each matrix)
-  std::vector<int32_t> h_unit0;      // first projection unit of each matrix
-  // zo_linear_perturbed's workspace: P_K ([P_hi ; P_lo] rows, K-major) and S_HL
+  // zo_linear_prepare / zo_linear_perturbed: P_K of every matrix ([P_hi ; P_lo] rows,
+  // K-major) at element offsets pk_off, S_HL and the partial sums of S (T rows each)
   __nv_bfloat16* d_pk = nullptr;
-  int64_t pk_ld = 0;
+  int64_t* d_pk_off = nullptr;
+  std::vector<int64_t> h_pk_off;
+  bool linear_ready = false;
   __nv_bfloat16* d_s_hl = nullptr;
-  int64_t s_cap = 0;
+  float* d_s_part = nullptr;
+  int64_t s_cap = 0, part_cap = 0;
   int64_t tc_tiles = 0;
   CUtensorMap* d_w_maps = nullptr;   // one TMA descriptor per W_i (device memory)
   CUtensorMap tm_a{}, tm_b{};        // descriptors of the stacked operands (kernel parameters)
@@ -153,7 +156,9 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_p_hl);
   cudaFree(c->d_tc);
   cudaFree(c->d_pk);
+  cudaFree(c->d_pk_off);
   cudaFree(c->d_s_hl);
+  cudaFree(c->d_s_part);
   cudaFree(c->d_w_maps);
   cudaFree(c->d_u_units);
   cudaFree(c->d_v_hl);
@@ -555,7 +560,6 @@ zo_status zo_create(zo_ctx** out, const zo_matrix* mats, int32_t n_mats, int32_t
     const int64_t tiles = ((mt.m + zo::kFmaTileRows - 1) / zo::kFmaTileRows) * ((mt.n + tn - 1) / tn);
     d.tile0 = prefix[i];
     prefix[i + 1] = prefix[i] + tiles;
-    c->h_unit0.push_back((int32_t)units.size());
     for (int64_t j0 = 0; j0 < mt.n; j0 += 128) units.push_back(make_int2(i, (int)j0));
     c->h_mats[i] = d;
   }
@@ -837,18 +841,69 @@ zo_status zo_step(zo_ctx* c, uint32_t t, int32_t adam_t, const float* losses, in
   return run_weight_pass(c);
 }
 
-zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, int64_t ldx,
-                              void* Y, int64_t ldy, uint32_t t, int32_t qa, float ca,
-                              int32_t qb, float cb, float eps) {
-  if (!c || !X || !Y) return ZO_ERR_INVALID_ARG;
+zo_status zo_linear_prepare(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t qb, float cb,
+                            float eps) {
+  if (!c) return ZO_ERR_INVALID_ARG;
   DeviceGuard guard(c->device);
   if (!c->tc_ok || !zo::linear_supported(c->r)) {
-    g_last_error = "zo_linear_perturbed needs the tensor-core path with r in {16, 32}";
+    g_last_error = "zo_linear_prepare needs the tensor-core path with r in {16, 32}";
     return ZO_ERR_UNSUPPORTED;
   }
-  if (mat < 0 || mat >= c->n_mats || qa < 0 || qa >= c->q || qb < -1 || qb >= c->q ||
-      !std::isfinite(ca) || !std::isfinite(cb) || !std::isfinite(eps)) {
-    g_last_error = "zo_linear_perturbed: matrix or query index out of range, or non-finite scalar";
+  if (qa < 0 || qa >= c->q || qb < -1 || qb >= c->q || !std::isfinite(ca) || !std::isfinite(cb) ||
+      !std::isfinite(eps)) {
+    g_last_error = "zo_linear_prepare: query index out of range or non-finite scalar";
+    return ZO_ERR_INVALID_ARG;
+  }
+  const int32_t r = c->r;
+  if (!c->d_pk) {
+    c->h_pk_off.assign(c->n_mats, 0);
+    int64_t total = 0;
+    for (int32_t i = 0; i < c->n_mats; ++i) {
+      c->h_pk_off[i] = total;
+      total += zo::linear_pk_elems(c->h_mats[i].n, r);
+    }
+    ZO_CUDA(cudaMalloc(&c->d_pk, sizeof(__nv_bfloat16) * total), "cudaMalloc(P_K)");
+    ZO_CUDA(cudaMalloc(&c->d_pk_off, sizeof(int64_t) * c->n_mats), "cudaMalloc(P_K offsets)");
+    ZO_CUDA(cudaMemcpy(c->d_pk_off, c->h_pk_off.data(), sizeof(int64_t) * c->n_mats,
+                       cudaMemcpyHostToDevice),
+            "upload P_K offsets");
+  }
+  // C_i = eps (ca Z_qa + cb Z_qb) for every matrix, P_i = C_i V_i^T, P_K = [P_hi ; P_lo]
+  zo::CoeffParams p{};
+  p.mode = zo::kCoeffPerturb;
+  p.seed = c->seed;
+  p.t = t;
+  p.r = r;
+  p.q = c->q;
+  p.qa = qa;
+  p.qb = qb;
+  p.ca = ca;
+  p.cb = cb;
+  p.eps = eps;
+  ZO_CUDA(zo::launch_coeff(c->d_mats, c->n_mats, p, c->stream), "coefficient kernel");
+  ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, r, c->d_c_hl, c->stream), "split C");
+  ZO_CUDA(zo::launch_project_tc(c->tm_v, c->tm_c, c->tm_p, c->d_tc, c->d_proj_units,
+                                c->n_proj_units, std::min<int32_t>(c->n_proj_units, c->sms), r,
+                                c->d_status, c->stream),
+          "tensor-core projection kernel");
+  ZO_CUDA(zo::launch_transpose_p(c->d_p_hl, c->d_tc, c->d_proj_units, c->n_proj_units,
+                                 c->d_pk_off, (int32_t)zo::tc_hl_width(r), r, c->d_pk, c->stream),
+          "P transpose");
+  c->launches += 4;
+  c->linear_ready = true;
+  return ZO_OK;
+}
+
+zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, int64_t ldx,
+                              void* Y, int64_t ldy) {
+  if (!c || !X || !Y) return ZO_ERR_INVALID_ARG;
+  DeviceGuard guard(c->device);
+  if (!c->linear_ready) {
+    g_last_error = "zo_linear_perturbed: call zo_linear_prepare first";
+    return ZO_ERR_INVALID_ARG;
+  }
+  if (mat < 0 || mat >= c->n_mats) {
+    g_last_error = "zo_linear_perturbed: matrix index out of range";
     return ZO_ERR_INVALID_ARG;
   }
   const zo::MatDesc& md = c->h_mats[mat];
@@ -864,65 +919,46 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
   }
   const int32_t r = c->r;
   const int64_t HLW = zo::tc_hl_width(r);
-  // workspace: P_K (2r x pk_ld) for the widest matrix, S_HL (T rows of 64)
-  if (!c->d_pk) {
-    int64_t nmax = 0;
-    for (const auto& d : c->h_mats) nmax = std::max(nmax, d.n);
-    c->pk_ld = (nmax + 63) / 64 * 64;
-    ZO_CUDA(cudaMalloc(&c->d_pk, sizeof(__nv_bfloat16) * 2 * r * c->pk_ld), "cudaMalloc(P_K)");
-  }
-  if (T > c->s_cap) {
+  int32_t k_split = 1, k_chunk = 1;
+  zo::linear_s_split(T, n, c->sms, &k_split, &k_chunk);
+  const int64_t part = (int64_t)k_split * T * r;
+  if (T > c->s_cap || part > c->part_cap) {
     ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
-    cudaFree(c->d_s_hl);
-    c->d_s_hl = nullptr;
-    c->s_cap = 0;
-    const int64_t cap = (T + 127) / 128 * 128;
-    ZO_CUDA(cudaMalloc(&c->d_s_hl, sizeof(__nv_bfloat16) * cap * HLW), "cudaMalloc(S_HL)");
-    c->s_cap = cap;
+    if (T > c->s_cap) {
+      cudaFree(c->d_s_hl);
+      c->d_s_hl = nullptr;
+      c->s_cap = 0;
+      const int64_t cap = (T + 127) / 128 * 128;
+      ZO_CUDA(cudaMalloc(&c->d_s_hl, sizeof(__nv_bfloat16) * cap * HLW), "cudaMalloc(S_HL)");
+      c->s_cap = cap;
+    }
+    if (part > c->part_cap) {
+      cudaFree(c->d_s_part);
+      c->d_s_part = nullptr;
+      c->part_cap = 0;
+      ZO_CUDA(cudaMalloc(&c->d_s_part, sizeof(float) * part), "cudaMalloc(partial S)");
+      c->part_cap = part;
+    }
   }
-  CUtensorMap tm_x{}, tm_pk{}, tm_s_st{}, tm_s_ld{}, tm_y{};
+  CUtensorMap tm_x{}, tm_pk{}, tm_s{}, tm_y{};
   const bool enc =
       encode_bf16_2d(&tm_x, const_cast<void*>(X), n, T, ldx * 2, 64, 128) &&
-      encode_bf16_2d(&tm_pk, c->d_pk, n, 2 * r, c->pk_ld * 2, 64, (uint32_t)(2 * r)) &&
-      encode_bf16_2d(&tm_s_st, c->d_s_hl, HLW, T, HLW * 2, 64, 32) &&
-      encode_bf16_2d(&tm_s_ld, c->d_s_hl, HLW, T, HLW * 2, 64, 128) &&
+      encode_bf16_2d(&tm_pk, c->d_pk + c->h_pk_off[mat], n, 2 * r, (n + 63) / 64 * 64 * 2, 64,
+                     (uint32_t)(2 * r)) &&
+      encode_bf16_2d(&tm_s, c->d_s_hl, HLW, T, HLW * 2, 64, 128) &&
       encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 64, 32);
   if (!enc) {
     g_last_error = "zo_linear_perturbed: cuTensorMapEncodeTiled rejected a descriptor";
     return ZO_ERR_CUDA;
   }
-  // C_i = eps (ca Z_qa + cb Z_qb), the coefficient zo_perturb would apply; P_i = C_i V_i^T
-  zo::CoeffParams p{};
-  p.mode = zo::kCoeffPerturb;
-  p.seed = c->seed;
-  p.t = t;
-  p.r = r;
-  p.q = c->q;
-  p.qa = qa;
-  p.qb = qb;
-  p.ca = ca;
-  p.cb = cb;
-  p.eps = eps;
-  ZO_CUDA(zo::launch_coeff(c->d_mats + mat, 1, p, c->stream), "coefficient kernel");
-  ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, r, c->d_c_hl, c->stream), "split C");
-  const int32_t unit0 = c->h_unit0[mat];
-  const int32_t n_units = (int32_t)((n + 127) / 128);
-  ZO_CUDA(zo::launch_project_tc(c->tm_v, c->tm_c, c->tm_p, c->d_tc, c->d_proj_units + unit0,
-                                n_units, std::min<int32_t>(n_units, c->sms), r, c->d_status,
-                                c->stream),
-          "tensor-core projection kernel");
-  ZO_CUDA(zo::launch_transpose_p(c->d_p_hl, c->h_tc[mat].p_row0, (int32_t)HLW, n, r, c->d_pk,
-                                 c->pk_ld, c->stream),
-          "P transpose");
-  // S = X P^T, then Y = X W^T + S U^T
-  const int32_t gs = std::min<int32_t>(zo::linear_tiles(T, 2 * r, true, r), c->sms);
-  ZO_CUDA(zo::launch_linear_s(tm_x, tm_pk, tm_s_st, T, n, r, gs, c->d_status, c->stream),
-          "S = X P^T kernel");
-  const int32_t gy = std::min<int32_t>(zo::linear_tiles(T, m, false, r), c->sms);
-  ZO_CUDA(zo::launch_linear_y(tm_x, c->d_w_maps + mat, tm_s_ld, c->tm_a, tm_y, T, m, n,
-                              c->h_tc[mat].u_row0, r, gy, c->d_status, c->stream),
+  // S = X P^T (split K, then the partial sums reduced into S_HL), Y = X W^T + S U^T
+  ZO_CUDA(zo::launch_linear_s(tm_x, tm_pk, T, n, r, k_split, k_chunk, c->d_s_part, c->d_s_hl,
+                              c->sms, c->d_status, c->stream),
+          "S = X P^T kernels");
+  ZO_CUDA(zo::launch_linear_y(tm_x, c->d_w_maps + mat, tm_s, c->tm_a, tm_y, T, m, n,
+                              c->h_tc[mat].u_row0, r, c->sms, c->d_status, c->stream),
           "perturbed linear kernel");
-  c->launches += 6;
+  c->launches += 3;
   return ZO_OK;
 }
 

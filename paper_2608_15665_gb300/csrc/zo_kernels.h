@@ -138,24 +138,28 @@ cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
 // ---- a linear layer at the perturbed weights, without a weight pass (zo_linear.cu) -----
 // Y = X (W + U C V^T)^T = X W^T + S U^T, S = X P^T, for bf16 contexts at r in {16, 32}.
 bool linear_supported(int32_t r);
-// Output tiles of the S GEMM (s_gemm, 2r columns) or of the Y GEMM (256 columns).
-int32_t linear_tiles(int64_t rows, int64_t cols, bool s_gemm, int32_t r);
-// P_K[k][j] = P_HL[p_row0 + j][k], k < 2r, j < n (rows [P_hi ; P_lo], row stride ld_k).
-cudaError_t launch_transpose_p(const __nv_bfloat16* p_hl, int64_t p_row0, int32_t hl_width,
-                               int64_t n, int32_t r, __nv_bfloat16* p_k, int64_t ld_k,
-                               cudaStream_t s);
+// The S GEMM's split of K = n into k_split ranges of k_chunk steps of 64 (~ one wave).
+void linear_s_split(int64_t T, int64_t n, int32_t sms, int32_t* k_split, int32_t* k_chunk);
+int32_t linear_y_tiles(int64_t T, int64_t m);
+// Elements of matrix i's P_K: 2r rows of n rounded up to 64.
+int64_t linear_pk_elems(int64_t n, int32_t r);
+// P_K of every matrix from P_HL (units = the projection units, pk_off = element offsets).
+cudaError_t launch_transpose_p(const __nv_bfloat16* p_hl, const TcMat* d_tc, const int2* d_units,
+                               int32_t n_units, const int64_t* d_pk_off, int32_t hl_width,
+                               int32_t r, __nv_bfloat16* p_k, cudaStream_t s);
 // S_HL rows [S_hi | S_lo | 0] of S = X P^T: tm_x over X (box 64 x 128), tm_pk over P_K
-// (box 64 x 2r), tm_s_out over S_HL (box 64 x 32).
-cudaError_t launch_linear_s(const CUtensorMap& tm_x, const CUtensorMap& tm_pk,
-                            const CUtensorMap& tm_s_out, int64_t T, int64_t n, int32_t r,
-                            int32_t grid, uint32_t* d_status, cudaStream_t s);
+// (box 64 x 2r); part = k_split x T x r fp32 workspace.
+cudaError_t launch_linear_s(const CUtensorMap& tm_x, const CUtensorMap& tm_pk, int64_t T,
+                            int64_t n, int32_t r, int32_t k_split, int32_t k_chunk, float* part,
+                            __nv_bfloat16* s_hl, int32_t sms, uint32_t* d_status,
+                            cudaStream_t s);
 // Y = X W^T + S U^T: d_w_map = W's descriptor (box 64 x 32), tm_s_in over S_HL (box
 // 64 x 128), tm_u over the U operand (box 64 x 128; W's rows from u_row0), tm_y over Y
 // (box 64 x 32).
 cudaError_t launch_linear_y(const CUtensorMap& tm_x, const CUtensorMap* d_w_map,
                             const CUtensorMap& tm_s_in, const CUtensorMap& tm_u,
                             const CUtensorMap& tm_y, int64_t T, int64_t m, int64_t n,
-                            int32_t u_row0, int32_t r, int32_t grid, uint32_t* d_status,
+                            int32_t u_row0, int32_t r, int32_t sms, uint32_t* d_status,
                             cudaStream_t s);
 
 // ---- refresh of tall panels at r = 16 ... 128: CholeskyQR2 (zo_cholqr.cu) ----------

@@ -7,17 +7,19 @@
 // Two tcgen05 GEMMs with one kernel template (both operands K-major in shared memory,
 // 128-byte swizzle, loaded by TMA; fp32 accumulators in TMEM; persistent CTAs over
 // output tiles of 128 rows of X):
-//   kModeS  S = X P^T with B = [P_hi ; P_lo] (2r rows, K-major, from P_K): N = 2r; the
-//           epilogue sums the two halves, S = D[:, :r] + D[:, r:], and writes S as bf16
-//           hi/lo rows [S_hi | S_lo | 0] of 64 elements (S_HL), the layout of the U
-//           operand.
+//   kModeS  partial S = X P^T over a range of K with B = [P_hi ; P_lo] (2r rows, K-major,
+//           from P_K): N = 2r, tiles = (128 rows of X) x (K range) so that a few row
+//           blocks still fill the SMs; the epilogue sums the two halves, D[:, :r] +
+//           D[:, r:], and writes the fp32 partial rows; reduce_s_kernel adds the partials
+//           and writes S as bf16 hi/lo rows [S_hi | S_lo | 0] of 64 elements (S_HL), the
+//           layout of the U operand.
 //   kModeY  Y = X W^T over K = n (single bf16 products, both operands exact in bf16)
 //           followed by one more K step from S_HL and the U operand, with the weight
 //           pass's three products S_hi U_hi + S_hi U_lo + S_lo U_hi (relative error
 //           ~2^-16 of the rank-r term); N = 256 columns of Y per tile; the epilogue
 //           rounds to bf16 and TMA-stores Y.
 // P_K is P_HL (the projection's rows [P_hi(j, :) | P_lo(j, :)], j < n) transposed by
-// transpose_p_kernel.  Ragged edges: TMA zero-fills loads past T, n and m and clips
+// transpose_p_kernel, for every matrix once per loss evaluation (zo_linear_prepare).  Ragged edges: TMA zero-fills loads past T, n and m and clips
 // stores.
 //
 // Roles of the 192 threads of a CTA:
@@ -31,6 +33,8 @@
 //                   staged 32 x 64 boxes.
 // Every mbarrier wait is bounded; on expiry the kernel records kDevTimeout in the status
 // word, lets the other roles stop, drains its copies and frees TMEM.
+#include <algorithm>
+
 #include <cuda.h>
 
 #include "zo_kernels.h"
@@ -76,7 +80,8 @@ __device__ __forceinline__ void lin_give_up(LinShared& sh, uint32_t* status) {
   *reinterpret_cast<volatile int*>(&sh.abort_flag) = 1;
 }
 
-// tm_a: X (box 64 x 128).  kModeS: tm_b = P_K (box 64 x 2r), tm_o = S_HL (box 64 x 32).
+// tm_a: X (box 64 x 128).  kModeS: tm_b = P_K (box 64 x 2r); K split into k_split
+// ranges of k_chunk steps; fp32 partials to part[(k range) x rows x R].
 // kModeY: w_map = W_i (box 64 x 32), tm_s = S_HL (box 64 x 128), tm_u = U operand (box
 // 64 x 128) with this matrix's rows from u_row0, tm_o = Y (box 64 x 32).
 template <int kMode, int R>
@@ -84,8 +89,8 @@ __global__ void __launch_bounds__(kLinThreads, 1)
 linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
               const CUtensorMap* __restrict__ w_map, const __grid_constant__ CUtensorMap tm_s,
               const __grid_constant__ CUtensorMap tm_u, const __grid_constant__ CUtensorMap tm_o,
-              int rows, int cols, int k_steps, int u_row0, uint32_t* __restrict__ status,
-              long long wait_cycles) {
+              int rows, int cols, int k_steps, int k_split, int k_chunk, int u_row0,
+              float* __restrict__ part, uint32_t* __restrict__ status, long long wait_cycles) {
   using Cfg = LinCfg<kMode, R>;
   static_assert(sizeof(LinShared) <= 1024, "barrier block");
   constexpr int kN = Cfg::kN;
@@ -97,9 +102,19 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
   LinShared& sh = *reinterpret_cast<LinShared*>(o_smem + Cfg::kOutBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int tiles_m = (cols + kN - 1) / kN;
+  // kModeY: tile = (row block, column block), K = all steps + the extension;
+  // kModeS: tile = (row block, K range)
+  const int tiles_m = kMode == kModeY ? (cols + kN - 1) / kN : k_split;
   const int n_tiles = ((rows + kBM - 1) / kBM) * tiles_m;
-  const int steps = k_steps + (kMode == kModeY ? 1 : 0);           // + the extension
+  auto k_range = [&](int nb, int& kb, int& ke) {
+    if (kMode == kModeY) {
+      kb = 0;
+      ke = k_steps + 1;                                             // + the extension
+    } else {
+      kb = nb * k_chunk;
+      ke = min(k_steps, kb + k_chunk);
+    }
+  };
   const volatile int* abort = &sh.abort_flag;
 
   if (threadIdx.x == 0) {
@@ -115,10 +130,10 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
     sh.abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tm_a);
-    prefetch_tmap(&tm_o);
     if constexpr (kMode == kModeS) {
       prefetch_tmap(&tm_b);
     } else {
+      prefetch_tmap(&tm_o);
       prefetch_tmap(w_map);
       prefetch_tmap(&tm_s);
       prefetch_tmap(&tm_u);
@@ -139,7 +154,9 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
     bool ok = true;
     for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
       const int tb = tile / tiles_m, nb = tile % tiles_m;
-      for (int k = 0; k < steps; ++k) {
+      int kb, ke;
+      k_range(nb, kb, ke);
+      for (int k = kb; k < ke; ++k) {
         const int s = (int)(n_st % Cfg::kStages);
         if (!mbar_wait_bounded(&sh.empty[s], (uint32_t)(((n_st / Cfg::kStages) & 1) ^ 1), abort,
                                wait_cycles)) {
@@ -186,7 +203,9 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
       }
       tc_fence_after();
       const uint32_t d = tmem + (uint32_t)(acc * kN);
-      for (int k = 0; k < steps; ++k) {
+      int kb, ke;
+      k_range(tile % tiles_m, kb, ke);
+      for (int k = kb; k < ke; ++k) {
         const int s = (int)(n_st % Cfg::kStages);
         if (!mbar_wait_bounded(&sh.full[s], (uint32_t)((n_st / Cfg::kStages) & 1), abort,
                                wait_cycles)) {
@@ -209,7 +228,7 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
             mma_bf16(d, sdesc_k_sw128(a_base + 32 * kk), sdesc_k_sw128(b_base + 32 * kk), idesc,
-                     (k > 0 || kk > 0) ? 1u : 0u);
+                     (k > kb || kk > 0) ? 1u : 0u);
         }
         mma_commit(&sh.empty[s]);
         ++n_st;
@@ -232,7 +251,7 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
     int64_t it = 0, n_box = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++it) {
-      const int tb = tile / tiles_m, nb = tile % tiles_m;
+      const int tb = tile / tiles_m, nb = tile % tiles_m;   // kModeS: nb = the K range
       const int acc = (int)(it & 1);
       if (!mbar_wait_bounded(&sh.acc_full[acc], (uint32_t)((it >> 1) & 1), abort, wait_cycles)) {
         ok = false;
@@ -241,7 +260,7 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
       tc_fence_after();
       const int y = tb * kBM + 32 * g;
       if constexpr (kMode == kModeS) {
-        // S = D[:, :R] + D[:, R:2R]; row [S_hi | S_lo | 0] of 64 elements
+        // partial S over this K range: D[:, :R] + D[:, R:2R], fp32, this lane's row
         uint32_t v[2 * R];
         if constexpr (R == 32) {
           uint32_t a[32], b[32];
@@ -260,30 +279,19 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sh.acc_empty[acc]);
-        if (lane == 0) bulk_wait_read_all();    // the previous tile's box has been stored
-        __syncwarp();
+        const int row = y + lane;
+        if (row < rows) {
+          float4* dst = reinterpret_cast<float4*>(part + ((int64_t)nb * rows + row) * R);
 #pragma unroll
-        for (int j = 0; j < R / 8; ++j) {
-          float x[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            x[e] = __uint_as_float(v[8 * j + e]) + __uint_as_float(v[R + 8 * j + e]);
-          uint4 hi, lo;
-          split8(x, hi, lo);
-          *reinterpret_cast<uint4*>(obox + lane * 128 + ((j ^ (lane & 7)) << 4)) = hi;
-          *reinterpret_cast<uint4*>(obox + lane * 128 + (((R / 8 + j) ^ (lane & 7)) << 4)) = lo;
+          for (int j = 0; j < R / 4; ++j) {
+            float4 q;
+            q.x = __uint_as_float(v[4 * j]) + __uint_as_float(v[R + 4 * j]);
+            q.y = __uint_as_float(v[4 * j + 1]) + __uint_as_float(v[R + 4 * j + 1]);
+            q.z = __uint_as_float(v[4 * j + 2]) + __uint_as_float(v[R + 4 * j + 2]);
+            q.w = __uint_as_float(v[4 * j + 3]) + __uint_as_float(v[R + 4 * j + 3]);
+            dst[j] = q;
+          }
         }
-#pragma unroll
-        for (int j = 2 * R / 8; j < 8; ++j)
-          *reinterpret_cast<uint4*>(obox + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-              make_uint4(0u, 0u, 0u, 0u);
-        fence_async_smem();
-        __syncwarp();
-        if (lane == 0) {
-          if (y < rows) tma_store_2d(&tm_o, 0, y, obox);
-          bulk_commit();
-        }
-        __syncwarp();
       } else {
         // 64 columns of Y at a time, alternating between the warp's two boxes
 #pragma unroll 1
@@ -337,38 +345,75 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
   }
 }
 
-// P_K[k][j] = P_HL[p_row0 + j][k] for k < 2r (rows [P_hi ; P_lo]), j < n: a 64 x 64 tile
-// per CTA through shared memory.
+// P_K of every matrix: P_K_i[k][j] = P_HL[p_row0_i + j][k] for k < 2r (rows [P_hi ; P_lo])
+// and j < n_i, at pk_off[i] with row stride ld_i = n_i rounded up to 64.  One CTA per
+// projection unit (matrix, 128 columns j), through shared memory.
 __global__ void __launch_bounds__(256)
-transpose_p_kernel(const __nv_bfloat16* __restrict__ p_hl, int64_t p_row0, int hl_width, int n,
-                   int r2, __nv_bfloat16* __restrict__ p_k, int64_t ld_k) {
-  __shared__ __nv_bfloat16 t[64][66];
-  const int j0 = blockIdx.x * 64;
-  for (int e = threadIdx.x; e < 64 * 64; e += blockDim.x) {
+transpose_p_kernel(const __nv_bfloat16* __restrict__ p_hl, const TcMat* __restrict__ tcm,
+                   const int2* __restrict__ units, const int64_t* __restrict__ pk_off,
+                   int hl_width, int r2, __nv_bfloat16* __restrict__ p_k) {
+  __shared__ __nv_bfloat16 t[128][66];
+  const int2 u = units[blockIdx.x];
+  const int64_t n = tcm[u.x].n;
+  const int64_t p_row0 = tcm[u.x].p_row0;
+  const int64_t ld = (n + 63) / 64 * 64;
+  const int64_t j0 = u.y;
+  __nv_bfloat16* dst = p_k + pk_off[u.x];
+  for (int e = threadIdx.x; e < 128 * 64; e += blockDim.x) {
     const int jj = e / 64, k = e % 64;
     t[jj][k] = (j0 + jj < n && k < r2) ? p_hl[(p_row0 + j0 + jj) * hl_width + k]
                                        : __float2bfloat16_rn(0.f);
   }
   __syncthreads();
-  for (int e = threadIdx.x; e < 64 * 64; e += blockDim.x) {
-    const int k = e / 64, jj = e % 64;
-    if (k < r2 && j0 + jj < n) p_k[(int64_t)k * ld_k + j0 + jj] = t[jj][k];
+  for (int e = threadIdx.x; e < 128 * 64; e += blockDim.x) {
+    const int k = e / 128, jj = e % 128;
+    if (k < r2 && j0 + jj < n) dst[(int64_t)k * ld + j0 + jj] = t[jj][k];
   }
+}
+
+// S_HL[row] = [hi | lo | 0] of the sum over the K ranges of the fp32 partial rows of S:
+// thread (row, g) adds columns 8 g .. 8 g + 7 and writes their hi and lo chunks (g = 0
+// also the zero chunks past 2R).
+template <int R>
+__global__ void __launch_bounds__(128)
+reduce_s_kernel(const float* __restrict__ part, int rows, int k_split,
+                __nv_bfloat16* __restrict__ s_hl) {
+  constexpr int kGroups = R / 8;
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)rows * kGroups) return;
+  const int row = (int)(idx / kGroups), g = (int)(idx % kGroups);
+  float x[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) x[e] = 0.f;
+  for (int ks = 0; ks < k_split; ++ks) {
+    const float4* src = reinterpret_cast<const float4*>(part + ((int64_t)ks * rows + row) * R + 8 * g);
+    const float4 a = src[0], b = src[1];
+    x[0] += a.x; x[1] += a.y; x[2] += a.z; x[3] += a.w;
+    x[4] += b.x; x[5] += b.y; x[6] += b.z; x[7] += b.w;
+  }
+  uint4 hi, lo;
+  split8(x, hi, lo);
+  uint4* out = reinterpret_cast<uint4*>(s_hl + (int64_t)row * 64);
+  out[g] = hi;
+  out[kGroups + g] = lo;
+  if (g == 0)
+    for (int z = 2 * kGroups; z < 8; ++z) out[z] = make_uint4(0u, 0u, 0u, 0u);
 }
 
 template <int kMode, int R>
 cudaError_t launch_linear_r(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
                             const CUtensorMap* w_map, const CUtensorMap& tm_s,
                             const CUtensorMap& tm_u, const CUtensorMap& tm_o, int rows, int cols,
-                            int k_steps, int u_row0, int grid, uint32_t* d_status,
-                            cudaStream_t s) {
+                            int k_steps, int k_split, int k_chunk, int u_row0, float* part,
+                            int grid, uint32_t* d_status, cudaStream_t s) {
   using Cfg = LinCfg<kMode, R>;
   cudaError_t e = cudaFuncSetAttribute(linear_kernel<kMode, R>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)Cfg::kSmem);
   if (e != cudaSuccess) return e;
   linear_kernel<kMode, R><<<grid, kLinThreads, Cfg::kSmem, s>>>(
-      tm_a, tm_b, w_map, tm_s, tm_u, tm_o, rows, cols, k_steps, u_row0, d_status, kWaitCycles);
+      tm_a, tm_b, w_map, tm_s, tm_u, tm_o, rows, cols, k_steps, k_split, k_chunk, u_row0, part,
+      d_status, kWaitCycles);
   return cudaGetLastError();
 }
 
@@ -376,40 +421,66 @@ cudaError_t launch_linear_r(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
 
 bool linear_supported(int32_t r) { return r == 16 || r == 32; }
 
-int32_t linear_tiles(int64_t rows, int64_t cols, bool s_gemm, int32_t r) {
-  const int64_t n = s_gemm ? 2 * r : 256;
-  return (int32_t)(((rows + kBM - 1) / kBM) * ((cols + n - 1) / n));
+void linear_s_split(int64_t T, int64_t n, int32_t sms, int32_t* k_split, int32_t* k_chunk) {
+  const int64_t k_steps = (n + 63) / 64;
+  const int64_t blocks = (T + kBM - 1) / kBM;
+  int64_t want = std::max<int64_t>(1, std::min<int64_t>(k_steps, (sms + blocks - 1) / blocks));
+  const int64_t chunk = (k_steps + want - 1) / want;
+  *k_chunk = (int32_t)chunk;
+  *k_split = (int32_t)((k_steps + chunk - 1) / chunk);   // every K range non-empty
 }
 
-cudaError_t launch_transpose_p(const __nv_bfloat16* p_hl, int64_t p_row0, int32_t hl_width,
-                               int64_t n, int32_t r, __nv_bfloat16* p_k, int64_t ld_k,
-                               cudaStream_t s) {
-  if (n <= 0) return cudaSuccess;
-  transpose_p_kernel<<<(unsigned)((n + 63) / 64), 256, 0, s>>>(p_hl, p_row0, hl_width, (int)n,
-                                                              2 * r, p_k, ld_k);
+int32_t linear_y_tiles(int64_t T, int64_t m) {
+  return (int32_t)(((T + kBM - 1) / kBM) * ((m + 255) / 256));
+}
+
+int64_t linear_pk_elems(int64_t n, int32_t r) { return 2 * (int64_t)r * ((n + 63) / 64 * 64); }
+
+cudaError_t launch_transpose_p(const __nv_bfloat16* p_hl, const TcMat* d_tc, const int2* d_units,
+                               int32_t n_units, const int64_t* d_pk_off, int32_t hl_width,
+                               int32_t r, __nv_bfloat16* p_k, cudaStream_t s) {
+  if (n_units <= 0) return cudaSuccess;
+  transpose_p_kernel<<<n_units, 256, 0, s>>>(p_hl, d_tc, d_units, d_pk_off, hl_width, 2 * r, p_k);
   return cudaGetLastError();
 }
 
-cudaError_t launch_linear_s(const CUtensorMap& tm_x, const CUtensorMap& tm_pk,
-                            const CUtensorMap& tm_s_out, int64_t T, int64_t n, int32_t r,
-                            int32_t grid, uint32_t* d_status, cudaStream_t s) {
+cudaError_t launch_linear_s(const CUtensorMap& tm_x, const CUtensorMap& tm_pk, int64_t T,
+                            int64_t n, int32_t r, int32_t k_split, int32_t k_chunk, float* part,
+                            __nv_bfloat16* s_hl, int32_t sms, uint32_t* d_status,
+                            cudaStream_t s) {
   const int k_steps = (int)((n + 63) / 64);
+  const int tiles = (int)((T + kBM - 1) / kBM) * k_split;
+  const int grid = std::min<int>(tiles, sms);
+  cudaError_t e;
   switch (r) {
-    case 16: return launch_linear_r<kModeS, 16>(tm_x, tm_pk, nullptr, tm_x, tm_x, tm_s_out, (int)T, 32, k_steps, 0, grid, d_status, s);
-    case 32: return launch_linear_r<kModeS, 32>(tm_x, tm_pk, nullptr, tm_x, tm_x, tm_s_out, (int)T, 64, k_steps, 0, grid, d_status, s);
+    case 16:
+      e = launch_linear_r<kModeS, 16>(tm_x, tm_pk, nullptr, tm_x, tm_x, tm_x, (int)T, 32, k_steps,
+                                       k_split, k_chunk, 0, part, grid, d_status, s);
+      if (e == cudaSuccess)
+        reduce_s_kernel<16><<<(unsigned)((T * 2 + 127) / 128), 128, 0, s>>>(part, (int)T, k_split, s_hl);
+      break;
+    case 32:
+      e = launch_linear_r<kModeS, 32>(tm_x, tm_pk, nullptr, tm_x, tm_x, tm_x, (int)T, 64, k_steps,
+                                       k_split, k_chunk, 0, part, grid, d_status, s);
+      if (e == cudaSuccess)
+        reduce_s_kernel<32><<<(unsigned)((T * 4 + 127) / 128), 128, 0, s>>>(part, (int)T, k_split, s_hl);
+      break;
     default: return cudaErrorInvalidValue;
   }
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
 }
 
 cudaError_t launch_linear_y(const CUtensorMap& tm_x, const CUtensorMap* d_w_map,
                             const CUtensorMap& tm_s_in, const CUtensorMap& tm_u,
                             const CUtensorMap& tm_y, int64_t T, int64_t m, int64_t n,
-                            int32_t u_row0, int32_t r, int32_t grid, uint32_t* d_status,
+                            int32_t u_row0, int32_t r, int32_t sms, uint32_t* d_status,
                             cudaStream_t s) {
   const int k_steps = (int)((n + 63) / 64);
+  const int grid = std::min<int>(linear_y_tiles(T, m), sms);
   switch (r) {
-    case 16: return launch_linear_r<kModeY, 16>(tm_x, tm_x, d_w_map, tm_s_in, tm_u, tm_y, (int)T, (int)m, k_steps, u_row0, grid, d_status, s);
-    case 32: return launch_linear_r<kModeY, 32>(tm_x, tm_x, d_w_map, tm_s_in, tm_u, tm_y, (int)T, (int)m, k_steps, u_row0, grid, d_status, s);
+    case 16: return launch_linear_r<kModeY, 16>(tm_x, tm_x, d_w_map, tm_s_in, tm_u, tm_y, (int)T, (int)m, k_steps, 1, k_steps, u_row0, nullptr, grid, d_status, s);
+    case 32: return launch_linear_r<kModeY, 32>(tm_x, tm_x, d_w_map, tm_s_in, tm_u, tm_y, (int)T, (int)m, k_steps, 1, k_steps, u_row0, nullptr, grid, d_status, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -66,13 +66,14 @@ def test_perturbed_linear_matches_oracle_and_leaves_W(lib, gpu, case, eps):
     before = snapshot(z)
     W_bits = [W.detach().clone() for W in z.weights]
     terms = [(1, 1.0), (2, -1.0)]
+    zb.zo_linear_prepare(z.ctx, 5, 1, 1.0, 2, -1.0, eps)
     for i, (m, n, _) in enumerate(spec):
         for T in tokens:
             X = _tokens(T, n, 17 * T + i, gpu)
             ldy = (m + 7) // 8 * 8
             Ybuf = torch.full((T, ldy), float("nan"), dtype=torch.bfloat16, device=gpu)
             Y = Ybuf[:, :m]
-            zb.zo_linear_perturbed(z.ctx, i, X, Y, 5, 1, 1.0, 2, -1.0, eps)
+            zb.zo_linear_perturbed(z.ctx, i, X, Y)
             z.sync()
             C = subzero.perturb_coeff(z.seed, base + i, 5, r, terms, f32(eps))
             zc = abs(f32(eps)) * 2.0
@@ -93,13 +94,18 @@ def test_perturbed_linear_single_query_and_repeat(lib, gpu):
     from paper_2608_15665_gb300 import binding as zb
     z, base = _context(gpu, "r32", seed=99)
     r, spec, _ = LINEAR_CASES["r32"]
-    before = snapshot(z)
     m, n, _ = spec[1]
     X = _tokens(64, n, 3, gpu)
     Y1 = torch.empty((64, m), dtype=torch.bfloat16, device=gpu)
     Y2 = torch.empty_like(Y1)
-    zb.zo_linear_perturbed(z.ctx, 1, X, Y1, 0, 3, -2.0, -1, 0.0, 1e-2)
-    zb.zo_linear_perturbed(z.ctx, 1, X, Y2, 0, 3, -2.0, -1, 0.0, 1e-2)
+    zb.zo_linear_prepare(z.ctx, 0, 3, -2.0, -1, 0.0, 1e-2)
+    # a weight pass after the prepare rewrites W and the pass's own C / P workspace; the
+    # prepared coefficient stays, and the layer sees the new W
+    z.perturb(7, 0, 1.0, -1, 0.0, 1e-3)
+    z.sync()
+    before = snapshot(z)
+    zb.zo_linear_perturbed(z.ctx, 1, X, Y1)
+    zb.zo_linear_perturbed(z.ctx, 1, X, Y2)
     z.sync()
     assert torch.equal(Y1.view(torch.int16), Y2.view(torch.int16))   # deterministic
     C = subzero.perturb_coeff(z.seed, base + 1, 0, r, [(3, -2.0)], f32(1e-2))
@@ -115,23 +121,27 @@ def test_perturbed_linear_rejections(lib, gpu):
     X = _tokens(8, 520, 1, gpu)
     Y = torch.empty((8, 304), dtype=torch.bfloat16, device=gpu)
     with pytest.raises(RuntimeError):
-        zb.zo_linear_perturbed(z.ctx, 3, X, Y, 0, 0, 1.0, -1, 0.0, 1e-3)            # no matrix 3
+        zb.zo_linear_perturbed(z.ctx, 0, X, Y)                                     # not prepared
     with pytest.raises(RuntimeError):
-        zb.zo_linear_perturbed(z.ctx, 0, X, Y, 0, 4, 1.0, -1, 0.0, 1e-3)            # query 4 of 4
+        zb.zo_linear_prepare(z.ctx, 0, 4, 1.0, -1, 0.0, 1e-3)                      # query 4 of 4
+    zb.zo_linear_prepare(z.ctx, 0, 0, 1.0, -1, 0.0, 1e-3)
+    with pytest.raises(RuntimeError):
+        zb.zo_linear_perturbed(z.ctx, 3, X, Y)                                     # no matrix 3
     Ybad = torch.empty((8, 312), dtype=torch.bfloat16, device=gpu)[:, 1:305]       # misaligned
     with pytest.raises(RuntimeError):
-        zb.zo_linear_perturbed(z.ctx, 0, X, Ybad, 0, 0, 1.0, -1, 0.0, 1e-3)
+        zb.zo_linear_perturbed(z.ctx, 0, X, Ybad)
     z.close()
     # an output width that is not a multiple of 8 (TMA stores write 16-byte chunks)
     w = [make_weight(300, 520, "bf16", 2, gpu)]
     zo = SubZeroPlus(w, 32, 4, 1)
     zo.init_subspace(0)
+    zb.zo_linear_prepare(zo.ctx, 0, 0, 1.0, -1, 0.0, 1e-3)
     with pytest.raises(RuntimeError):
-        zb.zo_linear_perturbed(zo.ctx, 0, X, Y[:, :300], 0, 0, 1.0, -1, 0.0, 1e-3)
+        zb.zo_linear_perturbed(zo.ctx, 0, X, Y[:, :300])
     zo.close()
     w = [make_weight(304, 520, "f32", 1, gpu)]
     zf = SubZeroPlus(w, 32, 4, 1)
     zf.init_subspace(0)
     with pytest.raises(RuntimeError):                                             # FMA path
-        zb.zo_linear_perturbed(zf.ctx, 0, X, Y, 0, 0, 1.0, -1, 0.0, 1e-3)
+        zb.zo_linear_prepare(zf.ctx, 0, 0, 1.0, -1, 0.0, 1e-3)
     zf.close()
