@@ -19,8 +19,9 @@
 //           ~2^-16 of the rank-r term); N = 256 columns of Y per tile; the epilogue
 //           rounds to bf16 and TMA-stores Y.
 // P_K is P_HL (the projection's rows [P_hi(j, :) | P_lo(j, :)], j < n) transposed by
-// transpose_p_kernel, for every matrix once per loss evaluation (zo_linear_prepare).  Ragged edges: TMA zero-fills loads past T, n and m and clips
-// stores.
+// transpose_p_kernel, for every matrix once per loss evaluation (zo_linear_prepare).
+// Ragged edges: TMA zero-fills loads past T, n and m; Y's stores are clipped to T rows and
+// m columns (m a multiple of 8, so that no 16-byte chunk reaches past Y's columns).
 //
 // Roles of the 192 threads of a CTA:
 //   warp 0, lane 0: TMA producer -- per K step one X box (64 x 128 rows) and the B rows
@@ -29,8 +30,8 @@
 //   warp 1, lane 0: MMA issuer (4 x K = 16 per K step, 3r/16 for the extension) into
 //                   one of two TMEM accumulators; warp 1 also owns TMEM.
 //   warps 2..5:     epilogue -- warp w owns rows 32 (w % 4) .. + 31 of the tile (its
-//                   TMEM lane group) and stores them 64 columns at a time through two
-//                   staged 32 x 64 boxes.
+//                   TMEM lane group); kModeY stores them 64 columns at a time through two
+//                   staged 32 x 64 boxes (TMA), kModeS writes its fp32 partial rows.
 // Every mbarrier wait is bounded; on expiry the kernel records kDevTimeout in the status
 // word, lets the other roles stop, drains its copies and frees TMEM.
 #include <algorithm>
