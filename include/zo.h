@@ -210,7 +210,8 @@ ZO_API zo_status zo_mezo_perturb(zo_ctx* ctx, uint32_t t, float coef);
  * zo_linear_prepare -- once per loss evaluation: C_i = eps (ca Z_i^(qa) + cb Z_i^(qb)) at
  *   step t (qb = -1: one term) for every matrix -- the coefficient zo_perturb(ctx, t, qa,
  *   ca, qb, cb, eps) would add to W_i -- and P_i = C_i V_i^T, kept for the calls below
- *   until the next zo_linear_prepare.
+ *   until the next zo_linear_prepare; zo_refresh (new U, V) discards it, and
+ *   zo_linear_perturbed then returns ZO_ERR_INVALID_ARG until the next prepare.
  * zo_linear_perturbed -- one layer: Y = X (W_i + U_i C_i V_i^T)^T = X W_i^T +
  *   (X V_i C_i^T) U_i^T.  X: T x n_i bf16, row stride ldx elements; Y: T x m_i bf16, row
  *   stride ldy (device, caller-owned, 16-byte aligned, strides multiples of 8; m_i a

@@ -683,6 +683,7 @@ zo_status zo_destroy(zo_ctx* c) {
 zo_status zo_refresh(zo_ctx* c, uint32_t refresh_idx, int32_t reset_moments) {
   if (!c) return ZO_ERR_INVALID_ARG;
   DeviceGuard guard(c->device);
+  c->linear_ready = false;   // a prepared P_K belongs to the old V
   const int n_levels = (int)c->up_off.size();
   for (int lv = 0; lv < n_levels; ++lv) {
     if (c->up_cnt[lv] == 0) continue;

@@ -127,6 +127,10 @@ def test_perturbed_linear_rejections(lib, gpu):
     zb.zo_linear_prepare(z.ctx, 0, 0, 1.0, -1, 0.0, 1e-3)
     with pytest.raises(RuntimeError):
         zb.zo_linear_perturbed(z.ctx, 3, X, Y)                                     # no matrix 3
+    z.refresh(1)                                                                   # new U, V
+    with pytest.raises(RuntimeError):
+        zb.zo_linear_perturbed(z.ctx, 0, X, Y)                                     # stale P
+    zb.zo_linear_prepare(z.ctx, 0, 0, 1.0, -1, 0.0, 1e-3)
     Ybad = torch.empty((8, 312), dtype=torch.bfloat16, device=gpu)[:, 1:305]       # misaligned
     with pytest.raises(RuntimeError):
         zb.zo_linear_perturbed(z.ctx, 0, X, Ybad)
