@@ -524,6 +524,15 @@ def run_linear(args):
     clk = clocks.stop()
     launches = zb.zo_kernel_launches(z.ctx) - launches0
     z.sync()
+    tile_rows = []
+    for i, (m, n) in enumerate(wl.shapes):
+        zb.zo_linear_perturbed(z.ctx, i, X[n], Y[i])
+        tile_rows.append(zb.zo_linear_tile_rows(z.ctx))
+    # for context: the same route with 128-row tiles throughout
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 1)
+    fused128_ms = timed(fused, K)
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 0)
+    z.sync()
     plain_ms = timed(lambda k: plain(), K)
     wpass_ms = timed(lambda k: (z.perturb(k, 0, 1.0, -1, 0.0, wl.eps), plain()), K)
     z.sync()
@@ -561,12 +570,13 @@ def run_linear(args):
         "ms_per_step": fused_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic",
         "config": {"workload": wl.name, "matrices": wl.n_mats, "tokens": T, "r": wl.r,
-                   "method": "linear",
+                   "method": "linear", "tile_rows": tile_rows,
                    "l2": "inputs larger than L2 (%.0f MB of weights)" % (sum(m * n for m, n in wl.shapes) * 2 / 1e6),
                    "parallelism": "single GPU"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "peak_kind": peak_kind, "traffic": None,
                      "kernel": "linear_kernel", "algorithmic_flops_per_step": flops},
+        "tile128_ms": fused128_ms,
         "plain_gemm_ms": plain_ms,
         "weight_pass_route_ms": wpass_ms,
         "e2e": {"value": flops / e2e_s / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": int(h2d),

@@ -36,6 +36,7 @@ ZO_OPT_SGD = 1
 ZO_OPTION_WPASS_PATH = 0
 ZO_OPTION_TIMING = 1
 ZO_OPTION_TEST_WAIT_TIMEOUT = 2
+ZO_OPTION_LINEAR_TILE = 3
 
 
 class ZoError(RuntimeError):
@@ -81,6 +82,7 @@ _SIGNATURES = {
     "zo_set_option": (_c.c_int32, [_c.c_void_p, _c.c_int32, _c.c_int64]),
     "zo_get_timing": (_c.c_int32, [_c.c_void_p, _c.POINTER(_c.c_double), _c.POINTER(_c.c_int64)]),
     "zo_wpass_path": (_c.c_int32, [_c.c_void_p]),
+    "zo_linear_tile_rows": (_c.c_int32, [_c.c_void_p]),
     "zo_kernel_launches": (_c.c_int64, [_c.c_void_p]),
     "zo_philox_fill": (_c.c_int32, [_c.c_uint64, _c.c_uint32, _c.c_uint32, _c.c_uint32,
                                     _c.c_void_p, _c.c_int64, _c.c_void_p]),
@@ -239,6 +241,10 @@ def zo_get_timing(ctx):
 
 def zo_wpass_path(ctx):
     return int(LIB.zo_wpass_path(ctx))
+
+
+def zo_linear_tile_rows(ctx):
+    return int(LIB.zo_linear_tile_rows(ctx))
 
 
 def zo_kernel_launches(ctx):

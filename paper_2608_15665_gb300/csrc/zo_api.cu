@@ -116,8 +116,11 @@ struct zo_ctx {
   int64_t* d_pk_off = nullptr;
   std::vector<int64_t> h_pk_off;
   bool linear_ready = false;
+  int linear_tile = 0;           // ZO_OPTION_LINEAR_TILE
+  int last_linear_rows = 0;      // rows per tile of the last Y GEMM
   __nv_bfloat16* d_s_hl = nullptr;
   float* d_s_part = nullptr;
+  uint32_t* d_s_count = nullptr;   // one counter per 32 rows of S_HL's capacity
   int64_t s_cap = 0, part_cap = 0;
   int64_t tc_tiles = 0;
   CUtensorMap* d_w_maps = nullptr;   // one TMA descriptor per W_i (device memory)
@@ -159,6 +162,7 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_pk_off);
   cudaFree(c->d_s_hl);
   cudaFree(c->d_s_part);
+  cudaFree(c->d_s_count);
   cudaFree(c->d_w_maps);
   cudaFree(c->d_u_units);
   cudaFree(c->d_v_hl);
@@ -927,10 +931,14 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
     if (T > c->s_cap) {
       cudaFree(c->d_s_hl);
+      cudaFree(c->d_s_count);
       c->d_s_hl = nullptr;
+      c->d_s_count = nullptr;
       c->s_cap = 0;
       const int64_t cap = (T + 127) / 128 * 128;
       ZO_CUDA(cudaMalloc(&c->d_s_hl, sizeof(__nv_bfloat16) * cap * HLW), "cudaMalloc(S_HL)");
+      ZO_CUDA(cudaMalloc(&c->d_s_count, sizeof(uint32_t) * (cap / 32)), "cudaMalloc(S counters)");
+      ZO_CUDA(cudaMemset(c->d_s_count, 0, sizeof(uint32_t) * (cap / 32)), "zero S counters");
       c->s_cap = cap;
     }
     if (part > c->part_cap) {
@@ -952,14 +960,16 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     g_last_error = "zo_linear_perturbed: cuTensorMapEncodeTiled rejected a descriptor";
     return ZO_ERR_CUDA;
   }
-  // S = X P^T (split K, then the partial sums reduced into S_HL), Y = X W^T + S U^T
+  // S = X P^T (split K, the partial sums reduced into S_HL), Y = X W^T + S U^T
   ZO_CUDA(zo::launch_linear_s(tm_x, tm_pk, T, n, r, k_split, k_chunk, c->d_s_part, c->d_s_hl,
-                              c->sms, c->d_status, c->stream),
+                              c->d_s_count, c->sms, c->d_status, c->stream),
           "S = X P^T kernels");
+  const int32_t rows = zo::linear_y_rows(T, m, c->sms, c->linear_tile);
   ZO_CUDA(zo::launch_linear_y(tm_x, c->d_w_maps + mat, tm_s, c->tm_a, tm_y, T, m, n,
-                              c->h_tc[mat].u_row0, r, c->sms, c->d_status, c->stream),
+                              c->h_tc[mat].u_row0, r, rows, c->sms, c->d_status, c->stream),
           "perturbed linear kernel");
-  c->launches += 3;
+  c->last_linear_rows = rows;
+  c->launches += 1 + zo::linear_s_launches(k_split);
   return ZO_OK;
 }
 
@@ -994,6 +1004,10 @@ zo_status zo_sync_status(zo_ctx* c) {
   if (s != 0) {
     ZO_CUDA(cudaMemset(c->d_status, 0, sizeof(uint32_t)), "clear status");
     if (s & zo::kDevTimeout) {
+      // a perturbed-linear S kernel cut short can leave its group counters part-counted
+      if (c->d_s_count)
+        ZO_CUDA(cudaMemset(c->d_s_count, 0, sizeof(uint32_t) * (c->s_cap / 32)),
+                "zero S counters");
       g_last_error = "a device-side wait ran out";
       return ZO_ERR_TIMEOUT;
     }
@@ -1031,6 +1045,11 @@ zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
     c->inject_wait = value != 0;
     return ZO_OK;
   }
+  if (option == ZO_OPTION_LINEAR_TILE) {
+    if (value < 0 || value > 2) return ZO_ERR_INVALID_ARG;
+    c->linear_tile = (int)value;
+    return ZO_OK;
+  }
   if (option == ZO_OPTION_TIMING) {
     if (value != 0 && value != 1) return ZO_ERR_INVALID_ARG;
     ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
@@ -1060,6 +1079,8 @@ zo_status zo_get_timing(zo_ctx* c, double* total_ms, int64_t* launches) {
 }
 
 int32_t zo_wpass_path(const zo_ctx* c) { return c ? c->last_path : 0; }
+
+int32_t zo_linear_tile_rows(const zo_ctx* c) { return c ? c->last_linear_rows : 0; }
 
 int64_t zo_kernel_launches(const zo_ctx* c) { return c ? c->launches : 0; }
 

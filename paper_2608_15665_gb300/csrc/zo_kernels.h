@@ -140,27 +140,35 @@ cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
 bool linear_supported(int32_t r);
 // The S GEMM's split of K = n into k_split ranges of k_chunk steps of 64 (~ one wave).
 void linear_s_split(int64_t T, int64_t n, int32_t sms, int32_t* k_split, int32_t* k_chunk);
-int32_t linear_y_tiles(int64_t T, int64_t m);
+// Rows of X per tile of the Y GEMM, 128 or 256: option 1 / 2 force one; 0 takes the
+// tiling with fewer waves of tiles over the SMs (a 256 x 256 tile costs ~1.6 of the
+// 128 x 256 one).
+int32_t linear_y_rows(int64_t T, int64_t m, int32_t sms, int32_t option);
 // Elements of matrix i's P_K: 2r rows of n rounded up to 64.
 int64_t linear_pk_elems(int64_t n, int32_t r);
 // P_K of every matrix from P_HL (units = the projection units, pk_off = element offsets).
 cudaError_t launch_transpose_p(const __nv_bfloat16* p_hl, const TcMat* d_tc, const int2* d_units,
                                int32_t n_units, const int64_t* d_pk_off, int32_t hl_width,
                                int32_t r, __nv_bfloat16* p_k, cudaStream_t s);
+// Kernels launch_linear_s launches for a split of k_split K ranges (1, or 2 with the
+// separate reduction).
+int32_t linear_s_launches(int32_t k_split);
 // S_HL rows [S_hi | S_lo | 0] of S = X P^T: tm_x over X (box 64 x 128), tm_pk over P_K
-// (box 64 x 2r); part = k_split x T x r fp32 workspace.
+// (box 64 x 2r); part = k_split x T x r fp32 workspace; s_count = one counter per 32 rows
+// of X, zero before the launch and zero again after it (a launch cut short by a wait
+// timeout can leave counts behind: zero them before the next).
 cudaError_t launch_linear_s(const CUtensorMap& tm_x, const CUtensorMap& tm_pk, int64_t T,
                             int64_t n, int32_t r, int32_t k_split, int32_t k_chunk, float* part,
-                            __nv_bfloat16* s_hl, int32_t sms, uint32_t* d_status,
-                            cudaStream_t s);
+                            __nv_bfloat16* s_hl, uint32_t* s_count, int32_t sms,
+                            uint32_t* d_status, cudaStream_t s);
 // Y = X W^T + S U^T: d_w_map = W's descriptor (box 64 x 32), tm_s_in over S_HL (box
 // 64 x 128), tm_u over the U operand (box 64 x 128; W's rows from u_row0), tm_y over Y
-// (box 64 x 32).
+// (box 64 x 32); tile_rows from linear_y_rows.
 cudaError_t launch_linear_y(const CUtensorMap& tm_x, const CUtensorMap* d_w_map,
                             const CUtensorMap& tm_s_in, const CUtensorMap& tm_u,
                             const CUtensorMap& tm_y, int64_t T, int64_t m, int64_t n,
-                            int32_t u_row0, int32_t r, int32_t sms, uint32_t* d_status,
-                            cudaStream_t s);
+                            int32_t u_row0, int32_t r, int32_t tile_rows, int32_t sms,
+                            uint32_t* d_status, cudaStream_t s);
 
 // ---- refresh of tall panels at r = 16 ... 128: CholeskyQR2 (zo_cholqr.cu) ----------
 constexpr int32_t kCqChunkRows = 1024;   // rows per partial Gram matrix

@@ -10,28 +10,42 @@
 //   kModeS  partial S = X P^T over a range of K with B = [P_hi ; P_lo] (2r rows, K-major,
 //           from P_K): N = 2r, tiles = (128 rows of X) x (K range) so that a few row
 //           blocks still fill the SMs; the epilogue sums the two halves, D[:, :r] +
-//           D[:, r:], and writes the fp32 partial rows; reduce_s_kernel adds the partials
-//           and writes S as bf16 hi/lo rows [S_hi | S_lo | 0] of 64 elements (S_HL), the
-//           layout of the U operand.
+//           D[:, r:], and writes the fp32 partial rows.  S leaves as bf16 hi/lo rows
+//           [S_hi | S_lo | 0] of 64 elements (S_HL), the layout of the U operand: with a
+//           single K range the epilogue writes S_HL directly; with up to kFusedSplits
+//           ranges the warp that finishes a 32-row group last (a counter per group,
+//           atomicInc wrapping back to 0) adds the group's partials in K-range order;
+//           with more, reduce_s_kernel does (one warp reading 32 x k_split partial rows
+//           would take k_split L2 round trips).
 //   kModeY  Y = X W^T over K = n (single bf16 products, both operands exact in bf16)
 //           followed by one more K step from S_HL and the U operand, with the weight
 //           pass's three products S_hi U_hi + S_hi U_lo + S_lo U_hi (relative error
 //           ~2^-16 of the rank-r term); N = 256 columns of Y per tile; the epilogue
 //           rounds to bf16 and TMA-stores Y.
+//   kModeY2 the same over 256 x 256 tiles: two M = 128 halves of X rows share each
+//           stage's W rows, so a stage (64 KB) carries twice the MMA work of a kModeY
+//           stage (48 KB) -- the operand bytes an SM takes in per flop fall by a third,
+//           and the 3-stage ring covers 1.5x the load latency.  Both halves'
+//           accumulators fill TMEM (2 x 256 columns), so the epilogue of a tile (eight
+//           warps) is not overlapped with the next tile's MMAs; chosen when the wave
+//           count favours it (linear_y_rows).
 // P_K is P_HL (the projection's rows [P_hi(j, :) | P_lo(j, :)], j < n) transposed by
 // transpose_p_kernel, for every matrix once per loss evaluation (zo_linear_prepare).
 // Ragged edges: TMA zero-fills loads past T, n and m; Y's stores are clipped to T rows and
 // m columns (m a multiple of 8, so that no 16-byte chunk reaches past Y's columns).
 //
-// Roles of the 192 threads of a CTA:
-//   warp 0, lane 0: TMA producer -- per K step one X box (64 x 128 rows) and the B rows
-//                   (W: N/32 boxes of 64 x 32; P_K: one box of 64 x 2r), into a ring
-//                   of kStages slots; kModeY ends each tile with the extension step.
-//   warp 1, lane 0: MMA issuer (4 x K = 16 per K step, 3r/16 for the extension) into
-//                   one of two TMEM accumulators; warp 1 also owns TMEM.
-//   warps 2..5:     epilogue -- warp w owns rows 32 (w % 4) .. + 31 of the tile (its
-//                   TMEM lane group); kModeY stores them 64 columns at a time through two
-//                   staged 32 x 64 boxes (TMA), kModeS writes its fp32 partial rows.
+// Roles of the threads of a CTA (192; kModeY2 320):
+//   warp 0, lane 0: TMA producer -- per K step one X box (64 x 128 rows) per half and
+//                   the B rows (W: N/32 boxes of 64 x 32; P_K: one box of 64 x 2r), into
+//                   a ring of kStages slots; the Y modes end each tile with the extension
+//                   step.
+//   warp 1, lane 0: MMA issuer (4 x K = 16 per K step and half, 3r/16 for the extension)
+//                   into one of two TMEM accumulators (kModeY2: the single pair of
+//                   halves); warp 1 also owns TMEM.
+//   warps 2..:      epilogue -- warp w owns rows 32 (w % 4) .. + 31 of a half (its TMEM
+//                   lane group; kModeY2 has eight warps, four per half); the Y modes store
+//                   them 64 columns at a time through staged 32 x 64 boxes (TMA), kModeS
+//                   writes its fp32 partial rows.
 // Every mbarrier wait is bounded; on expiry the kernel records kDevTimeout in the status
 // word, lets the other roles stop, drains its copies and frees TMEM.
 #include <algorithm>
@@ -48,25 +62,54 @@ namespace {
 using namespace sm100;
 using namespace tc;
 
-constexpr int kLinThreads = 192;
+constexpr int kFusedSplits = 4;   // most K ranges whose S partials the S kernel sums itself
 constexpr int kModeS = 0;
 constexpr int kModeY = 1;
+constexpr int kModeY2 = 2;
 
 template <int kMode, int R>
 struct LinCfg {
   static_assert(R == 16 || R == 32, "the U operand rows [hi | lo | 0] exist for r <= 32");
-  static constexpr int kN = kMode == kModeY ? 256 : 2 * R;          // tile columns
-  static constexpr int kStages = 4;
-  static constexpr int kABytes = kBM * 128;                          // 128 rows x 64 bf16
+  static constexpr bool kY = kMode != kModeS;
+  static constexpr int kHalves = kMode == kModeY2 ? 2 : 1;           // 128-row halves per tile
+  static constexpr int kTileRows = kHalves * kBM;
+  static constexpr int kN = kY ? 256 : 2 * R;                        // tile columns
+  static constexpr int kStages = kMode == kModeY2 ? 3 : 4;
+  static constexpr int kAccs = kMode == kModeY2 ? 1 : 2;             // accumulator buffers
+  static constexpr int kAccCols = kHalves * kN;                      // TMEM columns of one
+  static constexpr int kEpiWarps = kMode == kModeY2 ? 8 : 4;
+  static constexpr int kThreads = 64 + 32 * kEpiWarps;
+  static constexpr int kABytes = kTileRows * 128;                    // rows x 64 bf16
   static constexpr int kBBytes = kN * 128;                           // kN rows x 64 bf16
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kBoxBytes = 32 * 128;                         // 32 rows x 64 bf16
-  static constexpr int kOutBytes = 4 * 2 * kBoxBytes;                // two boxes per warp
-  static constexpr int kTmemCols = kN * 2 <= 32 ? 32 : kN * 2;       // two accumulators
+  static constexpr int kBoxesPerWarp = kMode == kModeY2 ? 1 : 2;
+  static constexpr int kOutBytes = kEpiWarps * kBoxesPerWarp * kBoxBytes;
+  static constexpr int kTmemCols = kAccs * kAccCols <= 32 ? 32 : kAccs * kAccCols;
   static constexpr size_t kSmem = (size_t)kStages * kStageBytes + kOutBytes + 1024 + 1024;
   static_assert(kSmem <= 227 * 1024, "shared memory per CTA");
   static_assert(kTmemCols <= 512, "TMEM columns");
+  static_assert(kABytes == kHalves * kPanelBytes, "one 128-row panel per half");
 };
+
+// S_HL row: [hi | lo] of the R sums in chunks of 8, then zero chunks up to 64 elements.
+template <int R>
+__device__ __forceinline__ void write_s_row(__nv_bfloat16* s_hl, int row, const float (&x)[R]) {
+  constexpr int kGroups = R / 8;
+  uint4* out = reinterpret_cast<uint4*>(s_hl + (int64_t)row * 64);
+#pragma unroll
+  for (int g = 0; g < kGroups; ++g) {
+    float c[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) c[e] = x[8 * g + e];
+    uint4 hi, lo;
+    split8(c, hi, lo);
+    out[g] = hi;
+    out[kGroups + g] = lo;
+  }
+#pragma unroll
+  for (int z = 2 * kGroups; z < 8; ++z) out[z] = make_uint4(0u, 0u, 0u, 0u);
+}
 
 struct LinShared {
   uint64_t full[4], empty[4];
@@ -82,16 +125,20 @@ __device__ __forceinline__ void lin_give_up(LinShared& sh, uint32_t* status) {
 }
 
 // tm_a: X (box 64 x 128).  kModeS: tm_b = P_K (box 64 x 2r); K split into k_split
-// ranges of k_chunk steps; fp32 partials to part[(k range) x rows x R].
+// ranges of k_chunk steps; fp32 partials to part[(k range) x rows x R], S_HL rows to
+// s_out, s_count = one zeroed counter per 32 rows (null: partials only, for
+// reduce_s_kernel).
 // kModeY: w_map = W_i (box 64 x 32), tm_s = S_HL (box 64 x 128), tm_u = U operand (box
 // 64 x 128) with this matrix's rows from u_row0, tm_o = Y (box 64 x 32).
 template <int kMode, int R>
-__global__ void __launch_bounds__(kLinThreads, 1)
+__global__ void __launch_bounds__(LinCfg<kMode, R>::kThreads, 1)
 linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
               const CUtensorMap* __restrict__ w_map, const __grid_constant__ CUtensorMap tm_s,
               const __grid_constant__ CUtensorMap tm_u, const __grid_constant__ CUtensorMap tm_o,
               int rows, int cols, int k_steps, int k_split, int k_chunk, int u_row0,
-              float* __restrict__ part, uint32_t* __restrict__ status, long long wait_cycles) {
+              float* __restrict__ part, __nv_bfloat16* __restrict__ s_out,
+              uint32_t* __restrict__ s_count, uint32_t* __restrict__ status,
+              long long wait_cycles) {
   using Cfg = LinCfg<kMode, R>;
   static_assert(sizeof(LinShared) <= 1024, "barrier block");
   constexpr int kN = Cfg::kN;
@@ -103,12 +150,12 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
   LinShared& sh = *reinterpret_cast<LinShared*>(o_smem + Cfg::kOutBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // kModeY: tile = (row block, column block), K = all steps + the extension;
+  // Y modes: tile = (row block, column block), K = all steps + the extension;
   // kModeS: tile = (row block, K range)
-  const int tiles_m = kMode == kModeY ? (cols + kN - 1) / kN : k_split;
-  const int n_tiles = ((rows + kBM - 1) / kBM) * tiles_m;
+  const int tiles_m = Cfg::kY ? (cols + kN - 1) / kN : k_split;
+  const int n_tiles = ((rows + Cfg::kTileRows - 1) / Cfg::kTileRows) * tiles_m;
   auto k_range = [&](int nb, int& kb, int& ke) {
-    if (kMode == kModeY) {
+    if (Cfg::kY) {
       kb = 0;
       ke = k_steps + 1;                                             // + the extension
     } else {
@@ -123,9 +170,9 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
       mbar_init(&sh.full[s], 1);
       mbar_init(&sh.empty[s], 1);
     }
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < Cfg::kAccs; ++s) {
       mbar_init(&sh.acc_full[s], 1);
-      mbar_init(&sh.acc_empty[s], 4);
+      mbar_init(&sh.acc_empty[s], Cfg::kEpiWarps);
     }
     mbar_init(&sh.drain, 1);
     sh.abort_flag = 0;
@@ -167,13 +214,17 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
         uint8_t* a_dst = st_smem + s * Cfg::kStageBytes;
         uint8_t* b_dst = a_dst + Cfg::kABytes;
         mbar_arrive_expect_tx(&sh.full[s], Cfg::kStageBytes);
-        if (kMode == kModeY && k == k_steps) {
+        if (Cfg::kY && k == k_steps) {
           // the extension: S_HL rows of the token block, U operand rows of the W block
-          tma_load_2d(a_dst, &tm_s, 0, tb * kBM, &sh.full[s]);
+          for (int h = 0; h < Cfg::kHalves; ++h)
+            tma_load_2d(a_dst + h * kPanelBytes, &tm_s, 0, tb * Cfg::kTileRows + h * kBM,
+                        &sh.full[s]);
           for (int h = 0; h < kN / kBM; ++h)
             tma_load_2d(b_dst + h * kPanelBytes, &tm_u, 0, u_row0 + nb * kN + h * kBM, &sh.full[s]);
         } else {
-          tma_load_2d(a_dst, &tm_a, 64 * k, tb * kBM, &sh.full[s]);
+          for (int h = 0; h < Cfg::kHalves; ++h)
+            tma_load_2d(a_dst + h * kPanelBytes, &tm_a, 64 * k, tb * Cfg::kTileRows + h * kBM,
+                        &sh.full[s]);
           if constexpr (kMode == kModeS) {
             tma_load_2d(b_dst, &tm_b, 64 * k, 0, &sh.full[s]);
           } else {
@@ -196,14 +247,14 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
     int64_t n_st = 0, it = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++it) {
-      const int acc = (int)(it & 1);
-      if (!mbar_wait_bounded(&sh.acc_empty[acc], (uint32_t)(((it >> 1) & 1) ^ 1), abort,
-                             wait_cycles)) {
+      const int acc = (int)(it % Cfg::kAccs);
+      const int64_t use = it / Cfg::kAccs;
+      if (!mbar_wait_bounded(&sh.acc_empty[acc], (uint32_t)((use & 1) ^ 1), abort, wait_cycles)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const uint32_t d = tmem + (uint32_t)(acc * kN);
+      const uint32_t d0 = tmem + (uint32_t)(acc * Cfg::kAccCols);
       int kb, ke;
       k_range(tile % tiles_m, kb, ke);
       for (int k = kb; k < ke; ++k) {
@@ -214,22 +265,27 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
           break;
         }
         tc_fence_after();
-        const uint32_t a_base = smem_u32(st_smem + s * Cfg::kStageBytes);
-        const uint32_t b_base = a_base + Cfg::kABytes;
-        if (kMode == kModeY && k == k_steps) {
-          // hi chunk kk at element 16 kk of an operand row, lo chunk at R + 16 kk
+        const uint32_t st_base = smem_u32(st_smem + s * Cfg::kStageBytes);
+        const uint32_t b_base = st_base + Cfg::kABytes;
 #pragma unroll
-          for (int kk = 0; kk < R / 16; ++kk) {
-            const uint32_t hi = (uint32_t)(16 * kk * 2), lo = (uint32_t)((R + 16 * kk) * 2);
-            mma_bf16(d, sdesc_k_sw128(a_base + hi), sdesc_k_sw128(b_base + hi), idesc, 1u);
-            mma_bf16(d, sdesc_k_sw128(a_base + hi), sdesc_k_sw128(b_base + lo), idesc, 1u);
-            mma_bf16(d, sdesc_k_sw128(a_base + lo), sdesc_k_sw128(b_base + hi), idesc, 1u);
+        for (int h = 0; h < Cfg::kHalves; ++h) {
+          const uint32_t d = d0 + (uint32_t)(h * kN);
+          const uint32_t a_base = st_base + (uint32_t)(h * kPanelBytes);
+          if (Cfg::kY && k == k_steps) {
+            // hi chunk kk at element 16 kk of an operand row, lo chunk at R + 16 kk
+#pragma unroll
+            for (int kk = 0; kk < R / 16; ++kk) {
+              const uint32_t hi = (uint32_t)(16 * kk * 2), lo = (uint32_t)((R + 16 * kk) * 2);
+              mma_bf16(d, sdesc_k_sw128(a_base + hi), sdesc_k_sw128(b_base + hi), idesc, 1u);
+              mma_bf16(d, sdesc_k_sw128(a_base + hi), sdesc_k_sw128(b_base + lo), idesc, 1u);
+              mma_bf16(d, sdesc_k_sw128(a_base + lo), sdesc_k_sw128(b_base + hi), idesc, 1u);
+            }
+          } else {
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              mma_bf16(d, sdesc_k_sw128(a_base + 32 * kk), sdesc_k_sw128(b_base + 32 * kk), idesc,
+                       (k > kb || kk > 0) ? 1u : 0u);
           }
-        } else {
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            mma_bf16(d, sdesc_k_sw128(a_base + 32 * kk), sdesc_k_sw128(b_base + 32 * kk), idesc,
-                     (k > kb || kk > 0) ? 1u : 0u);
         }
         mma_commit(&sh.empty[s]);
         ++n_st;
@@ -244,35 +300,38 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
       mma_commit(&sh.drain);
       mbar_wait_bounded(&sh.drain, 0u, nullptr, wait_cycles);
     }
-  } else if (warp >= 2 && warp <= 5) {
+  } else if (warp >= 2 && warp < 2 + Cfg::kEpiWarps) {
     // ------------------------------------------------------------ epilogue
     const int g = warp & 3;                      // TMEM lane group == rows 32 g .. + 31
+    const int half = (warp - 2) / 4;             // of the tile's 128-row halves
     const uint32_t lane_base = (uint32_t)(g * 32) << 16;
-    uint8_t* obox = o_smem + g * 2 * Cfg::kBoxBytes;
+    uint8_t* obox = o_smem + (warp - 2) * Cfg::kBoxesPerWarp * Cfg::kBoxBytes;
     int64_t it = 0, n_box = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++it) {
       const int tb = tile / tiles_m, nb = tile % tiles_m;   // kModeS: nb = the K range
-      const int acc = (int)(it & 1);
-      if (!mbar_wait_bounded(&sh.acc_full[acc], (uint32_t)((it >> 1) & 1), abort, wait_cycles)) {
+      const int acc = (int)(it % Cfg::kAccs);
+      const int64_t use = it / Cfg::kAccs;
+      if (!mbar_wait_bounded(&sh.acc_full[acc], (uint32_t)(use & 1), abort, wait_cycles)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const int y = tb * kBM + 32 * g;
+      const int y = tb * Cfg::kTileRows + half * kBM + 32 * g;
+      const uint32_t t_base = tmem + lane_base + (uint32_t)(acc * Cfg::kAccCols + half * kN);
       if constexpr (kMode == kModeS) {
         // partial S over this K range: D[:, :R] + D[:, R:2R], fp32, this lane's row
         uint32_t v[2 * R];
         if constexpr (R == 32) {
           uint32_t a[32], b[32];
-          tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * kN), a);
-          tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * kN + 32), b);
+          tmem_ld_32x32b_x32(t_base, a);
+          tmem_ld_32x32b_x32(t_base + 32u, b);
           tmem_ld_wait();
 #pragma unroll
           for (int e = 0; e < 32; ++e) { v[e] = a[e]; v[32 + e] = b[e]; }
         } else {
           uint32_t a[32];
-          tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * kN), a);
+          tmem_ld_32x32b_x32(t_base, a);
           tmem_ld_wait();
 #pragma unroll
           for (int e = 0; e < 32; ++e) v[e] = a[e];
@@ -281,33 +340,71 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
         __syncwarp();
         if (lane == 0) mbar_arrive(&sh.acc_empty[acc]);
         const int row = y + lane;
-        if (row < rows) {
-          float4* dst = reinterpret_cast<float4*>(part + ((int64_t)nb * rows + row) * R);
+        float x[R];
 #pragma unroll
-          for (int j = 0; j < R / 4; ++j) {
-            float4 q;
-            q.x = __uint_as_float(v[4 * j]) + __uint_as_float(v[R + 4 * j]);
-            q.y = __uint_as_float(v[4 * j + 1]) + __uint_as_float(v[R + 4 * j + 1]);
-            q.z = __uint_as_float(v[4 * j + 2]) + __uint_as_float(v[R + 4 * j + 2]);
-            q.w = __uint_as_float(v[4 * j + 3]) + __uint_as_float(v[R + 4 * j + 3]);
-            dst[j] = q;
+        for (int e = 0; e < R; ++e) x[e] = __uint_as_float(v[e]) + __uint_as_float(v[R + e]);
+        if (k_split == 1) {
+          if (row < rows) {
+#pragma unroll
+            for (int e = 0; e < R; ++e) x[e] = 0.f + x[e];     // as the sum over one range
+            write_s_row<R>(s_out, row, x);
+          }
+        } else {
+          if (row < rows) {
+            float4* dst = reinterpret_cast<float4*>(part + ((int64_t)nb * rows + row) * R);
+#pragma unroll
+            for (int j = 0; j < R / 4; ++j)
+              dst[j] = make_float4(x[4 * j], x[4 * j + 1], x[4 * j + 2], x[4 * j + 3]);
+          }
+          // the last of the k_split warps to finish this 32-row group sums its partials
+          if (s_count != nullptr) {
+            __threadfence();
+            __syncwarp();
+            uint32_t old = 0;
+            if (lane == 0) old = atomicInc(&s_count[tb * 4 + g], (uint32_t)(k_split - 1));
+            old = __shfl_sync(0xffffffffu, old, 0);
+            if (old == (uint32_t)(k_split - 1)) {
+              __threadfence();
+              if (row < rows) {
+#pragma unroll
+                for (int e = 0; e < R; ++e) x[e] = 0.f;
+                for (int ks = 0; ks < k_split; ++ks) {
+                  const float4* src =
+                      reinterpret_cast<const float4*>(part + ((int64_t)ks * rows + row) * R);
+#pragma unroll
+                  for (int j = 0; j < R / 4; ++j) {
+                    const float4 q = __ldcg(src + j);
+                    x[4 * j] += q.x;
+                    x[4 * j + 1] += q.y;
+                    x[4 * j + 2] += q.z;
+                    x[4 * j + 3] += q.w;
+                  }
+                }
+                write_s_row<R>(s_out, row, x);
+              }
+            }
           }
         }
       } else {
-        // 64 columns of Y at a time, alternating between the warp's two boxes
+        // 64 columns of Y at a time, through the warp's box(es) in turn
 #pragma unroll 1
-        for (int h = 0; h < kN / 64; ++h) {
+        for (int c = 0; c < kN / 64; ++c) {
           uint32_t v[2][32];
-          tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * kN + 64 * h), v[0]);
-          tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * kN + 64 * h + 32), v[1]);
+          tmem_ld_32x32b_x32(t_base + (uint32_t)(64 * c), v[0]);
+          tmem_ld_32x32b_x32(t_base + (uint32_t)(64 * c + 32), v[1]);
           tmem_ld_wait();
-          if (h == kN / 64 - 1) {
+          if (c == kN / 64 - 1) {
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&sh.acc_empty[acc]);
           }
-          uint8_t* box = obox + (int)(n_box & 1) * Cfg::kBoxBytes;
-          if (lane == 0) bulk_wait_read_1();     // the store that used this box has read it
+          uint8_t* box = obox + (int)(n_box % Cfg::kBoxesPerWarp) * Cfg::kBoxBytes;
+          if (lane == 0) {                       // the store that used this box has read it
+            if constexpr (Cfg::kBoxesPerWarp == 2)
+              bulk_wait_read_1();
+            else
+              bulk_wait_read_all();
+          }
           __syncwarp();
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
@@ -325,7 +422,7 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
           fence_async_smem();
           __syncwarp();
           if (lane == 0) {
-            const int x = nb * kN + 64 * h;
+            const int x = nb * kN + 64 * c;
             if (y < rows && x < cols) tma_store_2d(&tm_o, x, y, box);
             bulk_commit();
           }
@@ -372,9 +469,8 @@ transpose_p_kernel(const __nv_bfloat16* __restrict__ p_hl, const TcMat* __restri
   }
 }
 
-// S_HL[row] = [hi | lo | 0] of the sum over the K ranges of the fp32 partial rows of S:
-// thread (row, g) adds columns 8 g .. 8 g + 7 and writes their hi and lo chunks (g = 0
-// also the zero chunks past 2R).
+// S_HL[row] = [hi | lo | 0] of the sum over the K ranges of the fp32 partial rows of S
+// (k_split > kFusedSplits): thread (row, g) adds columns 8 g .. 8 g + 7 in K-range order.
 template <int R>
 __global__ void __launch_bounds__(128)
 reduce_s_kernel(const float* __restrict__ part, int rows, int k_split,
@@ -406,15 +502,16 @@ cudaError_t launch_linear_r(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
                             const CUtensorMap* w_map, const CUtensorMap& tm_s,
                             const CUtensorMap& tm_u, const CUtensorMap& tm_o, int rows, int cols,
                             int k_steps, int k_split, int k_chunk, int u_row0, float* part,
-                            int grid, uint32_t* d_status, cudaStream_t s) {
+                            __nv_bfloat16* s_out, uint32_t* s_count, int grid,
+                            uint32_t* d_status, cudaStream_t s) {
   using Cfg = LinCfg<kMode, R>;
   cudaError_t e = cudaFuncSetAttribute(linear_kernel<kMode, R>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)Cfg::kSmem);
   if (e != cudaSuccess) return e;
-  linear_kernel<kMode, R><<<grid, kLinThreads, Cfg::kSmem, s>>>(
+  linear_kernel<kMode, R><<<grid, Cfg::kThreads, Cfg::kSmem, s>>>(
       tm_a, tm_b, w_map, tm_s, tm_u, tm_o, rows, cols, k_steps, k_split, k_chunk, u_row0, part,
-      d_status, kWaitCycles);
+      s_out, s_count, d_status, kWaitCycles);
   return cudaGetLastError();
 }
 
@@ -425,14 +522,20 @@ bool linear_supported(int32_t r) { return r == 16 || r == 32; }
 void linear_s_split(int64_t T, int64_t n, int32_t sms, int32_t* k_split, int32_t* k_chunk) {
   const int64_t k_steps = (n + 63) / 64;
   const int64_t blocks = (T + kBM - 1) / kBM;
-  int64_t want = std::max<int64_t>(1, std::min<int64_t>(k_steps, (sms + blocks - 1) / blocks));
+  // at most one wave of tiles: a second, partial wave would double the kernel's time
+  int64_t want = std::max<int64_t>(1, std::min<int64_t>(k_steps, sms / blocks));
   const int64_t chunk = (k_steps + want - 1) / want;
   *k_chunk = (int32_t)chunk;
   *k_split = (int32_t)((k_steps + chunk - 1) / chunk);   // every K range non-empty
 }
 
-int32_t linear_y_tiles(int64_t T, int64_t m) {
-  return (int32_t)(((T + kBM - 1) / kBM) * ((m + 255) / 256));
+int32_t linear_y_rows(int64_t T, int64_t m, int32_t sms, int32_t option) {
+  if (option == 1) return 128;
+  if (option == 2) return 256;
+  const int64_t cols = (m + 255) / 256;
+  const int64_t waves128 = ((T + 127) / 128 * cols + sms - 1) / sms;
+  const int64_t waves256 = ((T + 255) / 256 * cols + sms - 1) / sms;
+  return 16 * waves256 < 10 * waves128 ? 256 : 128;
 }
 
 int64_t linear_pk_elems(int64_t n, int32_t r) { return 2 * (int64_t)r * ((n + 63) / 64 * 64); }
@@ -447,23 +550,25 @@ cudaError_t launch_transpose_p(const __nv_bfloat16* p_hl, const TcMat* d_tc, con
 
 cudaError_t launch_linear_s(const CUtensorMap& tm_x, const CUtensorMap& tm_pk, int64_t T,
                             int64_t n, int32_t r, int32_t k_split, int32_t k_chunk, float* part,
-                            __nv_bfloat16* s_hl, int32_t sms, uint32_t* d_status,
-                            cudaStream_t s) {
+                            __nv_bfloat16* s_hl, uint32_t* s_count, int32_t sms,
+                            uint32_t* d_status, cudaStream_t s) {
   const int k_steps = (int)((n + 63) / 64);
   const int tiles = (int)((T + kBM - 1) / kBM) * k_split;
   const int grid = std::min<int>(tiles, sms);
+  const bool fused = k_split <= kFusedSplits;
+  uint32_t* count = fused ? s_count : nullptr;
   cudaError_t e;
   switch (r) {
     case 16:
       e = launch_linear_r<kModeS, 16>(tm_x, tm_pk, nullptr, tm_x, tm_x, tm_x, (int)T, 32, k_steps,
-                                       k_split, k_chunk, 0, part, grid, d_status, s);
-      if (e == cudaSuccess)
+                                      k_split, k_chunk, 0, part, s_hl, count, grid, d_status, s);
+      if (e == cudaSuccess && !fused)
         reduce_s_kernel<16><<<(unsigned)((T * 2 + 127) / 128), 128, 0, s>>>(part, (int)T, k_split, s_hl);
       break;
     case 32:
       e = launch_linear_r<kModeS, 32>(tm_x, tm_pk, nullptr, tm_x, tm_x, tm_x, (int)T, 64, k_steps,
-                                       k_split, k_chunk, 0, part, grid, d_status, s);
-      if (e == cudaSuccess)
+                                      k_split, k_chunk, 0, part, s_hl, count, grid, d_status, s);
+      if (e == cudaSuccess && !fused)
         reduce_s_kernel<32><<<(unsigned)((T * 4 + 127) / 128), 128, 0, s>>>(part, (int)T, k_split, s_hl);
       break;
     default: return cudaErrorInvalidValue;
@@ -472,18 +577,27 @@ cudaError_t launch_linear_s(const CUtensorMap& tm_x, const CUtensorMap& tm_pk, i
   return cudaGetLastError();
 }
 
+int32_t linear_s_launches(int32_t k_split) { return k_split <= kFusedSplits ? 1 : 2; }
+
 cudaError_t launch_linear_y(const CUtensorMap& tm_x, const CUtensorMap* d_w_map,
                             const CUtensorMap& tm_s_in, const CUtensorMap& tm_u,
                             const CUtensorMap& tm_y, int64_t T, int64_t m, int64_t n,
-                            int32_t u_row0, int32_t r, int32_t sms, uint32_t* d_status,
-                            cudaStream_t s) {
+                            int32_t u_row0, int32_t r, int32_t tile_rows, int32_t sms,
+                            uint32_t* d_status, cudaStream_t s) {
+  if (tile_rows != 128 && tile_rows != 256) return cudaErrorInvalidValue;
   const int k_steps = (int)((n + 63) / 64);
-  const int grid = std::min<int>(linear_y_tiles(T, m), sms);
+  const int64_t tiles = (T + tile_rows - 1) / tile_rows * ((m + 255) / 256);
+  const int grid = (int)std::min<int64_t>(tiles, sms);
+#define ZO_LINEAR_Y(MODE, RR)                                                                  \
+  launch_linear_r<MODE, RR>(tm_x, tm_x, d_w_map, tm_s_in, tm_u, tm_y, (int)T, (int)m, k_steps, \
+                            1, k_steps, u_row0, nullptr, nullptr, nullptr, grid, d_status, s)
+  const bool wide = tile_rows == 256;
   switch (r) {
-    case 16: return launch_linear_r<kModeY, 16>(tm_x, tm_x, d_w_map, tm_s_in, tm_u, tm_y, (int)T, (int)m, k_steps, 1, k_steps, u_row0, nullptr, grid, d_status, s);
-    case 32: return launch_linear_r<kModeY, 32>(tm_x, tm_x, d_w_map, tm_s_in, tm_u, tm_y, (int)T, (int)m, k_steps, 1, k_steps, u_row0, nullptr, grid, d_status, s);
+    case 16: return wide ? ZO_LINEAR_Y(kModeY2, 16) : ZO_LINEAR_Y(kModeY, 16);
+    case 32: return wide ? ZO_LINEAR_Y(kModeY2, 32) : ZO_LINEAR_Y(kModeY, 32);
     default: return cudaErrorInvalidValue;
   }
+#undef ZO_LINEAR_Y
 }
 
 }  // namespace zo

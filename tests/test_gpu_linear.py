@@ -71,16 +71,23 @@ def test_perturbed_linear_matches_oracle_and_leaves_W(lib, gpu, case, eps):
         for T in tokens:
             X = _tokens(T, n, 17 * T + i, gpu)
             ldy = (m + 7) // 8 * 8
-            Ybuf = torch.full((T, ldy), float("nan"), dtype=torch.bfloat16, device=gpu)
-            Y = Ybuf[:, :m]
-            zb.zo_linear_perturbed(z.ctx, i, X, Y)
-            z.sync()
+            out = {}
+            for tile, rows in ((1, 128), (2, 256)):
+                zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, tile)
+                Ybuf = torch.full((T, ldy), float("nan"), dtype=torch.bfloat16, device=gpu)
+                zb.zo_linear_perturbed(z.ctx, i, X, Ybuf[:, :m])
+                z.sync()
+                assert zb.zo_linear_tile_rows(z.ctx) == rows
+                # the padding columns of Y's rows are not written
+                assert torch.isnan(Ybuf[:, m:].float()).all()
+                out[rows] = Ybuf[:, :m]
+            # 128- and 256-row tiles sum every output in the same order
+            assert torch.equal(out[128].view(torch.int16), out[256].view(torch.int16))
+            Y = out[256]
             C = subzero.perturb_coeff(z.seed, base + i, 5, r, terms, f32(eps))
             zc = abs(f32(eps)) * 2.0
             want = _check(Y, X, before["W"][i], before["U"][i], before["V"][i], C, zc,
                           f"{case} matrix {i} T={T} eps={eps}")
-            # the padding columns of Y's rows are not written
-            assert torch.isnan(Ybuf[:, m:].float()).all()
             if eps == 1e-1:
                 # the perturbation is visible: most outputs differ from the plain layer's
                 plain = rounding.round_to_bf16(to_f64(X) @ before["W"][i].T)
@@ -114,6 +121,29 @@ def test_perturbed_linear_single_query_and_repeat(lib, gpu):
     z.close()
 
 
+def test_perturbed_linear_long_token_block(lib, gpu):
+    """S = X P^T's three ways to S_HL: 257 and 300 tokens split K over many ranges (a
+    separate reduction kernel); 5000 tokens (40 row blocks) over 3 ranges, which the S
+    kernel sums itself through its per-group counters; 19500 tokens (more row blocks than
+    SMs) not at all, the epilogue writing S_HL directly while CTAs take several tiles.
+    The calls run in turn on one context, so the counters must come back to zero."""
+    from paper_2608_15665_gb300 import binding as zb
+    z, base = _context(gpu, "r16", seed=2024)
+    r, spec, _ = LINEAR_CASES["r16"]
+    m, n, _ = spec[2]
+    zb.zo_linear_prepare(z.ctx, 2, 0, 1.0, 3, -0.5, 1e-2)
+    before = snapshot(z)
+    C = subzero.perturb_coeff(z.seed, base + 2, 2, r, [(0, 1.0), (3, -0.5)], f32(1e-2))
+    for T in (257, 5000, 19500, 5000, 300):
+        X = _tokens(T, n, T, gpu)
+        Y = torch.empty((T, m), dtype=torch.bfloat16, device=gpu)
+        zb.zo_linear_perturbed(z.ctx, 2, X, Y)
+        z.sync()
+        _check(Y, X, before["W"][2], before["U"][2], before["V"][2], C, 2.0 * f32(1e-2),
+               f"long token block T={T}")
+    z.close()
+
+
 def test_perturbed_linear_rejections(lib, gpu):
     from paper_2608_15665_gb300 import binding as zb
     from paper_2608_15665_gb300.schedule import SubZeroPlus
@@ -127,6 +157,8 @@ def test_perturbed_linear_rejections(lib, gpu):
     zb.zo_linear_prepare(z.ctx, 0, 0, 1.0, -1, 0.0, 1e-3)
     with pytest.raises(RuntimeError):
         zb.zo_linear_perturbed(z.ctx, 3, X, Y)                                     # no matrix 3
+    with pytest.raises(RuntimeError):
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 3)                       # no tiling 3
     z.refresh(1)                                                                   # new U, V
     with pytest.raises(RuntimeError):
         zb.zo_linear_perturbed(z.ctx, 0, X, Y)                                     # stale P
