@@ -524,10 +524,11 @@ def run_linear(args):
     clk = clocks.stop()
     launches = zb.zo_kernel_launches(z.ctx) - launches0
     z.sync()
-    tile_rows = []
+    names = {1: "128x256", 2: "256x256", 3: "256x224"}
+    tiling = []
     for i, (m, n) in enumerate(wl.shapes):
         zb.zo_linear_perturbed(z.ctx, i, X[n], Y[i])
-        tile_rows.append(zb.zo_linear_tile_rows(z.ctx))
+        tiling.append(names[zb.zo_linear_tiling(z.ctx)])
     # for context: the same route with 128-row tiles throughout
     zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 1)
     fused128_ms = timed(fused, K)
@@ -570,7 +571,7 @@ def run_linear(args):
         "ms_per_step": fused_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic",
         "config": {"workload": wl.name, "matrices": wl.n_mats, "tokens": T, "r": wl.r,
-                   "method": "linear", "tile_rows": tile_rows,
+                   "method": "linear", "tiles": tiling,
                    "l2": "inputs larger than L2 (%.0f MB of weights)" % (sum(m * n for m, n in wl.shapes) * 2 / 1e6),
                    "parallelism": "single GPU"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",

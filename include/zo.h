@@ -101,11 +101,11 @@ enum {
                                      bounded wait (~0.1 s) runs out; that pass then reports
                                      ZO_ERR_TIMEOUT via zo_sync_status and leaves W partly
                                      updated.  Nothing faults; the context stays usable. */
-  ZO_OPTION_LINEAR_TILE = 3 /* tiles of zo_linear_perturbed's Y = X W^T + S U^T GEMM:
-                               0 = automatic (the tiling with fewer waves of tiles over the
-                               SMs, a 256-row tile counted as ~1.6 of a 128-row one),
-                               1 = 128 x 256 tiles, 2 = 256 x 256 tiles.  Both give
-                               bit-identical Y. */
+  ZO_OPTION_LINEAR_TILE = 3 /* tiles (rows of X x columns of Y) of zo_linear_perturbed's
+                               Y = X W^T + S U^T GEMM: 0 = automatic (the tiling with the
+                               least tile work per SM: waves of tiles x a tile's relative
+                               time), 1 = 128 x 256, 2 = 256 x 256, 3 = 256 x 224.  All
+                               give bit-identical Y. */
 };
 
 /* One trainable matrix W_i with its projection bases and Adam moments. */
@@ -246,9 +246,9 @@ ZO_API zo_status zo_get_timing(zo_ctx* ctx, double* total_ms, int64_t* launches)
    (1 = FMA on 32-row tiles, 2 = tcgen05, 3 = FMA on narrow tiles). */
 ZO_API int32_t zo_wpass_path(const zo_ctx* ctx);
 
-/* zo_linear_tile_rows -- rows of X per tile (128 or 256) of the Y GEMM that the last
- * zo_linear_perturbed launched; 0 before the first call or for a null ctx. */
-ZO_API int32_t zo_linear_tile_rows(const zo_ctx* ctx);
+/* zo_linear_tiling -- the tiling (1, 2 or 3, as ZO_OPTION_LINEAR_TILE) of the Y GEMM
+ * that the last zo_linear_perturbed launched; 0 before the first call or for a null ctx. */
+ZO_API int32_t zo_linear_tiling(const zo_ctx* ctx);
 
 /* zo_kernel_launches -- number of kernels this context has launched since zo_create. */
 ZO_API int64_t zo_kernel_launches(const zo_ctx* ctx);

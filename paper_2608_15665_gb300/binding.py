@@ -82,7 +82,7 @@ _SIGNATURES = {
     "zo_set_option": (_c.c_int32, [_c.c_void_p, _c.c_int32, _c.c_int64]),
     "zo_get_timing": (_c.c_int32, [_c.c_void_p, _c.POINTER(_c.c_double), _c.POINTER(_c.c_int64)]),
     "zo_wpass_path": (_c.c_int32, [_c.c_void_p]),
-    "zo_linear_tile_rows": (_c.c_int32, [_c.c_void_p]),
+    "zo_linear_tiling": (_c.c_int32, [_c.c_void_p]),
     "zo_kernel_launches": (_c.c_int64, [_c.c_void_p]),
     "zo_philox_fill": (_c.c_int32, [_c.c_uint64, _c.c_uint32, _c.c_uint32, _c.c_uint32,
                                     _c.c_void_p, _c.c_int64, _c.c_void_p]),
@@ -243,8 +243,8 @@ def zo_wpass_path(ctx):
     return int(LIB.zo_wpass_path(ctx))
 
 
-def zo_linear_tile_rows(ctx):
-    return int(LIB.zo_linear_tile_rows(ctx))
+def zo_linear_tiling(ctx):
+    return int(LIB.zo_linear_tiling(ctx))
 
 
 def zo_kernel_launches(ctx):

@@ -117,7 +117,7 @@ struct zo_ctx {
   std::vector<int64_t> h_pk_off;
   bool linear_ready = false;
   int linear_tile = 0;           // ZO_OPTION_LINEAR_TILE
-  int last_linear_rows = 0;      // rows per tile of the last Y GEMM
+  int last_linear_tiling = 0;    // tiling of the last Y GEMM (1..3)
   __nv_bfloat16* d_s_hl = nullptr;
   float* d_s_part = nullptr;
   uint32_t* d_s_count = nullptr;   // one counter per 32 rows of S_HL's capacity
@@ -327,7 +327,8 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
 // 2-D bf16 tensor map: `cols` contiguous elements per row, `rows` rows `row_bytes` apart,
 // boxes of box_cols x box_rows with the 128-byte swizzle.
 bool encode_bf16_2d(CUtensorMap* tm, void* base, uint64_t cols, uint64_t rows, uint64_t row_bytes,
-                    uint32_t box_cols, uint32_t box_rows) {
+                    uint32_t box_cols, uint32_t box_rows,
+                    CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   auto enc = tensor_map_encoder();
   if (!enc) return false;
   const cuuint64_t dims[2] = {cols, rows};
@@ -335,7 +336,7 @@ bool encode_bf16_2d(CUtensorMap* tm, void* base, uint64_t cols, uint64_t rows, u
   const cuuint32_t box[2] = {box_cols, box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -949,13 +950,16 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
       c->part_cap = part;
     }
   }
+  const int32_t tiling = zo::linear_y_tiling(T, m, c->sms, c->linear_tile);
+  const bool narrow_y = zo::linear_y_tile_cols(tiling) % 64 != 0;   // 32-column Y boxes
   CUtensorMap tm_x{}, tm_pk{}, tm_s{}, tm_y{};
   const bool enc =
       encode_bf16_2d(&tm_x, const_cast<void*>(X), n, T, ldx * 2, 64, 128) &&
       encode_bf16_2d(&tm_pk, c->d_pk + c->h_pk_off[mat], n, 2 * r, (n + 63) / 64 * 64 * 2, 64,
                      (uint32_t)(2 * r)) &&
       encode_bf16_2d(&tm_s, c->d_s_hl, HLW, T, HLW * 2, 64, 128) &&
-      encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 64, 32);
+      (narrow_y ? encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)
+                : encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 64, 32));
   if (!enc) {
     g_last_error = "zo_linear_perturbed: cuTensorMapEncodeTiled rejected a descriptor";
     return ZO_ERR_CUDA;
@@ -964,11 +968,10 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
   ZO_CUDA(zo::launch_linear_s(tm_x, tm_pk, T, n, r, k_split, k_chunk, c->d_s_part, c->d_s_hl,
                               c->d_s_count, c->sms, c->d_status, c->stream),
           "S = X P^T kernels");
-  const int32_t rows = zo::linear_y_rows(T, m, c->sms, c->linear_tile);
   ZO_CUDA(zo::launch_linear_y(tm_x, c->d_w_maps + mat, tm_s, c->tm_a, tm_y, T, m, n,
-                              c->h_tc[mat].u_row0, r, rows, c->sms, c->d_status, c->stream),
+                              c->h_tc[mat].u_row0, r, tiling, c->sms, c->d_status, c->stream),
           "perturbed linear kernel");
-  c->last_linear_rows = rows;
+  c->last_linear_tiling = tiling;
   c->launches += 1 + zo::linear_s_launches(k_split);
   return ZO_OK;
 }
@@ -1046,7 +1049,7 @@ zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
     return ZO_OK;
   }
   if (option == ZO_OPTION_LINEAR_TILE) {
-    if (value < 0 || value > 2) return ZO_ERR_INVALID_ARG;
+    if (value < 0 || value > 3) return ZO_ERR_INVALID_ARG;
     c->linear_tile = (int)value;
     return ZO_OK;
   }
@@ -1080,7 +1083,7 @@ zo_status zo_get_timing(zo_ctx* c, double* total_ms, int64_t* launches) {
 
 int32_t zo_wpass_path(const zo_ctx* c) { return c ? c->last_path : 0; }
 
-int32_t zo_linear_tile_rows(const zo_ctx* c) { return c ? c->last_linear_rows : 0; }
+int32_t zo_linear_tiling(const zo_ctx* c) { return c ? c->last_linear_tiling : 0; }
 
 int64_t zo_kernel_launches(const zo_ctx* c) { return c ? c->launches : 0; }
 

@@ -140,10 +140,12 @@ cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
 bool linear_supported(int32_t r);
 // The S GEMM's split of K = n into k_split ranges of k_chunk steps of 64 (~ one wave).
 void linear_s_split(int64_t T, int64_t n, int32_t sms, int32_t* k_split, int32_t* k_chunk);
-// Rows of X per tile of the Y GEMM, 128 or 256: option 1 / 2 force one; 0 takes the
-// tiling with fewer waves of tiles over the SMs (a 256 x 256 tile costs ~1.6 of the
-// 128 x 256 one).
-int32_t linear_y_rows(int64_t T, int64_t m, int32_t sms, int32_t option);
+// Tiling of the Y GEMM: 1 = 128 x 256, 2 = 256 x 256, 3 = 256 x 224 (rows of X x columns
+// of Y).  Option 1..3 forces one; 0 takes the one with the least tile work per SM (waves
+// of tiles x a tile's relative time).
+int32_t linear_y_tiling(int64_t T, int64_t m, int32_t sms, int32_t option);
+int32_t linear_y_tile_rows(int32_t tiling);
+int32_t linear_y_tile_cols(int32_t tiling);
 // Elements of matrix i's P_K: 2r rows of n rounded up to 64.
 int64_t linear_pk_elems(int64_t n, int32_t r);
 // P_K of every matrix from P_HL (units = the projection units, pk_off = element offsets).
@@ -163,11 +165,11 @@ cudaError_t launch_linear_s(const CUtensorMap& tm_x, const CUtensorMap& tm_pk, i
                             uint32_t* d_status, cudaStream_t s);
 // Y = X W^T + S U^T: d_w_map = W's descriptor (box 64 x 32), tm_s_in over S_HL (box
 // 64 x 128), tm_u over the U operand (box 64 x 128; W's rows from u_row0), tm_y over Y
-// (box 64 x 32); tile_rows from linear_y_rows.
+// (box 64 x 32, 128-byte swizzle; tiling 3: box 32 x 32, 64-byte swizzle).
 cudaError_t launch_linear_y(const CUtensorMap& tm_x, const CUtensorMap* d_w_map,
                             const CUtensorMap& tm_s_in, const CUtensorMap& tm_u,
                             const CUtensorMap& tm_y, int64_t T, int64_t m, int64_t n,
-                            int32_t u_row0, int32_t r, int32_t tile_rows, int32_t sms,
+                            int32_t u_row0, int32_t r, int32_t tiling, int32_t sms,
                             uint32_t* d_status, cudaStream_t s);
 
 // ---- refresh of tall panels at r = 16 ... 128: CholeskyQR2 (zo_cholqr.cu) ----------

@@ -27,8 +27,11 @@
 //           stage (48 KB) -- the operand bytes an SM takes in per flop fall by a third,
 //           and the 3-stage ring covers 1.5x the load latency.  Both halves'
 //           accumulators fill TMEM (2 x 256 columns), so the epilogue of a tile (eight
-//           warps) is not overlapped with the next tile's MMAs; chosen when the wave
-//           count favours it (linear_y_rows).
+//           warps) is not overlapped with the next tile's MMAs.
+//   kModeY2N the same over 256 x 224 tiles (halves 256 TMEM columns apart; Y stored 32
+//           columns at a time through 64-byte-swizzled boxes): 4096 columns make 19 of
+//           them, so 16 or 8 row blocks make exactly two or one wave on 152 SMs.
+//           linear_y_tiling picks the tiling with the fewest waves of tile work.
 // P_K is P_HL (the projection's rows [P_hi(j, :) | P_lo(j, :)], j < n) transposed by
 // transpose_p_kernel, for every matrix once per loss evaluation (zo_linear_prepare).
 // Ragged edges: TMA zero-fills loads past T, n and m; Y's stores are clipped to T rows and
@@ -66,23 +69,30 @@ constexpr int kFusedSplits = 4;   // most K ranges whose S partials the S kernel
 constexpr int kModeS = 0;
 constexpr int kModeY = 1;
 constexpr int kModeY2 = 2;
+constexpr int kModeY2N = 3;
 
 template <int kMode, int R>
 struct LinCfg {
   static_assert(R == 16 || R == 32, "the U operand rows [hi | lo | 0] exist for r <= 32");
   static constexpr bool kY = kMode != kModeS;
-  static constexpr int kHalves = kMode == kModeY2 ? 2 : 1;           // 128-row halves per tile
+  static constexpr bool kWide = kMode == kModeY2 || kMode == kModeY2N;
+  static constexpr int kHalves = kWide ? 2 : 1;                      // 128-row halves per tile
   static constexpr int kTileRows = kHalves * kBM;
-  static constexpr int kN = kY ? 256 : 2 * R;                        // tile columns
-  static constexpr int kStages = kMode == kModeY2 ? 3 : 4;
-  static constexpr int kAccs = kMode == kModeY2 ? 1 : 2;             // accumulator buffers
-  static constexpr int kAccCols = kHalves * kN;                      // TMEM columns of one
-  static constexpr int kEpiWarps = kMode == kModeY2 ? 8 : 4;
+  static constexpr int kN = kMode == kModeY2N ? 224 : kY ? 256 : 2 * R;   // tile columns
+  static constexpr int kHalfCols = kMode == kModeY2N ? 256 : kN;     // TMEM columns per half
+  static constexpr int kStages = kWide ? 3 : 4;
+  static constexpr int kAccs = kWide ? 1 : 2;                        // accumulator buffers
+  static constexpr int kAccCols = kHalves * kHalfCols;               // TMEM columns of one
+  static constexpr int kEpiWarps = kWide ? 8 : 4;
   static constexpr int kThreads = 64 + 32 * kEpiWarps;
   static constexpr int kABytes = kTileRows * 128;                    // rows x 64 bf16
-  static constexpr int kBBytes = kN * 128;                           // kN rows x 64 bf16
+  // B rows of a slot: the Y modes' extension step loads 256 U operand rows (two boxes)
+  static constexpr int kBRows = kY ? 256 : kN;
+  static constexpr int kBBytes = kBRows * 128;                       // 64 bf16 per row
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kBoxBytes = 32 * 128;                         // 32 rows x 64 bf16
+  static constexpr uint32_t kMainTx = kABytes + kN * 128;            // bytes of a K step
+  static constexpr int kCW = kN % 64 == 0 ? 64 : 32;                 // Y columns per store
+  static constexpr int kBoxBytes = 32 * kCW * 2;                     // 32 rows x kCW bf16
   static constexpr int kBoxesPerWarp = kMode == kModeY2 ? 1 : 2;
   static constexpr int kOutBytes = kEpiWarps * kBoxesPerWarp * kBoxBytes;
   static constexpr int kTmemCols = kAccs * kAccCols <= 32 ? 32 : kAccs * kAccCols;
@@ -90,6 +100,7 @@ struct LinCfg {
   static_assert(kSmem <= 227 * 1024, "shared memory per CTA");
   static_assert(kTmemCols <= 512, "TMEM columns");
   static_assert(kABytes == kHalves * kPanelBytes, "one 128-row panel per half");
+  static_assert(kN % 32 == 0 && kN <= kBRows && kN <= kHalfCols, "tile columns");
 };
 
 // S_HL row: [hi | lo] of the R sums in chunks of 8, then zero chunks up to 64 elements.
@@ -213,13 +224,14 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
         }
         uint8_t* a_dst = st_smem + s * Cfg::kStageBytes;
         uint8_t* b_dst = a_dst + Cfg::kABytes;
-        mbar_arrive_expect_tx(&sh.full[s], Cfg::kStageBytes);
+        mbar_arrive_expect_tx(&sh.full[s], (Cfg::kY && k == k_steps) ? (uint32_t)Cfg::kStageBytes
+                                                                     : Cfg::kMainTx);
         if (Cfg::kY && k == k_steps) {
           // the extension: S_HL rows of the token block, U operand rows of the W block
           for (int h = 0; h < Cfg::kHalves; ++h)
             tma_load_2d(a_dst + h * kPanelBytes, &tm_s, 0, tb * Cfg::kTileRows + h * kBM,
                         &sh.full[s]);
-          for (int h = 0; h < kN / kBM; ++h)
+          for (int h = 0; h < Cfg::kBRows / kBM; ++h)
             tma_load_2d(b_dst + h * kPanelBytes, &tm_u, 0, u_row0 + nb * kN + h * kBM, &sh.full[s]);
         } else {
           for (int h = 0; h < Cfg::kHalves; ++h)
@@ -229,7 +241,7 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
             tma_load_2d(b_dst, &tm_b, 64 * k, 0, &sh.full[s]);
           } else {
             for (int h = 0; h < kN / 32; ++h)
-              tma_load_2d(b_dst + h * Cfg::kBoxBytes, w_map, 64 * k, nb * kN + 32 * h, &sh.full[s]);
+              tma_load_2d(b_dst + h * 4096, w_map, 64 * k, nb * kN + 32 * h, &sh.full[s]);
           }
         }
         ++n_st;
@@ -269,7 +281,7 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
         const uint32_t b_base = st_base + Cfg::kABytes;
 #pragma unroll
         for (int h = 0; h < Cfg::kHalves; ++h) {
-          const uint32_t d = d0 + (uint32_t)(h * kN);
+          const uint32_t d = d0 + (uint32_t)(h * Cfg::kHalfCols);
           const uint32_t a_base = st_base + (uint32_t)(h * kPanelBytes);
           if (Cfg::kY && k == k_steps) {
             // hi chunk kk at element 16 kk of an operand row, lo chunk at R + 16 kk
@@ -318,7 +330,8 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
       }
       tc_fence_after();
       const int y = tb * Cfg::kTileRows + half * kBM + 32 * g;
-      const uint32_t t_base = tmem + lane_base + (uint32_t)(acc * Cfg::kAccCols + half * kN);
+      const uint32_t t_base =
+          tmem + lane_base + (uint32_t)(acc * Cfg::kAccCols + half * Cfg::kHalfCols);
       if constexpr (kMode == kModeS) {
         // partial S over this K range: D[:, :R] + D[:, R:2R], fp32, this lane's row
         uint32_t v[2 * R];
@@ -386,14 +399,15 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
           }
         }
       } else {
-        // 64 columns of Y at a time, through the warp's box(es) in turn
+        // kCW columns of Y at a time, through the warp's box(es) in turn
+        constexpr int kCW = Cfg::kCW;
 #pragma unroll 1
-        for (int c = 0; c < kN / 64; ++c) {
+        for (int c = 0; c < kN / kCW; ++c) {
           uint32_t v[2][32];
-          tmem_ld_32x32b_x32(t_base + (uint32_t)(64 * c), v[0]);
-          tmem_ld_32x32b_x32(t_base + (uint32_t)(64 * c + 32), v[1]);
+          tmem_ld_32x32b_x32(t_base + (uint32_t)(kCW * c), v[0]);
+          if constexpr (kCW == 64) tmem_ld_32x32b_x32(t_base + (uint32_t)(kCW * c + 32), v[1]);
           tmem_ld_wait();
-          if (c == kN / 64 - 1) {
+          if (c == kN / kCW - 1) {
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&sh.acc_empty[acc]);
@@ -406,8 +420,10 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
               bulk_wait_read_all();
           }
           __syncwarp();
+          // 16-byte chunk j of row `lane`: 128-byte swizzle (chunk ^ row % 8) for 64
+          // columns, 64-byte swizzle (chunk ^ (row / 2) % 4) for 32
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
+          for (int j = 0; j < kCW / 8; ++j) {
             uint32_t w[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
@@ -416,13 +432,14 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
                                         __uint_as_float(v[j >> 2][(j & 3) * 8 + 2 * e + 1]));
               w[e] = *reinterpret_cast<const uint32_t*>(&b2);
             }
-            *reinterpret_cast<uint4*>(box + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-                make_uint4(w[0], w[1], w[2], w[3]);
+            const int off = kCW == 64 ? lane * 128 + ((j ^ (lane & 7)) << 4)
+                                      : lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4);
+            *reinterpret_cast<uint4*>(box + off) = make_uint4(w[0], w[1], w[2], w[3]);
           }
           fence_async_smem();
           __syncwarp();
           if (lane == 0) {
-            const int x = nb * kN + 64 * c;
+            const int x = nb * kN + kCW * c;
             if (y < rows && x < cols) tma_store_2d(&tm_o, x, y, box);
             bulk_commit();
           }
@@ -529,14 +546,24 @@ void linear_s_split(int64_t T, int64_t n, int32_t sms, int32_t* k_split, int32_t
   *k_split = (int32_t)((k_steps + chunk - 1) / chunk);   // every K range non-empty
 }
 
-int32_t linear_y_rows(int64_t T, int64_t m, int32_t sms, int32_t option) {
-  if (option == 1) return 128;
-  if (option == 2) return 256;
-  const int64_t cols = (m + 255) / 256;
-  const int64_t waves128 = ((T + 127) / 128 * cols + sms - 1) / sms;
-  const int64_t waves256 = ((T + 255) / 256 * cols + sms - 1) / sms;
-  return 16 * waves256 < 10 * waves128 ? 256 : 128;
+int32_t linear_y_tiling(int64_t T, int64_t m, int32_t sms, int32_t option) {
+  if (option >= 1 && option <= 3) return option;
+  // waves of tiles x the time of one tile, relative to 256 x 256 (1000): 128 x 256 tiles
+  // run at ~1/1.6 of it, 256 x 224 tiles at ~0.9
+  auto cost = [&](int rows, int cols, int64_t per_tile) {
+    const int64_t tiles = (T + rows - 1) / rows * ((m + cols - 1) / cols);
+    return (tiles + sms - 1) / sms * per_tile;
+  };
+  int32_t best = 2;
+  int64_t c_best = cost(256, 256, 1000);
+  const int64_t c3 = cost(256, 224, 900), c1 = cost(128, 256, 625);
+  if (c3 < c_best) { best = 3; c_best = c3; }
+  if (c1 < c_best) best = 1;
+  return best;
 }
+
+int32_t linear_y_tile_rows(int32_t tiling) { return tiling == 1 ? 128 : 256; }
+int32_t linear_y_tile_cols(int32_t tiling) { return tiling == 3 ? 224 : 256; }
 
 int64_t linear_pk_elems(int64_t n, int32_t r) { return 2 * (int64_t)r * ((n + 63) / 64 * 64); }
 
@@ -582,19 +609,23 @@ int32_t linear_s_launches(int32_t k_split) { return k_split <= kFusedSplits ? 1 
 cudaError_t launch_linear_y(const CUtensorMap& tm_x, const CUtensorMap* d_w_map,
                             const CUtensorMap& tm_s_in, const CUtensorMap& tm_u,
                             const CUtensorMap& tm_y, int64_t T, int64_t m, int64_t n,
-                            int32_t u_row0, int32_t r, int32_t tile_rows, int32_t sms,
+                            int32_t u_row0, int32_t r, int32_t tiling, int32_t sms,
                             uint32_t* d_status, cudaStream_t s) {
-  if (tile_rows != 128 && tile_rows != 256) return cudaErrorInvalidValue;
+  if (tiling < 1 || tiling > 3) return cudaErrorInvalidValue;
   const int k_steps = (int)((n + 63) / 64);
-  const int64_t tiles = (T + tile_rows - 1) / tile_rows * ((m + 255) / 256);
+  const int64_t rows = linear_y_tile_rows(tiling), cols = linear_y_tile_cols(tiling);
+  const int64_t tiles = (T + rows - 1) / rows * ((m + cols - 1) / cols);
   const int grid = (int)std::min<int64_t>(tiles, sms);
 #define ZO_LINEAR_Y(MODE, RR)                                                                  \
   launch_linear_r<MODE, RR>(tm_x, tm_x, d_w_map, tm_s_in, tm_u, tm_y, (int)T, (int)m, k_steps, \
                             1, k_steps, u_row0, nullptr, nullptr, nullptr, grid, d_status, s)
-  const bool wide = tile_rows == 256;
-  switch (r) {
-    case 16: return wide ? ZO_LINEAR_Y(kModeY2, 16) : ZO_LINEAR_Y(kModeY, 16);
-    case 32: return wide ? ZO_LINEAR_Y(kModeY2, 32) : ZO_LINEAR_Y(kModeY, 32);
+  switch (r * 4 + tiling) {
+    case 16 * 4 + 1: return ZO_LINEAR_Y(kModeY, 16);
+    case 16 * 4 + 2: return ZO_LINEAR_Y(kModeY2, 16);
+    case 16 * 4 + 3: return ZO_LINEAR_Y(kModeY2N, 16);
+    case 32 * 4 + 1: return ZO_LINEAR_Y(kModeY, 32);
+    case 32 * 4 + 2: return ZO_LINEAR_Y(kModeY2, 32);
+    case 32 * 4 + 3: return ZO_LINEAR_Y(kModeY2N, 32);
     default: return cudaErrorInvalidValue;
   }
 #undef ZO_LINEAR_Y

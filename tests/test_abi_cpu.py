@@ -75,7 +75,7 @@ def test_calls_on_null_context_are_rejected(lib):
     assert L.zo_sync_status(None) == lib.ZO_ERR_INVALID_ARG
     assert L.zo_destroy(None) == lib.ZO_OK
     assert L.zo_wpass_path(None) == 0
-    assert L.zo_linear_tile_rows(None) == 0
+    assert L.zo_linear_tiling(None) == 0
 
 
 def test_rng_fills_validate_sizes(lib):

@@ -72,18 +72,19 @@ def test_perturbed_linear_matches_oracle_and_leaves_W(lib, gpu, case, eps):
             X = _tokens(T, n, 17 * T + i, gpu)
             ldy = (m + 7) // 8 * 8
             out = {}
-            for tile, rows in ((1, 128), (2, 256)):
-                zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, tile)
+            for tiling in (1, 2, 3):     # 128x256, 256x256, 256x224
+                zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, tiling)
                 Ybuf = torch.full((T, ldy), float("nan"), dtype=torch.bfloat16, device=gpu)
                 zb.zo_linear_perturbed(z.ctx, i, X, Ybuf[:, :m])
                 z.sync()
-                assert zb.zo_linear_tile_rows(z.ctx) == rows
+                assert zb.zo_linear_tiling(z.ctx) == tiling
                 # the padding columns of Y's rows are not written
                 assert torch.isnan(Ybuf[:, m:].float()).all()
-                out[rows] = Ybuf[:, :m]
-            # 128- and 256-row tiles sum every output in the same order
-            assert torch.equal(out[128].view(torch.int16), out[256].view(torch.int16))
-            Y = out[256]
+                out[tiling] = Ybuf[:, :m]
+            # every tiling sums each output in the same order
+            for tiling in (1, 3):
+                assert torch.equal(out[tiling].view(torch.int16), out[2].view(torch.int16))
+            Y = out[3]
             C = subzero.perturb_coeff(z.seed, base + i, 5, r, terms, f32(eps))
             zc = abs(f32(eps)) * 2.0
             want = _check(Y, X, before["W"][i], before["U"][i], before["V"][i], C, zc,
@@ -158,7 +159,7 @@ def test_perturbed_linear_rejections(lib, gpu):
     with pytest.raises(RuntimeError):
         zb.zo_linear_perturbed(z.ctx, 3, X, Y)                                     # no matrix 3
     with pytest.raises(RuntimeError):
-        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 3)                       # no tiling 3
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 4)                       # no tiling 4
     z.refresh(1)                                                                   # new U, V
     with pytest.raises(RuntimeError):
         zb.zo_linear_perturbed(z.ctx, 0, X, Y)                                     # stale P
