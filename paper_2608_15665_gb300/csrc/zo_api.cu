@@ -868,11 +868,21 @@ zo_status zo_linear_prepare(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t
       c->h_pk_off[i] = total;
       total += zo::linear_pk_elems(c->h_mats[i].n, r);
     }
-    ZO_CUDA(cudaMalloc(&c->d_pk, sizeof(__nv_bfloat16) * total), "cudaMalloc(P_K)");
-    ZO_CUDA(cudaMalloc(&c->d_pk_off, sizeof(int64_t) * c->n_mats), "cudaMalloc(P_K offsets)");
-    ZO_CUDA(cudaMemcpy(c->d_pk_off, c->h_pk_off.data(), sizeof(int64_t) * c->n_mats,
-                       cudaMemcpyHostToDevice),
-            "upload P_K offsets");
+    __nv_bfloat16* pk = nullptr;
+    int64_t* pk_off = nullptr;
+    cudaError_t e = cudaMalloc(&pk, sizeof(__nv_bfloat16) * total);
+    if (e == cudaSuccess) e = cudaMalloc(&pk_off, sizeof(int64_t) * c->n_mats);
+    // on the context's stream, ahead of the kernels that read it (the host copy stays)
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(pk_off, c->h_pk_off.data(), sizeof(int64_t) * c->n_mats,
+                          cudaMemcpyHostToDevice, c->stream);
+    if (e != cudaSuccess) {
+      cudaFree(pk);
+      cudaFree(pk_off);
+      return cuda_fail(e, "P_K workspace");
+    }
+    c->d_pk = pk;
+    c->d_pk_off = pk_off;
   }
   // C_i = eps (ca Z_qa + cb Z_qb) for every matrix, P_i = C_i V_i^T, P_K = [P_hi ; P_lo]
   zo::CoeffParams p{};
@@ -939,7 +949,10 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
       const int64_t cap = (T + 127) / 128 * 128;
       ZO_CUDA(cudaMalloc(&c->d_s_hl, sizeof(__nv_bfloat16) * cap * HLW), "cudaMalloc(S_HL)");
       ZO_CUDA(cudaMalloc(&c->d_s_count, sizeof(uint32_t) * (cap / 32)), "cudaMalloc(S counters)");
-      ZO_CUDA(cudaMemset(c->d_s_count, 0, sizeof(uint32_t) * (cap / 32)), "zero S counters");
+      // on the context's stream: a plain cudaMemset runs on the legacy default stream,
+      // which a non-blocking stream's kernels are not ordered after
+      ZO_CUDA(cudaMemsetAsync(c->d_s_count, 0, sizeof(uint32_t) * (cap / 32), c->stream),
+              "zero S counters");
       c->s_cap = cap;
     }
     if (part > c->part_cap) {
@@ -1005,12 +1018,14 @@ zo_status zo_sync_status(zo_ctx* c) {
   uint32_t s = 0;
   ZO_CUDA(cudaMemcpy(&s, c->d_status, sizeof(s), cudaMemcpyDeviceToHost), "read status");
   if (s != 0) {
-    ZO_CUDA(cudaMemset(c->d_status, 0, sizeof(uint32_t)), "clear status");
+    // cleared on the context's stream (ordered before its next kernels) and waited for
+    ZO_CUDA(cudaMemsetAsync(c->d_status, 0, sizeof(uint32_t), c->stream), "clear status");
+    // a perturbed-linear S kernel cut short can leave its group counters part-counted
+    if ((s & zo::kDevTimeout) && c->d_s_count)
+      ZO_CUDA(cudaMemsetAsync(c->d_s_count, 0, sizeof(uint32_t) * (c->s_cap / 32), c->stream),
+              "zero S counters");
+    ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
     if (s & zo::kDevTimeout) {
-      // a perturbed-linear S kernel cut short can leave its group counters part-counted
-      if (c->d_s_count)
-        ZO_CUDA(cudaMemset(c->d_s_count, 0, sizeof(uint32_t) * (c->s_cap / 32)),
-                "zero S counters");
       g_last_error = "a device-side wait ran out";
       return ZO_ERR_TIMEOUT;
     }
