@@ -223,7 +223,9 @@ ZO_API zo_status zo_mezo_perturb(zo_ctx* ctx, uint32_t t, float coef);
  *   multiple of 8, else ZO_ERR_SHAPE).  The dense product is exact in bf16 with fp32
  *   accumulation; the rank-r term carries the bf16 hi/lo split's ~2^-16 relative error;
  *   Y is rounded to bf16 once.  W_i is read, never written.  Asynchronous; device errors
- *   go to the status word.
+ *   go to the status word.  The GEMM's tiling follows ZO_OPTION_LINEAR_TILE (all tilings
+ *   give the same Y bits); the context keeps an S workspace sized for the most tokens
+ *   seen so far, and a call with more synchronises the stream to grow it.
  */
 ZO_API zo_status zo_linear_prepare(zo_ctx* ctx, uint32_t t, int32_t qa, float ca, int32_t qb,
                                    float cb, float eps);
