@@ -64,7 +64,7 @@ typedef enum zo_status {
   ZO_ERR_DTYPE = 4,         /* unknown weight dtype */
   ZO_ERR_CUDA = 5,          /* a CUDA runtime call failed (message: zo_last_error) */
   ZO_ERR_TIMEOUT = 6,       /* a bounded device-side wait ran out (zo_sync_status) */
-  ZO_ERR_UNSUPPORTED = 7,   /* valid request this build does not implement */
+  ZO_ERR_UNSUPPORTED = 7,   /* valid request the library does not implement */
   ZO_ERR_NOMEM = 8          /* workspace allocation failed */
 } zo_status;
 
@@ -127,7 +127,7 @@ typedef struct zo_ctx zo_ctx;
 /*
  * zo_create -- bind the caller's matrices into a context (Alg. 3 "Require" line).
  *   mats[n_mats]: copied; the pointers inside must stay valid until zo_destroy.
- *   r: subspace rank, 1 <= r <= min(m_i, n_i); this build supports r in {4, 8, 16, 32, 64, 128}.
+ *   r: subspace rank, 1 <= r <= min(m_i, n_i); the library supports r in {4, 8, 16, 32, 64, 128}.
  *   q: queries per step (K in the paper), 1 <= q <= 4096.
  *   seed: 64-bit base seed of the Philox key.
  *   matrix_index_base: matrix i of this table uses Philox matrix index base + i

@@ -18,7 +18,7 @@ Plain fp64 restatement of Sec. 4 of the paper:
 * ``run_schedule`` -- the Alg. 3 loop for one matrix: a refresh (Alg. 1) when
   t mod F == 0, the query passes, the Adam step fused with the final restore.
 
-Readings of points the paper leaves open (each also listed in the design doc):
+Readings of points the paper leaves open:
 * the Adam exponent t in Eq. (9) is the count of Adam updates including the
   current one (``adam_t`` >= 1), since Alg. 3 starts at t = 0;
 * moments are zeroed once (Alg. 3 first line) and kept across subspace

@@ -24,7 +24,9 @@ from oracle import rng, rounding
 
 REL = 1e-5
 UV_ABS = 1e-5
-# Box-Muller normals: fp32 log/sqrt/sincospi against fp64
+# Box-Muller normals: fp32 log/sqrt/sincospi against fp64.  With |log error| <= 1 ulp,
+# a correctly rounded sqrt and <= 1 ulp sin/cos, |dz| <= sqrt(-2 ln 2^-24) * (a few fp32
+# ulps) ~ 5.77 * 4 * 6e-8 ~ 1.4e-6
 NORMAL_ABS = 2e-6
 
 
