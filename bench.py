@@ -2,10 +2,11 @@
 """Benchmark of the SubZero+ weight path on GB300: ZO steps/s and weight-pass HBM GB/s.
 
 Default workload: the LLaMA-7B-shaped parameter set (224 bf16 matrices, 6.48 G
-parameters, r = 32, q = 4 queries, central differences -> 8 weight passes per
-step, subspace refresh every 25 steps).  One "step" is Alg. 3's iteration for
-every matrix: the 2q-1 perturbation passes, the subspace-Adam update fused with
-the last restore, and (when t mod F == 0) the batched QR refresh.  The losses
+parameters, r = 32, q = 4 queries, central differences -> 2q + 1 = 9 weight
+passes per step, subspace refresh every 25 steps).  One "step" is Alg. 3's
+iteration for every matrix: the 2q perturbation passes (+Z0, -2Z0, +Z0+Z1, ...,
+-2Z_{q-1}, a loss evaluation after each), the subspace-Adam update fused with the
+last restore, and (when t mod F == 0) the batched QR refresh.  The losses
 the forward passes would produce are synthetic (2.0 + 0.01 N(0,1)); the weights
 are N(0, 0.02^2) bf16.  25.9 GB of weights per pass is far larger than the
 129 MB L2, so every pass streams from HBM.
