@@ -196,6 +196,7 @@ def oracle_sample_step_seconds(wl, scheme, sample=((0, 1024),), seed_shift=0):
     from paper_2608_15665_gb300 import workloads
     t_pass = t_ref = 0.0
     el_sample = uv_sample = 0
+    used = []                                      # (matrix, rows actually sampled)
     cpu_s = wall_s = 0.0
     seed = wl.seed + seed_shift
     for i, n_rows in sample:
@@ -223,10 +224,11 @@ def oracle_sample_step_seconds(wl, scheme, sample=((0, 1024),), seed_shift=0):
         cpu_s += time.process_time() - c0
         el_sample += rows.size * n
         uv_sample += m + n
+        used.append((i, rows.size))
     step_s = t_pass * wl.params / el_sample
     refresh_s = t_ref * sum(m + n for m, n in wl.shapes) / uv_sample
     text = ("fp64 oracle, one step: all weight passes + estimator + Adam on "
-            + ", ".join(f"{r} rows of matrix {i} {wl.shapes[i][0]}x{wl.shapes[i][1]}" for i, r in sample)
+            + ", ".join(f"{r} rows of matrix {i} {wl.shapes[i][0]}x{wl.shapes[i][1]}" for i, r in used)
             + f" ({el_sample} of {wl.params} weights) and the refresh of those matrices; "
             f"extrapolated by weight count (refresh by m+n, amortized over F={wl.F})")
     cores = round(cpu_s / (t_pass + t_ref), 1) if t_pass + t_ref > 0 else 1.0
