@@ -83,3 +83,44 @@ def test_rng_fills_validate_sizes(lib):
     assert L.zo_philox_fill(1, 0, 0, 0, None, -1, None) == lib.ZO_ERR_INVALID_ARG
     assert L.zo_normal_fill(1, 0, 0, 0, None, 16, None) == lib.ZO_ERR_INVALID_ARG
     assert L.zo_philox_fill(1, 0, 0, 0, None, 0, None) == lib.ZO_OK   # empty: nothing launched
+
+
+def test_create_rejects_an_empty_set_and_a_null_output(lib):
+    arr = (lib.zo_matrix * 1)(_mat(lib))
+    ctx = ctypes.c_void_p(0x1234)
+    assert lib.LIB.zo_create(ctypes.byref(ctx), arr, 0, 8, 2, 1, 0, None) == lib.ZO_ERR_INVALID_ARG
+    assert not ctx.value                                       # *out cleared on failure
+    assert lib.LIB.zo_create(ctypes.byref(ctx), None, 1, 8, 2, 1, 0, None) == lib.ZO_ERR_INVALID_ARG
+    assert lib.LIB.zo_create(None, arr, 1, 8, 2, 1, 0, None) == lib.ZO_ERR_INVALID_ARG
+
+
+def test_create_without_a_device_fails_instead_of_falling_back(lib):
+    # a valid request on a machine with no visible GPU: the library has no CPU path, so the
+    # context is refused with ZO_ERR_CUDA (on a GPU machine the same call would build a
+    # context over the fake pointers, so it is not made there)
+    from conftest import cuda_available
+    if cuda_available():
+        pytest.skip("a GPU is visible")
+    st, ctx = _create_status(lib, [_mat(lib)])
+    assert st == lib.ZO_ERR_CUDA and not ctx.value
+    assert lib.LIB.zo_last_error()
+
+
+def _noalloc(lib, W=0x1000, m=64, n=64, ldw=64, dtype=0, U=0x2000, V=0x3000, r=8, qa=0, qb=-1,
+             ca=1.0, cb=0.0, eps=1e-3):
+    return lib.LIB.zo_perturb_noalloc(W, m, n, ldw, dtype, U, V, r, 1, 0, 0, qa, ca, qb, cb, eps,
+                                      None)
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(W=0), 1), (dict(U=0), 1), (dict(V=0), 1),               # null buffers
+    (dict(dtype=3), 4),                                           # unknown dtype
+    (dict(r=128), 2), (dict(r=5), 2),                             # ranks outside {4 ... 64}
+    (dict(m=4), 2), (dict(ldw=32), 2),                            # r > m, ldw < n
+    (dict(qa=-1), 1), (dict(qb=-2), 1), (dict(eps=float("inf")), 1),
+    (dict(W=0x1008), 3), (dict(ldw=66, dtype=1), 3),              # alignment
+    (dict(n=40000, ldw=40000, r=64), 2),                          # beyond the 8 MiB scratch
+])
+def test_noalloc_validates_on_the_host(lib, kw, status):
+    # every one of these is refused before any CUDA call, so it needs no device
+    assert _noalloc(lib, **kw) == status
