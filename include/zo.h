@@ -183,8 +183,10 @@ ZO_API zo_status zo_perturb(zo_ctx* ctx, uint32_t t, int32_t qa, float ca, int32
  *   W_i <- rnd(W_i + U_i (-lr D_i + restore_coef * eps * Z_i^(restore_query)) V_i^T)
  *     (Eq. (10) plus the restore; restore_query = -1 drops the restore term).
  * losses: n_losses fp32 values (2q central, q+1 forward, q direct); device memory
- *   unless losses_on_host != 0, in which case they are copied from host memory
- *   before the launch (the host buffer may be reused when the call returns).
+ *   unless losses_on_host != 0, in which case they are copied from host memory on the
+ *   context's stream before the launch.  A pageable host buffer may be reused as soon
+ *   as the call returns (the runtime stages it before returning); a page-locked one is
+ *   read only when the stream reaches the copy, so it must stay unchanged until then.
  * gamma_out: NULL or device array of n_mats floats receiving ||G_i||_F (Sec. 4.1).
  */
 ZO_API zo_status zo_step(zo_ctx* ctx, uint32_t t, int32_t adam_t, const float* losses, int32_t n_losses,

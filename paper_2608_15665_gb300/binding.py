@@ -190,7 +190,9 @@ def zo_perturb(ctx, t, qa, ca, qb, cb, eps):
 
 def zo_step(ctx, t, adam_t, losses, scheme, eps, lr, beta1, beta2, eps_adam, restore_query,
             restore_coef, optimizer=ZO_OPT_ADAM, gamma_out=None):
-    """losses: a CUDA fp32 tensor, or a CPU fp32 tensor / numpy array (copied by the library)."""
+    """losses: a CUDA fp32 tensor, or a CPU fp32 tensor / numpy array (copied by the library
+    on the context's stream; a page-locked CPU tensor is read only when the stream reaches
+    that copy, so keep it alive and unchanged until then)."""
     import numpy as np
     keep = None
     if hasattr(losses, "is_cuda") and losses.is_cuda:
