@@ -243,6 +243,8 @@ ZO_API zo_status zo_set_option(zo_ctx* ctx, int32_t option, int64_t value);
 /*
  * zo_get_timing -- with ZO_OPTION_TIMING on, the summed device time (ms) and count of
  * weight-pass kernel launches since the option was last set.  Synchronises the stream.
+ * The context holds a pair of CUDA events per timed launch until this call folds them
+ * into the totals (and reuses them), so long timed runs should call it now and then.
  */
 ZO_API zo_status zo_get_timing(zo_ctx* ctx, double* total_ms, int64_t* launches);
 
