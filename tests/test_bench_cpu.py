@@ -1,5 +1,6 @@
 """bench.py pieces that need no GPU: the reference arm (the fp64 oracle timed on the
-host cores) and the parsing of the clock record taken during the timed region."""
+host cores), the parsing of the clock record taken during the timed region, the code
+hash that keys the ncu-derived traffic, and the layer subsets used for profiling captures."""
 
 import json
 import os
@@ -107,3 +108,18 @@ def test_code_hash_ignores_comments_and_spacing(tmp_path, monkeypatch):
     assert bench._code_hash(["k.cu"]) == h0
     (csrc / "k.cu").write_text("int f(int x) { return x + 2; }\n")
     assert bench._code_hash(["k.cu"]) != h0
+
+
+def test_layer_subsets_keep_the_shapes_and_zero_init_of_their_layers():
+    import bench
+    from paper_2608_15665_gb300 import workloads
+    wl = workloads.get("llama7b_bf16_r32")
+    assert bench.subset(wl, 0) is wl
+    two = bench.subset(wl, 2)
+    assert two.shapes == wl.shapes[:14] and two.r == wl.r and two.q == wl.q
+    assert two.params == 2 * wl.params // 32
+    lora = workloads.get("lora_opt13b_f32_r4")
+    sub = bench.subset(lora, 3)
+    assert sub.shapes == lora.shapes[:12]
+    assert list(sub.zero_init) == [i for i in lora.zero_init if i < 12] and len(sub.zero_init) > 0
+    assert bench.subset(lora, 1000).shapes == lora.shapes    # more layers than there are: all
