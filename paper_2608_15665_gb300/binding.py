@@ -254,9 +254,24 @@ def zo_kernel_launches(ctx):
 
 
 def zo_perturb_noalloc(W, U, V, r, seed, matrix_index, t, qa, ca, qb, cb, eps, stream=None):
-    """One perturbation pass on one matrix with no device allocation (see include/zo.h)."""
+    """One perturbation pass on one matrix with no device allocation (see include/zo.h).
+    W: m x n bf16/fp32 with unit column stride; U (m x r) and V (n x r) contiguous fp32 --
+    checked here, since the C ABI cannot see the sizes behind its pointers."""
     import torch
-    dt = ZO_BF16 if W.dtype == torch.bfloat16 else ZO_F32 if W.dtype == torch.float32 else -1
+    if W.dtype == torch.bfloat16:
+        dt = ZO_BF16
+    elif W.dtype == torch.float32:
+        dt = ZO_F32
+    else:
+        raise ZoError(ZO_ERR_DTYPE, "zo_perturb_noalloc", str(W.dtype))
+    if W.dim() != 2 or W.stride(1) != 1:
+        raise ZoError(ZO_ERR_SHAPE, "zo_perturb_noalloc", "W must be 2-D with unit column stride")
+    for name, t_, rows in (("U", U, W.shape[0]), ("V", V, W.shape[1])):
+        if t_.dtype != torch.float32 or not t_.is_contiguous():
+            raise ZoError(ZO_ERR_DTYPE, "zo_perturb_noalloc", f"{name} must be contiguous fp32")
+        if tuple(t_.shape) != (rows, int(r)):
+            raise ZoError(ZO_ERR_SHAPE, "zo_perturb_noalloc",
+                          f"{name} has shape {tuple(t_.shape)}, expected {(rows, int(r))}")
     _check(LIB.zo_perturb_noalloc(_ptr(W), W.shape[0], W.shape[1], W.stride(0), dt, _ptr(U),
                                   _ptr(V), int(r), int(seed) & (2**64 - 1), int(matrix_index),
                                   int(t), int(qa), float(ca), int(qb), float(cb), float(eps),

@@ -9,7 +9,9 @@
 // P = C V^T, weight pass) on one matrix, with every piece of scratch -- the one-entry
 // matrix table, the tile prefix, the projection work list, C and P -- placed in the
 // file-scope array below.  That array is a fixed 8 MiB that every GPU which loads
-// this library keeps until the process exits.
+// this library keeps until the process exits.  The tables are written by a small kernel
+// that takes them as launch parameters, so a call makes no host-to-device copy: it is
+// four kernel launches on the caller's stream and nothing else.
 #include <algorithm>
 #include <cmath>
 #include <mutex>
@@ -50,6 +52,21 @@ Layout layout_for(int64_t n, int32_t r) {
 zo_status fail(zo_status st, const std::string& msg) {
   zo::set_last_error(msg);
   return st;
+}
+
+// Writes the one-entry matrix table, the tile prefix (0, tiles) and the projection work
+// list (matrix 0, first column 128 u) for u < n_units into the scratch array.
+__global__ void __launch_bounds__(256)
+noalloc_tables_kernel(zo::MatDesc d, int64_t tiles, int32_t n_units, zo::MatDesc* __restrict__ desc,
+                      int64_t* __restrict__ prefix, int2* __restrict__ units) {
+  const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (tid == 0) {
+    *desc = d;
+    prefix[0] = 0;
+    prefix[1] = tiles;
+  }
+  for (int64_t u = tid; u < n_units; u += (int64_t)gridDim.x * blockDim.x)
+    units[u] = make_int2(0, (int)(u * 128));
 }
 
 }  // namespace
@@ -105,7 +122,8 @@ extern "C" ZO_API zo_status zo_perturb_noalloc(void* W, int64_t m, int64_t n, in
     scratch = g_scratch_ptr[dev];
   }
 
-  // one-entry table, tile prefix and projection work list, written into the scratch
+  // one-entry table, tile prefix and projection work list, written into the scratch by
+  // the first of the call's kernels
   zo::MatDesc d{};
   d.W = W;
   d.m = m;
@@ -118,23 +136,16 @@ extern "C" ZO_API zo_status zo_perturb_noalloc(void* W, int64_t m, int64_t n, in
   d.C = scratch + L.C;
   d.P = scratch + L.P;
   d.tile0 = 0;
-  const int64_t prefix[2] = {0, tiles};
   const int64_t n_units = (n + 127) / 128;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   zo::MatDesc* d_desc = reinterpret_cast<zo::MatDesc*>(scratch + L.desc);
   int64_t* d_prefix = reinterpret_cast<int64_t*>(scratch + L.prefix);
   int2* d_units = reinterpret_cast<int2*>(scratch + L.units);
-  e = cudaMemcpyAsync(d_desc, &d, sizeof(d), cudaMemcpyHostToDevice, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(d_prefix, prefix, sizeof(prefix), cudaMemcpyHostToDevice, s);
-  // the work list is (0, 128 k), written in chunks from a small host buffer (a copy from
-  // pageable host memory has been staged when cudaMemcpyAsync returns, so it is reusable)
-  int2 chunk[256];
-  for (int64_t u0 = 0; e == cudaSuccess && u0 < n_units; u0 += 256) {
-    const int64_t cnt = std::min<int64_t>(256, n_units - u0);
-    for (int64_t k = 0; k < cnt; ++k) chunk[k] = make_int2(0, (int)((u0 + k) * 128));
-    e = cudaMemcpyAsync(d_units + u0, chunk, sizeof(int2) * cnt, cudaMemcpyHostToDevice, s);
-  }
-  if (e != cudaSuccess) return fail(ZO_ERR_CUDA, std::string("table upload: ") + cudaGetErrorString(e));
+  const int table_blocks = (int)std::min<int64_t>((n_units + 255) / 256, 64);
+  noalloc_tables_kernel<<<table_blocks, 256, 0, s>>>(d, tiles, (int32_t)n_units, d_desc, d_prefix,
+                                                      d_units);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(ZO_ERR_CUDA, std::string("table kernel: ") + cudaGetErrorString(e));
 
   zo::CoeffParams p{};
   p.mode = zo::kCoeffPerturb;

@@ -124,3 +124,31 @@ def _noalloc(lib, W=0x1000, m=64, n=64, ldw=64, dtype=0, U=0x2000, V=0x3000, r=8
 def test_noalloc_validates_on_the_host(lib, kw, status):
     # every one of these is refused before any CUDA call, so it needs no device
     assert _noalloc(lib, **kw) == status
+
+
+@pytest.mark.parametrize("what", ["U rows", "V rank", "U dtype", "V strided", "W strided",
+                                  "W dtype"])
+def test_noalloc_binding_checks_shapes_before_the_call(lib, what):
+    # the C ABI cannot see the sizes behind U and V; the binding refuses a U or V that does
+    # not hold m x r / n x r contiguous fp32 values, and a W without unit column stride,
+    # before the library is called (CPU tensors: nothing reaches a device)
+    import torch
+    m, n, r = 64, 96, 8
+    W = torch.zeros(m, n)
+    U = torch.zeros(m, r)
+    V = torch.zeros(n, r)
+    if what == "U rows":
+        U = torch.zeros(m - 1, r)
+    elif what == "V rank":
+        V = torch.zeros(n, 2 * r)
+    elif what == "U dtype":
+        U = U.double()
+    elif what == "V strided":
+        V = torch.zeros(n, 2 * r)[:, ::2]
+    elif what == "W strided":
+        W = torch.zeros(n, m).t()
+    else:
+        W = W.half()
+    with pytest.raises(lib.ZoError) as e:
+        lib.zo_perturb_noalloc(W, U, V, r, 1, 0, 0, 0, 1.0, -1, 0.0, 1e-3)
+    assert e.value.status in (lib.ZO_ERR_SHAPE, lib.ZO_ERR_DTYPE)
