@@ -88,7 +88,11 @@ enum {
 enum {
   ZO_OPTION_WPASS_PATH = 0, /* 0 = automatic: tcgen05 when every W is bf16 with n a
                                    multiple of 8 (its TMA stores write 16-byte chunks) and
-                                   r >= 16;
+                                   r >= 16 -- if such a set's tensor-core descriptors
+                                   cannot be built (cuTensorMapEncodeTiled rejects one, e.g.
+                                   a W row stride of 2^40 bytes or more), zo_perturb and
+                                   zo_step return ZO_ERR_UNSUPPORTED instead of running
+                                   another pass, and value 1 selects the FMA pass;
                                    else, at r in {4, 8}, the narrow-tile FMA pass when its
                                    tiles number at most half of the 32-row tiles (sets of
                                    thin matrices such as LoRA factors); else the FMA pass,
@@ -168,6 +172,10 @@ ZO_API zo_status zo_init_subspace(zo_ctx* ctx, uint32_t refresh_idx);
  * next (e.g. ca = +1, cb = -1 gives W += eps U (Z_(k+1) - Z_k) V^T); the sum is
  * formed in fp32 and W is rounded once (RNE) to its dtype.
  * 0 <= qa, qb < q.
+ * The update U C V^T is evaluated to fp32 grade on either path: the FMA pass in fp32;
+ * the tensor-core pass with U, P = C V^T (and, in the projection, V and C) held as
+ * power-of-two-scaled fp16 pairs hi + lo (~22 significant bits) and three products
+ * accumulated in fp32, which errs by ~2^-21 of sum |U| |C| |V|^T.
  */
 ZO_API zo_status zo_perturb(zo_ctx* ctx, uint32_t t, int32_t qa, float ca, int32_t qb, float cb,
                      float eps);
@@ -293,9 +301,13 @@ ZO_API zo_status zo_normal_fill(uint64_t seed, uint32_t x1, uint32_t x2, uint32_
  * floats -- is rejected with ZO_ERR_SHAPE before anything is launched.
  * The first call on a device looks up that array's device address (cudaGetSymbolAddress)
  * with the device current; make that first call before capturing any stream.
+ * A call copies nothing from the host: it launches four kernels on `stream` (the first
+ * writes the call's small tables into the array from its launch parameters).
  * All calls share the one array and rewrite everything they read from it before
  * reading it, so nothing needs clearing between calls -- but two calls whose work
  * overlaps on the GPU (different streams, or different host threads) race on it.
+ * U must hold m x r and V n x r contiguous fp32 values: the C ABI cannot check the sizes
+ * of the buffers behind the pointers.
  * Asynchronous on `stream` (void* cudaStream_t); errors as for zo_perturb.
  */
 ZO_API zo_status zo_perturb_noalloc(void* W, int64_t m, int64_t n, int64_t ldw, int32_t dtype,

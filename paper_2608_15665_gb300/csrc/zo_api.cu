@@ -103,11 +103,17 @@ struct zo_ctx {
   int64_t launches = 0;          // kernels launched by this context
   // tensor-core weight pass (all matrices bf16, r in {16, 32, 64, 128})
   bool tc_ok = false;
+  bool tc_failed = false;            // the set qualifies, but its setup failed (zo_last_error
+                                     // at zo_create); the automatic path then refuses to run
+  std::string tc_fail_msg;
   bool proj_tc = false;              // the projection's descriptors are in place
   int sms = 0;
-  void* d_u_op = nullptr;            // stacked U operand of every U_i, 128-row padded
-                                     // (rows [hi | lo | 0] for r <= 32, chunk-major for r >= 64)
-  __nv_bfloat16* d_p_hl = nullptr;   // stacked [hi | lo] rows of every P_i^T, 128-row padded
+  void* d_u_op = nullptr;            // stacked U operand of every U_i, 128-row padded: the fp16
+                                     // pair of U 2^14 (rows [hi | lo | 0] for r <= 32,
+                                     // chunk-major for r >= 64)
+  uint16_t* d_p_hl = nullptr;        // stacked [hi | lo] fp16 rows of every P_i^T 2^(e_P,i),
+                                     // 128-row padded
+  float* d_pinv = nullptr;           // 2^-(e_P,i) of the current pass, one per matrix
   zo::TcMat* d_tc = nullptr;
   std::vector<zo::TcMat> h_tc;       // host copy (operand rows of each matrix)
   // zo_linear_prepare / zo_linear_perturbed: P_K of every matrix ([P_hi ; P_lo] rows,
@@ -116,6 +122,10 @@ struct zo_ctx {
   int64_t* d_pk_off = nullptr;
   std::vector<int64_t> h_pk_off;
   bool linear_ready = false;
+  __nv_bfloat16* d_u_lin = nullptr;  // the U operand as a bf16 pair (rows as d_u_op at r <= 32)
+  CUtensorMap tm_u_lin{};
+  bool u_lin_valid = false;          // d_u_lin holds the current U (cleared by every refresh)
+  int64_t u_rows = 0;                // rows of the stacked U operand
   int linear_tile = 0;           // ZO_OPTION_LINEAR_TILE
   int last_linear_tiling = 0;    // tiling of the last Y GEMM (1..3)
   __nv_bfloat16* d_s_hl = nullptr;
@@ -127,8 +137,8 @@ struct zo_ctx {
   CUtensorMap tm_a{}, tm_b{};        // descriptors of the stacked operands (kernel parameters)
   int2* d_u_units = nullptr;
   int32_t n_u_units = 0;
-  __nv_bfloat16* d_v_hl = nullptr;   // [hi | lo] rows of every V_i, rows as P_HL
-  __nv_bfloat16* d_c_hl = nullptr;   // [hi | lo] rows of every C_i, r rows each
+  uint16_t* d_v_hl = nullptr;        // fp16 [hi | lo] rows of every V_i 2^14, rows as P_HL
+  uint16_t* d_c_hl = nullptr;        // fp16 [hi | lo] rows of every C_i 2^(e_C,i), r rows each
   CUtensorMap tm_v{}, tm_c{}, tm_p{};  // V_HL, C_HL, and P_HL in 32-row boxes
   bool timing = false;
   std::vector<cudaEvent_t> ev_start, ev_stop;
@@ -167,6 +177,8 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_u_units);
   cudaFree(c->d_v_hl);
   cudaFree(c->d_c_hl);
+  cudaFree(c->d_pinv);
+  cudaFree(c->d_u_lin);
   for (auto e : c->ev_start) cudaEventDestroy(e);
   for (auto e : c->ev_stop) cudaEventDestroy(e);
   delete c;
@@ -257,6 +269,13 @@ zo_status record_stop(zo_ctx* c) {
 }
 
 bool tc_path(const zo_ctx* c) { return c->tc_ok && (c->path_option == 0 || c->path_option == 2); }
+// The automatic path on a set that qualifies for the tensor cores but could not be set up
+// for them: refused (ZO_ERR_UNSUPPORTED) instead of running the FMA pass unasked.
+bool tc_refused(const zo_ctx* c) { return c->tc_failed && c->path_option == 0; }
+zo_status refuse_tc(const zo_ctx* c) {
+  g_last_error = c->tc_fail_msg;
+  return ZO_ERR_UNSUPPORTED;
+}
 bool narrow_path(const zo_ctx* c) {
   return c->narrow_ok && (c->path_option == 3 || (c->path_option == 0 && c->narrow_auto));
 }
@@ -280,7 +299,8 @@ zo_status run_weight_pass(zo_ctx* c) {
   }
   if (use_tc) {
     // setup_tc keeps tc_ok only with the projection's descriptors in place (proj_tc)
-    ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, c->r, c->d_c_hl, c->stream), "split C");
+    ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, c->r, c->d_c_hl, c->d_pinv, c->stream),
+            "split C");
     ++c->launches;
     const int grid = std::min<int>(c->n_proj_units, c->sms);
     ZO_CUDA(zo::launch_project_tc(c->tm_v, c->tm_c, c->tm_p, c->d_tc, c->d_proj_units,
@@ -297,8 +317,8 @@ zo_status run_weight_pass(zo_ctx* c) {
     const int grid = (int)std::min<int64_t>(c->tc_tiles, c->sms);
     const bool inject = c->inject_wait;
     c->inject_wait = false;
-    ZO_CUDA(zo::launch_wpass_tc(c->tm_a, c->d_u_op, c->tm_b, c->d_w_maps, c->d_tc, c->n_mats, c->tc_tiles,
-                                grid, c->r, c->d_status, inject, c->stream),
+    ZO_CUDA(zo::launch_wpass_tc(c->tm_a, c->d_u_op, c->tm_b, c->d_w_maps, c->d_tc, c->d_pinv,
+                                c->n_mats, c->tc_tiles, grid, c->r, c->d_status, inject, c->stream),
             "tensor-core weight-pass kernel");
     c->last_path = 2;
   } else {
@@ -324,20 +344,30 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
-// 2-D bf16 tensor map: `cols` contiguous elements per row, `rows` rows `row_bytes` apart,
-// boxes of box_cols x box_rows with the 128-byte swizzle.
-bool encode_bf16_2d(CUtensorMap* tm, void* base, uint64_t cols, uint64_t rows, uint64_t row_bytes,
-                    uint32_t box_cols, uint32_t box_rows,
-                    CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
+// 2-D tensor map of 16-bit elements (bf16, or fp16 with f16 = true): `cols` contiguous
+// elements per row, `rows` rows `row_bytes` apart, boxes of box_cols x box_rows with the
+// 128-byte swizzle.
+bool encode_16b_2d(CUtensorMap* tm, void* base, uint64_t cols, uint64_t rows, uint64_t row_bytes,
+                   uint32_t box_cols, uint32_t box_rows, bool f16,
+                   CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   auto enc = tensor_map_encoder();
   if (!enc) return false;
   const cuuint64_t dims[2] = {cols, rows};
   const cuuint64_t strides[1] = {row_bytes};
   const cuuint32_t box[2] = {box_cols, box_rows};
   const cuuint32_t estr[2] = {1, 1};
-  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
+  return enc(tm, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base,
+             dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+bool encode_bf16_2d(CUtensorMap* tm, void* base, uint64_t cols, uint64_t rows, uint64_t row_bytes,
+                    uint32_t box_cols, uint32_t box_rows,
+                    CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
+  return encode_16b_2d(tm, base, cols, rows, row_bytes, box_cols, box_rows, false, swizzle);
+}
+bool encode_f16_2d(CUtensorMap* tm, void* base, uint64_t cols, uint64_t rows, uint64_t row_bytes,
+                   uint32_t box_cols, uint32_t box_rows) {
+  return encode_16b_2d(tm, base, cols, rows, row_bytes, box_cols, box_rows, true);
 }
 
 // Tile table of the narrow-tile FMA pass (r in {4, 8}).
@@ -390,10 +420,20 @@ zo_status setup_narrow(zo_ctx* c, const zo_matrix* mats) {
 // the context does not qualify: an fp32 matrix, r outside {16, 32, 64, 128}, or a
 // width n not a multiple of 8 -- TMA stores write whole 16-byte chunks, and the chunk
 // that holds a row's last element would also overwrite the caller's elements past n.
+// A set that qualifies but whose descriptors or row counts the tensor-core pass cannot
+// take gets tc_failed instead: the automatic path then returns ZO_ERR_UNSUPPORTED rather
+// than running the FMA pass in its place; ZO_OPTION_WPASS_PATH = 1 selects that pass.
 zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
   if (!zo::wpass_tc_supported(c->r)) return ZO_OK;
   for (int32_t i = 0; i < c->n_mats; ++i)
     if (mats[i].dtype != ZO_BF16 || mats[i].n % 8 != 0) return ZO_OK;
+  auto refuse = [&](const char* why) {
+    c->tc_failed = true;
+    c->tc_fail_msg = std::string("the tensor-core weight pass could not be set up (") + why +
+                     "); set ZO_OPTION_WPASS_PATH = 1 to run the FMA pass instead";
+    g_last_error = c->tc_fail_msg;
+    return ZO_OK;
+  };
   const int64_t BM = zo::tc_tile_rows(), BN = zo::tc_tile_cols();
   const int64_t HLW = zo::tc_hl_width(c->r);
   std::vector<zo::TcMat> tc(c->n_mats);
@@ -413,14 +453,18 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
     prows += (n + BN - 1) / BN * BN;
     for (int64_t r0 = 0; r0 < m; r0 += 128) uunits.push_back(make_int2(i, (int)r0));
   }
-  if (urows >= (int64_t(1) << 31) || prows >= (int64_t(1) << 31)) return ZO_OK;
+  if (urows >= (int64_t(1) << 31) || prows >= (int64_t(1) << 31))
+    return refuse("more than 2^31 stacked operand rows");
   c->h_tc = tc;
+  c->u_rows = urows;
   ZO_CUDA(cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, c->device), "SM count");
   const int64_t u_bytes = zo::tc_u_operand_bytes(c->r, urows);
   ZO_CUDA(cudaMalloc(&c->d_u_op, u_bytes), "cudaMalloc(U hi/lo)");
-  ZO_CUDA(cudaMalloc(&c->d_p_hl, sizeof(__nv_bfloat16) * prows * HLW), "cudaMalloc(P hi/lo)");
+  ZO_CUDA(cudaMalloc(&c->d_p_hl, sizeof(uint16_t) * prows * HLW), "cudaMalloc(P hi/lo)");
   ZO_CUDA(cudaMemset(c->d_u_op, 0, u_bytes), "memset");
-  ZO_CUDA(cudaMemset(c->d_p_hl, 0, sizeof(__nv_bfloat16) * prows * HLW), "memset");
+  ZO_CUDA(cudaMemset(c->d_p_hl, 0, sizeof(uint16_t) * prows * HLW), "memset");
+  ZO_CUDA(cudaMalloc(&c->d_pinv, sizeof(float) * c->n_mats), "cudaMalloc(P scales)");
+  ZO_CUDA(cudaMemset(c->d_pinv, 0, sizeof(float) * c->n_mats), "memset");
   ZO_CUDA(cudaMalloc(&c->d_tc, sizeof(zo::TcMat) * c->n_mats), "cudaMalloc(tile table)");
   ZO_CUDA(cudaMemcpy(c->d_tc, tc.data(), sizeof(zo::TcMat) * c->n_mats, cudaMemcpyHostToDevice),
           "upload tile table");
@@ -430,14 +474,20 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
           "upload units");
   c->n_u_units = (int32_t)uunits.size();
   std::vector<CUtensorMap> wmaps(c->n_mats);
-  bool ok = encode_bf16_2d(&c->tm_b, c->d_p_hl, HLW, prows, HLW * 2, 64, 128);
+  bool ok = encode_f16_2d(&c->tm_b, c->d_p_hl, HLW, prows, HLW * 2, 64, 128);
   if (ok && !zo::wpass_tc_u_in_tmem(c->r))   // r <= 32: U rows read by TMA
-    ok = encode_bf16_2d(&c->tm_a, c->d_u_op, HLW, urows, HLW * 2, 64, 128);
-  for (int32_t i = 0; ok && i < c->n_mats; ++i)
+    ok = encode_f16_2d(&c->tm_a, c->d_u_op, HLW, urows, HLW * 2, 64, 128);
+  int32_t bad_w = -1;
+  for (int32_t i = 0; ok && i < c->n_mats; ++i) {
     ok = encode_bf16_2d(&wmaps[i], mats[i].W, mats[i].n, mats[i].m, mats[i].ldw * 2, 64, 32);
+    if (!ok) bad_w = i;
+  }
   if (!ok) {
-    g_last_error = "cuTensorMapEncodeTiled unavailable or rejected a descriptor; using the FMA pass";
-    return ZO_OK;
+    const std::string why = bad_w >= 0 ? "cuTensorMapEncodeTiled rejected the descriptor of W_" +
+                                             std::to_string(bad_w)
+                                       : std::string("cuTensorMapEncodeTiled unavailable or "
+                                                     "rejected an operand descriptor");
+    return refuse(why.c_str());
   }
   ZO_CUDA(cudaMalloc(&c->d_w_maps, sizeof(CUtensorMap) * c->n_mats), "cudaMalloc(tensor maps)");
   ZO_CUDA(cudaMemcpy(c->d_w_maps, wmaps.data(), sizeof(CUtensorMap) * c->n_mats,
@@ -447,17 +497,17 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
   c->tc_ok = true;
   // the projection P = C V^T on the tensor cores (every tensor-core rank): V_HL, C_HL
   const int64_t crows = (int64_t)c->n_mats * c->r;
-  ZO_CUDA(cudaMalloc(&c->d_v_hl, sizeof(__nv_bfloat16) * prows * HLW), "cudaMalloc(V hi/lo)");
-  ZO_CUDA(cudaMemset(c->d_v_hl, 0, sizeof(__nv_bfloat16) * prows * HLW), "memset");
-  ZO_CUDA(cudaMalloc(&c->d_c_hl, sizeof(__nv_bfloat16) * crows * HLW), "cudaMalloc(C hi/lo)");
-  ZO_CUDA(cudaMemset(c->d_c_hl, 0, sizeof(__nv_bfloat16) * crows * HLW), "memset");
+  ZO_CUDA(cudaMalloc(&c->d_v_hl, sizeof(uint16_t) * prows * HLW), "cudaMalloc(V hi/lo)");
+  ZO_CUDA(cudaMemset(c->d_v_hl, 0, sizeof(uint16_t) * prows * HLW), "memset");
+  ZO_CUDA(cudaMalloc(&c->d_c_hl, sizeof(uint16_t) * crows * HLW), "cudaMalloc(C hi/lo)");
+  ZO_CUDA(cudaMemset(c->d_c_hl, 0, sizeof(uint16_t) * crows * HLW), "memset");
   c->proj_tc = zo::project_tc_supported(c->r) &&
-               encode_bf16_2d(&c->tm_v, c->d_v_hl, HLW, prows, HLW * 2, 64, 128) &&
-               encode_bf16_2d(&c->tm_c, c->d_c_hl, HLW, crows, HLW * 2, 64, (uint32_t)c->r) &&
-               encode_bf16_2d(&c->tm_p, c->d_p_hl, HLW, prows, HLW * 2, 64, 32);
+               encode_f16_2d(&c->tm_v, c->d_v_hl, HLW, prows, HLW * 2, 64, 128) &&
+               encode_f16_2d(&c->tm_c, c->d_c_hl, HLW, crows, HLW * 2, 64, (uint32_t)c->r) &&
+               encode_f16_2d(&c->tm_p, c->d_p_hl, HLW, prows, HLW * 2, 64, 32);
   if (!c->proj_tc) {
-    g_last_error = "cuTensorMapEncodeTiled rejected a projection descriptor; using the FMA pass";
     c->tc_ok = false;
+    return refuse("cuTensorMapEncodeTiled rejected a projection descriptor");
   }
   return ZO_OK;
 }
@@ -715,6 +765,7 @@ zo_status zo_refresh(zo_ctx* c, uint32_t refresh_idx, int32_t reset_moments) {
     ZO_CUDA(zo::launch_zero_moments(c->d_mats, c->n_mats, c->r, c->stream), "zero moments");
     ++c->launches;
   }
+  c->u_lin_valid = false;   // the linear route's bf16 U operand belongs to the old U
   if (c->tc_ok) {
     ZO_CUDA(zo::launch_split_u(c->d_mats, c->d_tc, c->d_u_units, c->n_u_units, c->r, c->d_u_op,
                                c->stream),
@@ -742,6 +793,7 @@ zo_status zo_perturb(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t qb, fl
     g_last_error = "zo_perturb: query index out of range or non-finite scalar";
     return ZO_ERR_INVALID_ARG;
   }
+  if (tc_refused(c)) return refuse_tc(c);
   zo::CoeffParams p{};
   p.mode = zo::kCoeffPerturb;
   p.seed = c->seed;
@@ -815,6 +867,7 @@ zo_status zo_step(zo_ctx* c, uint32_t t, int32_t adam_t, const float* losses, in
     inv_bc1 = 1.0 / (1.0 - std::pow((double)beta1, (double)adam_t));
     inv_bc2 = 1.0 / (1.0 - std::pow((double)beta2, (double)adam_t));
   }
+  if (tc_refused(c)) return refuse_tc(c);
   const float* d_losses = losses;
   if (losses_on_host) {
     ZO_CUDA(cudaMemcpyAsync(c->d_losses, losses, sizeof(float) * n_losses, cudaMemcpyHostToDevice,
@@ -884,6 +937,33 @@ zo_status zo_linear_prepare(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t
     c->d_pk = pk;
     c->d_pk_off = pk_off;
   }
+  if (!c->d_u_lin) {
+    // the route's U operand: the bf16 pair of U in rows laid out like d_u_op's (r <= 32)
+    const int64_t HLW = zo::tc_hl_width(r);
+    const size_t bytes = sizeof(__nv_bfloat16) * (size_t)c->u_rows * HLW;
+    __nv_bfloat16* u_lin = nullptr;
+    cudaError_t e = cudaMalloc(&u_lin, bytes);
+    // padding rows and columns stay zero; on the context's stream, before the split
+    if (e == cudaSuccess) e = cudaMemsetAsync(u_lin, 0, bytes, c->stream);
+    if (e != cudaSuccess) {
+      cudaFree(u_lin);
+      return cuda_fail(e, "linear U operand");
+    }
+    if (!encode_bf16_2d(&c->tm_u_lin, u_lin, HLW, c->u_rows, HLW * 2, 64, 128)) {
+      cudaFree(u_lin);
+      g_last_error = "zo_linear_prepare: cuTensorMapEncodeTiled rejected the U operand descriptor";
+      return ZO_ERR_CUDA;
+    }
+    c->d_u_lin = u_lin;
+    c->u_lin_valid = false;
+  }
+  if (!c->u_lin_valid) {
+    ZO_CUDA(zo::launch_split_u_bf16(c->d_mats, c->d_tc, c->d_u_units, c->n_u_units, r, c->d_u_lin,
+                                    c->stream),
+            "split U into a bf16 pair");
+    ++c->launches;
+    c->u_lin_valid = true;
+  }
   // C_i = eps (ca Z_qa + cb Z_qb) for every matrix, P_i = C_i V_i^T, P_K = [P_hi ; P_lo]
   zo::CoeffParams p{};
   p.mode = zo::kCoeffPerturb;
@@ -897,13 +977,14 @@ zo_status zo_linear_prepare(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t
   p.cb = cb;
   p.eps = eps;
   ZO_CUDA(zo::launch_coeff(c->d_mats, c->n_mats, p, c->stream), "coefficient kernel");
-  ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, r, c->d_c_hl, c->stream), "split C");
+  ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, r, c->d_c_hl, c->d_pinv, c->stream), "split C");
   ZO_CUDA(zo::launch_project_tc(c->tm_v, c->tm_c, c->tm_p, c->d_tc, c->d_proj_units,
                                 c->n_proj_units, std::min<int32_t>(c->n_proj_units, c->sms), r,
                                 c->d_status, c->stream),
           "tensor-core projection kernel");
   ZO_CUDA(zo::launch_transpose_p(c->d_p_hl, c->d_tc, c->d_proj_units, c->n_proj_units,
-                                 c->d_pk_off, (int32_t)zo::tc_hl_width(r), r, c->d_pk, c->stream),
+                                 c->d_pk_off, c->d_pinv, (int32_t)zo::tc_hl_width(r), r, c->d_pk,
+                                 c->stream),
           "P transpose");
   c->launches += 4;
   c->linear_ready = true;
@@ -981,7 +1062,7 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
   ZO_CUDA(zo::launch_linear_s(tm_x, tm_pk, T, n, r, k_split, k_chunk, c->d_s_part, c->d_s_hl,
                               c->d_s_count, c->sms, c->d_status, c->stream),
           "S = X P^T kernels");
-  ZO_CUDA(zo::launch_linear_y(tm_x, c->d_w_maps + mat, tm_s, c->tm_a, tm_y, T, m, n,
+  ZO_CUDA(zo::launch_linear_y(tm_x, c->d_w_maps + mat, tm_s, c->tm_u_lin, tm_y, T, m, n,
                               c->h_tc[mat].u_row0, r, tiling, c->sms, c->d_status, c->stream),
           "perturbed linear kernel");
   c->last_linear_tiling = tiling;

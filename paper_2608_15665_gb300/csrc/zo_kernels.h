@@ -97,39 +97,46 @@ cudaError_t launch_mezo(const MatDesc* d_mats, int32_t n_mats, const int64_t* d_
 // ---- weight pass, tcgen05 path (zo_wpass_tc.cu: r <= 32, zo_wpass_tmem.cu: r >= 64) -----
 bool wpass_tc_supported(int32_t r);
 bool wpass_tc_u_in_tmem(int32_t r);   // the U operand is read from Tensor Memory (r >= 64)
-int32_t tc_hl_width(int32_t r);       // bf16 elements per hi/lo operand row
+int32_t tc_hl_width(int32_t r);       // 16-bit elements per hi/lo operand row
 int32_t tc_tile_rows();
 int32_t tc_tile_cols();
 // Bytes of the stacked U operand for `rows` rows (both layouts below fit).
 int64_t tc_u_operand_bytes(int32_t r, int64_t rows);
-// The U operand of every matrix from U (after a refresh); units = (matrix, first row) x
-// 128 rows.  r <= 32: rows [hi | lo | 0] of tc_hl_width(r) bf16, read by TMA (tm_a);
-// r >= 64: chunk-major per 128-row block, read into Tensor Memory (zo_wpass_tmem.cu).
+// The U operand of every matrix from U (after a refresh): the fp16 pair of U 2^kUVScaleExp
+// (zo_tc_common.cuh); units = (matrix, first row) x 128 rows.  r <= 32: rows [hi | lo | 0]
+// of tc_hl_width(r) fp16, read by TMA (tm_a); r >= 64: chunk-major per 128-row block, read
+// into Tensor Memory (zo_wpass_tmem.cu).
 cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                            int32_t n_units, int32_t r, void* u_op, cudaStream_t s);
-// tm_a is used for r <= 32, u_op for r >= 64.
+// The perturbed-linear route's U operand (r in {16, 32}): rows [hi | lo | 0] of the bf16
+// pair of U, unscaled, laid out as the r <= 32 U operand above.
+cudaError_t launch_split_u_bf16(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                                int32_t n_units, int32_t r, __nv_bfloat16* u_lin, cudaStream_t s);
+// tm_a is used for r <= 32, u_op for r >= 64; d_pinv[i] = 2^-(e_P,i) from launch_split_c.
 cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const void* u_op, const CUtensorMap& tm_b,
-                            const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
-                            int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
-                            bool inject_wait, cudaStream_t s);
+                            const CUtensorMap* d_w_maps, const TcMat* d_tc, const float* d_pinv,
+                            int32_t n_mats, int64_t n_tiles, int32_t grid, int32_t r,
+                            uint32_t* d_status, bool inject_wait, cudaStream_t s);
 // r >= 64 (zo_wpass_tmem.cu)
 cudaError_t launch_split_u_chunks(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                                   int32_t n_units, int32_t r, uint4* u_t, cudaStream_t s);
 cudaError_t launch_wpass_tmem(const uint4* u_t, const CUtensorMap& tm_b,
-                              const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
-                              int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
-                              bool inject_wait, cudaStream_t s);
+                              const CUtensorMap* d_w_maps, const TcMat* d_tc, const float* d_pinv,
+                              int32_t n_mats, int64_t n_tiles, int32_t grid, int32_t r,
+                              uint32_t* d_status, bool inject_wait, cudaStream_t s);
 
 // ---- projection P = C V^T on the tensor cores, r >= 16 (zo_project_tc.cu) ---------
 bool project_tc_supported(int32_t r);
-// V_HL rows [hi | lo] of V (after a refresh); units = the projection units (matrix, first row)
+// V_HL rows [hi | lo] of the fp16 pair of V 2^kUVScaleExp (after a refresh); units = the
+// projection units (matrix, first row)
 cudaError_t launch_split_v(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                           int32_t n_units, int32_t r, __nv_bfloat16* v_hl, cudaStream_t s);
-// C_HL rows [hi | lo] of C (every pass), r rows per matrix at matrix * r
-cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, __nv_bfloat16* c_hl,
-                           cudaStream_t s);
-// P_HL = [hi | lo] of V C^T: tm_v over V_HL (box 64 x 128), tm_c over C_HL (box 64 x r),
-// tm_p over P_HL (box 64 x 32)
+                           int32_t n_units, int32_t r, uint16_t* v_hl, cudaStream_t s);
+// C_HL rows [hi | lo] of the fp16 pair of C_i 2^(e_C,i) (every pass), r rows per matrix at
+// matrix * r, and pinv[i] = 2^-(e_P,i), e_P,i = e_C,i + p_scale_offset(r)
+cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, uint16_t* c_hl,
+                           float* pinv, cudaStream_t s);
+// P_HL = [hi | lo] of the fp16 pair of (V C^T) 2^(e_P,i): tm_v over V_HL (box 64 x 128),
+// tm_c over C_HL (box 64 x r), tm_p over P_HL (box 64 x 32)
 cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
                               const CUtensorMap& tm_p, const TcMat* d_tc, const int2* d_units,
                               int32_t n_units, int32_t grid, int32_t r, uint32_t* d_status,
@@ -148,10 +155,11 @@ int32_t linear_y_tile_rows(int32_t tiling);
 int32_t linear_y_tile_cols(int32_t tiling);
 // Elements of matrix i's P_K: 2r rows of n rounded up to 64.
 int64_t linear_pk_elems(int64_t n, int32_t r);
-// P_K of every matrix from P_HL (units = the projection units, pk_off = element offsets).
-cudaError_t launch_transpose_p(const __nv_bfloat16* p_hl, const TcMat* d_tc, const int2* d_units,
-                               int32_t n_units, const int64_t* d_pk_off, int32_t hl_width,
-                               int32_t r, __nv_bfloat16* p_k, cudaStream_t s);
+// P_K of every matrix ([P_hi ; P_lo], the bf16 pair of P) from P_HL and pinv (units = the
+// projection units, pk_off = element offsets).
+cudaError_t launch_transpose_p(const uint16_t* p_hl, const TcMat* d_tc, const int2* d_units,
+                               int32_t n_units, const int64_t* d_pk_off, const float* d_pinv,
+                               int32_t hl_width, int32_t r, __nv_bfloat16* p_k, cudaStream_t s);
 // Kernels launch_linear_s launches for a split of k_split K ranges (1, or 2 with the
 // separate reduction).
 int32_t linear_s_launches(int32_t k_split);
@@ -164,7 +172,7 @@ cudaError_t launch_linear_s(const CUtensorMap& tm_x, const CUtensorMap& tm_pk, i
                             __nv_bfloat16* s_hl, uint32_t* s_count, int32_t sms,
                             uint32_t* d_status, cudaStream_t s);
 // Y = X W^T + S U^T: d_w_map = W's descriptor (box 64 x 32), tm_s_in over S_HL (box
-// 64 x 128), tm_u over the U operand (box 64 x 128; W's rows from u_row0), tm_y over Y
+// 64 x 128), tm_u over the bf16 U operand (box 64 x 128; W's rows from u_row0), tm_y over Y
 // (box 64 x 32, 128-byte swizzle; tiling 3: box 32 x 32, 64-byte swizzle).
 cudaError_t launch_linear_y(const CUtensorMap& tm_x, const CUtensorMap* d_w_map,
                             const CUtensorMap& tm_s_in, const CUtensorMap& tm_u,

@@ -288,14 +288,14 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
 #pragma unroll
             for (int kk = 0; kk < R / 16; ++kk) {
               const uint32_t hi = (uint32_t)(16 * kk * 2), lo = (uint32_t)((R + 16 * kk) * 2);
-              mma_bf16(d, sdesc_k_sw128(a_base + hi), sdesc_k_sw128(b_base + hi), idesc, 1u);
-              mma_bf16(d, sdesc_k_sw128(a_base + hi), sdesc_k_sw128(b_base + lo), idesc, 1u);
-              mma_bf16(d, sdesc_k_sw128(a_base + lo), sdesc_k_sw128(b_base + hi), idesc, 1u);
+              mma_f16(d, sdesc_k_sw128(a_base + hi), sdesc_k_sw128(b_base + hi), idesc, 1u);
+              mma_f16(d, sdesc_k_sw128(a_base + hi), sdesc_k_sw128(b_base + lo), idesc, 1u);
+              mma_f16(d, sdesc_k_sw128(a_base + lo), sdesc_k_sw128(b_base + hi), idesc, 1u);
             }
           } else {
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-              mma_bf16(d, sdesc_k_sw128(a_base + 32 * kk), sdesc_k_sw128(b_base + 32 * kk), idesc,
+              mma_f16(d, sdesc_k_sw128(a_base + 32 * kk), sdesc_k_sw128(b_base + 32 * kk), idesc,
                        (k > kb || kk > 0) ? 1u : 0u);
           }
         }
@@ -460,24 +460,38 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
   }
 }
 
-// P_K of every matrix: P_K_i[k][j] = P_HL[p_row0_i + j][k] for k < 2r (rows [P_hi ; P_lo])
-// and j < n_i, at pk_off[i] with row stride ld_i = n_i rounded up to 64.  One CTA per
-// projection unit (matrix, 128 columns j), through shared memory.
+// P_K of every matrix: rows [P_hi ; P_lo] of the bf16 pair of P_i (P_hi = bf16(P),
+// P_lo = bf16(P - P_hi)), K-major: P_K_i[k][j] and P_K_i[r + k][j] for k < r, j < n_i, at
+// pk_off[i] with row stride ld_i = n_i rounded up to 64.  P comes from the projection's
+// scaled fp16 pair, P = (hi + lo) pinv[i] (exact in fp32 up to the pair's rounding).  One
+// CTA per projection unit (matrix, 128 columns j), through shared memory.
 __global__ void __launch_bounds__(256)
-transpose_p_kernel(const __nv_bfloat16* __restrict__ p_hl, const TcMat* __restrict__ tcm,
+transpose_p_kernel(const uint16_t* __restrict__ p_hl, const TcMat* __restrict__ tcm,
                    const int2* __restrict__ units, const int64_t* __restrict__ pk_off,
-                   int hl_width, int r2, __nv_bfloat16* __restrict__ p_k) {
+                   const float* __restrict__ pinv, int hl_width, int r2,
+                   __nv_bfloat16* __restrict__ p_k) {
   __shared__ __nv_bfloat16 t[128][66];
   const int2 u = units[blockIdx.x];
   const int64_t n = tcm[u.x].n;
   const int64_t p_row0 = tcm[u.x].p_row0;
   const int64_t ld = (n + 63) / 64 * 64;
   const int64_t j0 = u.y;
+  const int r = r2 / 2;
+  const float unscale = pinv[u.x];
   __nv_bfloat16* dst = p_k + pk_off[u.x];
-  for (int e = threadIdx.x; e < 128 * 64; e += blockDim.x) {
-    const int jj = e / 64, k = e % 64;
-    t[jj][k] = (j0 + jj < n && k < r2) ? p_hl[(p_row0 + j0 + jj) * hl_width + k]
-                                       : __float2bfloat16_rn(0.f);
+  for (int e = threadIdx.x; e < 128 * 32; e += blockDim.x) {
+    const int jj = e / 32, k = e % 32;
+    if (k < r) {
+      float x = 0.f;
+      if (j0 + jj < n) {
+        const uint16_t* row = p_hl + (p_row0 + j0 + jj) * hl_width;
+        x = (__half2float(__ushort_as_half(row[k])) + __half2float(__ushort_as_half(row[r + k]))) *
+            unscale;
+      }
+      const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+      t[jj][k] = hi;
+      t[jj][r + k] = __float2bfloat16_rn(x - __bfloat162float(hi));
+    }
   }
   __syncthreads();
   for (int e = threadIdx.x; e < 128 * 64; e += blockDim.x) {
@@ -567,11 +581,12 @@ int32_t linear_y_tile_cols(int32_t tiling) { return tiling == 3 ? 224 : 256; }
 
 int64_t linear_pk_elems(int64_t n, int32_t r) { return 2 * (int64_t)r * ((n + 63) / 64 * 64); }
 
-cudaError_t launch_transpose_p(const __nv_bfloat16* p_hl, const TcMat* d_tc, const int2* d_units,
-                               int32_t n_units, const int64_t* d_pk_off, int32_t hl_width,
-                               int32_t r, __nv_bfloat16* p_k, cudaStream_t s) {
-  if (n_units <= 0) return cudaSuccess;
-  transpose_p_kernel<<<n_units, 256, 0, s>>>(p_hl, d_tc, d_units, d_pk_off, hl_width, 2 * r, p_k);
+cudaError_t launch_transpose_p(const uint16_t* p_hl, const TcMat* d_tc, const int2* d_units,
+                               int32_t n_units, const int64_t* d_pk_off, const float* d_pinv,
+                               int32_t hl_width, int32_t r, __nv_bfloat16* p_k, cudaStream_t s) {
+  if (n_units <= 0 || r > 32) return n_units <= 0 ? cudaSuccess : cudaErrorInvalidValue;
+  transpose_p_kernel<<<n_units, 256, 0, s>>>(p_hl, d_tc, d_units, d_pk_off, d_pinv, hl_width, 2 * r,
+                                             p_k);
   return cudaGetLastError();
 }
 

@@ -1,8 +1,10 @@
 // The U operand of the r <= 32 tensor-core weight pass (zo_wpass_tc.cu): rows
-// [bf16 hi(U) | bf16 lo(U) | 0 ...], formed once per refresh, stacked per matrix in 128-row
-// blocks and read by TMA.  x = hi + lo with hi = bf16(x), lo = bf16(x - hi).  Also the
-// dispatch of the split by rank (r >= 64: the chunk-major U of zo_wpass_tmem.cu).  P^T =
-// V C^T, the other operand, comes from the tensor-core projection (zo_project_tc.cu).
+// [hi(U s) | lo(U s) | 0 ...] in fp16 with s = 2^kUVScaleExp (zo_tc_common.cuh), formed once
+// per refresh, stacked per matrix in 128-row blocks and read by TMA.  The perturbed-linear
+// route (zo_linear.cu) reads the same rows as a bf16 pair, hi = bf16(x), lo = bf16(x - hi),
+// unscaled, from a buffer of its own: there U meets the bf16 X and W in one accumulator.
+// Also the dispatch of the split by rank (r >= 64: the chunk-major U of zo_wpass_tmem.cu).
+// P^T = V C^T, the other operand, comes from the tensor-core projection (zo_project_tc.cu).
 #include "zo_kernels.h"
 #include "zo_tc_common.cuh"
 
@@ -18,7 +20,7 @@ using namespace tc;
 // operand, with coalesced 16-byte stores.  Padding columns of a row stay at the zero they
 // were set to.
 template <int R>
-__device__ __forceinline__ void write_rows(const uint4* Os, __nv_bfloat16* dst_rows, int rows) {
+__device__ __forceinline__ void write_rows(const uint4* Os, uint16_t* dst_rows, int rows) {
   constexpr int kVecPerRow = hl_width(R) * 2 / 16;   // 8 or 16 chunks per row
   uint4* dst = reinterpret_cast<uint4*>(dst_rows);
   for (int e = threadIdx.x; e < rows * kVecPerRow; e += blockDim.x) {
@@ -27,11 +29,12 @@ __device__ __forceinline__ void write_rows(const uint4* Os, __nv_bfloat16* dst_r
   }
 }
 
-// U_HL[u_row0 + i] = [bf16 hi(U[i, :]) | bf16 lo(U[i, :]) | 0 ...]  (row width hl_width(R))
-template <int R>
+// dst[u_row0 + i] = [hi | lo | 0 ...] of row i of U (row width hl_width(R)): the fp16 pair
+// of U 2^kUVScaleExp (kF16) or the bf16 pair of U.
+template <int R, bool kF16>
 __global__ void __launch_bounds__(128)
 split_u_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
-               const int2* __restrict__ units, __nv_bfloat16* __restrict__ u_hl) {
+               const int2* __restrict__ units, uint16_t* __restrict__ dst) {
   constexpr int kVecPerRow = hl_width(R) * 2 / 16;
   extern __shared__ uint4 su_smem[];
   uint4* Os = su_smem;                                     // 128 x kVecPerRow
@@ -48,25 +51,26 @@ split_u_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
       const float4 a = src[2 * g], b = src[2 * g + 1];
       const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
       uint4 hi, lo;
-      split8(x, hi, lo);
+      if constexpr (kF16) split8_f16(x, exp2i(kUVScaleExp), hi, lo);
+      else split8(x, hi, lo);
       orow[g ^ (tid & 7)] = hi;
       orow[(R / 8 + g) ^ (tid & 7)] = lo;
     }
   }
   __syncthreads();
-  write_rows<R>(Os, u_hl + ((int64_t)tcm[u.x].u_row0 + i0) * hl_width(R), rows);
+  write_rows<R>(Os, dst + ((int64_t)tcm[u.x].u_row0 + i0) * hl_width(R), rows);
 }
 
-template <int R>
+template <int R, bool kF16>
 cudaError_t launch_split_u_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                             int32_t n_units, __nv_bfloat16* u_hl, cudaStream_t s) {
+                             int32_t n_units, uint16_t* dst, cudaStream_t s) {
   const size_t smem = 128 * (size_t)hl_width(R) * 2;
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(split_u_kernel<R>,
+    cudaError_t e = cudaFuncSetAttribute(split_u_kernel<R, kF16>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
-  split_u_kernel<R><<<n_units, 128, smem, s>>>(d_mats, d_tc, d_units, u_hl);
+  split_u_kernel<R, kF16><<<n_units, 128, smem, s>>>(d_mats, d_tc, d_units, dst);
   return cudaGetLastError();
 }
 
@@ -76,10 +80,20 @@ cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2*
                            int32_t n_units, int32_t r, void* u_op, cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
-    case 16: return launch_split_u_r<16>(d_mats, d_tc, d_units, n_units, static_cast<__nv_bfloat16*>(u_op), s);
-    case 32: return launch_split_u_r<32>(d_mats, d_tc, d_units, n_units, static_cast<__nv_bfloat16*>(u_op), s);
+    case 16: return launch_split_u_r<16, true>(d_mats, d_tc, d_units, n_units, static_cast<uint16_t*>(u_op), s);
+    case 32: return launch_split_u_r<32, true>(d_mats, d_tc, d_units, n_units, static_cast<uint16_t*>(u_op), s);
     case 64:
     case 128: return launch_split_u_chunks(d_mats, d_tc, d_units, n_units, r, static_cast<uint4*>(u_op), s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_split_u_bf16(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
+                                int32_t n_units, int32_t r, __nv_bfloat16* u_lin, cudaStream_t s) {
+  if (n_units <= 0) return cudaSuccess;
+  switch (r) {
+    case 16: return launch_split_u_r<16, false>(d_mats, d_tc, d_units, n_units, reinterpret_cast<uint16_t*>(u_lin), s);
+    case 32: return launch_split_u_r<32, false>(d_mats, d_tc, d_units, n_units, reinterpret_cast<uint16_t*>(u_lin), s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -5,10 +5,11 @@
 // At r = 128 the projection is an r^2-deep contraction per column of P -- 2 r^2 flops
 // per row of V, 37 GFLOP per pass on the LLaMA-7B set -- so it runs as a GEMM on
 // tcgen05.mma: D (128 rows of V x r columns) = V_tile . C^T with M = 128, N = K = r.
-// Both operands are split x = hi + lo in bf16 like the weight pass's operands and the
-// products hi.hi + hi.lo + lo.hi accumulate in fp32 in Tensor Memory (relative error
-// ~2^-16 against the summed terms); the epilogue splits D into the bf16 hi/lo rows of
-// P_HL.  V_HL ([hi | lo] rows of V) is formed once per refresh, C_HL once per pass.
+// Both operands are scaled fp16 pairs like the weight pass's operands (V 2^kUVScaleExp,
+// C_i 2^(e_C,i); zo_tc_common.cuh) and the products hi.hi + hi.lo + lo.hi accumulate in
+// fp32 in Tensor Memory (relative error ~2^-21 against the summed terms); the epilogue
+// rescales D to P_i 2^(e_P,i) and splits it into the fp16 hi/lo rows of P_HL.  V_HL
+// ([hi | lo] rows of V) is formed once per refresh, C_HL and e_C,i once per pass.
 //
 // Roles of the 192 threads of a CTA (one CTA per SM, each over a contiguous range of
 // 128-row units, so C_HL is reloaded only when the matrix changes):
@@ -18,7 +19,7 @@
 //   warp 1, lane 0: MMA issuer -- 3 * r/16 tcgen05.mma (M=128, N=r, K=16) per unit into
 //                   one of two TMEM accumulators; warp 1 also owns the TMEM allocation.
 //   warps 2..5:     epilogue -- warp w owns 32 rows (its TMEM lane group): tcgen05.ld
-//                   the fp32 row of D, split it into bf16 hi/lo, write them as 32 x 64
+//                   the fp32 row of D, scale and split it into fp16 hi/lo, write them as 32 x 64
 //                   boxes of P_HL into shared memory (128-byte swizzle) and TMA-store
 //                   them, 64 columns of D at a time (one hi and one lo box staged).
 // Every mbarrier wait is bounded; on expiry the kernel records kDevTimeout in the
@@ -173,7 +174,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
     }
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA issuer
-    constexpr uint32_t idesc = idesc_bf16_f32(kBM, R);
+    constexpr uint32_t idesc = idesc_f16_f32(kBM, R);
     int64_t it = 0, n_c = 0;
     int prev_i = -1;
     bool ok = true;
@@ -211,9 +212,9 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
             sdesc_k_sw128(b_base + (e_hi / 64) * Cfg::kCPanelBytes + (e_hi % 64) * 2);
         const uint64_t b_lo =
             sdesc_k_sw128(b_base + (e_lo / 64) * Cfg::kCPanelBytes + (e_lo % 64) * 2);
-        mma_bf16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
-        mma_bf16(d, a_hi, b_lo, idesc, 1u);
-        mma_bf16(d, a_lo, b_hi, idesc, 1u);
+        mma_f16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
+        mma_f16(d, a_hi, b_lo, idesc, 1u);
+        mma_f16(d, a_lo, b_hi, idesc, 1u);
       }
       mma_commit(&sh.v_empty[vs]);
       if (last_c) mma_commit(&sh.c_empty);
@@ -230,6 +231,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
     const int g = warp & 3;                      // TMEM lane group == rows 32 g .. + 31
     const uint32_t lane_base = (uint32_t)(g * 32) << 16;
     uint8_t* obox = o_smem + g * Cfg::kWarpOutBytes;   // this warp's boxes
+    // D = 2^(kUVScaleExp + e_C) P^T; P_HL holds P 2^(e_C + p_scale_offset(R))
+    const float p_scale = exp2i(p_scale_offset(R) - kUVScaleExp);
     int64_t it = 0;
     bool ok = true;
     for (int u = u_begin; u < u_end; ++u, ++it) {
@@ -258,7 +261,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
 #pragma unroll
           for (int e = 0; e < 8; ++e) x[e] = __uint_as_float(v[8 * j + e]);
           uint4 hi, lo;
-          split8(x, hi, lo);
+          split8_f16(x, p_scale, hi, lo);
           *reinterpret_cast<uint4*>(obox + lane * 128 + ((j ^ (lane & 7)) << 4)) = hi;
           *reinterpret_cast<uint4*>(obox + lane * 128 + (((R / 8 + j) ^ (lane & 7)) << 4)) = lo;
         }
@@ -290,7 +293,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
 #pragma unroll
             for (int e = 0; e < 8; ++e) x[e] = __uint_as_float(v[j >> 2][(j & 3) * 8 + e]);
             uint4 hi, lo;
-            split8(x, hi, lo);
+            split8_f16(x, p_scale, hi, lo);
             const int sw = (j ^ (lane & 7)) << 4;
             *reinterpret_cast<uint4*>(obox + lane * 128 + sw) = hi;
             *reinterpret_cast<uint4*>(obox + Cfg::kOutBoxBytes + lane * 128 + sw) = lo;
@@ -323,14 +326,16 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
   }
 }
 
-// Rows [bf16 hi(x) | bf16 lo(x)] of V (units = (matrix, first row) x 128 rows, into V_HL at
-// p_row0) or of C (one CTA per matrix, r rows into C_HL at matrix * r).  Each thread
-// splits one row; the rows are staged in shared memory with the 16-byte chunk index XOR
-// (row & 7) and written with coalesced 16-byte stores.
+// Rows [hi | lo] of the scaled fp16 pair of V (units = (matrix, first row) x 128 rows, into
+// V_HL at p_row0; scale 2^kUVScaleExp) or of C (one CTA per matrix, r rows into C_HL at
+// matrix * r; scale 2^(e_C,i), found here from max |C_i|, with pinv[i] = 2^-(e_P,i) written
+// for the weight pass).  Each thread splits one row; the rows are staged in shared memory
+// with the 16-byte chunk index XOR (row & 7) and written with coalesced 16-byte stores.
 template <int R, bool kC>
 __global__ void __launch_bounds__(128)
 split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
-                  const int2* __restrict__ units, __nv_bfloat16* __restrict__ dst) {
+                  const int2* __restrict__ units, uint16_t* __restrict__ dst,
+                  float* __restrict__ pinv) {
   constexpr int kVecPerRow = 2 * R * 2 / 16;     // 16-byte chunks of [hi | lo]
   constexpr int kSw = kVecPerRow >= 8 ? 7 : kVecPerRow - 1;   // chunk swizzle within a row
   constexpr int kStride = hl_width(R) / 8;       // chunks per row of V_HL / C_HL
@@ -353,6 +358,28 @@ split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tc
     src = mats[i].V;
     dst_row0 = (int64_t)tcm[i].p_row0 + row0;
   }
+  float scale = exp2i(kUVScaleExp);
+  if constexpr (kC) {
+    // e_C,i from the largest |C_i|: every thread takes the max of its row, then the block's
+    __shared__ float wmax[4];
+    float amax = 0.f;
+    if (tid < rows) {
+      const float4* s4 = reinterpret_cast<const float4*>(src + (int64_t)tid * R);
+#pragma unroll
+      for (int g = 0; g < R / 4; ++g) {
+        const float4 a = s4[g];
+        amax = fmaxf(amax, fmaxf(fmaxf(fabsf(a.x), fabsf(a.y)), fmaxf(fabsf(a.z), fabsf(a.w))));
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+    if ((tid & 31) == 0) wmax[tid >> 5] = amax;
+    __syncthreads();
+    amax = fmaxf(fmaxf(wmax[0], wmax[1]), fmaxf(wmax[2], wmax[3]));
+    const int e_c = coeff_scale_exp(amax);
+    scale = exp2i(e_c);
+    if (tid == 0) pinv[i] = exp2i(-(e_c + p_scale_offset(R)));
+  }
   if (tid < rows) {
     const float4* s4 = reinterpret_cast<const float4*>(src + (row0 + tid) * R);
     uint4* orow = Os + tid * kVecPerRow;
@@ -361,7 +388,7 @@ split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tc
       const float4 a = s4[2 * g], b = s4[2 * g + 1];
       const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
       uint4 hi, lo;
-      split8(x, hi, lo);
+      split8_f16(x, scale, hi, lo);
       orow[g ^ (tid & kSw)] = hi;
       orow[(R / 8 + g) ^ (tid & kSw)] = lo;
     }
@@ -390,14 +417,14 @@ cudaError_t launch_project_tc_r(const CUtensorMap& tm_v, const CUtensorMap& tm_c
 
 template <int R, bool kC>
 cudaError_t launch_split_rows_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                                int32_t n_blocks, __nv_bfloat16* dst, cudaStream_t s) {
+                                int32_t n_blocks, uint16_t* dst, float* pinv, cudaStream_t s) {
   constexpr size_t smem = 128 * (size_t)(2 * R * 2);
   if (smem > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(split_rows_kernel<R, kC>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
-  split_rows_kernel<R, kC><<<n_blocks, 128, smem, s>>>(d_mats, d_tc, d_units, dst);
+  split_rows_kernel<R, kC><<<n_blocks, 128, smem, s>>>(d_mats, d_tc, d_units, dst, pinv);
   return cudaGetLastError();
 }
 
@@ -406,25 +433,25 @@ cudaError_t launch_split_rows_r(const MatDesc* d_mats, const TcMat* d_tc, const 
 bool project_tc_supported(int32_t r) { return r == 16 || r == 32 || r == 64 || r == 128; }
 
 cudaError_t launch_split_v(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                           int32_t n_units, int32_t r, __nv_bfloat16* v_hl, cudaStream_t s) {
+                           int32_t n_units, int32_t r, uint16_t* v_hl, cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
-    case 16: return launch_split_rows_r<16, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
-    case 32: return launch_split_rows_r<32, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
-    case 64: return launch_split_rows_r<64, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
-    case 128: return launch_split_rows_r<128, false>(d_mats, d_tc, d_units, n_units, v_hl, s);
+    case 16: return launch_split_rows_r<16, false>(d_mats, d_tc, d_units, n_units, v_hl, nullptr, s);
+    case 32: return launch_split_rows_r<32, false>(d_mats, d_tc, d_units, n_units, v_hl, nullptr, s);
+    case 64: return launch_split_rows_r<64, false>(d_mats, d_tc, d_units, n_units, v_hl, nullptr, s);
+    case 128: return launch_split_rows_r<128, false>(d_mats, d_tc, d_units, n_units, v_hl, nullptr, s);
     default: return cudaErrorInvalidValue;
   }
 }
 
-cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, __nv_bfloat16* c_hl,
-                           cudaStream_t s) {
+cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, uint16_t* c_hl,
+                           float* pinv, cudaStream_t s) {
   if (n_mats <= 0) return cudaSuccess;
   switch (r) {
-    case 16: return launch_split_rows_r<16, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
-    case 32: return launch_split_rows_r<32, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
-    case 64: return launch_split_rows_r<64, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
-    case 128: return launch_split_rows_r<128, true>(d_mats, nullptr, nullptr, n_mats, c_hl, s);
+    case 16: return launch_split_rows_r<16, true>(d_mats, nullptr, nullptr, n_mats, c_hl, pinv, s);
+    case 32: return launch_split_rows_r<32, true>(d_mats, nullptr, nullptr, n_mats, c_hl, pinv, s);
+    case 64: return launch_split_rows_r<64, true>(d_mats, nullptr, nullptr, n_mats, c_hl, pinv, s);
+    case 128: return launch_split_rows_r<128, true>(d_mats, nullptr, nullptr, n_mats, c_hl, pinv, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -5,6 +5,7 @@
 #pragma once
 
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cstdint>
 
 #include "zo_kernels.h"
@@ -104,8 +105,59 @@ __device__ __forceinline__ void give_up(Shared& sh, uint32_t* status) {
   *reinterpret_cast<volatile int*>(&sh.abort_flag) = 1;
 }
 
+// ---- fp16 operands of the weight pass and the projection -------------------------------
+// The tensor-core operands U, P = C V^T (and, in the projection, V and C) are held as
+// pairs of fp16 values, x s = hi + lo with hi = f16(x s), lo = f16(x s - hi), where s is a
+// power of two that puts x s into fp16's normal range.  fp16 carries an 11-bit
+// significand, so hi + lo keeps ~22 bits of x (relative representation error <= 2^-22,
+// against 2^-17 for a bf16 pair) and the three products hi.hi + hi.lo + lo.hi that the
+// MMAs accumulate in fp32 drop only lo.lo (~2^-22): the update U P then errs by ~2^-21 of
+// sum |U| |P|, the grade of an fp32 evaluation, at the MMA count of the bf16 pair.
+// Scales (all exact powers of two, undone in fp32 by the consumer):
+//   U, V:  2^kUVScaleExp  (|U|, |V| <= 1 for column-orthonormal bases)
+//   C_i:   2^(e_C,i) with e_C,i = 14 - E, max |C_i| < 2^E, so |C_i s| < 2^14
+//   P_i:   2^(e_C,i + p_scale_offset(r)): |P_kj| <= ||C_k,:|| ||V_j,:|| <= sqrt(r) max |C|,
+//          so |P_i s| <= 2^15 (fp16 holds up to 65504)
+// The weight pass multiplies its accumulator by pinv_i 2^-kUVScaleExp, pinv_i = 2^-(e_P,i).
+constexpr int kUVScaleExp = 14;
+__host__ __device__ constexpr int p_scale_offset(int r) {   // 1 - ceil(log2(r) / 2)
+  return r <= 16 ? -1 : r <= 64 ? -2 : -3;
+}
+constexpr int kScaleExpMax = 100;   // |e_C| bound: keeps every scale a normal fp32 value
+
+// 2^e as an fp32 value, -126 <= e <= 127 (exact).
+__device__ __forceinline__ float exp2i(int e) { return __int_as_float((e + 127) << 23); }
+
+// e_C of a coefficient matrix whose largest magnitude is amax (>= 0): 14 - E with
+// amax < 2^E; a zero or fp32-subnormal amax takes the largest exponent, a non-finite one 0.
+__device__ __forceinline__ int coeff_scale_exp(float amax) {
+  const int biased = (__float_as_int(amax) >> 23) & 0xFF;
+  if (biased == 0) return kScaleExpMax;
+  if (biased == 0xFF) return 0;
+  const int e = 14 - (biased - 126);
+  return e > kScaleExpMax ? kScaleExpMax : e < -kScaleExpMax ? -kScaleExpMax : e;
+}
+
+// s x = hi + lo in fp16 for 8 consecutive fp32 values, packed two per 32-bit word (lower
+// half = first element).  s x - hi is exact in fp32.
+__device__ __forceinline__ void split8_f16(const float (&x)[8], float s, uint4& hi, uint4& lo) {
+  uint32_t hw[4], lw[4];
+#pragma unroll
+  for (int pr = 0; pr < 4; ++pr) {
+    const float a = x[2 * pr] * s, b = x[2 * pr + 1] * s;
+    const __half2 h2 = __floats2half2_rn(a, b);
+    const float2 hf = __half22float2(h2);
+    const __half2 l2 = __floats2half2_rn(a - hf.x, b - hf.y);
+    hw[pr] = *reinterpret_cast<const uint32_t*>(&h2);
+    lw[pr] = *reinterpret_cast<const uint32_t*>(&l2);
+  }
+  hi = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+  lo = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+}
+
 // x = hi + lo for 8 consecutive fp32 values: hi = bf16(x), lo = bf16(x - hi), packed two
-// per 32-bit word (lower half = first element).
+// per 32-bit word (lower half = first element).  (The perturbed-linear route's operands,
+// which meet the bf16 X and W in the same accumulator.)
 __device__ __forceinline__ void split8(const float (&x)[8], uint4& hi, uint4& lo) {
   uint32_t hw[4], lw[4];
 #pragma unroll

@@ -9,10 +9,12 @@
 // The contraction U (128 x r) . P (r x 128) of a 128 x 128 tile is r-deep, so it
 // costs 2r flops per weight against 4 bytes of HBM traffic; past r = 16 that is
 // more than the fp32 FMA pipes deliver at HBM speed, so it runs on tcgen05.mma.
-// To keep fp32-grade accuracy of the update with bf16 tensor-core inputs, both
-// operands are split x = hi + lo (hi = bf16(x), lo = bf16(x - hi)) and the tile
-// accumulates hi.hi + hi.lo + lo.hi in fp32 in Tensor Memory (relative error of
-// the product ~2^-16 instead of 2^-8).
+// To keep fp32-grade accuracy of the update with 16-bit tensor-core inputs, both
+// operands are held as power-of-two-scaled fp16 pairs x s = hi + lo (hi = f16(x s),
+// lo = f16(x s - hi); the scales in zo_tc_common.cuh) and the tile accumulates
+// hi.hi + hi.lo + lo.hi in fp32 in Tensor Memory: relative error of the product
+// ~2^-21 of sum |U| |P|, against 2^-16 for a bf16 pair and 2^-8 for plain bf16.  The
+// epilogue undoes the scales with one fp32 multiply-add per weight.
 //
 // Roles of the 224 threads of a CTA (one CTA per SM, persistent over the chunks of 4
 // tiles b, b + G, b + 2G, ... of the interleaved walk, G = number of CTAs):
@@ -26,8 +28,8 @@
 //                   tile into one of two TMEM accumulators; warp 1 also owns
 //                   the TMEM allocation.
 //   warps 2..5:     epilogue -- each warp owns 32 rows (its TMEM lane group):
-//                   tcgen05.ld the fp32 update, add it to the W rows in shared
-//                   memory, round to bf16 in place, TMA-store its rows.
+//                   tcgen05.ld the fp32 update, scale it and add it to the W rows
+//                   in shared memory, round to bf16 in place, TMA-store its rows.
 // Every mbarrier wait is bounded; on expiry the kernel records kDevTimeout in
 // the status word, lets the other roles stop, drains its copies and frees TMEM.
 #include <cuda.h>
@@ -62,9 +64,9 @@ struct TcCfg {
 template <int R>
 __global__ void __launch_bounds__(kThreads, 1)
 wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
-                const CUtensorMap* __restrict__ w_maps, const TcMat* __restrict__ mats, int n_mats,
-                int64_t n_tiles, uint32_t* __restrict__ status, long long wait_cycles,
-                int inject_wait) {
+                const CUtensorMap* __restrict__ w_maps, const TcMat* __restrict__ mats,
+                const float* __restrict__ pinv, int n_mats, int64_t n_tiles,
+                uint32_t* __restrict__ status, long long wait_cycles, int inject_wait) {
   using Cfg = TcCfg<R>;
   static_assert(Cfg::kWStages >= 2 && Cfg::kWStages <= 4, "W ring must fit Shared::w_full");
   static_assert(Cfg::kAStages >= 1 && Cfg::kAStages <= 2, "A ring must fit Shared::a_full");
@@ -198,7 +200,7 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
         mbar_wait_bounded(&sh.b_full[bi], (uint32_t)((b_iss[bi] - 1) & 1), nullptr, wait_cycles);
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA issuer
-    constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN);
+    constexpr uint32_t idesc = idesc_f16_f32(kBM, kBN);
     int64_t it = 0, a_it = 0;
     int prev_i = -1;
     int64_t prev_rb = -1;
@@ -247,9 +249,9 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
         const uint32_t off_lo = (uint32_t)((e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
         const uint64_t a_hi = sdesc_k_sw128(a_base + off_hi), a_lo = sdesc_k_sw128(a_base + off_lo);
         const uint64_t b_hi = sdesc_k_sw128(b_base + off_hi), b_lo = sdesc_k_sw128(b_base + off_lo);
-        mma_bf16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
-        mma_bf16(d, a_hi, b_lo, idesc, 1u);
-        mma_bf16(d, a_lo, b_hi, idesc, 1u);
+        mma_f16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
+        mma_f16(d, a_hi, b_lo, idesc, 1u);
+        mma_f16(d, a_lo, b_hi, idesc, 1u);
       }
       mma_commit(&sh.b_empty[sb]);
       if (last_a) mma_commit(&sh.a_empty[sa]);
@@ -273,6 +275,8 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
     for (; ti.valid(); ti.next(), ++it) {
       const TcMat& mt = mats[ti.i];
       const int acc = (int)(it & 1);
+      // the accumulator holds 2^(kUVScaleExp + e_P) U P: back to U P in the add
+      const float wscale = pinv[ti.i] * exp2i(-kUVScaleExp);
       // test hook (zo_set_option ZO_OPTION_TEST_WAIT_TIMEOUT): CTA 0's epilogue first waits
       // on a barrier that nothing arrives on, so its bounded wait runs out
       if (inject_wait && blockIdx.x == 0 && it == 0 &&
@@ -306,9 +310,10 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
           uint32_t wv[4] = {raw.x, raw.y, raw.z, raw.w};
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            const float lo = __uint_as_float(wv[e] << 16) + __uint_as_float(v[j4 * 8 + 2 * e]);
-            const float hi = __uint_as_float(wv[e] & 0xFFFF0000u) +
-                             __uint_as_float(v[j4 * 8 + 2 * e + 1]);
+            const float lo = fmaf(__uint_as_float(v[j4 * 8 + 2 * e]), wscale,
+                                  __uint_as_float(wv[e] << 16));
+            const float hi = fmaf(__uint_as_float(v[j4 * 8 + 2 * e + 1]), wscale,
+                                  __uint_as_float(wv[e] & 0xFFFF0000u));
             const __nv_bfloat162 h2 = __floats2bfloat162_rn(lo, hi);
             wv[e] = *reinterpret_cast<const uint32_t*>(&h2);
           }
@@ -349,16 +354,16 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
 
 template <int R>
 cudaError_t launch_tc_r(const CUtensorMap& tm_a, const CUtensorMap& tm_b, const CUtensorMap* w_maps,
-                        const TcMat* mats, int n_mats, int64_t n_tiles, int grid, uint32_t* status,
-                        bool inject_wait, cudaStream_t s) {
+                        const TcMat* mats, const float* pinv, int n_mats, int64_t n_tiles, int grid,
+                        uint32_t* status, bool inject_wait, cudaStream_t s) {
   const size_t smem = TcCfg<R>::kSmem;
   cudaError_t e = cudaFuncSetAttribute(wpass_tc_kernel<R>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   // with the test hook armed the wait limit is ~0.1 s so the test ends quickly
   const long long wait = inject_wait ? kTestWaitCycles : kWaitCycles;
-  wpass_tc_kernel<R><<<grid, kThreads, smem, s>>>(tm_a, tm_b, w_maps, mats, n_mats, n_tiles, status,
-                                                  wait, inject_wait ? 1 : 0);
+  wpass_tc_kernel<R><<<grid, kThreads, smem, s>>>(tm_a, tm_b, w_maps, mats, pinv, n_mats, n_tiles,
+                                                  status, wait, inject_wait ? 1 : 0);
   return cudaGetLastError();
 }
 
@@ -370,23 +375,23 @@ int32_t tc_hl_width(int32_t r) { return hl_width(r); }
 int32_t tc_tile_rows() { return kBM; }
 int32_t tc_tile_cols() { return kBN; }
 int64_t tc_u_operand_bytes(int32_t r, int64_t rows) {
-  const int64_t row_layout = rows * hl_width(r) * 2;        // bf16 [hi | lo | 0] rows
+  const int64_t row_layout = rows * hl_width(r) * 2;        // 16-bit [hi | lo | 0] rows
   const int64_t chunk_layout = rows * r * 4;                // R 32-bit words per row
   return row_layout > chunk_layout ? row_layout : chunk_layout;
 }
 
 cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const void* u_op, const CUtensorMap& tm_b,
-                            const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
-                            int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
-                            bool inject_wait, cudaStream_t s) {
+                            const CUtensorMap* d_w_maps, const TcMat* d_tc, const float* d_pinv,
+                            int32_t n_mats, int64_t n_tiles, int32_t grid, int32_t r,
+                            uint32_t* d_status, bool inject_wait, cudaStream_t s) {
   if (n_tiles <= 0) return cudaSuccess;
   switch (r) {
-    case 16: return launch_tc_r<16>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
-    case 32: return launch_tc_r<32>(tm_a, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
+    case 16: return launch_tc_r<16>(tm_a, tm_b, d_w_maps, d_tc, d_pinv, n_mats, n_tiles, grid, d_status, inject_wait, s);
+    case 32: return launch_tc_r<32>(tm_a, tm_b, d_w_maps, d_tc, d_pinv, n_mats, n_tiles, grid, d_status, inject_wait, s);
     case 64:
     case 128:
-      return launch_wpass_tmem(static_cast<const uint4*>(u_op), tm_b, d_w_maps, d_tc, n_mats, n_tiles,
-                               grid, r, d_status, inject_wait, s);
+      return launch_wpass_tmem(static_cast<const uint4*>(u_op), tm_b, d_w_maps, d_tc, d_pinv, n_mats,
+                               n_tiles, grid, r, d_status, inject_wait, s);
     default: return cudaErrorInvalidValue;
   }
 }

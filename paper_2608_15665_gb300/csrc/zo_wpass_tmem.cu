@@ -2,7 +2,8 @@
 // Tensor Memory: W_i <- rnd_bf16(W_i + U_i P_i) for every bf16 matrix in one persistent
 // launch (the fused form of Alg. 2's "W_i <- W_i + eps U_i Z_i V_i^T", Eq. (4), and of
 // the update of Eq. (10)).  The r <= 32 kernel, with both operands in shared memory, and
-// the operand split (hi.hi + hi.lo + lo.hi in fp32) are described in zo_wpass_tc.cu.
+// the operand split (scaled fp16 pairs, hi.hi + hi.lo + lo.hi in fp32) are described in
+// zo_wpass_tc.cu.
 //
 // Why Tensor Memory for U: at r = 64 and 128 the 3r/16 MMAs of a 128 x 128 tile (12 and
 // 24) read their operands at up to 128 B/clk from shared memory, the SM's whole shared-
@@ -71,9 +72,9 @@ struct TmemCfg {
 template <int R>
 __global__ void __launch_bounds__(TmemCfg<R>::kThreads, 1)
 wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtensorMap tm_b,
-                const CUtensorMap* __restrict__ w_maps, const TcMat* __restrict__ mats, int n_mats,
-                int64_t n_tiles, uint32_t* __restrict__ status, long long wait_cycles,
-                int inject_wait) {
+                const CUtensorMap* __restrict__ w_maps, const TcMat* __restrict__ mats,
+                const float* __restrict__ pinv, int n_mats, int64_t n_tiles,
+                uint32_t* __restrict__ status, long long wait_cycles, int inject_wait) {
   using Cfg = TmemCfg<R>;
   static_assert(Cfg::kWStages >= 2 && Cfg::kWStages <= 4, "W ring must fit Shared::w_full");
   static_assert(Cfg::kBStages >= 2 && Cfg::kBStages <= 4, "P ring must fit Shared::b_full");
@@ -182,7 +183,7 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
     // ------------------------------------------------------------ U tiles into TMEM
     // Warp w may address TMEM lanes 32 (w % 4) .. + 31 only, so the four loader warps
     // cover the tile's 128 rows; lane t writes row 32 (w % 4) + t: its R words of
-    // [hi | lo] (two bf16 per 32-bit column, lower half first).  U_T keeps chunk j of
+    // [hi | lo] (two fp16 per 32-bit column, lower half first).  U_T keeps chunk j of
     // the block's 128 rows contiguous, so each 16-byte load of the warp is one 512-byte
     // access.
     const int q = warp & 3;
@@ -244,7 +245,7 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
     if (!ok && lane == 0) give_up(sh, status);
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA issuer
-    constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN);
+    constexpr uint32_t idesc = idesc_f16_f32(kBM, kBN);
     int64_t it = 0, a_it = 0;
     int prev_i = -1;
     int64_t prev_rb = -1;
@@ -289,9 +290,9 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
         const uint32_t off_hi = (uint32_t)((e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
         const uint32_t off_lo = (uint32_t)((e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
         const uint64_t b_hi = sdesc_k_sw128(b_base + off_hi), b_lo = sdesc_k_sw128(b_base + off_lo);
-        mma_bf16_ts(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
-        mma_bf16_ts(d, a_hi, b_lo, idesc, 1u);
-        mma_bf16_ts(d, a_lo, b_hi, idesc, 1u);
+        mma_f16_ts(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
+        mma_f16_ts(d, a_hi, b_lo, idesc, 1u);
+        mma_f16_ts(d, a_lo, b_hi, idesc, 1u);
       }
       mma_commit(&sh.b_empty[sb]);
       if (last_a) mma_commit(&sh.a_empty[sa]);
@@ -319,6 +320,8 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
     for (; ti.valid(); ti.next(), ++it) {
       const TcMat& mt = mats[ti.i];
       const int acc = (int)(it & 1);
+      // the accumulator holds 2^(kUVScaleExp + e_P) U P: back to U P in the add
+      const float wscale = pinv[ti.i] * exp2i(-kUVScaleExp);
       // test hook (zo_set_option ZO_OPTION_TEST_WAIT_TIMEOUT): CTA 0's epilogue first waits
       // on a barrier that nothing arrives on, so its bounded wait runs out
       if (inject_wait && blockIdx.x == 0 && it == 0 &&
@@ -354,10 +357,10 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
           uint32_t wv[4] = {raw.x, raw.y, raw.z, raw.w};
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            const float lo = __uint_as_float(wv[e] << 16) +
-                             __uint_as_float(v[j >> 2][(j & 3) * 8 + 2 * e]);
-            const float hi = __uint_as_float(wv[e] & 0xFFFF0000u) +
-                             __uint_as_float(v[j >> 2][(j & 3) * 8 + 2 * e + 1]);
+            const float lo = fmaf(__uint_as_float(v[j >> 2][(j & 3) * 8 + 2 * e]), wscale,
+                                  __uint_as_float(wv[e] << 16));
+            const float hi = fmaf(__uint_as_float(v[j >> 2][(j & 3) * 8 + 2 * e + 1]), wscale,
+                                  __uint_as_float(wv[e] & 0xFFFF0000u));
             const __nv_bfloat162 h2 = __floats2bfloat162_rn(lo, hi);
             wv[e] = *reinterpret_cast<const uint32_t*>(&h2);
           }
@@ -408,7 +411,8 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
 }
 
 // U_T: the U operand in the layout the TMEM loaders read.  Row i of the stacked operand
-// is [bf16 hi(U[i, :]) | bf16 lo(U[i, :])] = R 32-bit words = R/4 chunks of 16 bytes;
+// is [hi | lo] of the fp16 pair of U[i, :] 2^kUVScaleExp = R 32-bit words = R/4 chunks of
+// 16 bytes;
 // within each 128-row block chunk j of all 128 rows is contiguous:
 //   U_T[(block * (R/4) + j) * 128 + (i % 128)] = chunk j of row i,
 // so one warp reads 512 contiguous bytes per chunk (one row per lane), and this kernel
@@ -431,7 +435,7 @@ split_u_chunks_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict_
     const float4 a = src[2 * g], b = src[2 * g + 1];
     const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
     uint4 hi, lo;
-    split8(x, hi, lo);
+    split8_f16(x, exp2i(kUVScaleExp), hi, lo);
     dst[(int64_t)g * 128] = hi;
     dst[(int64_t)(R / 8 + g) * 128] = lo;
   }
@@ -439,15 +443,15 @@ split_u_chunks_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict_
 
 template <int R>
 cudaError_t launch_tmem_r(const uint4* u_t, const CUtensorMap& tm_b, const CUtensorMap* w_maps,
-                          const TcMat* mats, int n_mats, int64_t n_tiles, int grid, uint32_t* status,
-                          bool inject_wait, cudaStream_t s) {
+                          const TcMat* mats, const float* pinv, int n_mats, int64_t n_tiles, int grid,
+                          uint32_t* status, bool inject_wait, cudaStream_t s) {
   const size_t smem = TmemCfg<R>::kSmem;
   cudaError_t e = cudaFuncSetAttribute(wpass_tmem_kernel<R>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const long long wait = inject_wait ? kTestWaitCycles : kWaitCycles;
-  wpass_tmem_kernel<R><<<grid, TmemCfg<R>::kThreads, smem, s>>>(u_t, tm_b, w_maps, mats, n_mats,
-                                                                 n_tiles, status, wait,
+  wpass_tmem_kernel<R><<<grid, TmemCfg<R>::kThreads, smem, s>>>(u_t, tm_b, w_maps, mats, pinv,
+                                                                 n_mats, n_tiles, status, wait,
                                                                  inject_wait ? 1 : 0);
   return cudaGetLastError();
 }
@@ -466,13 +470,13 @@ cudaError_t launch_split_u_chunks(const MatDesc* d_mats, const TcMat* d_tc, cons
 }
 
 cudaError_t launch_wpass_tmem(const uint4* u_t, const CUtensorMap& tm_b,
-                              const CUtensorMap* d_w_maps, const TcMat* d_tc, int32_t n_mats,
-                              int64_t n_tiles, int32_t grid, int32_t r, uint32_t* d_status,
-                              bool inject_wait, cudaStream_t s) {
+                              const CUtensorMap* d_w_maps, const TcMat* d_tc, const float* d_pinv,
+                              int32_t n_mats, int64_t n_tiles, int32_t grid, int32_t r,
+                              uint32_t* d_status, bool inject_wait, cudaStream_t s) {
   if (n_tiles <= 0) return cudaSuccess;
   switch (r) {
-    case 64: return launch_tmem_r<64>(u_t, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
-    case 128: return launch_tmem_r<128>(u_t, tm_b, d_w_maps, d_tc, n_mats, n_tiles, grid, d_status, inject_wait, s);
+    case 64: return launch_tmem_r<64>(u_t, tm_b, d_w_maps, d_tc, d_pinv, n_mats, n_tiles, grid, d_status, inject_wait, s);
+    case 128: return launch_tmem_r<128>(u_t, tm_b, d_w_maps, d_tc, d_pinv, n_mats, n_tiles, grid, d_status, inject_wait, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -53,3 +53,36 @@ def test_wait_hook_needs_the_tensor_core_pass(lib, gpu):
         zb.zo_set_option(z.ctx, zb.ZO_OPTION_TEST_WAIT_TIMEOUT, 1)
     assert e.value.status == zb.ZO_ERR_UNSUPPORTED
     z.close()
+
+
+def test_rejected_tensor_core_descriptor_is_refused_not_downgraded(lib, gpu):
+    # A bf16 set at r = 16 qualifies for the tensor-core pass.  A W row stride of 2^40
+    # bytes is one cuTensorMapEncodeTiled rejects (strides must stay below 2^40), so the
+    # context cannot build that pass.  zo_create still succeeds, but the automatic path
+    # refuses zo_perturb / zo_step with ZO_ERR_UNSUPPORTED (naming the remedy) instead of
+    # running the FMA pass in its place, and nothing is launched.  The context is only
+    # created and destroyed: no kernel ever touches this W.
+    import torch
+    from paper_2608_15665_gb300 import binding as zb
+    m, n, r = 16, 64, 16
+    W = torch.zeros(m, n, dtype=torch.bfloat16, device=gpu)
+    bufs = [torch.zeros(m, r, device=gpu), torch.zeros(n, r, device=gpu),
+            torch.zeros(r, r, device=gpu), torch.zeros(r, r, device=gpu)]
+    mat = zb.zo_matrix(W.data_ptr(), m, n, 2 ** 39, zb.ZO_BF16, 0, *[b.data_ptr() for b in bufs])
+    ctx = zb.zo_create([mat], r, 2, 1)
+    try:
+        with pytest.raises(zb.ZoError) as e:
+            zb.zo_perturb(ctx, 0, 0, 1.0, -1, 0.0, 1e-3)
+        assert e.value.status == zb.ZO_ERR_UNSUPPORTED
+        assert "ZO_OPTION_WPASS_PATH" in str(e.value) and "W_0" in str(e.value)
+        losses = torch.full((4,), 2.0, device=gpu)
+        with pytest.raises(zb.ZoError) as e:
+            zb.zo_step(ctx, 0, 1, losses, zb.ZO_SCHEME_CENTRAL, 1e-3, 1e-3, 0.9, 0.95, 1e-8, 1, 1.0)
+        assert e.value.status == zb.ZO_ERR_UNSUPPORTED
+        assert zb.zo_kernel_launches(ctx) == 0
+        # the tensor-core path cannot be forced either
+        with pytest.raises(zb.ZoError) as e:
+            zb.zo_set_option(ctx, zb.ZO_OPTION_WPASS_PATH, 2)
+        assert e.value.status == zb.ZO_ERR_UNSUPPORTED
+    finally:
+        zb.zo_destroy(ctx)
