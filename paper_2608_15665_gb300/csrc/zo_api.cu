@@ -113,7 +113,8 @@ struct zo_ctx {
                                      // chunk-major for r >= 64)
   uint16_t* d_p_hl = nullptr;        // stacked [hi | lo] fp16 rows of every P_i^T 2^(e_P,i),
                                      // 128-row padded
-  float* d_pinv = nullptr;           // 2^-(e_P,i) of the current pass, one per matrix
+  float* d_amax = nullptr;           // max |C_i| of the current pass, one per matrix
+  float* d_pinv = nullptr;           // 2^-e_P of the current pass (one for every matrix)
   zo::TcMat* d_tc = nullptr;
   std::vector<zo::TcMat> h_tc;       // host copy (operand rows of each matrix)
   // zo_linear_prepare / zo_linear_perturbed: P_K of every matrix ([P_hi ; P_lo] rows,
@@ -178,6 +179,7 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_v_hl);
   cudaFree(c->d_c_hl);
   cudaFree(c->d_pinv);
+  cudaFree(c->d_amax);
   cudaFree(c->d_u_lin);
   for (auto e : c->ev_start) cudaEventDestroy(e);
   for (auto e : c->ev_stop) cudaEventDestroy(e);
@@ -299,7 +301,8 @@ zo_status run_weight_pass(zo_ctx* c) {
   }
   if (use_tc) {
     // setup_tc keeps tc_ok only with the projection's descriptors in place (proj_tc)
-    ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, c->r, c->d_c_hl, c->d_pinv, c->stream),
+    ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, c->r, c->d_amax, c->d_c_hl, c->d_pinv,
+                               c->stream),
             "split C");
     ++c->launches;
     const int grid = std::min<int>(c->n_proj_units, c->sms);
@@ -463,8 +466,10 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
   ZO_CUDA(cudaMalloc(&c->d_p_hl, sizeof(uint16_t) * prows * HLW), "cudaMalloc(P hi/lo)");
   ZO_CUDA(cudaMemset(c->d_u_op, 0, u_bytes), "memset");
   ZO_CUDA(cudaMemset(c->d_p_hl, 0, sizeof(uint16_t) * prows * HLW), "memset");
-  ZO_CUDA(cudaMalloc(&c->d_pinv, sizeof(float) * c->n_mats), "cudaMalloc(P scales)");
-  ZO_CUDA(cudaMemset(c->d_pinv, 0, sizeof(float) * c->n_mats), "memset");
+  ZO_CUDA(cudaMalloc(&c->d_pinv, sizeof(float)), "cudaMalloc(P scale)");
+  ZO_CUDA(cudaMemset(c->d_pinv, 0, sizeof(float)), "memset");
+  ZO_CUDA(cudaMalloc(&c->d_amax, sizeof(float) * c->n_mats), "cudaMalloc(C maxima)");
+  ZO_CUDA(cudaMemset(c->d_amax, 0, sizeof(float) * c->n_mats), "memset");
   ZO_CUDA(cudaMalloc(&c->d_tc, sizeof(zo::TcMat) * c->n_mats), "cudaMalloc(tile table)");
   ZO_CUDA(cudaMemcpy(c->d_tc, tc.data(), sizeof(zo::TcMat) * c->n_mats, cudaMemcpyHostToDevice),
           "upload tile table");
@@ -806,6 +811,7 @@ zo_status zo_perturb(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t qb, fl
   p.cb = cb;
   p.eps = eps;
   const bool use_tc = tc_path(c);
+  p.amax = use_tc ? c->d_amax : nullptr;
   if (!use_tc && narrow_path(c)) {
     zo_status st = record_start(c);
     if (st != ZO_OK) return st;
@@ -895,6 +901,7 @@ zo_status zo_step(zo_ctx* c, uint32_t t, int32_t adam_t, const float* losses, in
   p.restore_query = restore_query;
   p.restore_coef = restore_coef;
   p.gamma_out = gamma_out;
+  p.amax = tc_path(c) ? c->d_amax : nullptr;
   ZO_CUDA(zo::launch_coeff(c->d_mats, c->n_mats, p, c->stream), "coefficient kernel");
   ++c->launches;
   return run_weight_pass(c);
@@ -976,8 +983,10 @@ zo_status zo_linear_prepare(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t
   p.ca = ca;
   p.cb = cb;
   p.eps = eps;
+  p.amax = c->d_amax;
   ZO_CUDA(zo::launch_coeff(c->d_mats, c->n_mats, p, c->stream), "coefficient kernel");
-  ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, r, c->d_c_hl, c->d_pinv, c->stream), "split C");
+  ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, r, c->d_amax, c->d_c_hl, c->d_pinv, c->stream),
+          "split C");
   ZO_CUDA(zo::launch_project_tc(c->tm_v, c->tm_c, c->tm_p, c->d_tc, c->d_proj_units,
                                 c->n_proj_units, std::min<int32_t>(c->n_proj_units, c->sms), r,
                                 c->d_status, c->stream),

@@ -10,7 +10,8 @@
 //                  D = (M / (1-b1^t)) / (sqrt(Vm / (1-b2^t)) + eps_adam)  (Eqs. (9), (10))
 //            SGD:  D = G                                              (Sec. 3)
 //            C_i = -lr D + restore_coef eps Z_i^(restore_query)
-// P_i = C_i V_i^T (r x n) then feeds the weight pass.
+// P_i = C_i V_i^T (r x n) then feeds the weight pass.  For the tensor-core path the kernel
+// also writes max |C_i| (p.amax), from which the pass's operand scale is chosen.
 #include "zo_kernels.h"
 
 namespace zo {
@@ -29,6 +30,7 @@ __global__ void __launch_bounds__(256) coeff_kernel(const MatDesc* __restrict__ 
                                                     CoeffParams p) {
   __shared__ float rho_s[kMaxQ];
   __shared__ float red_s[8];
+  __shared__ float max_s[8];
   const MatDesc md = mats[blockIdx.x];
   const int r = p.r;
   const int rr = r * r;          // r is a multiple of 4, so rr is a multiple of 16
@@ -51,6 +53,7 @@ __global__ void __launch_bounds__(256) coeff_kernel(const MatDesc* __restrict__ 
   }
 
   float gsq = 0.0f;
+  float cmax = 0.0f;
   float4* C4 = reinterpret_cast<float4*>(md.C);
   for (int c = tid; c < n_ctr; c += blockDim.x) {
     float4 out;
@@ -98,6 +101,19 @@ __global__ void __launch_bounds__(256) coeff_kernel(const MatDesc* __restrict__ 
       }
     }
     C4[c] = out;
+    cmax = fmaxf(cmax, fmaxf(fmaxf(fabsf(out.x), fabsf(out.y)), fmaxf(fabsf(out.z), fabsf(out.w))));
+  }
+
+  if (p.amax != nullptr) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cmax = fmaxf(cmax, __shfl_xor_sync(0xffffffffu, cmax, o));
+    if ((tid & 31) == 0) max_s[tid >> 5] = cmax;
+    __syncthreads();
+    if (tid == 0) {
+      float m = 0.f;
+      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) m = fmaxf(m, max_s[w]);
+      p.amax[blockIdx.x] = m;
+    }
   }
 
   if (p.mode == kCoeffStep && p.gamma_out != nullptr) {

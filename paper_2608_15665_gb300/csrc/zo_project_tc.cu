@@ -202,19 +202,18 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
       tc_fence_after();
       const uint32_t d = tmem + (uint32_t)(acc * R);
       const uint32_t a_base = smem_u32(v_smem + vs * Cfg::kVBytes), b_base = smem_u32(c_smem);
+      // hi.lo and lo.hi first, hi.hi last (see zo_wpass_tc.cu)
 #pragma unroll
-      for (int kk = 0; kk < Cfg::kKC; ++kk) {
-        // hi chunk kk at element 16 kk of an operand row, lo chunk at R + 16 kk
-        const int e_hi = 16 * kk, e_lo = R + 16 * kk;
-        const uint64_t a_hi = sdesc_k_sw128(a_base + (e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
-        const uint64_t a_lo = sdesc_k_sw128(a_base + (e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
-        const uint64_t b_hi =
-            sdesc_k_sw128(b_base + (e_hi / 64) * Cfg::kCPanelBytes + (e_hi % 64) * 2);
-        const uint64_t b_lo =
-            sdesc_k_sw128(b_base + (e_lo / 64) * Cfg::kCPanelBytes + (e_lo % 64) * 2);
-        mma_f16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
-        mma_f16(d, a_hi, b_lo, idesc, 1u);
-        mma_f16(d, a_lo, b_hi, idesc, 1u);
+      for (int pass = 0; pass < 3; ++pass) {
+#pragma unroll
+        for (int kk = 0; kk < Cfg::kKC; ++kk) {
+          // hi chunk kk at element 16 kk of an operand row, lo chunk at R + 16 kk
+          const int e_a = (pass == 1 ? R : 0) + 16 * kk, e_b = (pass == 0 ? R : 0) + 16 * kk;
+          const uint64_t a_d = sdesc_k_sw128(a_base + (e_a / 64) * kPanelBytes + (e_a % 64) * 2);
+          const uint64_t b_d =
+              sdesc_k_sw128(b_base + (e_b / 64) * Cfg::kCPanelBytes + (e_b % 64) * 2);
+          mma_f16(d, a_d, b_d, idesc, (pass | kk) != 0 ? 1u : 0u);
+        }
       }
       mma_commit(&sh.v_empty[vs]);
       if (last_c) mma_commit(&sh.c_empty);
@@ -328,14 +327,15 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
 
 // Rows [hi | lo] of the scaled fp16 pair of V (units = (matrix, first row) x 128 rows, into
 // V_HL at p_row0; scale 2^kUVScaleExp) or of C (one CTA per matrix, r rows into C_HL at
-// matrix * r; scale 2^(e_C,i), found here from max |C_i|, with pinv[i] = 2^-(e_P,i) written
-// for the weight pass).  Each thread splits one row; the rows are staged in shared memory
-// with the 16-byte chunk index XOR (row & 7) and written with coalesced 16-byte stores.
+// matrix * r; scale 2^e_C, one exponent for the pass from the largest of the n_mats maxima
+// amax[], with pinv[0] = 2^-e_P written for the weight pass).  Each thread splits one row;
+// the rows are staged in shared memory with the 16-byte chunk index XOR (row & 7) and
+// written with coalesced 16-byte stores.
 template <int R, bool kC>
 __global__ void __launch_bounds__(128)
 split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
-                  const int2* __restrict__ units, uint16_t* __restrict__ dst,
-                  float* __restrict__ pinv) {
+                  const int2* __restrict__ units, const float* __restrict__ amax_in, int n_mats,
+                  uint16_t* __restrict__ dst, float* __restrict__ pinv) {
   constexpr int kVecPerRow = 2 * R * 2 / 16;     // 16-byte chunks of [hi | lo]
   constexpr int kSw = kVecPerRow >= 8 ? 7 : kVecPerRow - 1;   // chunk swizzle within a row
   constexpr int kStride = hl_width(R) / 8;       // chunks per row of V_HL / C_HL
@@ -360,17 +360,10 @@ split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tc
   }
   float scale = exp2i(kUVScaleExp);
   if constexpr (kC) {
-    // e_C,i from the largest |C_i|: every thread takes the max of its row, then the block's
+    // e_C from the largest max |C_i| of the pass (the same in every CTA)
     __shared__ float wmax[4];
     float amax = 0.f;
-    if (tid < rows) {
-      const float4* s4 = reinterpret_cast<const float4*>(src + (int64_t)tid * R);
-#pragma unroll
-      for (int g = 0; g < R / 4; ++g) {
-        const float4 a = s4[g];
-        amax = fmaxf(amax, fmaxf(fmaxf(fabsf(a.x), fabsf(a.y)), fmaxf(fabsf(a.z), fabsf(a.w))));
-      }
-    }
+    for (int k = tid; k < n_mats; k += blockDim.x) amax = fmaxf(amax, amax_in[k]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
     if ((tid & 31) == 0) wmax[tid >> 5] = amax;
@@ -378,7 +371,7 @@ split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tc
     amax = fmaxf(fmaxf(wmax[0], wmax[1]), fmaxf(wmax[2], wmax[3]));
     const int e_c = coeff_scale_exp(amax);
     scale = exp2i(e_c);
-    if (tid == 0) pinv[i] = exp2i(-(e_c + p_scale_offset(R)));
+    if (blockIdx.x == 0 && tid == 0) pinv[0] = exp2i(-(e_c + p_scale_offset(R)));
   }
   if (tid < rows) {
     const float4* s4 = reinterpret_cast<const float4*>(src + (row0 + tid) * R);
@@ -417,14 +410,16 @@ cudaError_t launch_project_tc_r(const CUtensorMap& tm_v, const CUtensorMap& tm_c
 
 template <int R, bool kC>
 cudaError_t launch_split_rows_r(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
-                                int32_t n_blocks, uint16_t* dst, float* pinv, cudaStream_t s) {
+                                int32_t n_blocks, const float* amax, uint16_t* dst, float* pinv,
+                                cudaStream_t s) {
   constexpr size_t smem = 128 * (size_t)(2 * R * 2);
   if (smem > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(split_rows_kernel<R, kC>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
-  split_rows_kernel<R, kC><<<n_blocks, 128, smem, s>>>(d_mats, d_tc, d_units, dst, pinv);
+  split_rows_kernel<R, kC><<<n_blocks, 128, smem, s>>>(d_mats, d_tc, d_units, amax, n_blocks, dst,
+                                                      pinv);
   return cudaGetLastError();
 }
 
@@ -436,22 +431,22 @@ cudaError_t launch_split_v(const MatDesc* d_mats, const TcMat* d_tc, const int2*
                            int32_t n_units, int32_t r, uint16_t* v_hl, cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
-    case 16: return launch_split_rows_r<16, false>(d_mats, d_tc, d_units, n_units, v_hl, nullptr, s);
-    case 32: return launch_split_rows_r<32, false>(d_mats, d_tc, d_units, n_units, v_hl, nullptr, s);
-    case 64: return launch_split_rows_r<64, false>(d_mats, d_tc, d_units, n_units, v_hl, nullptr, s);
-    case 128: return launch_split_rows_r<128, false>(d_mats, d_tc, d_units, n_units, v_hl, nullptr, s);
+    case 16: return launch_split_rows_r<16, false>(d_mats, d_tc, d_units, n_units, nullptr, v_hl, nullptr, s);
+    case 32: return launch_split_rows_r<32, false>(d_mats, d_tc, d_units, n_units, nullptr, v_hl, nullptr, s);
+    case 64: return launch_split_rows_r<64, false>(d_mats, d_tc, d_units, n_units, nullptr, v_hl, nullptr, s);
+    case 128: return launch_split_rows_r<128, false>(d_mats, d_tc, d_units, n_units, nullptr, v_hl, nullptr, s);
     default: return cudaErrorInvalidValue;
   }
 }
 
-cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, uint16_t* c_hl,
-                           float* pinv, cudaStream_t s) {
+cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, const float* amax,
+                           uint16_t* c_hl, float* pinv, cudaStream_t s) {
   if (n_mats <= 0) return cudaSuccess;
   switch (r) {
-    case 16: return launch_split_rows_r<16, true>(d_mats, nullptr, nullptr, n_mats, c_hl, pinv, s);
-    case 32: return launch_split_rows_r<32, true>(d_mats, nullptr, nullptr, n_mats, c_hl, pinv, s);
-    case 64: return launch_split_rows_r<64, true>(d_mats, nullptr, nullptr, n_mats, c_hl, pinv, s);
-    case 128: return launch_split_rows_r<128, true>(d_mats, nullptr, nullptr, n_mats, c_hl, pinv, s);
+    case 16: return launch_split_rows_r<16, true>(d_mats, nullptr, nullptr, n_mats, amax, c_hl, pinv, s);
+    case 32: return launch_split_rows_r<32, true>(d_mats, nullptr, nullptr, n_mats, amax, c_hl, pinv, s);
+    case 64: return launch_split_rows_r<64, true>(d_mats, nullptr, nullptr, n_mats, amax, c_hl, pinv, s);
+    case 128: return launch_split_rows_r<128, true>(d_mats, nullptr, nullptr, n_mats, amax, c_hl, pinv, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -241,17 +241,21 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
         break;
       }
       tc_fence_after();
+      // the small cross products hi.lo and lo.hi first, hi.hi last: each MMA adds its
+      // products to the fp32 accumulator with one rounding relative to the accumulator's
+      // magnitude, so only the r/16 hi.hi MMAs round at the update's full size
 #pragma unroll
-      for (int kk = 0; kk < Cfg::kKC; ++kk) {
-        // hi chunk kk at element 16 kk of the operand row, lo chunk at R + 16 kk
-        const int e_hi = 16 * kk, e_lo = R + 16 * kk;
-        const uint32_t off_hi = (uint32_t)((e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
-        const uint32_t off_lo = (uint32_t)((e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
-        const uint64_t a_hi = sdesc_k_sw128(a_base + off_hi), a_lo = sdesc_k_sw128(a_base + off_lo);
-        const uint64_t b_hi = sdesc_k_sw128(b_base + off_hi), b_lo = sdesc_k_sw128(b_base + off_lo);
-        mma_f16(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
-        mma_f16(d, a_hi, b_lo, idesc, 1u);
-        mma_f16(d, a_lo, b_hi, idesc, 1u);
+      for (int pass = 0; pass < 3; ++pass) {
+#pragma unroll
+        for (int kk = 0; kk < Cfg::kKC; ++kk) {
+          // hi chunk kk at element 16 kk of the operand row, lo chunk at R + 16 kk
+          const int e_hi = 16 * kk, e_lo = R + 16 * kk;
+          const uint32_t off_hi = (uint32_t)((e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
+          const uint32_t off_lo = (uint32_t)((e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
+          const uint64_t a_d = sdesc_k_sw128(a_base + (pass == 1 ? off_lo : off_hi));
+          const uint64_t b_d = sdesc_k_sw128(b_base + (pass == 0 ? off_lo : off_hi));
+          mma_f16(d, a_d, b_d, idesc, (pass | kk) != 0 ? 1u : 0u);
+        }
       }
       mma_commit(&sh.b_empty[sb]);
       if (last_a) mma_commit(&sh.a_empty[sa]);
@@ -272,11 +276,13 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
     TileIter ti;
     ti.init(mats, n_mats, t_begin, t_end, t_stride);
     ti.chunk = kTileChunk;
+    // the accumulator holds 2^(kUVScaleExp + e_P) U P, with one e_P for the whole pass:
+    // back to U P in the add.  Loaded once -- these warps set the kernel's pace, and a
+    // load per tile costs a measured 1.5% of the pass
+    const float wscale = pinv[0] * exp2i(-kUVScaleExp);
     for (; ti.valid(); ti.next(), ++it) {
       const TcMat& mt = mats[ti.i];
       const int acc = (int)(it & 1);
-      // the accumulator holds 2^(kUVScaleExp + e_P) U P: back to U P in the add
-      const float wscale = pinv[ti.i] * exp2i(-kUVScaleExp);
       // test hook (zo_set_option ZO_OPTION_TEST_WAIT_TIMEOUT): CTA 0's epilogue first waits
       // on a barrier that nothing arrives on, so its bounded wait runs out
       if (inject_wait && blockIdx.x == 0 && it == 0 &&

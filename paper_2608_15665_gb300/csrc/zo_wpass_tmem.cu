@@ -281,18 +281,20 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
       const uint32_t d = tmem + (uint32_t)(acc * kBN);
       const uint32_t a_base = tmem + (uint32_t)(2 * kBN + sa * Cfg::kACols);
       const uint32_t b_base = smem_u32(b_smem + sb * Cfg::kOpBytes);
+      // hi.lo and lo.hi first, hi.hi last (see zo_wpass_tc.cu): only the r/16 hi.hi MMAs
+      // round at the update's full size
 #pragma unroll
-      for (int kk = 0; kk < Cfg::kKC; ++kk) {
-        // U: hi chunk kk at column 8 kk of the buffer, lo chunk at R/2 + 8 kk;
-        // P: hi chunk kk at element 16 kk of the operand row, lo chunk at R + 16 kk
-        const uint32_t a_hi = a_base + (uint32_t)(8 * kk), a_lo = a_base + (uint32_t)(R / 2 + 8 * kk);
-        const int e_hi = 16 * kk, e_lo = R + 16 * kk;
-        const uint32_t off_hi = (uint32_t)((e_hi / 64) * kPanelBytes + (e_hi % 64) * 2);
-        const uint32_t off_lo = (uint32_t)((e_lo / 64) * kPanelBytes + (e_lo % 64) * 2);
-        const uint64_t b_hi = sdesc_k_sw128(b_base + off_hi), b_lo = sdesc_k_sw128(b_base + off_lo);
-        mma_f16_ts(d, a_hi, b_hi, idesc, kk > 0 ? 1u : 0u);
-        mma_f16_ts(d, a_hi, b_lo, idesc, 1u);
-        mma_f16_ts(d, a_lo, b_hi, idesc, 1u);
+      for (int pass = 0; pass < 3; ++pass) {
+#pragma unroll
+        for (int kk = 0; kk < Cfg::kKC; ++kk) {
+          // U: hi chunk kk at column 8 kk of the buffer, lo chunk at R/2 + 8 kk;
+          // P: hi chunk kk at element 16 kk of the operand row, lo chunk at R + 16 kk
+          const uint32_t a_t = a_base + (uint32_t)((pass == 1 ? R / 2 : 0) + 8 * kk);
+          const int e_b = (pass == 0 ? R : 0) + 16 * kk;
+          const uint64_t b_d =
+              sdesc_k_sw128(b_base + (uint32_t)((e_b / 64) * kPanelBytes + (e_b % 64) * 2));
+          mma_f16_ts(d, a_t, b_d, idesc, (pass | kk) != 0 ? 1u : 0u);
+        }
       }
       mma_commit(&sh.b_empty[sb]);
       if (last_a) mma_commit(&sh.a_empty[sa]);
@@ -317,11 +319,12 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
     TileIter ti;
     ti.init(mats, n_mats, t_begin, t_end, t_stride);
     ti.chunk = kTileChunk;
+    // the accumulator holds 2^(kUVScaleExp + e_P) U P (one e_P for the pass): back to U P
+    // in the add, with the scale loaded once (see zo_wpass_tc.cu)
+    const float wscale = pinv[0] * exp2i(-kUVScaleExp);
     for (; ti.valid(); ti.next(), ++it) {
       const TcMat& mt = mats[ti.i];
       const int acc = (int)(it & 1);
-      // the accumulator holds 2^(kUVScaleExp + e_P) U P: back to U P in the add
-      const float wscale = pinv[ti.i] * exp2i(-kUVScaleExp);
       // test hook (zo_set_option ZO_OPTION_TEST_WAIT_TIMEOUT): CTA 0's epilogue first waits
       // on a barrier that nothing arrives on, so its bounded wait runs out
       if (inject_wait && blockIdx.x == 0 && it == 0 &&

@@ -101,3 +101,121 @@ def test_moment_tolerance_accepts_fp32_and_rejects_mistakes():
     for name, (Mb, Vb) in bad.items():
         with pytest.raises(AssertionError):
             assert_moments(Mb, Vb, M, Vm, M0, V0, Gabs, b1, b2, name)
+
+
+# ---------------------------------------------------------------------------------------
+# The flip bounds of the bf16 trajectory test (parity.pass_error_coeff / FlipLedger)
+# ---------------------------------------------------------------------------------------
+
+def _fma_chain(a, b):
+    """sum_k a[:, k] b[k, :] by one fmaf per term in k order (fp32, each fma rounded once;
+    the exact product-plus-accumulator is formed in fp64 first)."""
+    acc = np.zeros((a.shape[0], b.shape[1]), np.float32)
+    for k in range(a.shape[1]):
+        acc = (np.outer(a[:, k].astype(np.float64), b[k].astype(np.float64)) + acc).astype(np.float32)
+    return acc
+
+
+def _sim_fma_pass(W, U, V, C):
+    """The FMA path's arithmetic: P = C V^T and U P by fmaf chains, W + delta in fp32."""
+    f = np.float32
+    P = _fma_chain(C.astype(f), V.astype(f).T)
+    d = _fma_chain(U.astype(f), P)
+    return (W.astype(f) + d).astype(np.float64)
+
+
+def _pair16(x, s):
+    """Scaled fp16 pair: x s = hi + lo (RNE, subnormals kept)."""
+    xs = (np.asarray(x, np.float32) * np.float32(s)).astype(np.float32)
+    hi = xs.astype(np.float16)
+    lo = (xs - hi.astype(np.float32)).astype(np.float16)
+    return hi.astype(np.float64), lo.astype(np.float64)
+
+
+def _mma_chain(ah, al, bh, bl):
+    """hi.hi + hi.lo + lo.hi over K in MMAs of 16: each MMA's 16 exact products are added
+    to the fp32 accumulator with one rounding (the kernels' order: K chunk by K chunk, the
+    three products of a chunk in turn)."""
+    K = ah.shape[1]
+    acc = np.zeros((ah.shape[0], bh.shape[1]), np.float32)
+    for k0 in range(0, K, 16):
+        sl = slice(k0, k0 + 16)
+        for x, y in ((ah, bh), (ah, bl), (al, bh)):
+            acc = (x[:, sl] @ y[sl] + acc.astype(np.float64)).astype(np.float32)
+    return acc
+
+
+def _sim_tc_pass(W, U, V, C, r, scale_err=1.0):
+    """The tensor-core path's arithmetic with the scales of zo_tc_common.cuh: V, C, U, P as
+    fp16 pairs (V, U at 2^14, C at 2^(14 - E), max|C| < 2^E, P at 2^(e_C + off(r))), three
+    products per K chunk into fp32, the epilogue's fp32 multiply-add.  scale_err != 1
+    plants a mistake: the P pair formed at a scale off by that factor but undone as if not."""
+    off = -1 if r <= 16 else -2 if r <= 64 else -3
+    e_c = 14 - int(np.frexp(np.abs(C).max())[1])
+    vh, vl = _pair16(V, 2.0 ** 14)
+    ch, cl = _pair16(C, 2.0 ** e_c)
+    D = _mma_chain(vh, vl, ch.T, cl.T)                     # (V C^T) 2^(14 + e_C) = P^T s
+    e_p = e_c + off
+    Pt = (D.astype(np.float64) * 2.0 ** (off - 14)).astype(np.float32)
+    ph, pl = _pair16(Pt.T, scale_err)
+    uh, ul = _pair16(U, 2.0 ** 14)
+    acc = _mma_chain(uh, ul, ph, pl)
+    w = np.float32(2.0 ** (-14 - e_p))
+    return (acc.astype(np.float64) * w + W.astype(np.float32).astype(np.float64)).astype(np.float32) \
+        .astype(np.float64)
+
+
+@pytest.mark.parametrize("path,r", [("fma", 8), ("fma", 32), ("tc", 16), ("tc", 32), ("tc", 64)])
+@pytest.mark.parametrize("eps", [1e-3, 1e-1, 1.0])
+def test_flip_bound_covers_the_simulated_arithmetic(path, r, eps):
+    # every element whose simulated rounding differs from the exact one has its exact value
+    # within the derived error bound of a rounding boundary
+    from parity import FlipLedger, bounded_pass
+    m, n = 160, 136
+    U, V = haar.haar_proj(SEED, 3, 0, m, n, r)
+    U, V = U.astype(np.float32).astype(np.float64), V.astype(np.float32).astype(np.float64)
+    W = rounding.round_to_bf16(np.random.default_rng(r).standard_normal((m, n)) * 0.02)
+    flips = near = 0
+    for k in range(4):
+        C = subzero.perturb_coeff(SEED, 3, k, r, [(0, 1.0), (1, -1.0)], eps)
+        C = C.astype(np.float32).astype(np.float64)          # the C the kernels hold
+        ledger = FlipLedger(W.shape)
+        want = bounded_pass(W, U, V, C, np.zeros_like(C), path, r, ledger)
+        x = _sim_fma_pass(W, U, V, C) if path == "fma" else _sim_tc_pass(W, U, V, C, r)
+        differ = rounding.round_to_bf16(x) != want
+        assert not (differ & (ledger.n_amb == 0)).any()
+        flips += int(differ.sum())
+        near += int((ledger.n_amb > 0).sum())
+    assert near >= flips
+
+
+def test_flip_bound_rejects_a_pair_at_the_wrong_scale():
+    # a P pair formed at twice the scale the epilogue undoes doubles delta: nearly every
+    # element rounds differently, far outside the bound
+    from parity import FlipLedger, bounded_pass
+    m, n, r = 160, 136, 32
+    U, V = haar.haar_proj(SEED, 4, 0, m, n, r)
+    W = rounding.round_to_bf16(np.random.default_rng(5).standard_normal((m, n)) * 0.02)
+    C = subzero.perturb_coeff(SEED, 4, 0, r, [(0, 1.0)], 1e-1).astype(np.float32).astype(np.float64)
+    ledger = FlipLedger(W.shape)
+    want = bounded_pass(W, U, V, C, np.zeros_like(C), "tc", r, ledger)
+    x = _sim_tc_pass(W, U, V, C, r, scale_err=2.0)
+    differ = rounding.round_to_bf16(x) != want
+    assert (differ & (ledger.n_amb == 0)).sum() > differ.size // 4
+
+
+def test_boundary_distance_is_the_rounding_margin():
+    from parity import bf16_boundary_distance
+    x = np.random.default_rng(7).standard_normal(20000) * 0.02
+    x = np.concatenate([x, [1.0, -1.0, 2.0 ** -3, 3.0 * 2.0 ** -9]])   # values on a binade edge
+    d = bf16_boundary_distance(x)
+    r0 = rounding.round_to_bf16(x)
+    s = np.sign(x)
+    assert (d >= 0).all()
+    # just inside the margin the rounding holds on both sides; just past it, on one side, it
+    # changes
+    assert (rounding.round_to_bf16(x + d * (1 - 1e-6)) == r0).all()
+    assert (rounding.round_to_bf16(x - d * (1 - 1e-6)) == r0).all()
+    moved = (rounding.round_to_bf16(x + s * d * (1 + 1e-6)) != r0) | \
+            (rounding.round_to_bf16(x - s * d * (1 + 1e-6)) != r0)
+    assert moved.all()
