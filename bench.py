@@ -77,6 +77,11 @@ def parse_args():
                         "for profiling captures); 0 = all")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-secondary", action="store_true",
+                   help="skip the second measurement on the 32B-shaped set (default workload only)")
+    p.add_argument("--oracle-sample", action="store_true",
+                   help="internal: print one timing of the oracle's bounded sample as JSON and exit "
+                        "(run in a single-thread subprocess for cpu_baseline.single_thread)")
     return p.parse_args()
 
 
@@ -182,6 +187,12 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------------------- oracle timing
+def oracle_sample(wl):
+    """The bounded sample both oracle legs time: 1024 rows of matrix 0 and, where the set
+    has one, 1024 rows of matrix 4 (the first wide projection of a LLaMA-shaped layer)."""
+    return ((0, 1024), (4, 1024)) if wl.n_mats > 4 else ((0, 1024),)
+
+
 def oracle_sample_step_seconds(wl, scheme, sample=((0, 1024),), seed_shift=0):
     """Time the fp64 oracle, as it stands, on a bounded sample of one step: for each
     (matrix, n_rows) in ``sample``, the refresh of that matrix (Alg. 1 on its full m x r
@@ -230,17 +241,54 @@ def oracle_sample_step_seconds(wl, scheme, sample=((0, 1024),), seed_shift=0):
     text = ("fp64 oracle, one step: all weight passes + estimator + Adam on "
             + ", ".join(f"{r} rows of matrix {i} {wl.shapes[i][0]}x{wl.shapes[i][1]}" for i, r in used)
             + f" ({el_sample} of {wl.params} weights) and the refresh of those matrices; "
-            f"extrapolated by weight count (refresh by m+n, amortized over F={wl.F})")
+            f"EXTRAPOLATED to the whole set by weight count (refresh by m+n, amortized over "
+            f"F={wl.F})")
     cores = round(cpu_s / (t_pass + t_ref), 1) if t_pass + t_ref > 0 else 1.0
-    return step_s, refresh_s, text, cores
+    return step_s, refresh_s, text, cores, t_pass + t_ref
+
+
+def oracle_single_thread(wl_name, scheme):
+    """The same oracle sample timed in a fresh interpreter pinned to one BLAS / OpenMP
+    thread (a spawned process: nothing CUDA is inherited).  Returns its JSON or None."""
+    env = dict(os.environ)
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "NUMEXPR_NUM_THREADS",
+              "VECLIB_MAXIMUM_THREADS"):
+        env[k] = "1"
+    for k in ("RANK", "LOCAL_RANK", "WORLD_SIZE"):
+        env.pop(k, None)
+    try:
+        res = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-sample",
+                              "--workload", wl_name, "--scheme", scheme],
+                             capture_output=True, text=True, env=env, timeout=600)
+        return json.loads(res.stdout.strip().splitlines()[-1]) if res.returncode == 0 else None
+    except Exception:
+        return None
+
+
+def run_oracle_sample(args):
+    from paper_2608_15665_gb300 import workloads
+    wl = workloads.get(args.workload)
+    step_s, refresh_s, text, cores, _ = oracle_sample_step_seconds(wl, args.scheme,
+                                                                   sample=oracle_sample(wl))
+    print(json.dumps({"value": 1.0 / (step_s + refresh_s / wl.F), "cores": cores}), flush=True)
 
 
 def cpu_baseline(wl, scheme):
-    step_s, refresh_s, text, cores = oracle_sample_step_seconds(wl, scheme,
-                                                                sample=((0, 1024), (4, 1024)))
+    step_s, refresh_s, text, cores, _ = oracle_sample_step_seconds(wl, scheme,
+                                                                   sample=oracle_sample(wl))
     per_step = step_s + refresh_s / wl.F
+    one = oracle_single_thread(wl.name, scheme)
     return {"value": 1.0 / per_step, "unit": "ZO steps/s", "cores": cores,
-            "host_cores": os.cpu_count(), "kind": "oracle", "sample": text}
+            "host_cores": os.cpu_count(), "kind": "oracle", "sample": text, "extrapolated": True,
+            "single_thread": ({"value": one["value"], "unit": "ZO steps/s", "cores": one["cores"],
+                               "threads": "1 BLAS / OpenMP thread"} if one else None)}
+
+
+def amortise_refresh(window_ms, K, t0, F, refresh_ms):
+    """ms per step of a window of K steps t0 .. t0 + K - 1 with the refreshes it held (steps
+    t with t mod F == 0) replaced by refresh_ms / F per step."""
+    n_ref = sum(1 for t in range(t0, t0 + K) if t % F == 0)
+    return (window_ms - n_ref * refresh_ms) / K + refresh_ms / F
 
 
 # --------------------------------------------------------------------------- reference arm
@@ -250,13 +298,14 @@ def run_reference(args):
         return
     from paper_2608_15665_gb300 import workloads
     wl = workloads.get(args.workload)
-    times, cores = [], []
+    times, cores, sample_s = [], [], []
     for s in range(args.warmup + args.steps):
-        step_s, refresh_s, text, c = oracle_sample_step_seconds(wl, args.scheme, sample=((0, 512),),
-                                                                seed_shift=s)
+        step_s, refresh_s, text, c, spent = oracle_sample_step_seconds(
+            wl, args.scheme, sample=oracle_sample(wl), seed_shift=s)
         if s >= args.warmup:
             times.append(step_s + refresh_s / wl.F)
             cores.append(c)
+            sample_s.append(spent)
     per_step = sum(times) / len(times)
     value = 1.0 / per_step
     passes = 2 * wl.q + 1 if args.scheme == "central" else wl.q + 1
@@ -269,9 +318,15 @@ def run_reference(args):
                    "q": wl.q, "scheme": args.scheme, "passes_per_step": passes,
                    "refresh_every": wl.F},
         "cpu_baseline": {"value": value, "unit": "ZO steps/s", "cores": max(cores),
-                         "host_cores": os.cpu_count(), "kind": "oracle", "sample": text},
+                         "host_cores": os.cpu_count(), "kind": "oracle", "sample": text,
+                         "extrapolated": True},
         "e2e": {"value": value, "unit": "ZO steps/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
+        # ms_per_step is the whole set's step, extrapolated from the timed sample; the time
+        # this run actually spent per step is the sample's
+        "extrapolation": {"sample_seconds_per_step": sum(sample_s) / len(sample_s),
+                          "weights_sampled_of": [sum(min(r, wl.shapes[i][0]) * wl.shapes[i][1]
+                                                     for i, r in oracle_sample(wl)), wl.params]},
     }
     print(json.dumps(line), flush=True)
 
@@ -305,7 +360,7 @@ def run_ours(args):
     calls, (rq, rc) = step_plan(args.scheme, wl.q)
     passes = len(calls) + 1
     K, W = args.steps, args.warmup
-    table = workloads.loss_table(wl, args.scheme, steps=W + 2 * K)
+    table = workloads.loss_table(wl, args.scheme, steps=W + 2 * K + 1)
     table_dev = torch.from_numpy(table).to(dev)
 
     if args.method == "mezo":
@@ -380,25 +435,45 @@ def run_ours(args):
     refresh_ms = max_over_ranks(r0.elapsed_time(r1))
     z.sync()
 
+    # Both timed windows are reported with the refresh amortised: a window of K steps holds
+    # floor-or-ceil(K / F) refreshes depending on where it starts, so the refreshes it
+    # happened to contain are replaced by refresh_ms / F per step (Alg. 3 refreshes every F
+    # steps).  The raw window figures stay in "window".
+    def amortised_ms(window_ms, t0):
+        if args.method == "mezo":                 # no subspace, no refresh
+            return window_ms / K
+        return amortise_refresh(window_ms, K, t0, wl.F, refresh_ms)
+
     # ---- end to end through the public API with host buffers -------------------------
     e2e = None
     if not args.no_e2e:
-        host_losses = torch.from_numpy(table[W + K:W + 2 * K].copy()).pin_memory()
+        host_losses = torch.from_numpy(table[W + K:W + 2 * K + 1].copy()).pin_memory()
         gamma = torch.zeros(wl.n_mats, dtype=torch.float32, device=dev)
         gamma_host = torch.zeros(wl.n_mats, dtype=torch.float32).pin_memory()
+        # one untimed step through the host path first (first use of the pinned buffers)
+        do_step(W + K, host_losses[0].numpy(), gamma)
+        gamma_host.copy_(gamma)
+        e_clocks = ClockSampler(local)
+        e_clocks.start()
         barrier()
         t0 = time.perf_counter()
-        for k, t in enumerate(range(W + K, W + 2 * K)):
-            do_step(t, host_losses[k].numpy(), gamma)
+        for k, t in enumerate(range(W + K + 1, W + 2 * K + 1)):
+            do_step(t, host_losses[k + 1].numpy(), gamma)
             gamma_host.copy_(gamma)            # the step's result back on the host (syncs)
         barrier()
         e2e_s = max_over_ranks(time.perf_counter() - t0)
-        e2e = {"value": world * K / e2e_s, "unit": "ZO steps/s",
+        e_clk = e_clocks.stop()
+        e2e_ms = amortised_ms(e2e_s * 1e3, W + K + 1)
+        e2e = {"value": world * 1e3 / e2e_ms, "unit": "ZO steps/s",
                "h2d_bytes_per_step": int(table.shape[1] * 4),
-               "d2h_bytes_per_step": int(wl.n_mats * 4)}
+               "d2h_bytes_per_step": int(wl.n_mats * 4),
+               "ms_per_step": e2e_ms,
+               "window": {"value": world * K / e2e_s, "ms_per_step": e2e_s * 1e3 / K},
+               "clocks": e_clk}
     z.sync()
 
-    value = world * K / (elapsed_ms / 1e3)
+    step_ms = amortised_ms(elapsed_ms, W)
+    value = world * 1e3 / step_ms
     bytes_pass = wl.bytes_per_pass()
     peak, peak_kind = measured_peaks()
     avg_launch_s = (wpass_ms / wpass_n) / 1e3 if wpass_n else float("nan")
@@ -407,7 +482,7 @@ def run_ours(args):
     l2_resident = bytes_pass / 2 < L2_BYTES
     line = {
         "metric": METRIC, "value": value, "unit": "ZO steps/s", "n_gpus": world, "steps": K,
-        "warmup": W, "ms_per_step": elapsed_ms / K, "higher_is_better": True, "scaling": "weak",
+        "warmup": W, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": wl0.name, "matrices": wl.n_mats, "params": wl.params,
                    "weights": "bf16 N(0,0.02^2)" if wl.dtype == "bf16" else "f32 N(0,0.02^2)",
@@ -420,6 +495,11 @@ def run_ours(args):
                    "parallelism": f"layer partition x{world}" if world > 1 else "single GPU"},
         "weight_pass_gbs": passes * bytes_pass * K / (elapsed_ms / 1e3) / 1e9,
         "refresh_ms": refresh_ms,
+        "window": {"value": world * K / (elapsed_ms / 1e3), "ms_per_step": elapsed_ms / K,
+                   "refreshes": sum(1 for t in range(W, W + K) if t % wl.F == 0)
+                   if args.method != "mezo" else 0,
+                   "note": "value and ms_per_step replace the refreshes this window held by "
+                           "refresh_ms / F per step"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "traffic": TRAFFIC_BY_SOURCE.get((src, wl.name)),
@@ -455,14 +535,84 @@ def run_ours(args):
         line["config"].pop("r"); line["config"].pop("q")
     if e2e:
         line["e2e"] = e2e
+    z.close()
+    if (world == 1 and args.method == "subzero" and args.workload == "llama7b_bf16_r32"
+            and not args.layers and not args.no_secondary):
+        # the second shape the weight pass is held to: the 32B-shaped set (r = 64, q = 8)
+        del weights, z
+        torch.cuda.empty_cache()
+        line["secondary"] = {"dense32b_bf16_r64": secondary_32b(dev, local, peak)}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl0, args.scheme)
-    z.close()
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.barrier()
         dist.destroy_process_group()
+
+
+def secondary_32b(dev, local, peak):
+    """A short measurement of the weight pass on the 32B-shaped set (448 bf16 matrices,
+    31.2 G parameters, r = 64, q = 8, central scheme: 17 passes per step, refresh every 5):
+    one warm-up step (with its refresh), then 2 timed steps with the weight-pass launches
+    timed by CUDA events, and one refresh timed on its own."""
+    import torch
+    from paper_2608_15665_gb300 import binding as zb
+    from paper_2608_15665_gb300 import workloads
+    from paper_2608_15665_gb300.schedule import SubZeroPlus, step_plan
+    wl = workloads.get("dense32b_bf16_r64")
+    weights = [workloads.init_weight(wl, i, dev) for i in range(wl.n_mats)]
+    z = SubZeroPlus(weights, wl.r, wl.q, wl.seed)
+    calls, (rq, rc) = step_plan("central", wl.q)
+    K = 2
+    table = torch.from_numpy(workloads.loss_table(wl, "central", steps=1 + K)).to(dev)
+
+    def do_step(t):
+        if t % wl.F == 0:
+            z.refresh(t // wl.F, reset_moments=(t == 0))
+        for (qa, ca), second in calls:
+            qb, cb = second if second is not None else (-1, 0.0)
+            z.perturb(t, qa, ca, qb, cb, wl.eps)
+        z.step(t, t + 1, table[t], "central", wl.eps, wl.lr, wl.beta1, wl.beta2, wl.eps_adam, rq, rc)
+
+    do_step(0)
+    z.sync()
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_TIMING, 1)
+    clocks = ClockSampler(local)
+    clocks.start()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for t in range(1, 1 + K):
+        do_step(t)
+    e1.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    window_ms = e0.elapsed_time(e1)
+    wpass_ms, wpass_n = zb.zo_get_timing(z.ctx)
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_TIMING, 0)
+    path = zb.zo_wpass_path(z.ctx)
+    r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    r0.record()
+    z.refresh(1)
+    r1.record()
+    torch.cuda.synchronize()
+    refresh_ms = r0.elapsed_time(r1)
+    z.sync()
+    z.close()
+    del weights, z
+    torch.cuda.empty_cache()
+    avg_s = (wpass_ms / wpass_n) / 1e3
+    achieved = wl.bytes_per_pass() / avg_s / 1e9
+    step_ms = window_ms / K + refresh_ms / wl.F
+    return {"workload": wl.name, "matrices": wl.n_mats, "params": wl.params, "r": wl.r, "q": wl.q,
+            "passes_per_step": 2 * wl.q + 1, "refresh_every": wl.F, "steps_timed": K,
+            "kernel": {2: "wpass_tmem", 1: "wpass_fma"}.get(path, "?"),
+            "avg_launch_ms": avg_s * 1e3, "launches_timed": wpass_n,
+            "algorithmic_bytes_per_launch": wl.bytes_per_pass(),
+            "achieved_gbs": achieved, "peak_gbs": peak, "frac": achieved / peak,
+            "zo_steps_s": 1e3 / step_ms, "ms_per_step": step_ms, "refresh_ms": refresh_ms,
+            "clocks": clk}
 
 
 def run_linear(args):
@@ -594,7 +744,9 @@ def run_linear(args):
 
 def main():
     args = parse_args()
-    if args.impl == "reference":
+    if args.oracle_sample:
+        run_oracle_sample(args)
+    elif args.impl == "reference":
         run_reference(args)
     elif args.method == "linear":
         run_linear(args)

@@ -160,6 +160,30 @@ __device__ __forceinline__ void split8_f16(const float (&x)[8], float s, uint4& 
   lo = make_uint4(lw[0], lw[1], lw[2], lw[3]);
 }
 
+// The weight-pass epilogue's arithmetic for two neighbouring bf16 weights w (packed, lower
+// half = first) and their fp32 updates a, b: rnd_bf16(w + s a), rnd_bf16(w' + s b), as one
+// packed fp32 multiply-add (fma.rn.f32x2: each lane an IEEE fp32 fma, round to nearest)
+// and one packed conversion.  s2 holds {s, s}.
+__device__ __forceinline__ uint64_t splat2(float s) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %1};" : "=l"(r) : "f"(s));
+  return r;
+}
+__device__ __forceinline__ uint32_t bf16x2_add_scaled(uint32_t w, uint32_t a, uint32_t b, uint64_t s2) {
+  uint32_t out;
+  asm("{\n\t.reg .b64 x, c, d;\n\t.reg .b32 l, h;\n\t"
+      "mov.b64 x, {%1, %2};\n\t"
+      "shl.b32 l, %3, 16;\n\t"
+      "and.b32 h, %3, 0xFFFF0000;\n\t"
+      "mov.b64 c, {l, h};\n\t"
+      "fma.rn.f32x2 d, x, %4, c;\n\t"
+      "mov.b64 {l, h}, d;\n\t"
+      "cvt.rn.bf16x2.f32 %0, h, l;\n\t}"
+      : "=r"(out)
+      : "r"(a), "r"(b), "r"(w), "l"(s2));
+  return out;
+}
+
 // x = hi + lo for 8 consecutive fp32 values: hi = bf16(x), lo = bf16(x - hi), packed two
 // per 32-bit word (lower half = first element).  (The perturbed-linear route's operands,
 // which meet the bf16 X and W in the same accumulator.)

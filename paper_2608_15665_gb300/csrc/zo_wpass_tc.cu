@@ -279,7 +279,7 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
     // the accumulator holds 2^(kUVScaleExp + e_P) U P, with one e_P for the whole pass:
     // back to U P in the add.  Loaded once -- these warps set the kernel's pace, and a
     // load per tile costs a measured 1.5% of the pass
-    const float wscale = pinv[0] * exp2i(-kUVScaleExp);
+    const uint64_t wscale2 = splat2(pinv[0] * exp2i(-kUVScaleExp));
     for (; ti.valid(); ti.next(), ++it) {
       const TcMat& mt = mats[ti.i];
       const int acc = (int)(it & 1);
@@ -315,14 +315,8 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
           uint4 raw = *p;
           uint32_t wv[4] = {raw.x, raw.y, raw.z, raw.w};
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float lo = fmaf(__uint_as_float(v[j4 * 8 + 2 * e]), wscale,
-                                  __uint_as_float(wv[e] << 16));
-            const float hi = fmaf(__uint_as_float(v[j4 * 8 + 2 * e + 1]), wscale,
-                                  __uint_as_float(wv[e] & 0xFFFF0000u));
-            const __nv_bfloat162 h2 = __floats2bfloat162_rn(lo, hi);
-            wv[e] = *reinterpret_cast<const uint32_t*>(&h2);
-          }
+          for (int e = 0; e < 4; ++e)
+            wv[e] = bf16x2_add_scaled(wv[e], v[j4 * 8 + 2 * e], v[j4 * 8 + 2 * e + 1], wscale2);
           *p = make_uint4(wv[0], wv[1], wv[2], wv[3]);
         }
       }

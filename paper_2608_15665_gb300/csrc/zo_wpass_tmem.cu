@@ -321,7 +321,7 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
     ti.chunk = kTileChunk;
     // the accumulator holds 2^(kUVScaleExp + e_P) U P (one e_P for the pass): back to U P
     // in the add, with the scale loaded once (see zo_wpass_tc.cu)
-    const float wscale = pinv[0] * exp2i(-kUVScaleExp);
+    const uint64_t wscale2 = splat2(pinv[0] * exp2i(-kUVScaleExp));
     for (; ti.valid(); ti.next(), ++it) {
       const TcMat& mt = mats[ti.i];
       const int acc = (int)(it & 1);
@@ -359,14 +359,9 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
           uint4 raw = *p;
           uint32_t wv[4] = {raw.x, raw.y, raw.z, raw.w};
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float lo = fmaf(__uint_as_float(v[j >> 2][(j & 3) * 8 + 2 * e]), wscale,
-                                  __uint_as_float(wv[e] << 16));
-            const float hi = fmaf(__uint_as_float(v[j >> 2][(j & 3) * 8 + 2 * e + 1]), wscale,
-                                  __uint_as_float(wv[e] & 0xFFFF0000u));
-            const __nv_bfloat162 h2 = __floats2bfloat162_rn(lo, hi);
-            wv[e] = *reinterpret_cast<const uint32_t*>(&h2);
-          }
+          for (int e = 0; e < 4; ++e)
+            wv[e] = bf16x2_add_scaled(wv[e], v[j >> 2][(j & 3) * 8 + 2 * e],
+                                      v[j >> 2][(j & 3) * 8 + 2 * e + 1], wscale2);
           *p = make_uint4(wv[0], wv[1], wv[2], wv[3]);
         }
       }

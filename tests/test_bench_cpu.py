@@ -123,3 +123,36 @@ def test_layer_subsets_keep_the_shapes_and_zero_init_of_their_layers():
     assert sub.shapes == lora.shapes[:12]
     assert list(sub.zero_init) == [i for i in lora.zero_init if i < 12] and len(sub.zero_init) > 0
     assert bench.subset(lora, 1000).shapes == lora.shapes    # more layers than there are: all
+
+
+def test_refresh_amortisation_does_not_depend_on_the_window():
+    import bench
+    F, K, step, ref = 25, 20, 36.0, 1.3
+    # a window without a refresh and one with a refresh give the same amortised step
+    w0 = K * step                               # steps 5 .. 24
+    w1 = K * step + ref                         # steps 20 .. 39 (holds t = 25)
+    a0 = bench.amortise_refresh(w0, K, 5, F, ref)
+    a1 = bench.amortise_refresh(w1, K, 20, F, ref)
+    assert a0 == pytest.approx(step + ref / F) and a1 == pytest.approx(a0)
+    # two refreshes in a window of 30 steps at F = 25 (t = 25 and t = 50)
+    assert bench.amortise_refresh(30 * step + 2 * ref, 30, 25, F, ref) == pytest.approx(a0)
+
+
+def test_both_oracle_legs_time_the_same_sample():
+    import bench
+    from paper_2608_15665_gb300 import workloads
+    assert bench.oracle_sample(workloads.get("llama7b_bf16_r32")) == ((0, 1024), (4, 1024))
+    assert bench.oracle_sample(workloads.get("single256_f32_r8")) == ((0, 1024),)
+    res = run_bench(["--impl", "reference", "--steps", "1", "--warmup", "0",
+                     "--workload", "single256_f32_r8"])
+    line = json.loads(res.stdout.strip())
+    assert line["cpu_baseline"]["extrapolated"] is True
+    assert "EXTRAPOLATED" in line["cpu_baseline"]["sample"]
+    ex = line["extrapolation"]
+    assert ex["weights_sampled_of"] == [256 * 256, 256 * 256] and ex["sample_seconds_per_step"] > 0
+
+
+def test_single_thread_oracle_sample_runs_in_its_own_process():
+    import bench
+    one = bench.oracle_single_thread("single256_f32_r8", "central")
+    assert one is not None and one["value"] > 0 and 0 < one["cores"] <= 1.5
