@@ -43,8 +43,8 @@ L2_BYTES = 129e6          # GB300 L2 capacity
 TRAFFIC_BY_SOURCE = {
     # code hash (comments ignored) -> dram read + write bytes of one launch, from ncu
     # --metrics dram__bytes_read.sum,dram__bytes_write.sum on a small case, scaled by weights
-    # profiles/wpass_tc_r32_llama7b_2layers.md: 1.5775 GB on the 2-layer subset, x16.0
-    ("d85d2a44b97e1c78", "llama7b_bf16_r32"): 25.25e9,
+    # profiles/wpass_tc_r32_llama7b_2layers.md: 1.5779 GB on the 2-layer subset, x16.0
+    ("7b7c8c0aed88fc85", "llama7b_bf16_r32"): 25.25e9,
     # profiles/wpass_tmem_r128_llama7b_2layers.md: 1.6377 GB on the 2-layer subset, x16.0
     ("d85d2a44b97e1c78", "llama7b_bf16_r128_q99"): 26.20e9,
     # profiles/wpass_tmem_r64_dense32b_1layer.md: 1.9266 GB on the 1-layer subset, x64.0
@@ -284,6 +284,24 @@ def cpu_baseline(wl, scheme):
                                "threads": "1 BLAS / OpenMP thread"} if one else None)}
 
 
+def max_over_ranks(x, world, device):
+    """The largest x over the ranks (one all_reduce MAX on the process group); x itself on
+    one rank.  The job takes as long as its slowest rank."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_steps_per_second(ms_per_step, world):
+    """Whole-job ZO steps/s of a layer-partitioned run: every rank steps its own partition
+    (weak scaling), so the job completes `world` partitions' steps per ms_per_step."""
+    return world * 1e3 / ms_per_step
+
+
 def amortise_refresh(window_ms, K, t0, F, refresh_ms):
     """ms per step of a window of K steps t0 .. t0 + K - 1 with the refreshes it held (steps
     t with t mod F == 0) replaced by refresh_ms / F per step."""
@@ -393,12 +411,8 @@ def run_ours(args):
             dist.barrier()
         torch.cuda.synchronize()
 
-    def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+    def max_ranks(x):
+        return max_over_ranks(x, world, dev)
 
     for t in range(W):
         do_step(t, table_dev[t])
@@ -418,7 +432,7 @@ def run_ours(args):
     ev1.record()
     barrier()
     clk = clocks.stop()
-    elapsed_ms = max_over_ranks(ev0.elapsed_time(ev1))
+    elapsed_ms = max_ranks(ev0.elapsed_time(ev1))
     wpass_ms, wpass_n = zb.zo_get_timing(z.ctx)
     launches = zb.zo_kernel_launches(z.ctx) - launches0
     zb.zo_set_option(z.ctx, zb.ZO_OPTION_TIMING, 0)
@@ -432,7 +446,7 @@ def run_ours(args):
     z.refresh((W + K) // wl.F)
     r1.record()
     barrier()
-    refresh_ms = max_over_ranks(r0.elapsed_time(r1))
+    refresh_ms = max_ranks(r0.elapsed_time(r1))
     z.sync()
 
     # Both timed windows are reported with the refresh amortised: a window of K steps holds
@@ -461,10 +475,10 @@ def run_ours(args):
             do_step(t, host_losses[k + 1].numpy(), gamma)
             gamma_host.copy_(gamma)            # the step's result back on the host (syncs)
         barrier()
-        e2e_s = max_over_ranks(time.perf_counter() - t0)
+        e2e_s = max_ranks(time.perf_counter() - t0)
         e_clk = e_clocks.stop()
         e2e_ms = amortised_ms(e2e_s * 1e3, W + K + 1)
-        e2e = {"value": world * 1e3 / e2e_ms, "unit": "ZO steps/s",
+        e2e = {"value": job_steps_per_second(e2e_ms, world), "unit": "ZO steps/s",
                "h2d_bytes_per_step": int(table.shape[1] * 4),
                "d2h_bytes_per_step": int(wl.n_mats * 4),
                "ms_per_step": e2e_ms,
@@ -473,7 +487,7 @@ def run_ours(args):
     z.sync()
 
     step_ms = amortised_ms(elapsed_ms, W)
-    value = world * 1e3 / step_ms
+    value = job_steps_per_second(step_ms, world)
     bytes_pass = wl.bytes_per_pass()
     peak, peak_kind = measured_peaks()
     avg_launch_s = (wpass_ms / wpass_n) / 1e3 if wpass_n else float("nan")

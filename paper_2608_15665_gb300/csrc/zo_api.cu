@@ -114,7 +114,7 @@ struct zo_ctx {
   uint16_t* d_p_hl = nullptr;        // stacked [hi | lo] fp16 rows of every P_i^T 2^(e_P,i),
                                      // 128-row padded
   float* d_amax = nullptr;           // max |C_i| of the current pass, one per matrix
-  float* d_pinv = nullptr;           // 2^-e_P of the current pass (one for every matrix)
+  float* d_pinv = nullptr;           // 2^-(e_P,i) of the current pass, one per matrix
   zo::TcMat* d_tc = nullptr;
   std::vector<zo::TcMat> h_tc;       // host copy (operand rows of each matrix)
   // zo_linear_prepare / zo_linear_perturbed: P_K of every matrix ([P_hi ; P_lo] rows,
@@ -466,8 +466,8 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
   ZO_CUDA(cudaMalloc(&c->d_p_hl, sizeof(uint16_t) * prows * HLW), "cudaMalloc(P hi/lo)");
   ZO_CUDA(cudaMemset(c->d_u_op, 0, u_bytes), "memset");
   ZO_CUDA(cudaMemset(c->d_p_hl, 0, sizeof(uint16_t) * prows * HLW), "memset");
-  ZO_CUDA(cudaMalloc(&c->d_pinv, sizeof(float)), "cudaMalloc(P scale)");
-  ZO_CUDA(cudaMemset(c->d_pinv, 0, sizeof(float)), "memset");
+  ZO_CUDA(cudaMalloc(&c->d_pinv, sizeof(float) * c->n_mats), "cudaMalloc(P scales)");
+  ZO_CUDA(cudaMemset(c->d_pinv, 0, sizeof(float) * c->n_mats), "memset");
   ZO_CUDA(cudaMalloc(&c->d_amax, sizeof(float) * c->n_mats), "cudaMalloc(C maxima)");
   ZO_CUDA(cudaMemset(c->d_amax, 0, sizeof(float) * c->n_mats), "memset");
   ZO_CUDA(cudaMalloc(&c->d_tc, sizeof(zo::TcMat) * c->n_mats), "cudaMalloc(tile table)");

@@ -115,7 +115,7 @@ cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2*
 // pair of U, unscaled, laid out as the r <= 32 U operand above.
 cudaError_t launch_split_u_bf16(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                                 int32_t n_units, int32_t r, __nv_bfloat16* u_lin, cudaStream_t s);
-// tm_a is used for r <= 32, u_op for r >= 64; d_pinv[0] = 2^-e_P from launch_split_c.
+// tm_a is used for r <= 32, u_op for r >= 64; d_pinv[i] = 2^-(e_P,i) from launch_split_c.
 cudaError_t launch_wpass_tc(const CUtensorMap& tm_a, const void* u_op, const CUtensorMap& tm_b,
                             const CUtensorMap* d_w_maps, const TcMat* d_tc, const float* d_pinv,
                             int32_t n_mats, int64_t n_tiles, int32_t grid, int32_t r,
@@ -134,9 +134,9 @@ bool project_tc_supported(int32_t r);
 // projection units (matrix, first row)
 cudaError_t launch_split_v(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                            int32_t n_units, int32_t r, uint16_t* v_hl, cudaStream_t s);
-// C_HL rows [hi | lo] of the fp16 pair of C_i 2^e_C (every pass), r rows per matrix at
-// matrix * r, with e_C from max_i amax[i] (the coefficient kernel's per-matrix maxima), and
-// pinv[0] = 2^-e_P, e_P = e_C + p_scale_offset(r)
+// C_HL rows [hi | lo] of the fp16 pair of C_i 2^(e_C,i) (every pass), r rows per matrix at
+// matrix * r, with e_C,i from amax[i] = max |C_i| (the coefficient kernel's), and
+// pinv[i] = 2^-(e_P,i), e_P,i = e_C,i + p_scale_offset(r)
 cudaError_t launch_split_c(const MatDesc* d_mats, int32_t n_mats, int32_t r, const float* amax,
                            uint16_t* c_hl, float* pinv, cudaStream_t s);
 // P_HL = [hi | lo] of the fp16 pair of (V C^T) 2^(e_P,i): tm_v over V_HL (box 64 x 128),

@@ -463,7 +463,7 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
 // P_K of every matrix: rows [P_hi ; P_lo] of the bf16 pair of P_i (P_hi = bf16(P),
 // P_lo = bf16(P - P_hi)), K-major: P_K_i[k][j] and P_K_i[r + k][j] for k < r, j < n_i, at
 // pk_off[i] with row stride ld_i = n_i rounded up to 64.  P comes from the projection's
-// scaled fp16 pair, P = (hi + lo) pinv[0] (exact in fp32 up to the pair's rounding).  One
+// scaled fp16 pair, P = (hi + lo) pinv[i] (exact in fp32 up to the pair's rounding).  One
 // CTA per projection unit (matrix, 128 columns j), through shared memory.
 __global__ void __launch_bounds__(256)
 transpose_p_kernel(const uint16_t* __restrict__ p_hl, const TcMat* __restrict__ tcm,
@@ -477,7 +477,7 @@ transpose_p_kernel(const uint16_t* __restrict__ p_hl, const TcMat* __restrict__ 
   const int64_t ld = (n + 63) / 64 * 64;
   const int64_t j0 = u.y;
   const int r = r2 / 2;
-  const float unscale = pinv[0];
+  const float unscale = pinv[u.x];
   __nv_bfloat16* dst = p_k + pk_off[u.x];
   for (int e = threadIdx.x; e < 128 * 32; e += blockDim.x) {
     const int jj = e / 32, k = e % 32;

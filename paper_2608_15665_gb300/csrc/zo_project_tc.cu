@@ -327,14 +327,14 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
 
 // Rows [hi | lo] of the scaled fp16 pair of V (units = (matrix, first row) x 128 rows, into
 // V_HL at p_row0; scale 2^kUVScaleExp) or of C (one CTA per matrix, r rows into C_HL at
-// matrix * r; scale 2^e_C, one exponent for the pass from the largest of the n_mats maxima
-// amax[], with pinv[0] = 2^-e_P written for the weight pass).  Each thread splits one row;
+// matrix * r; scale 2^(e_C,i) from the coefficient kernel's max |C_i| = amax[i], with
+// pinv[i] = 2^-(e_P,i) written for the weight pass).  Each thread splits one row;
 // the rows are staged in shared memory with the 16-byte chunk index XOR (row & 7) and
 // written with coalesced 16-byte stores.
 template <int R, bool kC>
 __global__ void __launch_bounds__(128)
 split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tcm,
-                  const int2* __restrict__ units, const float* __restrict__ amax_in, int n_mats,
+                  const int2* __restrict__ units, const float* __restrict__ amax_in,
                   uint16_t* __restrict__ dst, float* __restrict__ pinv) {
   constexpr int kVecPerRow = 2 * R * 2 / 16;     // 16-byte chunks of [hi | lo]
   constexpr int kSw = kVecPerRow >= 8 ? 7 : kVecPerRow - 1;   // chunk swizzle within a row
@@ -360,18 +360,9 @@ split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tc
   }
   float scale = exp2i(kUVScaleExp);
   if constexpr (kC) {
-    // e_C from the largest max |C_i| of the pass (the same in every CTA)
-    __shared__ float wmax[4];
-    float amax = 0.f;
-    for (int k = tid; k < n_mats; k += blockDim.x) amax = fmaxf(amax, amax_in[k]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
-    if ((tid & 31) == 0) wmax[tid >> 5] = amax;
-    __syncthreads();
-    amax = fmaxf(fmaxf(wmax[0], wmax[1]), fmaxf(wmax[2], wmax[3]));
-    const int e_c = coeff_scale_exp(amax);
+    const int e_c = coeff_scale_exp(amax_in[i]);
     scale = exp2i(e_c);
-    if (blockIdx.x == 0 && tid == 0) pinv[0] = exp2i(-(e_c + p_scale_offset(R)));
+    if (tid == 0) pinv[i] = exp2i(-(e_c + p_scale_offset(R)));
   }
   if (tid < rows) {
     const float4* s4 = reinterpret_cast<const float4*>(src + (row0 + tid) * R);
@@ -418,8 +409,7 @@ cudaError_t launch_split_rows_r(const MatDesc* d_mats, const TcMat* d_tc, const 
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
-  split_rows_kernel<R, kC><<<n_blocks, 128, smem, s>>>(d_mats, d_tc, d_units, amax, n_blocks, dst,
-                                                      pinv);
+  split_rows_kernel<R, kC><<<n_blocks, 128, smem, s>>>(d_mats, d_tc, d_units, amax, dst, pinv);
   return cudaGetLastError();
 }
 

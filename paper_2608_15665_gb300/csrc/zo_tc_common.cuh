@@ -27,6 +27,9 @@ constexpr int kTileChunk = 4;                    // consecutive tiles per CTA vi
 __host__ __device__ constexpr int hl_width(int r) { return 2 * r > 64 ? 2 * r : 64; }
 
 struct Shared {
+  // scale of the tile in W stage s (written by the W producer before it arms w_full[s],
+  // read by the epilogue after its wait on w_full[s])
+  float w_scale[4];
   uint64_t w_full[4], w_empty[4];
   uint64_t a_full[2], a_empty[2];
   uint64_t b_full[4], b_empty[4];
@@ -115,15 +118,13 @@ __device__ __forceinline__ void give_up(Shared& sh, uint32_t* status) {
 // sum |U| |P|, the grade of an fp32 evaluation, at the MMA count of the bf16 pair.
 // Scales (all exact powers of two, undone in fp32 by the consumer):
 //   U, V:  2^kUVScaleExp  (|U|, |V| <= 1 for column-orthonormal bases)
-//   C_i:   2^e_C with e_C = 14 - E, max_i max |C_i| < 2^E, so |C_i s| < 2^14 -- one exponent
-//          for every matrix of the pass (from the per-matrix maxima the coefficient kernel
-//          writes), so the weight pass undoes a single scale
-//   P_i:   2^e_P, e_P = e_C + p_scale_offset(r): |P_kj| <= ||C_k,:|| ||V_j,:|| <= sqrt(r)
-//          max |C|, so |P_i s| <= 2^15 (fp16 holds up to 65504)
-// The weight pass multiplies its accumulator by pinv 2^-kUVScaleExp, pinv = 2^-e_P.  A pair
-// keeps its ~22 bits while its lo part is a normal fp16 (|x s| >= ~2^-3): for the update of
-// a matrix whose C is up to ~2^12 times smaller than the largest C of the pass; the C of one
-// pass share eps and the scale of their Gaussians (or of the Adam direction).
+//   C_i:   2^(e_C,i) with e_C,i = 14 - E, max |C_i| < 2^E (from the maximum the coefficient
+//          kernel writes), so |C_i s| < 2^14
+//   P_i:   2^(e_P,i), e_P,i = e_C,i + p_scale_offset(r): |P_kj| <= ||C_k,:|| ||V_j,:|| <=
+//          sqrt(r) max |C_i|, so |P_i s| <= 2^15 (fp16 holds up to 65504)
+// The weight pass multiplies its accumulator by pinv_i 2^-kUVScaleExp, pinv_i = 2^-(e_P,i).
+// Each matrix's scale depends on its own C alone, so a set split over several contexts (or
+// ranks) gets the same bits as one context over the whole set.
 constexpr int kUVScaleExp = 14;
 __host__ __device__ constexpr int p_scale_offset(int r) {   // 1 - ceil(log2(r) / 2)
   return r <= 16 ? -1 : r <= 64 ? -2 : -3;

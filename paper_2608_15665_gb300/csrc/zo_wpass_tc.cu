@@ -139,6 +139,9 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
         const int s = (int)(n_w % Cfg::kWStages);
         const uint32_t ph = (uint32_t)((n_w / Cfg::kWStages) & 1);
         if (!mbar_wait_bounded(&sh.w_empty[s], ph ^ 1u, abort, wait_cycles)) { ok = false; break; }
+        // the tile's scale rides with its W stage: the epilogue warps, which set the pace,
+        // then read it from shared memory instead of waiting on a global load
+        sh.w_scale[s] = pinv[ti.i] * exp2i(-kUVScaleExp);
         mbar_arrive_expect_tx(&sh.w_full[s], kWStageBytes);
         uint8_t* dst = w_smem + s * kWStageBytes;
         for (int g = 0; g < 4; ++g)
@@ -276,10 +279,6 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
     TileIter ti;
     ti.init(mats, n_mats, t_begin, t_end, t_stride);
     ti.chunk = kTileChunk;
-    // the accumulator holds 2^(kUVScaleExp + e_P) U P, with one e_P for the whole pass:
-    // back to U P in the add.  Loaded once -- these warps set the kernel's pace, and a
-    // load per tile costs a measured 1.5% of the pass
-    const uint64_t wscale2 = splat2(pinv[0] * exp2i(-kUVScaleExp));
     for (; ti.valid(); ti.next(), ++it) {
       const TcMat& mt = mats[ti.i];
       const int acc = (int)(it & 1);
@@ -302,6 +301,8 @@ wpass_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
         break;
       }
       uint8_t* stage = w_smem + s * kWStageBytes;
+      // the accumulator holds 2^(kUVScaleExp + e_P,i) U P: back to U P in the add
+      const uint64_t wscale2 = splat2(sh.w_scale[s]);
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         uint32_t v[32];

@@ -142,6 +142,8 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
       const int s = (int)(n_w % Cfg::kWStages);
       const uint32_t ph = (uint32_t)((n_w / Cfg::kWStages) & 1);
       if (!mbar_wait_bounded(&sh.w_empty[s], ph ^ 1u, abort, wait_cycles)) { ok = false; break; }
+      // the tile's scale rides with its W stage (see zo_wpass_tc.cu)
+      sh.w_scale[s] = pinv[ti.i] * exp2i(-kUVScaleExp);
       mbar_arrive_expect_tx(&sh.w_full[s], kWStageBytes);
       uint8_t* dst = w_smem + s * kWStageBytes;
       for (int g = 0; g < 4; ++g)
@@ -319,9 +321,6 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
     TileIter ti;
     ti.init(mats, n_mats, t_begin, t_end, t_stride);
     ti.chunk = kTileChunk;
-    // the accumulator holds 2^(kUVScaleExp + e_P) U P (one e_P for the pass): back to U P
-    // in the add, with the scale loaded once (see zo_wpass_tc.cu)
-    const uint64_t wscale2 = splat2(pinv[0] * exp2i(-kUVScaleExp));
     for (; ti.valid(); ti.next(), ++it) {
       const TcMat& mt = mats[ti.i];
       const int acc = (int)(it & 1);
@@ -344,6 +343,8 @@ wpass_tmem_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
         break;
       }
       uint8_t* stage = w_smem + s * kWStageBytes;
+      // the accumulator holds 2^(kUVScaleExp + e_P,i) U P: back to U P in the add
+      const uint64_t wscale2 = splat2(sh.w_scale[s]);
 #pragma unroll
       for (int hh = 0; hh < Cfg::kBoxesPerWarp; ++hh) {
         const int h = h0 + hh;

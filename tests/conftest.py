@@ -10,6 +10,19 @@ if ROOT not in sys.path:
 GOLDEN = os.path.join(ROOT, "tests", "golden")
 
 
+def pytest_terminal_summary(terminalreporter):
+    # how many weight elements passed only because the tolerance is taken at the scale of
+    # the update's operands rather than of the result alone (tests/parity.py)
+    mod = sys.modules.get("parity")
+    if mod is None or not mod.WEIGHT_TOTALS["compared"]:
+        return
+    t = mod.WEIGHT_TOTALS
+    terminalreporter.write_line(
+        f"parity: {t['compared']} weight elements compared with the oracle, {t['differ']} differ, "
+        f"{t['widened_only']} of them within 1 ulp / rel 1e-5 only at the operand scale "
+        f"(max(|W_oracle|, |W_before|, |U||C||V|^T)), not at |W_oracle| alone")
+
+
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (sm_103a) and the built library")
     config.addinivalue_line("markers", "slow: long-running CPU test")

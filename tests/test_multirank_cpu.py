@@ -4,8 +4,10 @@ The weight path shards by matrix with no data exchange: each rank owns a block
 of global matrix indices and regenerates every Z and Omega from the shared seed
 and the global index.  This checks, across two real processes, that the
 partitions are disjoint and cover the set, that a rank's random streams equal
-those a single process computes for the same global indices, and that the
-max-over-ranks reduction used for timing works."""
+those a single process computes for the same global indices, and that bench.py's
+timing reduction -- the max over ranks of the timed region and the whole-job
+throughput world x K / slowest rank -- works over the process group, with a stub
+standing in for the library (each rank reports its own region length)."""
 
 import os
 
@@ -38,8 +40,15 @@ def _worker(rank, world, port, result_path):
     dist.all_gather(oms, om)
     t = torch.tensor([float(rank + 1)], dtype=torch.float64)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    # bench.py's reduction: a stub timed region per rank (the slower rank 1 sets the pace)
+    import bench
+    K, F, refresh_ms = 20, 25, 1.3
+    stub_ms = 700.0 + 50.0 * rank
+    slowest = bench.max_over_ranks(stub_ms, world, "cpu")
+    value = bench.job_steps_per_second(bench.amortise_refresh(slowest, K, 5, F, refresh_ms), world)
     if rank == 0:
-        torch.save({"idx": gathered, "z": zs, "om": oms, "max": float(t.item())}, result_path)
+        torch.save({"idx": gathered, "z": zs, "om": oms, "max": float(t.item()),
+                    "slowest": slowest, "value": value}, result_path)
     dist.barrier()
     dist.destroy_process_group()
 
@@ -63,6 +72,8 @@ def test_partition_over_two_gloo_ranks(tmp_path):
         assert np.array_equal(res["om"][r].numpy(), rng.gen_omega(wl.seed, g0, 0, "U", 8, wl.r))
     assert not np.array_equal(res["z"][0].numpy(), res["z"][1].numpy())
     assert res["max"] == 2.0
+    assert res["slowest"] == 750.0
+    assert res["value"] == pytest.approx(2 * 1e3 / (750.0 / 20 + 1.3 / 25))
 
 
 def test_partition_rejects_bad_rank():
