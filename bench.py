@@ -41,14 +41,12 @@ FALLBACK_HBM_GBS = 6800.0
 # source it was taken on (reported as null once the source differs).
 L2_BYTES = 129e6          # GB300 L2 capacity
 TRAFFIC_BY_SOURCE = {
-    # code hash (comments ignored) -> dram read + write bytes of one launch, from ncu
-    # --metrics dram__bytes_read.sum,dram__bytes_write.sum on a small case, scaled by weights
+    # code hash of the kernel that runs (comments ignored) -> dram read + write bytes of one
+    # launch, from an ncu capture on a small case of the same workload, scaled by weights
     # profiles/wpass_tc_r32_llama7b_2layers.md: 1.5779 GB on the 2-layer subset, x16.0
-    ("7b7c8c0aed88fc85", "llama7b_bf16_r32"): 25.25e9,
-    # profiles/wpass_tmem_r128_llama7b_2layers.md: 1.6377 GB on the 2-layer subset, x16.0
-    ("d85d2a44b97e1c78", "llama7b_bf16_r128_q99"): 26.20e9,
-    # profiles/wpass_tmem_r64_dense32b_1layer.md: 1.9266 GB on the 1-layer subset, x64.0
-    ("d85d2a44b97e1c78", "dense32b_bf16_r64"): 123.30e9,
+    ("a733f29ccdac1cbd", "llama7b_bf16_r32"): 25.25e9,
+    # profiles/wpass_pair_r128_llama7b_2layers.md: 1.6390 GB on the 2-layer subset, x16.0
+    ("541634a914c93b6a", "llama7b_bf16_r128_q99"): 26.22e9,
 }
 # thread instructions per weight of the full-space SPSA kernel (ncu), keyed by source hash
 INSTR_PER_WEIGHT_BY_SOURCE = {
@@ -77,6 +75,9 @@ def parse_args():
                         "for profiling captures); 0 = all")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--single-sm", action="store_true",
+                   help="r = 128: run the single-SM weight-pass kernel instead of the SM-pair one "
+                        "(ZO_OPTION_PAIR_MMA = 0; the two give the same bits)")
     p.add_argument("--no-secondary", action="store_true",
                    help="skip the second measurement on the 32B-shaped set (default workload only)")
     p.add_argument("--oracle-sample", action="store_true",
@@ -110,10 +111,12 @@ def _code_hash(names):
     return h.hexdigest()[:16]
 
 
-def kernel_source_hash():
-    """Code hash of the tensor-core weight-pass kernels and the headers they include."""
-    return _code_hash(("zo_wpass_tc.cu", "zo_wpass_tmem.cu", "zo_tc_common.cuh", "zo_sm100.cuh",
-                       "zo_device.cuh"))
+def kernel_source_hash(r=32):
+    """Code hash of the tensor-core weight-pass kernel that runs at rank r (r <= 32:
+    zo_wpass_tc.cu, r = 64: zo_wpass_tmem.cu, r = 128: zo_wpass_pair.cu) and the headers
+    it includes."""
+    kernel = "zo_wpass_tc.cu" if r <= 32 else "zo_wpass_tmem.cu" if r == 64 else "zo_wpass_pair.cu"
+    return _code_hash((kernel, "zo_tc_common.cuh", "zo_sm100.cuh", "zo_device.cuh"))
 
 
 def subset(wl, layers):
@@ -375,6 +378,8 @@ def run_ours(args):
                for i in range(wl.n_mats)]
     z = SubZeroPlus(weights, wl.r, wl.q, part["seed"],
                     matrix_index_base=part["matrix_index_base"])
+    if args.single_sm:
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_PAIR_MMA, 0)
     calls, (rq, rc) = step_plan(args.scheme, wl.q)
     passes = len(calls) + 1
     K, W = args.steps, args.warmup
@@ -492,7 +497,7 @@ def run_ours(args):
     peak, peak_kind = measured_peaks()
     avg_launch_s = (wpass_ms / wpass_n) / 1e3 if wpass_n else float("nan")
     achieved = bytes_pass / avg_launch_s / 1e9
-    src = kernel_source_hash()
+    src = kernel_source_hash(64 if (wl.r == 128 and args.single_sm) else wl.r)
     l2_resident = bytes_pass / 2 < L2_BYTES
     line = {
         "metric": METRIC, "value": value, "unit": "ZO steps/s", "n_gpus": world, "steps": K,
@@ -517,7 +522,9 @@ def run_ours(args):
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "traffic": TRAFFIC_BY_SOURCE.get((src, wl.name)),
-                     "kernel": {1: "wpass_fma", 2: "wpass_tmem" if wl.r >= 64 else "wpass_tc",
+                     "kernel": {1: "wpass_fma",
+                                2: ("wpass_tmem" if args.single_sm else "wpass_pair") if wl.r == 128
+                                else "wpass_tmem" if wl.r == 64 else "wpass_tc",
                                 3: "wpass_narrow"}.get(path, "?"),
                      "algorithmic_bytes_per_launch": bytes_pass,
                      "avg_launch_ms": avg_launch_s * 1e3, "launches_timed": wpass_n},

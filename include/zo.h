@@ -105,11 +105,15 @@ enum {
                                      bounded wait (~0.1 s) runs out; that pass then reports
                                      ZO_ERR_TIMEOUT via zo_sync_status and leaves W partly
                                      updated.  Nothing faults; the context stays usable. */
-  ZO_OPTION_LINEAR_TILE = 3 /* tiles (rows of X x columns of Y) of zo_linear_perturbed's
+  ZO_OPTION_LINEAR_TILE = 3, /* tiles (rows of X x columns of Y) of zo_linear_perturbed's
                                Y = X W^T + S U^T GEMM: 0 = automatic (the tiling with the
                                least tile work per SM: waves of tiles x a tile's relative
                                time), 1 = 128 x 256, 2 = 256 x 256, 3 = 256 x 224.  All
                                give bit-identical Y. */
+  ZO_OPTION_PAIR_MMA = 4    /* tensor-core weight pass at r = 128: 1 (default) = M = 256 MMAs
+                               across the two SMs of a cluster (each SM holds and reads half
+                               of every P tile), 0 = the single-SM kernel.  Both give
+                               bit-identical weights. */
 };
 
 /* One trainable matrix W_i with its projection bases and Adam moments. */

@@ -37,6 +37,7 @@ ZO_OPTION_WPASS_PATH = 0
 ZO_OPTION_TIMING = 1
 ZO_OPTION_TEST_WAIT_TIMEOUT = 2
 ZO_OPTION_LINEAR_TILE = 3
+ZO_OPTION_PAIR_MMA = 4
 
 
 class ZoError(RuntimeError):

@@ -134,6 +134,14 @@ struct zo_ctx {
   uint32_t* d_s_count = nullptr;   // one counter per 32 rows of S_HL's capacity
   int64_t s_cap = 0, part_cap = 0;
   int64_t tc_tiles = 0;
+  // r = 128: the weight pass on SM pairs (256-row tiles numbered in d_tc_pair), unless
+  // ZO_OPTION_PAIR_MMA = 0 selects the single-SM kernel
+  bool pair_ok = false;
+  int pair_option = 1;
+  zo::TcMat* d_tc_pair = nullptr;
+  int64_t pair_tiles = 0;
+  int32_t n_pairs = 0;
+  CUtensorMap tm_b64{};              // P_HL in 64 x 64 boxes (one SM's half of a P tile)
   CUtensorMap* d_w_maps = nullptr;   // one TMA descriptor per W_i (device memory)
   CUtensorMap tm_a{}, tm_b{};        // descriptors of the stacked operands (kernel parameters)
   int2* d_u_units = nullptr;
@@ -169,6 +177,7 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_u_op);
   cudaFree(c->d_p_hl);
   cudaFree(c->d_tc);
+  cudaFree(c->d_tc_pair);
   cudaFree(c->d_pk);
   cudaFree(c->d_pk_off);
   cudaFree(c->d_s_hl);
@@ -320,9 +329,18 @@ zo_status run_weight_pass(zo_ctx* c) {
     const int grid = (int)std::min<int64_t>(c->tc_tiles, c->sms);
     const bool inject = c->inject_wait;
     c->inject_wait = false;
-    ZO_CUDA(zo::launch_wpass_tc(c->tm_a, c->d_u_op, c->tm_b, c->d_w_maps, c->d_tc, c->d_pinv,
-                                c->n_mats, c->tc_tiles, grid, c->r, c->d_status, inject, c->stream),
-            "tensor-core weight-pass kernel");
+    if (c->pair_ok && c->pair_option == 1) {
+      ZO_CUDA(zo::launch_wpass_pair(static_cast<const uint4*>(c->d_u_op), c->tm_b64, c->d_w_maps,
+                                    c->d_tc_pair, c->d_pinv, c->n_mats, c->pair_tiles,
+                                    (int32_t)std::min<int64_t>(c->pair_tiles, c->n_pairs),
+                                    c->d_status, inject, c->stream),
+              "tensor-core weight-pass kernel (SM pairs)");
+    } else {
+      ZO_CUDA(zo::launch_wpass_tc(c->tm_a, c->d_u_op, c->tm_b, c->d_w_maps, c->d_tc, c->d_pinv,
+                                  c->n_mats, c->tc_tiles, grid, c->r, c->d_status, inject,
+                                  c->stream),
+              "tensor-core weight-pass kernel");
+    }
     c->last_path = 2;
   } else {
     ZO_CUDA(zo::launch_wpass_fma(c->d_mats, c->n_mats, c->d_tile_prefix, c->n_tiles, c->r,
@@ -439,9 +457,13 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
   };
   const int64_t BM = zo::tc_tile_rows(), BN = zo::tc_tile_cols();
   const int64_t HLW = zo::tc_hl_width(c->r);
-  std::vector<zo::TcMat> tc(c->n_mats);
+  // at r = 128 the U operand is padded to the SM pair's 256-row tiles (the second 128-row
+  // block of a ragged pair tile reads zeros), which the single-SM kernel reads as well
+  const bool pair = zo::wpass_pair_supported(c->r);
+  const int64_t UPAD = pair ? zo::pair_tile_rows() : BM;
+  std::vector<zo::TcMat> tc(c->n_mats), tcp;
   std::vector<int2> uunits;
-  int64_t urows = 0, prows = 0, tiles = 0;
+  int64_t urows = 0, prows = 0, tiles = 0, ptiles = 0;
   for (int32_t i = 0; i < c->n_mats; ++i) {
     const int64_t m = mats[i].m, n = mats[i].n;
     tc[i].m = m;
@@ -452,7 +474,13 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
     tc[i].p_row0 = (int32_t)prows;
     tc[i].pad = 0;
     tiles += ((m + BM - 1) / BM) * tc[i].tiles_n;
-    urows += (m + BM - 1) / BM * BM;
+    if (pair) {
+      zo::TcMat tp = tc[i];
+      tp.tile0 = ptiles;
+      ptiles += ((m + UPAD - 1) / UPAD) * tp.tiles_n;
+      tcp.push_back(tp);
+    }
+    urows += (m + UPAD - 1) / UPAD * UPAD;
     prows += (n + BN - 1) / BN * BN;
     for (int64_t r0 = 0; r0 < m; r0 += 128) uunits.push_back(make_int2(i, (int)r0));
   }
@@ -473,6 +501,12 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
   ZO_CUDA(cudaMalloc(&c->d_tc, sizeof(zo::TcMat) * c->n_mats), "cudaMalloc(tile table)");
   ZO_CUDA(cudaMemcpy(c->d_tc, tc.data(), sizeof(zo::TcMat) * c->n_mats, cudaMemcpyHostToDevice),
           "upload tile table");
+  if (pair) {
+    ZO_CUDA(cudaMalloc(&c->d_tc_pair, sizeof(zo::TcMat) * c->n_mats), "cudaMalloc(pair tile table)");
+    ZO_CUDA(cudaMemcpy(c->d_tc_pair, tcp.data(), sizeof(zo::TcMat) * c->n_mats,
+                       cudaMemcpyHostToDevice),
+            "upload pair tile table");
+  }
   ZO_CUDA(cudaMalloc(&c->d_u_units, sizeof(int2) * uunits.size()), "cudaMalloc(units)");
   ZO_CUDA(cudaMemcpy(c->d_u_units, uunits.data(), sizeof(int2) * uunits.size(),
                      cudaMemcpyHostToDevice),
@@ -500,6 +534,14 @@ zo_status setup_tc(zo_ctx* c, const zo_matrix* mats) {
           "upload tensor maps");
   c->tc_tiles = tiles;
   c->tc_ok = true;
+  if (pair) {
+    // every pair is persistent over its share of the tiles: launch only as many pairs as
+    // fit on the device at once
+    c->n_pairs = zo::wpass_pair_max_pairs();
+    c->pair_tiles = ptiles;
+    c->pair_ok = c->n_pairs > 0 && encode_f16_2d(&c->tm_b64, c->d_p_hl, HLW, prows, HLW * 2, 64, 64);
+    if (!c->pair_ok) return refuse("the SM-pair weight pass could not be set up");
+  }
   // the projection P = C V^T on the tensor cores (every tensor-core rank): V_HL, C_HL
   const int64_t crows = (int64_t)c->n_mats * c->r;
   ZO_CUDA(cudaMalloc(&c->d_v_hl, sizeof(uint16_t) * prows * HLW), "cudaMalloc(V hi/lo)");
@@ -1156,6 +1198,15 @@ zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
   if (option == ZO_OPTION_LINEAR_TILE) {
     if (value < 0 || value > 3) return ZO_ERR_INVALID_ARG;
     c->linear_tile = (int)value;
+    return ZO_OK;
+  }
+  if (option == ZO_OPTION_PAIR_MMA) {
+    if (value != 0 && value != 1) return ZO_ERR_INVALID_ARG;
+    if (value == 1 && !c->pair_ok) {
+      g_last_error = "the SM-pair weight pass needs the tensor-core path at r = 128";
+      return ZO_ERR_UNSUPPORTED;
+    }
+    c->pair_option = (int)value;
     return ZO_OK;
   }
   if (option == ZO_OPTION_TIMING) {

@@ -128,6 +128,17 @@ cudaError_t launch_wpass_tmem(const uint4* u_t, const CUtensorMap& tm_b,
                               int32_t n_mats, int64_t n_tiles, int32_t grid, int32_t r,
                               uint32_t* d_status, bool inject_wait, cudaStream_t s);
 
+// r = 128 on SM pairs (zo_wpass_pair.cu): tiles of 256 rows (pair_tile_rows()) numbered in
+// d_tc's tile0 / tiles_n, the U operand padded to 256-row blocks per matrix, tm_b64 over
+// P_HL with 64 x 64 boxes; 2 n_pairs CTAs in clusters of two.
+bool wpass_pair_supported(int32_t r);
+int32_t pair_tile_rows();
+int32_t wpass_pair_max_pairs();   // co-resident clusters of the kernel (0 if unknown)
+cudaError_t launch_wpass_pair(const uint4* u_t, const CUtensorMap& tm_b64,
+                              const CUtensorMap* d_w_maps, const TcMat* d_tc, const float* d_pinv,
+                              int32_t n_mats, int64_t n_pair_tiles, int32_t n_pairs,
+                              uint32_t* d_status, bool inject_wait, cudaStream_t s);
+
 // ---- projection P = C V^T on the tensor cores, r >= 16 (zo_project_tc.cu) ---------
 bool project_tc_supported(int32_t r);
 // V_HL rows [hi | lo] of the fp16 pair of V 2^kUVScaleExp (after a refresh); units = the

@@ -268,6 +268,35 @@ def test_tensor_core_rings_wrap(lib, gpu, r):
     z.close()
 
 
+@pytest.mark.parametrize("shapes", [
+    [(300, 520, None), (130, 1000, 1008), (1030, 136, None)],
+    # a pair tile's second 128 rows empty (m = 128), exactly full (m = 256), one row into the
+    # second pair tile (m = 257), and 200 rows of a single column block
+    [(128, 256, None), (256, 384, None), (257, 136, 144), (200, 128, None)],
+], ids=["ragged", "edges"])
+def test_sm_pair_and_single_sm_passes_are_bit_identical(lib, gpu, shapes):
+    # r = 128: the weight pass as M = 256 MMAs across an SM pair (the default) and as the
+    # single-SM kernel sum the same products in the same order: a pass and a step give the
+    # same bits (both are also checked against the oracle above)
+    from paper_2608_15665_gb300 import binding as zb
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    out = {}
+    for option in (1, 0):
+        weights = [make_weight(m, n, "bf16", 700 + k, gpu, ldw) for k, (m, n, ldw) in enumerate(shapes)]
+        z = SubZeroPlus(weights, 128, 4, 5151, matrix_index_base=3)
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_PAIR_MMA, option)
+        z.init_subspace(0)
+        z.perturb(0, 0, 1.0, 1, -1.0, 1e-1)
+        z.step(0, 1, np.array([2.01, 1.99, 2.0, 2.02, 1.98, 2.0, 2.03, 2.01], np.float32),
+               "central", 1e-1, 1e-2, 0.9, 0.95, 1e-8, 3, 1.0)
+        z.sync()
+        assert zb.zo_wpass_path(z.ctx) == 2
+        out[option] = [W.clone() for W in z.weights]
+        z.close()
+    for i, (a, b) in enumerate(zip(out[1], out[0])):
+        assert torch.equal(a, b), f"matrix {i}: SM-pair and single-SM weight passes differ"
+
+
 @pytest.mark.parametrize("case", list(TC_CASES))
 def test_tensor_core_and_fma_paths_agree(lib, gpu, case):
     # one pass from the same state on both paths: each is within 1 ulp (at the operand
