@@ -47,6 +47,8 @@ TRAFFIC_BY_SOURCE = {
     ("a733f29ccdac1cbd", "llama7b_bf16_r32"): 25.25e9,
     # profiles/wpass_pair_r128_llama7b_2layers.md: 1.6390 GB on the 2-layer subset, x16.0
     ("541634a914c93b6a", "llama7b_bf16_r128_q99"): 26.22e9,
+    # profiles/wpass_tmem_r64_dense32b_1layer.md: 1.9271 GB on the 1-layer subset, x64.0
+    ("5d6c6cd8669a0a74", "dense32b_bf16_r64"): 123.33e9,
 }
 # thread instructions per weight of the full-space SPSA kernel (ncu), keyed by source hash
 INSTR_PER_WEIGHT_BY_SOURCE = {
