@@ -634,6 +634,7 @@ def secondary_32b(dev, local, peak):
             "avg_launch_ms": avg_s * 1e3, "launches_timed": wpass_n,
             "algorithmic_bytes_per_launch": wl.bytes_per_pass(),
             "achieved_gbs": achieved, "peak_gbs": peak, "frac": achieved / peak,
+            "traffic": TRAFFIC_BY_SOURCE.get((kernel_source_hash(wl.r), wl.name)),
             "zo_steps_s": 1e3 / step_ms, "ms_per_step": step_ms, "refresh_ms": refresh_ms,
             "clocks": clk}
 
