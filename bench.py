@@ -118,7 +118,10 @@ def kernel_source_hash(r=32):
     zo_wpass_tc.cu, r = 64: zo_wpass_tmem.cu, r = 128: zo_wpass_pair.cu) and the headers
     it includes."""
     kernel = "zo_wpass_tc.cu" if r <= 32 else "zo_wpass_tmem.cu" if r == 64 else "zo_wpass_pair.cu"
-    return _code_hash((kernel, "zo_tc_common.cuh", "zo_sm100.cuh", "zo_device.cuh"))
+    headers = ("zo_tc_common.cuh", "zo_sm100.cuh", "zo_device.cuh")
+    if r == 128:
+        headers += ("zo_cluster.cuh",)
+    return _code_hash((kernel,) + headers)
 
 
 def subset(wl, layers):
@@ -701,14 +704,17 @@ def run_linear(args):
     clk = clocks.stop()
     launches = zb.zo_kernel_launches(z.ctx) - launches0
     z.sync()
-    names = {1: "128x256", 2: "256x256", 3: "256x224"}
+    names = {1: "128x256", 2: "256x256", 3: "256x224", 4: "256x256 pair", 5: "256x240 pair",
+             6: "256x224 pair", 7: "256x192 pair", 8: "256x128 pair"}
     tiling = []
     for i, (m, n) in enumerate(wl.shapes):
         zb.zo_linear_perturbed(z.ctx, i, X[n], Y[i])
         tiling.append(names[zb.zo_linear_tiling(z.ctx)])
-    # for context: the same route with 128-row tiles throughout
+    # for context: the same route with the single-CTA 128 x 256 and 256 x 224 tiles throughout
     zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 1)
     fused128_ms = timed(fused, K)
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 3)
+    fused224_ms = timed(fused, K)
     zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 0)
     z.sync()
     plain_ms = timed(lambda k: plain(), K)
@@ -753,8 +759,10 @@ def run_linear(args):
                    "parallelism": "single GPU"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "peak_kind": peak_kind, "traffic": None,
-                     "kernel": "linear_kernel", "algorithmic_flops_per_step": flops},
+                     "kernel": "linear_pair_kernel" if any("pair" in t for t in tiling)
+                     else "linear_kernel", "algorithmic_flops_per_step": flops},
         "tile128_ms": fused128_ms,
+        "tile224_single_cta_ms": fused224_ms,
         "plain_gemm_ms": plain_ms,
         "weight_pass_route_ms": wpass_ms,
         "e2e": {"value": flops / e2e_s / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": int(h2d),

@@ -106,10 +106,12 @@ enum {
                                      ZO_ERR_TIMEOUT via zo_sync_status and leaves W partly
                                      updated.  Nothing faults; the context stays usable. */
   ZO_OPTION_LINEAR_TILE = 3, /* tiles (rows of X x columns of Y) of zo_linear_perturbed's
-                               Y = X W^T + S U^T GEMM: 0 = automatic (the tiling with the
-                               least tile work per SM: waves of tiles x a tile's relative
-                               time), 1 = 128 x 256, 2 = 256 x 256, 3 = 256 x 224.  All
-                               give bit-identical Y. */
+                               Y = X W^T + S U^T GEMM: 0 = automatic (the SM-pair tiling
+                               with the fewest waves x a tile's time; the single-CTA ones
+                               if no 2-CTA cluster fits), 1 = 128 x 256, 2 = 256 x 256,
+                               3 = 256 x 224 on single CTAs, 4 .. 8 = 256 x 256, 240, 224,
+                               192, 128 on SM pairs (M = 256 MMAs across a 2-CTA cluster).
+                               All give bit-identical Y. */
   ZO_OPTION_PAIR_MMA = 4    /* tensor-core weight pass at r = 128: 1 (default) = M = 256 MMAs
                                across the two SMs of a cluster (each SM holds and reads half
                                of every P tile), 0 = the single-SM kernel.  Both give
@@ -264,8 +266,8 @@ ZO_API zo_status zo_get_timing(zo_ctx* ctx, double* total_ms, int64_t* launches)
    (1 = FMA on 32-row tiles, 2 = tcgen05, 3 = FMA on narrow tiles). */
 ZO_API int32_t zo_wpass_path(const zo_ctx* ctx);
 
-/* zo_linear_tiling -- the tiling (1, 2 or 3, as ZO_OPTION_LINEAR_TILE) of the Y GEMM
- * that the last zo_linear_perturbed launched; 0 before the first call or for a null ctx. */
+/* zo_linear_tiling -- the tiling (1 .. 8, as ZO_OPTION_LINEAR_TILE) of the Y GEMM that
+ * the last zo_linear_perturbed launched; 0 before the first call or for a null ctx. */
 ZO_API int32_t zo_linear_tiling(const zo_ctx* ctx);
 
 /* zo_kernel_launches -- number of kernels this context has launched since zo_create. */

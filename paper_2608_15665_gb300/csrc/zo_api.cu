@@ -128,7 +128,8 @@ struct zo_ctx {
   bool u_lin_valid = false;          // d_u_lin holds the current U (cleared by every refresh)
   int64_t u_rows = 0;                // rows of the stacked U operand
   int linear_tile = 0;           // ZO_OPTION_LINEAR_TILE
-  int last_linear_tiling = 0;    // tiling of the last Y GEMM (1..3)
+  int last_linear_tiling = 0;    // tiling of the last Y GEMM (1..3, or a pair tiling)
+  int linear_pairs = -1;         // co-resident clusters of the pair Y GEMM (-1: not asked)
   __nv_bfloat16* d_s_hl = nullptr;
   float* d_s_part = nullptr;
   uint32_t* d_s_count = nullptr;   // one counter per 32 rows of S_HL's capacity
@@ -1095,16 +1096,36 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
       c->part_cap = part;
     }
   }
-  const int32_t tiling = zo::linear_y_tiling(T, m, c->sms, c->linear_tile);
-  const bool narrow_y = zo::linear_y_tile_cols(tiling) % 64 != 0;   // 32-column Y boxes
-  CUtensorMap tm_x{}, tm_pk{}, tm_s{}, tm_y{};
-  const bool enc =
+  // the Y GEMM's tiling: automatic = the pair tiling with the fewest waves (the single-CTA
+  // tilings if no cluster of the pair kernel fits), or the one ZO_OPTION_LINEAR_TILE names
+  if (c->linear_pairs < 0) c->linear_pairs = std::max(0, (int)zo::linear_pair_max_pairs());
+  int32_t tiling = c->linear_tile;
+  if (tiling == 0)
+    tiling = c->linear_pairs > 0 ? zo::linear_pair_tiling(T, m, c->linear_pairs)
+                                 : zo::linear_y_tiling(T, m, c->sms, 0);
+  const int32_t pair_n = zo::linear_pair_cols(tiling);
+  if (pair_n > 0 && c->linear_pairs <= 0) {
+    g_last_error = "zo_linear_perturbed: no cluster of the SM-pair GEMM fits on this device";
+    return ZO_ERR_UNSUPPORTED;
+  }
+  const bool narrow_y = pair_n == 0 && zo::linear_y_tile_cols(tiling) % 64 != 0;
+  CUtensorMap tm_x{}, tm_pk{}, tm_s{}, tm_y{}, tm_w{}, tm_u{};
+  bool enc =
       encode_bf16_2d(&tm_x, const_cast<void*>(X), n, T, ldx * 2, 64, 128) &&
       encode_bf16_2d(&tm_pk, c->d_pk + c->h_pk_off[mat], n, 2 * r, (n + 63) / 64 * 64 * 2, 64,
                      (uint32_t)(2 * r)) &&
-      encode_bf16_2d(&tm_s, c->d_s_hl, HLW, T, HLW * 2, 64, 128) &&
-      (narrow_y ? encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)
-                : encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 64, 32));
+      encode_bf16_2d(&tm_s, c->d_s_hl, HLW, T, HLW * 2, 64, 128);
+  if (pair_n > 0) {
+    // W_i and the U operand in boxes of N/2 rows (each CTA of a pair loads half of the
+    // tile's B rows), Y in 32 x 16 boxes
+    enc = enc && encode_bf16_2d(&tm_w, md.W, n, m, md.ldw * 2, 64, (uint32_t)(pair_n / 2)) &&
+          encode_bf16_2d(&tm_u, c->d_u_lin, HLW, c->u_rows, HLW * 2, 64, (uint32_t)(pair_n / 2)) &&
+          encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 16, 32, CU_TENSOR_MAP_SWIZZLE_32B);
+  } else {
+    enc = enc && (narrow_y ? encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 32, 32,
+                                            CU_TENSOR_MAP_SWIZZLE_64B)
+                           : encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 64, 32));
+  }
   if (!enc) {
     g_last_error = "zo_linear_perturbed: cuTensorMapEncodeTiled rejected a descriptor";
     return ZO_ERR_CUDA;
@@ -1113,9 +1134,15 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
   ZO_CUDA(zo::launch_linear_s(tm_x, tm_pk, T, n, r, k_split, k_chunk, c->d_s_part, c->d_s_hl,
                               c->d_s_count, c->sms, c->d_status, c->stream),
           "S = X P^T kernels");
-  ZO_CUDA(zo::launch_linear_y(tm_x, c->d_w_maps + mat, tm_s, c->tm_u_lin, tm_y, T, m, n,
-                              c->h_tc[mat].u_row0, r, tiling, c->sms, c->d_status, c->stream),
-          "perturbed linear kernel");
+  if (pair_n > 0) {
+    ZO_CUDA(zo::launch_linear_pair(tm_x, tm_w, tm_s, tm_u, tm_y, T, m, n, c->h_tc[mat].u_row0, r,
+                                   tiling, c->linear_pairs, c->d_status, c->stream),
+            "perturbed linear kernel (SM pairs)");
+  } else {
+    ZO_CUDA(zo::launch_linear_y(tm_x, c->d_w_maps + mat, tm_s, c->tm_u_lin, tm_y, T, m, n,
+                                c->h_tc[mat].u_row0, r, tiling, c->sms, c->d_status, c->stream),
+            "perturbed linear kernel");
+  }
   c->last_linear_tiling = tiling;
   c->launches += 1 + zo::linear_s_launches(k_split);
   return ZO_OK;
@@ -1196,7 +1223,7 @@ zo_status zo_set_option(zo_ctx* c, int32_t option, int64_t value) {
     return ZO_OK;
   }
   if (option == ZO_OPTION_LINEAR_TILE) {
-    if (value < 0 || value > 3) return ZO_ERR_INVALID_ARG;
+    if (value < 0 || value >= zo::kLinearPairTiling0 + 5) return ZO_ERR_INVALID_ARG;
     c->linear_tile = (int)value;
     return ZO_OK;
   }

@@ -195,6 +195,23 @@ cudaError_t launch_linear_y(const CUtensorMap& tm_x, const CUtensorMap* d_w_map,
                             int32_t u_row0, int32_t r, int32_t tiling, int32_t sms,
                             uint32_t* d_status, cudaStream_t s);
 
+// The Y GEMM on SM pairs (zo_linear_pair.cu): 256 x N tiles (rows of X x columns of Y),
+// M = 256 MMAs across a 2-CTA cluster, two accumulators per SM.  Tilings
+// kLinearPairTiling0 + 0 .. 4 are N = 256, 240, 224, 192, 128.
+constexpr int32_t kLinearPairTiling0 = 4;
+int32_t linear_pair_cols(int32_t tiling);        // N of a pair tiling, 0 for the others
+int32_t linear_pair_max_pairs();                 // co-resident clusters (0 if unknown)
+// The pair tiling with the least tile work per pair (waves of tiles x a tile's time).
+int32_t linear_pair_tiling(int64_t T, int64_t m, int32_t n_pairs);
+// tm_x over X (box 64 x 128), tm_w over W_i (box 64 x N/2), tm_s over S_HL (box 64 x 128),
+// tm_u over the bf16 U operand (box 64 x N/2; W_i's rows from u_row0), tm_y over Y (box
+// 16 x 32, 32-byte swizzle).
+cudaError_t launch_linear_pair(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
+                               const CUtensorMap& tm_s, const CUtensorMap& tm_u,
+                               const CUtensorMap& tm_y, int64_t T, int64_t m, int64_t n,
+                               int32_t u_row0, int32_t r, int32_t tiling, int32_t n_pairs,
+                               uint32_t* d_status, cudaStream_t s);
+
 // ---- refresh of tall panels at r = 16 ... 128: CholeskyQR2 (zo_cholqr.cu) ----------
 constexpr int32_t kCqChunkRows = 1024;   // rows per partial Gram matrix
 struct CqPanel {

@@ -1,0 +1,459 @@
+// The Y GEMM of the perturbed linear layer (Y = X W_i^T + S U_i^T, the forward of Alg. 3
+// at W' = W + eps U Z V^T, Eq. (4) form, with W left as it is) on SM pairs: M = 256
+// tcgen05.mma.cta_group::2 across the two SMs of a cluster.
+//
+// Pair tile = 256 rows of X (tokens) x N columns of Y (rows of W_i); CTA c of the cluster
+// holds rows 128 c .. 128 c + 127 of the tile (its half of the A operand, its accumulator
+// lanes) and rows N/2 c .. N/2 c + N/2 - 1 of the B operand (W rows, then U operand rows);
+// the leader's MMAs read both halves of B.  Each SM then stages 128 x 64 + N/2 x 64 bf16
+// per K step for 128 x N x 64 multiply-adds, and holds a 128 x N fp32 accumulator -- two
+// of them fit its Tensor Memory (N <= 256), so a tile's epilogue runs while the MMAs of
+// the pair's next tile accumulate into the other one.
+//
+// K steps: n / 64 steps of X and W (single bf16 products, both operands exact in bf16),
+// then one step of the rank-r term from S_HL = [S_hi | S_lo | 0] (A) and the U operand
+// [U_hi | U_lo | 0] (B) with the three products S_hi U_hi + S_hi U_lo + S_lo U_hi -- the
+// same MMAs, in the same order, as the single-CTA kernels of zo_linear.cu, so each 128-row
+// half of a pair tile gets the bits those kernels give.
+// N (a multiple of 16, 128 .. 256) is chosen by the host so that the tiles fill whole
+// waves of the resident pairs (224 for 4096 columns at 4096 tokens: 19 x 16 = 304 tiles =
+// 4 waves of 76 pairs; 240 for 11008 columns).
+//
+// Roles (320 threads per CTA, one CTA per SM):
+//   warp 0, lane 0: TMA producer of this CTA's halves, kStages stages; both halves of a
+//                   stage complete their bytes on the leader's full barrier (the TMA's
+//                   .cta_group::2 form), which the leader's producer arms for both.
+//   warp 1:         Tensor Memory (.cta_group::2, in both CTAs); in the leader lane 0
+//                   issues every MMA of the pair into one of two accumulators.
+//   warps 2..9:     epilogue of this CTA's 128 rows: warp w reads TMEM lanes 32 (w % 4) ..
+//                   + 31, every other 16-column chunk, rounds to bf16 and stores 32 x 16
+//                   boxes of Y (32-byte swizzle) by TMA.
+// Barriers: in each CTA empty[s] and acc_full[a] (arrived in both CTAs by the leader's
+// multicast commits); in the leader full[s] (bytes of both halves) and acc_empty[a] (the
+// sixteen epilogue warps of the pair, the peer's through its shared::cluster address).
+// Every wait is bounded; a give-up sets the abort flag of both CTAs and kDevTimeout in
+// the status word, the producers wait (bounded) for the leader's release of every stage
+// they filled, the MMA thread for its last MMAs, and TMEM is freed after a cluster barrier.
+#include <algorithm>
+
+#include <cuda.h>
+
+#include "zo_cluster.cuh"
+#include "zo_kernels.h"
+#include "zo_sm100.cuh"
+#include "zo_tc_common.cuh"
+
+namespace zo {
+namespace {
+
+using namespace sm100;
+using namespace tc;
+using namespace cta2;
+
+constexpr int kPairRows = 2 * kBM;   // 256 rows of X per pair tile
+
+template <int N>
+struct PairLin {
+  static_assert(N % 16 == 0 && N >= 128 && N <= 256, "pair tile columns");
+  static constexpr int kHalfN = N / 2;                        // B rows per CTA (multiple of 8)
+  static constexpr int kPanels = 2;                           // 64-element K panels per stage
+  static constexpr int kAPanel = kBM * 128;                   // 128 rows x 64 bf16
+  static constexpr int kBPanel = kHalfN * 128;                // N/2 rows x 64 bf16
+  static constexpr int kABytes = kPanels * kAPanel;
+  static constexpr int kStageBytes = kPanels * (kAPanel + kBPanel);   // a multiple of 1024
+  static constexpr int kEpiWarps = 8;
+  static constexpr int kBoxBytes = 32 * 16 * 2;               // 32 rows x 16 bf16 of Y
+  static constexpr int kOutBytes = kEpiWarps * kBoxBytes;
+  static constexpr int kStagesFit = (227 * 1024 - kOutBytes - 2048) / kStageBytes;
+  static constexpr int kStages = kStagesFit < 8 ? kStagesFit : 8;
+  static constexpr int kThreads = 64 + 32 * kEpiWarps;
+  static constexpr int kAccStride = 256;                      // TMEM columns between the two
+  static constexpr int kTmemCols = 512;
+  static constexpr int kChunks = N / 16;                      // 16-column chunks of a row
+  static constexpr size_t kSmem = (size_t)kStages * kStageBytes + kOutBytes + 1024 + 1024;
+  static_assert(kStages >= 3, "operand ring");
+  static_assert(kSmem <= 227 * 1024, "shared memory per CTA");
+  static_assert(kAccStride + N <= kTmemCols, "two accumulators in TMEM");
+};
+
+struct LinPairShared {
+  uint64_t full[8], empty[8];
+  uint64_t acc_full[2], acc_empty[2];
+  uint64_t drain;          // one commit after the leader's last MMA
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+__device__ __forceinline__ void lp_give_up(LinPairShared& sh, uint32_t* status) {
+  atomicOr(status, (uint32_t)kDevTimeout);
+  *reinterpret_cast<volatile int*>(&sh.abort_flag) = 1;
+  store_peer(&sh.abort_flag, 1);
+}
+
+// 32 lanes x 16 consecutive 32-bit columns: thread t gets lane (base lane + t)
+__device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&v)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+        "=r"(v[14]), "=r"(v[15])
+      : "r"(taddr));
+}
+
+// Pair tile t -> (row block tb, column block nb): column stripes of `group` column blocks,
+// each walked row block by row block (group = the column blocks: plain row-major order).
+// Stripes about one wave of tiles wide keep the wave's W rows few enough to stay in L2
+// while every row block of X passes them.
+struct StripeOrder {
+  int tiles_n, row_blocks, group;
+  __device__ void decode(int64_t t, int& tb, int& nb) const {
+    const int64_t per = (int64_t)row_blocks * group;
+    const int full = tiles_n / group;
+    if (t < (int64_t)full * per) {
+      const int stripe = (int)(t / per), rem = (int)(t % per);
+      tb = rem / group;
+      nb = stripe * group + rem % group;
+    } else {
+      const int rem = (int)(t - (int64_t)full * per);
+      const int last = tiles_n - full * group;
+      tb = rem / last;
+      nb = full * group + rem % last;
+    }
+  }
+};
+
+// tm_x: X (box 64 x 128), tm_w: W_i (box 64 x N/2), tm_s: S_HL (box 64 x 128), tm_u: the
+// route's U operand (box 64 x N/2; this matrix's rows from u_row0), tm_y: Y (box 16 x 32,
+// 32-byte swizzle).  rows = T, cols = m, k_steps = ceil(n / 64).
+template <int N, int R>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairLin<N>::kThreads, 1)
+linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
+                   const __grid_constant__ CUtensorMap tm_s, const __grid_constant__ CUtensorMap tm_u,
+                   const __grid_constant__ CUtensorMap tm_y, int rows, int cols, int k_steps,
+                   int u_row0, int group, uint32_t* __restrict__ status, long long wait_cycles) {
+  using Cfg = PairLin<N>;
+  constexpr int S = Cfg::kStages;
+  static_assert(sizeof(LinPairShared) <= 1024, "barrier block");
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* st_smem = smem;                                    // stages: [A half | B half]
+  uint8_t* o_smem = st_smem + S * Cfg::kStageBytes;           // one Y box per epilogue warp
+  LinPairShared& sh = *reinterpret_cast<LinPairShared*>(o_smem + Cfg::kOutBytes);
+
+  const uint32_t rank = cluster_rank();
+  const bool leader = rank == 0;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+  const int tiles_n = (cols + N - 1) / N;
+  const int row_blocks = (rows + kPairRows - 1) / kPairRows;
+  const int64_t n_tiles = (int64_t)row_blocks * tiles_n;
+  const StripeOrder order{tiles_n, row_blocks, group < 1 || group > tiles_n ? tiles_n : group};
+  const volatile int* abort = &sh.abort_flag;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&sh.full[s], 1);              // the leader's producer (bytes of both halves)
+      mbar_init(&sh.empty[s], 1);             // the leader's commit
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&sh.acc_full[a], 1);
+      mbar_init(&sh.acc_empty[a], 2 * Cfg::kEpiWarps);
+    }
+    mbar_init(&sh.drain, 1);
+    sh.abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tm_x);
+    prefetch_tmap(&tm_w);
+    prefetch_tmap(&tm_s);
+    prefetch_tmap(&tm_u);
+    prefetch_tmap(&tm_y);
+  }
+  if (warp == 1) tmem_alloc_pair(&sh.tmem_base, Cfg::kTmemCols);
+  tc_fence_before();
+  cluster_sync_all();                         // both CTAs' barriers and TMEM exist
+  tc_fence_after();
+  const uint32_t tmem = sh.tmem_base;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------ TMA producer (each CTA)
+    int s = 0;
+    uint32_t ph = 0;
+    int64_t n_st = 0;
+    bool ok = true;
+    const int k_stages = (k_steps + Cfg::kPanels - 1) / Cfg::kPanels;
+    for (int64_t tile = pair; tile < n_tiles && ok; tile += n_pairs) {
+      int tb, nb;
+      order.decode(tile, tb, nb);
+      const int y_a = tb * kPairRows + kBM * (int)rank;
+      const int y_b = nb * N + Cfg::kHalfN * (int)rank;
+      for (int k = 0; k <= k_stages; ++k) {
+        if (!mbar_wait_bounded(&sh.empty[s], ph ^ 1u, abort, wait_cycles)) {
+          ok = false;
+          break;
+        }
+        uint8_t* a_dst = st_smem + s * Cfg::kStageBytes;
+        uint8_t* b_dst = a_dst + Cfg::kABytes;
+        if (k < k_stages) {
+          // panels past n read TMA's zero fill
+          if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * Cfg::kStageBytes);
+#pragma unroll
+          for (int p = 0; p < Cfg::kPanels; ++p) {
+            const int x = 64 * (Cfg::kPanels * k + p);
+            tma_load_2d_to_leader(a_dst + p * Cfg::kAPanel, &tm_x, x, y_a, &sh.full[s]);
+            tma_load_2d_to_leader(b_dst + p * Cfg::kBPanel, &tm_w, x, y_b, &sh.full[s]);
+          }
+        } else {                               // the rank-r step: S_HL rows, U operand rows
+          if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * (Cfg::kAPanel + Cfg::kBPanel));
+          tma_load_2d_to_leader(a_dst, &tm_s, 0, y_a, &sh.full[s]);
+          tma_load_2d_to_leader(b_dst, &tm_u, 0, u_row0 + y_b, &sh.full[s]);
+        }
+        ++n_st;
+        if (++s == S) { s = 0; ph ^= 1u; }
+      }
+    }
+    if (!ok) lp_give_up(sh, status);
+    // tail: the leader's MMAs have released every stage this CTA filled
+    for (int q = 0; q < S; ++q) {
+      const int64_t k = last_in_slot(n_st, q, S);
+      if (k >= 0) mbar_wait_bounded(&sh.empty[q], (uint32_t)((k / S) & 1), nullptr, wait_cycles);
+    }
+  } else if (warp == 1 && lane == 0 && leader) {
+    // ------------------------------------------------------------ MMA issuer (leader)
+    constexpr uint32_t idesc = idesc_bf16_f32(kPairRows, N);
+    // descriptors advance by their 16-byte address units: 32 bytes per K = 16 step, one
+    // panel per 64 elements of K
+    constexpr uint64_t kStepK = 32 >> 4, kPanelA = Cfg::kAPanel >> 4, kPanelB = Cfg::kBPanel >> 4;
+    const int k_stages = (k_steps + Cfg::kPanels - 1) / Cfg::kPanels;
+    int s = 0;
+    uint32_t ph = 0;
+    int64_t n_st = 0, it = 0;
+    bool ok = true;
+    for (int64_t tile = pair; tile < n_tiles && ok; tile += n_pairs, ++it) {
+      const int acc = (int)(it & 1);
+      if (!mbar_wait_bounded(&sh.acc_empty[acc], (uint32_t)(((it >> 1) & 1) ^ 1), abort,
+                             wait_cycles)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();                          // the epilogue's reads of this accumulator
+      const uint32_t d = tmem + (uint32_t)(acc * Cfg::kAccStride);
+      for (int k = 0; k <= k_stages; ++k) {
+        // the operands arrive by TMA on this barrier: its wait orders the MMAs' reads
+        if (!mbar_wait_bounded(&sh.full[s], ph, abort, wait_cycles)) {
+          ok = false;
+          break;
+        }
+        const uint64_t a0 = sdesc_k_sw128(smem_u32(st_smem + s * Cfg::kStageBytes));
+        const uint64_t b0 = sdesc_k_sw128(smem_u32(st_smem + s * Cfg::kStageBytes + Cfg::kABytes));
+        if (k < k_stages) {
+#pragma unroll
+          for (int p = 0; p < Cfg::kPanels; ++p)
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              mma_pair_ss(d, a0 + p * kPanelA + kk * kStepK, b0 + p * kPanelB + kk * kStepK, idesc,
+                          (k > 0 || p > 0 || kk > 0) ? 1u : 0u);
+        } else {
+          // hi chunk kk at element 16 kk of an operand row, lo chunk at R + 16 kk
+#pragma unroll
+          for (int kk = 0; kk < R / 16; ++kk) {
+            const uint64_t hi = kk * kStepK, lo = (R / 16 + kk) * kStepK;
+            mma_pair_ss(d, a0 + hi, b0 + hi, idesc, 1u);
+            mma_pair_ss(d, a0 + hi, b0 + lo, idesc, 1u);
+            mma_pair_ss(d, a0 + lo, b0 + hi, idesc, 1u);
+          }
+        }
+        commit_both(&sh.empty[s]);
+        ++n_st;
+        if (++s == S) { s = 0; ph ^= 1u; }
+      }
+      if (!ok) break;
+      commit_both(&sh.acc_full[acc]);
+    }
+    if (!ok) lp_give_up(sh, status);
+    if (n_st > 0) {
+      // every MMA of the pair -- a tile left half-way included -- has completed before
+      // TMEM is released
+      commit_both(&sh.drain);
+      mbar_wait_bounded(&sh.drain, 0u, nullptr, wait_cycles);
+    }
+  } else if (warp >= 2 && warp < 2 + Cfg::kEpiWarps) {
+    // ------------------------------------------------------------ epilogue (each CTA)
+    const int e = warp - 2;
+    const int g = warp & 3;                      // TMEM lane group == rows 32 g .. + 31
+    const int h = e >> 2;                        // chunks h, h + 2, ...
+    const uint32_t lane_base = (uint32_t)(g * 32) << 16;
+    uint8_t* box = o_smem + e * Cfg::kBoxBytes;
+    int64_t it = 0;
+    bool ok = true;
+    for (int64_t tile = pair; tile < n_tiles; tile += n_pairs, ++it) {
+      int tb, nb;
+      order.decode(tile, tb, nb);
+      const int acc = (int)(it & 1);
+      if (!mbar_wait_bounded(&sh.acc_full[acc], (uint32_t)((it >> 1) & 1), abort, wait_cycles)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const int y = tb * kPairRows + kBM * (int)rank + 32 * g;
+      const uint32_t t_base = tmem + lane_base + (uint32_t)(acc * Cfg::kAccStride);
+#pragma unroll 1
+      for (int c = h; c < Cfg::kChunks; c += 2) {
+        uint32_t v[16];
+        tmem_ld_32x32b_x16(t_base + (uint32_t)(16 * c), v);
+        tmem_ld_wait();
+        if (c + 2 >= Cfg::kChunks) {             // this warp's last read of the accumulator
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) arrive_leader(&sh.acc_empty[acc]);
+        }
+        if (lane == 0) bulk_wait_read_all();     // the box's previous store has read it
+        __syncwarp();
+        uint32_t w[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const __nv_bfloat162 b2 =
+              __floats2bfloat162_rn(__uint_as_float(v[2 * q]), __uint_as_float(v[2 * q + 1]));
+          w[q] = *reinterpret_cast<const uint32_t*>(&b2);
+        }
+        // 16-byte chunk j of row `lane` (32-byte rows): 32-byte swizzle, chunk ^ (row / 4) % 2
+#pragma unroll
+        for (int j = 0; j < 2; ++j)
+          *reinterpret_cast<uint4*>(box + lane * 32 + ((j ^ ((lane >> 2) & 1)) << 4)) =
+              make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          const int x = nb * N + 16 * c;
+          if (y < rows && x < cols) tma_store_2d(&tm_y, x, y, box);
+          bulk_commit();
+        }
+        __syncwarp();
+      }
+    }
+    if (!ok && lane == 0) lp_give_up(sh, status);
+    if (lane == 0) bulk_wait_all();
+  }
+
+  tc_fence_before();
+  cluster_sync_all();                          // neither CTA frees TMEM or exits early
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, Cfg::kTmemCols);
+  }
+}
+
+template <int N, int R>
+cudaError_t launch_pair_nr(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
+                           const CUtensorMap& tm_s, const CUtensorMap& tm_u,
+                           const CUtensorMap& tm_y, int rows, int cols, int k_steps, int u_row0,
+                           int group, int n_pairs, uint32_t* d_status, cudaStream_t s) {
+  using Cfg = PairLin<N>;
+  cudaError_t e = cudaFuncSetAttribute(linear_pair_kernel<N, R>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::kSmem);
+  if (e != cudaSuccess) return e;
+  linear_pair_kernel<N, R><<<2 * n_pairs, Cfg::kThreads, Cfg::kSmem, s>>>(
+      tm_x, tm_w, tm_s, tm_u, tm_y, rows, cols, k_steps, u_row0, group, d_status, kWaitCycles);
+  return cudaGetLastError();
+}
+
+template <int N>
+int max_pairs_n() {
+  using Cfg = PairLin<N>;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2, 1, 1);
+  cfg.blockDim = dim3(Cfg::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmem;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = 2;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  if (cudaFuncSetAttribute(linear_pair_kernel<N, 32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)Cfg::kSmem) != cudaSuccess)
+    return 0;
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, linear_pair_kernel<N, 32>, &cfg) != cudaSuccess)
+    return 0;
+  return clusters;
+}
+
+constexpr int kPairCols[] = {256, 240, 224, 192, 128};
+
+}  // namespace
+
+int32_t linear_pair_cols(int32_t tiling) {
+  return tiling >= kLinearPairTiling0 && tiling < kLinearPairTiling0 + 5
+             ? kPairCols[tiling - kLinearPairTiling0]
+             : 0;
+}
+
+int32_t linear_pair_max_pairs() {
+  // every N has the same threads and (within a stage) the same shared-memory class: one
+  // CTA per SM; the smallest count over the tilings is the safe one
+  int p = max_pairs_n<256>();
+  p = std::min(p, max_pairs_n<240>());
+  p = std::min(p, max_pairs_n<224>());
+  p = std::min(p, max_pairs_n<192>());
+  p = std::min(p, max_pairs_n<128>());
+  return p;
+}
+
+int32_t linear_pair_tiling(int64_t T, int64_t m, int32_t n_pairs) {
+  // waves of pair tiles x the time of one tile (proportional to N, plus a fixed share for
+  // the tile's ramp) -- the fewest-waves choice among the supported N
+  int32_t best = kLinearPairTiling0;
+  int64_t c_best = -1;
+  const int64_t row_blocks = (T + kPairRows - 1) / kPairRows;
+  for (int i = 0; i < 5; ++i) {
+    const int64_t N = kPairCols[i];
+    const int64_t tiles = row_blocks * ((m + N - 1) / N);
+    const int64_t waves = (tiles + n_pairs - 1) / n_pairs;
+    const int64_t c = waves * (N + 8);
+    if (c_best < 0 || c < c_best) {
+      c_best = c;
+      best = kLinearPairTiling0 + i;
+    }
+  }
+  return best;
+}
+
+cudaError_t launch_linear_pair(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
+                               const CUtensorMap& tm_s, const CUtensorMap& tm_u,
+                               const CUtensorMap& tm_y, int64_t T, int64_t m, int64_t n,
+                               int32_t u_row0, int32_t r, int32_t tiling, int32_t n_pairs,
+                               uint32_t* d_status, cudaStream_t s) {
+  const int32_t N = linear_pair_cols(tiling);
+  if (N == 0 || n_pairs <= 0 || (r != 16 && r != 32)) return cudaErrorInvalidValue;
+  const int k_steps = (int)((n + 63) / 64);
+  const int64_t tiles = (T + kPairRows - 1) / kPairRows * ((m + N - 1) / N);
+  const int pairs = (int)std::min<int64_t>(tiles, n_pairs);
+  // column stripes as wide as one wave of pairs spread over every row block: a wave then
+  // shares its few W rows across all of X (measured on the LLaMA-7B shapes: 4 column blocks
+  // per stripe at 4096 tokens beat row-major order by 4% (4096 x 4096), 15% (11008 x 4096)
+  // and 2% (4096 x 11008))
+  const int64_t row_blocks = (T + kPairRows - 1) / kPairRows;
+  const int group = (int)std::max<int64_t>(1, pairs / row_blocks);
+#define ZO_PAIR_Y(NN, RR)                                                                     \
+  launch_pair_nr<NN, RR>(tm_x, tm_w, tm_s, tm_u, tm_y, (int)T, (int)m, k_steps, u_row0, group, \
+                         pairs, d_status, s)
+  switch (N * 64 + r) {
+    case 256 * 64 + 16: return ZO_PAIR_Y(256, 16);
+    case 256 * 64 + 32: return ZO_PAIR_Y(256, 32);
+    case 240 * 64 + 16: return ZO_PAIR_Y(240, 16);
+    case 240 * 64 + 32: return ZO_PAIR_Y(240, 32);
+    case 224 * 64 + 16: return ZO_PAIR_Y(224, 16);
+    case 224 * 64 + 32: return ZO_PAIR_Y(224, 32);
+    case 192 * 64 + 16: return ZO_PAIR_Y(192, 16);
+    case 192 * 64 + 32: return ZO_PAIR_Y(192, 32);
+    case 128 * 64 + 16: return ZO_PAIR_Y(128, 16);
+    case 128 * 64 + 32: return ZO_PAIR_Y(128, 32);
+    default: return cudaErrorInvalidValue;
+  }
+#undef ZO_PAIR_Y
+}
+
+}  // namespace zo

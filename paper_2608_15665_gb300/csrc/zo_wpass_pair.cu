@@ -40,6 +40,7 @@
 #include <cuda.h>
 
 #include "zo_kernels.h"
+#include "zo_cluster.cuh"
 #include "zo_sm100.cuh"
 #include "zo_tc_common.cuh"
 
@@ -48,6 +49,7 @@ namespace {
 
 using namespace sm100;
 using namespace tc;
+using namespace cta2;
 
 constexpr int kR = 128;
 constexpr int kPM = 256;                                   // pair tile rows
@@ -82,62 +84,10 @@ struct PairShared {
   uint32_t tmem_base;
 };
 
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-// shared::cluster address of `p` (a variable of this CTA's shared memory) in CTA `rank`
-__device__ __forceinline__ uint32_t map_to(const void* p, uint32_t rank) {
-  uint32_t a;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(p)), "r"(rank));
-  return a;
-}
-// arrive on the barrier at the same offset in the leader CTA
-__device__ __forceinline__ void arrive_leader(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(map_to(bar, 0)) : "memory");
-}
-// TMA load of a box into this CTA's shared memory whose bytes complete on the barrier at
-// the same offset in the leader CTA
-__device__ __forceinline__ void tma_load_2d_to_leader(void* smem_dst, const void* tmap, int32_t x,
-                                                      int32_t y, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(map_to(bar, 0))
-      : "memory");
-}
 __device__ __forceinline__ void give_up_pair(PairShared& sh, uint32_t* status) {
   atomicOr(status, (uint32_t)kDevTimeout);
   *reinterpret_cast<volatile int*>(&sh.abort_flag) = 1;
-  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(map_to(&sh.abort_flag, cluster_rank() ^ 1u)),
-               "r"(1)
-               : "memory");
-}
-// every thread of both CTAs (non-aligned forms: the role branches above may leave a warp
-// diverged; each warp reconverges first)
-__device__ __forceinline__ void cluster_sync_all() {
-  __syncwarp();
-  asm volatile("barrier.cluster.arrive.release;" ::: "memory");
-  asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
-}
-__device__ __forceinline__ void mma_pair_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
-                                            uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// arrive once on the barrier at this offset in both CTAs when the pair's MMAs so far complete
-__device__ __forceinline__ void commit_both(uint64_t* bar) {
-  const uint16_t mask = 3;
-  asm volatile(
-      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-      " [%0], %1;" ::"r"(smem_u32(bar)),
-      "h"(mask)
-      : "memory");
+  store_peer(&sh.abort_flag, 1);
 }
 
 // The pair tiles of one pair: chunks of kTileChunk consecutive pair tiles b, b + G, ...
@@ -224,13 +174,7 @@ wpass_pair_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
     fence_mbar_init();
     prefetch_tmap(&tm_b64);
   }
-  if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     smem_u32(&sh.tmem_base)),
-                 "r"(kTmemCols)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
-  }
+  if (warp == 1) tmem_alloc_pair(&sh.tmem_base, kTmemCols);
   tc_fence_before();
   cluster_sync_all();                          // both CTAs' barriers and TMEM exist
   tc_fence_after();
@@ -489,8 +433,7 @@ wpass_pair_kernel(const uint4* __restrict__ u_t, const __grid_constant__ CUtenso
   cluster_sync_all();                          // neither CTA frees TMEM or exits early
   if (warp == 1) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
-                 : "memory");
+    tmem_dealloc_pair(tmem, kTmemCols);
   }
 }
 

@@ -18,6 +18,10 @@ from parity import NORMAL_ABS, to_f64
 
 pytestmark = pytest.mark.gpu
 
+# ZO_OPTION_LINEAR_TILE values: 1..3 single-CTA tiles, 4..8 SM-pair tiles (N = 256, 240,
+# 224, 192, 128 columns of Y)
+TILINGS = (1, 2, 3, 4, 5, 6, 7, 8)
+
 # (r, [(m, n, ldw)], token counts)
 LINEAR_CASES = {
     "r32": (32, [(304, 520, None), (264, 2048, None), (1032, 72, 80)], (1, 130, 300)),
@@ -72,7 +76,8 @@ def test_perturbed_linear_matches_oracle_and_leaves_W(lib, gpu, case, eps):
             X = _tokens(T, n, 17 * T + i, gpu)
             ldy = (m + 7) // 8 * 8
             out = {}
-            for tiling in (1, 2, 3):     # 128x256, 256x256, 256x224
+            # 128x256, 256x256, 256x224 on single CTAs; 256 x (256, 240, 224, 192, 128) on SM pairs
+            for tiling in TILINGS:
                 zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, tiling)
                 Ybuf = torch.full((T, ldy), float("nan"), dtype=torch.bfloat16, device=gpu)
                 zb.zo_linear_perturbed(z.ctx, i, X, Ybuf[:, :m])
@@ -82,8 +87,8 @@ def test_perturbed_linear_matches_oracle_and_leaves_W(lib, gpu, case, eps):
                 assert torch.isnan(Ybuf[:, m:].float()).all()
                 out[tiling] = Ybuf[:, :m]
             # every tiling sums each output in the same order
-            for tiling in (1, 3):
-                assert torch.equal(out[tiling].view(torch.int16), out[2].view(torch.int16))
+            for tiling in TILINGS:
+                assert torch.equal(out[tiling].view(torch.int16), out[2].view(torch.int16)), tiling
             Y = out[3]
             C = subzero.perturb_coeff(z.seed, base + i, 5, r, terms, f32(eps))
             zc = abs(f32(eps)) * 2.0
@@ -116,6 +121,7 @@ def test_perturbed_linear_single_query_and_repeat(lib, gpu):
     zb.zo_linear_perturbed(z.ctx, 1, X, Y2)
     z.sync()
     assert torch.equal(Y1.view(torch.int16), Y2.view(torch.int16))   # deterministic
+    assert zb.zo_linear_tiling(z.ctx) >= 4        # the automatic choice runs on SM pairs
     C = subzero.perturb_coeff(z.seed, base + 1, 0, r, [(3, -2.0)], f32(1e-2))
     _check(Y1, X, before["W"][1], before["U"][1], before["V"][1], C, 2.0 * f32(1e-2),
            "single query")
@@ -159,7 +165,7 @@ def test_perturbed_linear_rejections(lib, gpu):
     with pytest.raises(RuntimeError):
         zb.zo_linear_perturbed(z.ctx, 3, X, Y)                                     # no matrix 3
     with pytest.raises(RuntimeError):
-        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 4)                       # no tiling 4
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 9)                       # no tiling 9
     z.refresh(1)                                                                   # new U, V
     with pytest.raises(RuntimeError):
         zb.zo_linear_perturbed(z.ctx, 0, X, Y)                                     # stale P
