@@ -104,14 +104,21 @@ enum {
                                      CTA first waits on a barrier nothing arrives on, so its
                                      bounded wait (~0.1 s) runs out; that pass then reports
                                      ZO_ERR_TIMEOUT via zo_sync_status and leaves W partly
-                                     updated.  Nothing faults; the context stays usable. */
+                                     updated.  If an SM-pair zo_linear_perturbed call comes
+                                     first, it takes the hook instead: its Y tiles wait for
+                                     S rows that are never counted as written, give up after
+                                     ~0.1 s and leave Y partly written.  Nothing faults; the
+                                     context stays usable. */
   ZO_OPTION_LINEAR_TILE = 3, /* tiles (rows of X x columns of Y) of zo_linear_perturbed's
                                Y = X W^T + S U^T GEMM: 0 = automatic (the SM-pair tiling
-                               with the fewest waves x a tile's time; the single-CTA ones
-                               if no 2-CTA cluster fits), 1 = 128 x 256, 2 = 256 x 256,
-                               3 = 256 x 224 on single CTAs, 4 .. 8 = 256 x 256, 240, 224,
-                               192, 128 on SM pairs (M = 256 MMAs across a 2-CTA cluster).
-                               All give bit-identical Y. */
+                               whose busiest pair has the least operand traffic; the
+                               single-CTA ones if no 2-CTA cluster fits), 1 = 128 x 256,
+                               2 = 256 x 256, 3 = 256 x 224 on single CTAs (S = X P^T by a
+                               separate split-K kernel), 4 .. 8 = 256 x 256, 240, 224, 192,
+                               128 on SM pairs (M = 256 MMAs across a 2-CTA cluster, S in
+                               the same launch).  The tilings of one family give
+                               bit-identical Y; the two families may differ in the last
+                               bits of S (one K range against split-K partial sums). */
   ZO_OPTION_PAIR_MMA = 4    /* tensor-core weight pass at r = 128: 1 (default) = M = 256 MMAs
                                across the two SMs of a cluster (each SM holds and reads half
                                of every P tile), 0 = the single-SM kernel.  Both give

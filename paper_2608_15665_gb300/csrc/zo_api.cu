@@ -133,6 +133,10 @@ struct zo_ctx {
   __nv_bfloat16* d_s_hl = nullptr;
   float* d_s_part = nullptr;
   uint32_t* d_s_count = nullptr;   // one counter per 32 rows of S_HL's capacity
+  // the SM-pair route's row-block counters (one per 256 rows of S_HL's capacity) and the
+  // epoch of its last call
+  uint32_t* d_s_flags = nullptr;
+  uint32_t lin_epoch = 0;
   int64_t s_cap = 0, part_cap = 0;
   int64_t tc_tiles = 0;
   // r = 128: the weight pass on SM pairs (256-row tiles numbered in d_tc_pair), unless
@@ -184,6 +188,7 @@ void free_ctx(zo_ctx* c) {
   cudaFree(c->d_s_hl);
   cudaFree(c->d_s_part);
   cudaFree(c->d_s_count);
+  cudaFree(c->d_s_flags);
   cudaFree(c->d_w_maps);
   cudaFree(c->d_u_units);
   cudaFree(c->d_v_hl);
@@ -1076,16 +1081,23 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     if (T > c->s_cap) {
       cudaFree(c->d_s_hl);
       cudaFree(c->d_s_count);
+      cudaFree(c->d_s_flags);
       c->d_s_hl = nullptr;
       c->d_s_count = nullptr;
+      c->d_s_flags = nullptr;
       c->s_cap = 0;
       const int64_t cap = (T + 127) / 128 * 128;
       ZO_CUDA(cudaMalloc(&c->d_s_hl, sizeof(__nv_bfloat16) * cap * HLW), "cudaMalloc(S_HL)");
       ZO_CUDA(cudaMalloc(&c->d_s_count, sizeof(uint32_t) * (cap / 32)), "cudaMalloc(S counters)");
+      ZO_CUDA(cudaMalloc(&c->d_s_flags, sizeof(uint32_t) * (cap / 256 + 1)),
+              "cudaMalloc(S row-block counters)");
       // on the context's stream: a plain cudaMemset runs on the legacy default stream,
       // which a non-blocking stream's kernels are not ordered after
       ZO_CUDA(cudaMemsetAsync(c->d_s_count, 0, sizeof(uint32_t) * (cap / 32), c->stream),
               "zero S counters");
+      ZO_CUDA(cudaMemsetAsync(c->d_s_flags, 0, sizeof(uint32_t) * (cap / 256 + 1), c->stream),
+              "zero S row-block counters");
+      c->lin_epoch = 0;
       c->s_cap = cap;
     }
     if (part > c->part_cap) {
@@ -1101,7 +1113,7 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
   if (c->linear_pairs < 0) c->linear_pairs = std::max(0, (int)zo::linear_pair_max_pairs());
   int32_t tiling = c->linear_tile;
   if (tiling == 0)
-    tiling = c->linear_pairs > 0 ? zo::linear_pair_tiling(T, m, c->linear_pairs)
+    tiling = c->linear_pairs > 0 ? zo::linear_pair_tiling(T, m, c->r, c->linear_pairs)
                                  : zo::linear_y_tiling(T, m, c->sms, 0);
   const int32_t pair_n = zo::linear_pair_cols(tiling);
   if (pair_n > 0 && c->linear_pairs <= 0) {
@@ -1109,7 +1121,7 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     return ZO_ERR_UNSUPPORTED;
   }
   const bool narrow_y = pair_n == 0 && zo::linear_y_tile_cols(tiling) % 64 != 0;
-  CUtensorMap tm_x{}, tm_pk{}, tm_s{}, tm_y{}, tm_w{}, tm_u{};
+  CUtensorMap tm_x{}, tm_pk{}, tm_s{}, tm_y{}, tm_w{}, tm_u{}, tm_pk_half{};
   bool enc =
       encode_bf16_2d(&tm_x, const_cast<void*>(X), n, T, ldx * 2, 64, 128) &&
       encode_bf16_2d(&tm_pk, c->d_pk + c->h_pk_off[mat], n, 2 * r, (n + 63) / 64 * 64 * 2, 64,
@@ -1120,7 +1132,10 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     // tile's B rows), Y in 32 x 16 boxes
     enc = enc && encode_bf16_2d(&tm_w, md.W, n, m, md.ldw * 2, 64, (uint32_t)(pair_n / 2)) &&
           encode_bf16_2d(&tm_u, c->d_u_lin, HLW, c->u_rows, HLW * 2, 64, (uint32_t)(pair_n / 2)) &&
-          encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 16, 32, CU_TENSOR_MAP_SWIZZLE_32B);
+          encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 16, 32, CU_TENSOR_MAP_SWIZZLE_32B) &&
+          // P_K in boxes of r rows: CTA 0 of a pair loads P_hi, CTA 1 P_lo
+          encode_bf16_2d(&tm_pk_half, c->d_pk + c->h_pk_off[mat], n, 2 * r, (n + 63) / 64 * 64 * 2,
+                         64, (uint32_t)r);
   } else {
     enc = enc && (narrow_y ? encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 32, 32,
                                             CU_TENSOR_MAP_SWIZZLE_64B)
@@ -1130,21 +1145,33 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     g_last_error = "zo_linear_perturbed: cuTensorMapEncodeTiled rejected a descriptor";
     return ZO_ERR_CUDA;
   }
-  // S = X P^T (split K, the partial sums reduced into S_HL), Y = X W^T + S U^T
-  ZO_CUDA(zo::launch_linear_s(tm_x, tm_pk, T, n, r, k_split, k_chunk, c->d_s_part, c->d_s_hl,
-                              c->d_s_count, c->sms, c->d_status, c->stream),
-          "S = X P^T kernels");
   if (pair_n > 0) {
-    ZO_CUDA(zo::launch_linear_pair(tm_x, tm_w, tm_s, tm_u, tm_y, T, m, n, c->h_tc[mat].u_row0, r,
-                                   tiling, c->linear_pairs, c->d_status, c->stream),
+    // one launch: S = X P^T in its S tiles (one per 256 rows), then Y = X W^T + S U^T
+    if (c->lin_epoch + 1 >= zo::kLinearPairEpochs) {
+      // the epochs start again: no counter may hold an old call's complete count
+      ZO_CUDA(cudaMemsetAsync(c->d_s_flags, 0, sizeof(uint32_t) * (c->s_cap / 256 + 1), c->stream),
+              "zero S row-block counters");
+      c->lin_epoch = 0;
+    }
+    ++c->lin_epoch;
+    const bool inject = c->inject_wait;    // the test hook is one-shot
+    c->inject_wait = false;
+    ZO_CUDA(zo::launch_linear_pair(tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk_half, T, m, n,
+                                   c->h_tc[mat].u_row0, r, tiling, c->linear_pairs, c->d_s_hl,
+                                   c->d_s_flags, c->lin_epoch, inject, c->d_status, c->stream),
             "perturbed linear kernel (SM pairs)");
+    c->launches += 1;
   } else {
+    // S = X P^T (split K, the partial sums reduced into S_HL), Y = X W^T + S U^T
+    ZO_CUDA(zo::launch_linear_s(tm_x, tm_pk, T, n, r, k_split, k_chunk, c->d_s_part, c->d_s_hl,
+                                c->d_s_count, c->sms, c->d_status, c->stream),
+            "S = X P^T kernels");
     ZO_CUDA(zo::launch_linear_y(tm_x, c->d_w_maps + mat, tm_s, c->tm_u_lin, tm_y, T, m, n,
                                 c->h_tc[mat].u_row0, r, tiling, c->sms, c->d_status, c->stream),
             "perturbed linear kernel");
+    c->launches += 1 + zo::linear_s_launches(k_split);
   }
   c->last_linear_tiling = tiling;
-  c->launches += 1 + zo::linear_s_launches(k_split);
   return ZO_OK;
 }
 
@@ -1179,10 +1206,16 @@ zo_status zo_sync_status(zo_ctx* c) {
   if (s != 0) {
     // cleared on the context's stream (ordered before its next kernels) and waited for
     ZO_CUDA(cudaMemsetAsync(c->d_status, 0, sizeof(uint32_t), c->stream), "clear status");
-    // a perturbed-linear S kernel cut short can leave its group counters part-counted
+    // a perturbed-linear S kernel cut short can leave its group counters part-counted, and
+    // an SM-pair launch its row-block counters
     if ((s & zo::kDevTimeout) && c->d_s_count)
       ZO_CUDA(cudaMemsetAsync(c->d_s_count, 0, sizeof(uint32_t) * (c->s_cap / 32), c->stream),
               "zero S counters");
+    if ((s & zo::kDevTimeout) && c->d_s_flags) {
+      ZO_CUDA(cudaMemsetAsync(c->d_s_flags, 0, sizeof(uint32_t) * (c->s_cap / 256 + 1), c->stream),
+              "zero S row-block counters");
+      c->lin_epoch = 0;
+    }
     ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
     if (s & zo::kDevTimeout) {
       g_last_error = "a device-side wait ran out";

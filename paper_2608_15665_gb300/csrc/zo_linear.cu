@@ -56,6 +56,7 @@
 #include <cuda.h>
 
 #include "zo_kernels.h"
+#include "zo_linear_common.cuh"
 #include "zo_sm100.cuh"
 #include "zo_tc_common.cuh"
 
@@ -64,6 +65,7 @@ namespace {
 
 using namespace sm100;
 using namespace tc;
+using namespace lin;
 
 constexpr int kFusedSplits = 4;   // most K ranges whose S partials the S kernel sums itself
 constexpr int kModeS = 0;
@@ -102,25 +104,6 @@ struct LinCfg {
   static_assert(kABytes == kHalves * kPanelBytes, "one 128-row panel per half");
   static_assert(kN % 32 == 0 && kN <= kBRows && kN <= kHalfCols, "tile columns");
 };
-
-// S_HL row: [hi | lo] of the R sums in chunks of 8, then zero chunks up to 64 elements.
-template <int R>
-__device__ __forceinline__ void write_s_row(__nv_bfloat16* s_hl, int row, const float (&x)[R]) {
-  constexpr int kGroups = R / 8;
-  uint4* out = reinterpret_cast<uint4*>(s_hl + (int64_t)row * 64);
-#pragma unroll
-  for (int g = 0; g < kGroups; ++g) {
-    float c[8];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) c[e] = x[8 * g + e];
-    uint4 hi, lo;
-    split8(c, hi, lo);
-    out[g] = hi;
-    out[kGroups + g] = lo;
-  }
-#pragma unroll
-  for (int z = 2 * kGroups; z < 8; ++z) out[z] = make_uint4(0u, 0u, 0u, 0u);
-}
 
 struct LinShared {
   uint64_t full[4], empty[4];

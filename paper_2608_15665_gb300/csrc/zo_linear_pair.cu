@@ -40,6 +40,7 @@
 
 #include "zo_cluster.cuh"
 #include "zo_kernels.h"
+#include "zo_linear_common.cuh"
 #include "zo_sm100.cuh"
 #include "zo_tc_common.cuh"
 
@@ -49,6 +50,7 @@ namespace {
 using namespace sm100;
 using namespace tc;
 using namespace cta2;
+using namespace lin;
 
 constexpr int kPairRows = 2 * kBM;   // 256 rows of X per pair tile
 
@@ -84,6 +86,41 @@ struct LinPairShared {
   int abort_flag;
 };
 
+// Row-block counters of the S tiles: (call epoch << 4) | finished S-tile epilogue warps.
+// A warp of call e moves the counter to (e, count + 1), or to (e, 1) from an older call's
+// value (release, GPU scope); the Y tiles of call e wait for (e, 8) (acquire).  Calls
+// whose T covers fewer row blocks leave the others' counters behind, which the epoch
+// makes harmless.
+__device__ __forceinline__ void count_s_warp(uint32_t* f, uint32_t epoch) {
+  uint32_t cur;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(cur) : "l"(f) : "memory");
+  for (;;) {
+    const uint32_t want = (cur >> 4) == epoch ? cur + 1 : (epoch << 4) + 1;
+    uint32_t prev;
+    asm volatile("atom.release.gpu.global.cas.b32 %0, [%1], %2, %3;"
+                 : "=r"(prev) : "l"(f), "r"(cur), "r"(want) : "memory");
+    if (prev == cur) return;
+    cur = prev;
+  }
+}
+__device__ __forceinline__ bool wait_s_rows(const uint32_t* f, uint32_t epoch,
+                                            const volatile int* abort, long long limit_cycles) {
+  const uint32_t target = (epoch << 4) + kLinearPairCountsPerCall;
+  const long long t0 = clock64();
+  for (;;) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(f) : "memory");
+    if (v == target) return true;
+    if (*abort) return false;
+    if (clock64() - t0 > limit_cycles) return false;
+    __nanosleep(64);
+  }
+}
+// generic-proxy global writes <-> later async-proxy (TMA) reads
+__device__ __forceinline__ void fence_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
 __device__ __forceinline__ void lp_give_up(LinPairShared& sh, uint32_t* status) {
   atomicOr(status, (uint32_t)kDevTimeout);
   *reinterpret_cast<volatile int*>(&sh.abort_flag) = 1;
@@ -101,6 +138,8 @@ __device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&v)
       : "r"(taddr));
 }
 
+// The launch's tiles: first one S tile per row block (S = X P^T for its 256 rows, written
+// to S_HL), then the Y tiles in stripe order.
 // Pair tile t -> (row block tb, column block nb): column stripes of `group` column blocks,
 // each walked row block by row block (group = the column blocks: plain row-major order).
 // Stripes about one wave of tiles wide keep the wave's W rows few enough to stay in L2
@@ -123,15 +162,38 @@ struct StripeOrder {
   }
 };
 
+// The launch's tiles: first one S tile per row block (S = X P^T for its 256 rows, written
+// to S_HL), then the Y tiles in stripe order.
+struct PairTiles {
+  int row_blocks;
+  StripeOrder order;
+  __device__ bool decode(int64_t t, int& tb, int& nb) const {   // true: an S tile
+    if (t < row_blocks) {
+      tb = (int)t;
+      nb = 0;
+      return true;
+    }
+    order.decode(t - row_blocks, tb, nb);
+    return false;
+  }
+};
+
 // tm_x: X (box 64 x 128), tm_w: W_i (box 64 x N/2), tm_s: S_HL (box 64 x 128), tm_u: the
 // route's U operand (box 64 x N/2; this matrix's rows from u_row0), tm_y: Y (box 16 x 32,
-// 32-byte swizzle).  rows = T, cols = m, k_steps = ceil(n / 64).
+// 32-byte swizzle), tm_pk: P_K = [P_hi ; P_lo] (box 64 x R: CTA c loads rows R c ..).
+// rows = T, cols = m, k_steps = ceil(n / 64).  s_hl: the S_HL rows the S tiles write;
+// s_count[tb]: the row block's counter (count_s_warp); epoch: this call's (1 .. 2^28 - 1),
+// which its S tiles write; wait_epoch: the one its Y tiles wait for (= epoch; the test hook
+// passes one that never comes, so that every Y tile's bounded wait runs out).
 template <int N, int R>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairLin<N>::kThreads, 1)
 linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
                    const __grid_constant__ CUtensorMap tm_s, const __grid_constant__ CUtensorMap tm_u,
-                   const __grid_constant__ CUtensorMap tm_y, int rows, int cols, int k_steps,
-                   int u_row0, int group, uint32_t* __restrict__ status, long long wait_cycles) {
+                   const __grid_constant__ CUtensorMap tm_y, const __grid_constant__ CUtensorMap tm_pk,
+                   int rows, int cols, int k_steps, int u_row0, int group,
+                   __nv_bfloat16* __restrict__ s_hl, uint32_t* __restrict__ s_count,
+                   uint32_t epoch, uint32_t wait_epoch, uint32_t* __restrict__ status,
+                   long long wait_cycles) {
   using Cfg = PairLin<N>;
   constexpr int S = Cfg::kStages;
   static_assert(sizeof(LinPairShared) <= 1024, "barrier block");
@@ -148,8 +210,9 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
   const int64_t pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
   const int tiles_n = (cols + N - 1) / N;
   const int row_blocks = (rows + kPairRows - 1) / kPairRows;
-  const int64_t n_tiles = (int64_t)row_blocks * tiles_n;
-  const StripeOrder order{tiles_n, row_blocks, group < 1 || group > tiles_n ? tiles_n : group};
+  const int64_t n_tiles = (int64_t)row_blocks * (tiles_n + 1);
+  const PairTiles tiles{row_blocks,
+                        StripeOrder{tiles_n, row_blocks, group < 1 || group > tiles_n ? tiles_n : group}};
   const volatile int* abort = &sh.abort_flag;
 
   if (threadIdx.x == 0) {
@@ -169,6 +232,7 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
     prefetch_tmap(&tm_s);
     prefetch_tmap(&tm_u);
     prefetch_tmap(&tm_y);
+    prefetch_tmap(&tm_pk);
   }
   if (warp == 1) tmem_alloc_pair(&sh.tmem_base, Cfg::kTmemCols);
   tc_fence_before();
@@ -185,17 +249,26 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
     const int k_stages = (k_steps + Cfg::kPanels - 1) / Cfg::kPanels;
     for (int64_t tile = pair; tile < n_tiles && ok; tile += n_pairs) {
       int tb, nb;
-      order.decode(tile, tb, nb);
+      const bool s_tile = tiles.decode(tile, tb, nb);
       const int y_a = tb * kPairRows + kBM * (int)rank;
       const int y_b = nb * N + Cfg::kHalfN * (int)rank;
-      for (int k = 0; k <= k_stages; ++k) {
+      for (int k = 0; k < k_stages + (s_tile ? 0 : 1); ++k) {
         if (!mbar_wait_bounded(&sh.empty[s], ph ^ 1u, abort, wait_cycles)) {
           ok = false;
           break;
         }
         uint8_t* a_dst = st_smem + s * Cfg::kStageBytes;
         uint8_t* b_dst = a_dst + Cfg::kABytes;
-        if (k < k_stages) {
+        if (s_tile) {
+          // X panels and this CTA's R rows of P_K (P_hi in CTA 0, P_lo in CTA 1)
+          if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * Cfg::kPanels * (Cfg::kAPanel + R * 128));
+#pragma unroll
+          for (int p = 0; p < Cfg::kPanels; ++p) {
+            const int x = 64 * (Cfg::kPanels * k + p);
+            tma_load_2d_to_leader(a_dst + p * Cfg::kAPanel, &tm_x, x, y_a, &sh.full[s]);
+            tma_load_2d_to_leader(b_dst + p * Cfg::kBPanel, &tm_pk, x, R * (int)rank, &sh.full[s]);
+          }
+        } else if (k < k_stages) {
           // panels past n read TMA's zero fill
           if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * Cfg::kStageBytes);
 #pragma unroll
@@ -205,6 +278,13 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
             tma_load_2d_to_leader(b_dst + p * Cfg::kBPanel, &tm_w, x, y_b, &sh.full[s]);
           }
         } else {                               // the rank-r step: S_HL rows, U operand rows
+          // this row block's S rows: written by its S tile (both CTAs' epilogues) earlier in
+          // this launch
+          if (!wait_s_rows(s_count + tb, wait_epoch, abort, wait_cycles)) {
+            ok = false;
+            break;
+          }
+          fence_async_global();
           if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * (Cfg::kAPanel + Cfg::kBPanel));
           tma_load_2d_to_leader(a_dst, &tm_s, 0, y_a, &sh.full[s]);
           tma_load_2d_to_leader(b_dst, &tm_u, 0, u_row0 + y_b, &sh.full[s]);
@@ -222,6 +302,7 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
   } else if (warp == 1 && lane == 0 && leader) {
     // ------------------------------------------------------------ MMA issuer (leader)
     constexpr uint32_t idesc = idesc_bf16_f32(kPairRows, N);
+    constexpr uint32_t idesc_s = idesc_bf16_f32(kPairRows, 2 * R);
     // descriptors advance by their 16-byte address units: 32 bytes per K = 16 step, one
     // panel per 64 elements of K
     constexpr uint64_t kStepK = 32 >> 4, kPanelA = Cfg::kAPanel >> 4, kPanelB = Cfg::kBPanel >> 4;
@@ -231,6 +312,8 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
     int64_t n_st = 0, it = 0;
     bool ok = true;
     for (int64_t tile = pair; tile < n_tiles && ok; tile += n_pairs, ++it) {
+      int tb, nb;
+      const bool s_tile = tiles.decode(tile, tb, nb);
       const int acc = (int)(it & 1);
       if (!mbar_wait_bounded(&sh.acc_empty[acc], (uint32_t)(((it >> 1) & 1) ^ 1), abort,
                              wait_cycles)) {
@@ -239,7 +322,7 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
       }
       tc_fence_after();                          // the epilogue's reads of this accumulator
       const uint32_t d = tmem + (uint32_t)(acc * Cfg::kAccStride);
-      for (int k = 0; k <= k_stages; ++k) {
+      for (int k = 0; k < k_stages + (s_tile ? 0 : 1); ++k) {
         // the operands arrive by TMA on this barrier: its wait orders the MMAs' reads
         if (!mbar_wait_bounded(&sh.full[s], ph, abort, wait_cycles)) {
           ok = false;
@@ -247,7 +330,15 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
         }
         const uint64_t a0 = sdesc_k_sw128(smem_u32(st_smem + s * Cfg::kStageBytes));
         const uint64_t b0 = sdesc_k_sw128(smem_u32(st_smem + s * Cfg::kStageBytes + Cfg::kABytes));
-        if (k < k_stages) {
+        if (s_tile) {
+          // D[:, :R] = X P_hi^T, D[:, R:2R] = X P_lo^T
+#pragma unroll
+          for (int p = 0; p < Cfg::kPanels; ++p)
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              mma_pair_ss(d, a0 + p * kPanelA + kk * kStepK, b0 + p * kPanelB + kk * kStepK, idesc_s,
+                          (k > 0 || p > 0 || kk > 0) ? 1u : 0u);
+        } else if (k < k_stages) {
 #pragma unroll
           for (int p = 0; p < Cfg::kPanels; ++p)
 #pragma unroll
@@ -289,7 +380,7 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
     bool ok = true;
     for (int64_t tile = pair; tile < n_tiles; tile += n_pairs, ++it) {
       int tb, nb;
-      order.decode(tile, tb, nb);
+      const bool s_tile = tiles.decode(tile, tb, nb);
       const int acc = (int)(it & 1);
       if (!mbar_wait_bounded(&sh.acc_full[acc], (uint32_t)((it >> 1) & 1), abort, wait_cycles)) {
         ok = false;
@@ -298,6 +389,38 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
       tc_fence_after();
       const int y = tb * kPairRows + kBM * (int)rank + 32 * g;
       const uint32_t t_base = tmem + lane_base + (uint32_t)(acc * Cfg::kAccStride);
+      if (s_tile) {
+        // S = D[:, :R] + D[:, R:2R] for this lane's row, written as its S_HL row; four warps
+        // per CTA (one per TMEM lane group), then each counts itself done for the row block
+        if (h == 0) {
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(t_base, v);
+          float x[R];
+          if constexpr (R == 32) {
+            uint32_t w[32];
+            tmem_ld_32x32b_x32(t_base + 32u, w);
+            tmem_ld_wait();
+#pragma unroll
+            for (int q = 0; q < R; ++q) x[q] = 0.f + (__uint_as_float(v[q]) + __uint_as_float(w[q]));
+          } else {
+            tmem_ld_wait();
+#pragma unroll
+            for (int q = 0; q < R; ++q) x[q] = 0.f + (__uint_as_float(v[q]) + __uint_as_float(v[R + q]));
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) arrive_leader(&sh.acc_empty[acc]);
+          if (y + lane < rows) write_s_row<R>(s_hl, y + lane, x);
+          fence_async_global();
+          __threadfence();
+          __syncwarp();
+          if (lane == 0) count_s_warp(s_count + tb, epoch);
+        } else {
+          __syncwarp();
+          if (lane == 0) arrive_leader(&sh.acc_empty[acc]);
+        }
+        continue;
+      }
 #pragma unroll 1
       for (int c = h; c < Cfg::kChunks; c += 2) {
         uint32_t v[16];
@@ -347,14 +470,17 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
 template <int N, int R>
 cudaError_t launch_pair_nr(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
                            const CUtensorMap& tm_s, const CUtensorMap& tm_u,
-                           const CUtensorMap& tm_y, int rows, int cols, int k_steps, int u_row0,
-                           int group, int n_pairs, uint32_t* d_status, cudaStream_t s) {
+                           const CUtensorMap& tm_y, const CUtensorMap& tm_pk, int rows, int cols,
+                           int k_steps, int u_row0, int group, __nv_bfloat16* s_hl,
+                           uint32_t* s_count, uint32_t epoch, bool inject_wait, int n_pairs,
+                           uint32_t* d_status, cudaStream_t s) {
   using Cfg = PairLin<N>;
   cudaError_t e = cudaFuncSetAttribute(linear_pair_kernel<N, R>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::kSmem);
   if (e != cudaSuccess) return e;
   linear_pair_kernel<N, R><<<2 * n_pairs, Cfg::kThreads, Cfg::kSmem, s>>>(
-      tm_x, tm_w, tm_s, tm_u, tm_y, rows, cols, k_steps, u_row0, group, d_status, kWaitCycles);
+      tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk, rows, cols, k_steps, u_row0, group, s_hl, s_count,
+      epoch, inject_wait ? epoch + 1 : epoch, d_status, inject_wait ? kTestWaitCycles : kWaitCycles);
   return cudaGetLastError();
 }
 
@@ -402,17 +528,23 @@ int32_t linear_pair_max_pairs() {
   return p;
 }
 
-int32_t linear_pair_tiling(int64_t T, int64_t m, int32_t n_pairs) {
-  // waves of pair tiles x the time of one tile (proportional to N, plus a fixed share for
-  // the tile's ramp) -- the fewest-waves choice among the supported N
+int32_t linear_pair_tiling(int64_t T, int64_t m, int32_t r, int32_t n_pairs) {
+  // the busiest pair's work, tiles dealt round-robin (the row blocks' S tiles first); a tile
+  // costs the bytes an SM takes in per 128 elements of K, at ~64 B per cycle the rate that
+  // bounds these tiles: 32 KB of X plus N/2 rows of W (Y tiles), or r rows of P_K (S tiles)
   int32_t best = kLinearPairTiling0;
   int64_t c_best = -1;
   const int64_t row_blocks = (T + kPairRows - 1) / kPairRows;
+  const int64_t pairs = std::max<int32_t>(1, n_pairs);
   for (int i = 0; i < 5; ++i) {
     const int64_t N = kPairCols[i];
-    const int64_t tiles = row_blocks * ((m + N - 1) / N);
-    const int64_t waves = (tiles + n_pairs - 1) / n_pairs;
-    const int64_t c = waves * (N + 8);
+    const int64_t total = row_blocks * ((m + N - 1) / N + 1);
+    int64_t c = 0;
+    for (int64_t p = 0; p < std::min(pairs, total); ++p) {
+      const int64_t n_tiles = (total - p + pairs - 1) / pairs;      // tiles p, p + pairs, ...
+      const int64_t n_s = p < row_blocks ? (row_blocks - p + pairs - 1) / pairs : 0;
+      c = std::max(c, n_s * (512 + 4 * r) + (n_tiles - n_s) * (512 + 2 * N));
+    }
     if (c_best < 0 || c < c_best) {
       c_best = c;
       best = kLinearPairTiling0 + i;
@@ -423,13 +555,15 @@ int32_t linear_pair_tiling(int64_t T, int64_t m, int32_t n_pairs) {
 
 cudaError_t launch_linear_pair(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
                                const CUtensorMap& tm_s, const CUtensorMap& tm_u,
-                               const CUtensorMap& tm_y, int64_t T, int64_t m, int64_t n,
-                               int32_t u_row0, int32_t r, int32_t tiling, int32_t n_pairs,
-                               uint32_t* d_status, cudaStream_t s) {
+                               const CUtensorMap& tm_y, const CUtensorMap& tm_pk, int64_t T,
+                               int64_t m, int64_t n, int32_t u_row0, int32_t r, int32_t tiling,
+                               int32_t n_pairs, __nv_bfloat16* s_hl, uint32_t* s_count,
+                               uint32_t epoch, bool inject_wait, uint32_t* d_status,
+                               cudaStream_t s) {
   const int32_t N = linear_pair_cols(tiling);
   if (N == 0 || n_pairs <= 0 || (r != 16 && r != 32)) return cudaErrorInvalidValue;
   const int k_steps = (int)((n + 63) / 64);
-  const int64_t tiles = (T + kPairRows - 1) / kPairRows * ((m + N - 1) / N);
+  const int64_t tiles = (T + kPairRows - 1) / kPairRows * ((m + N - 1) / N + 1);
   const int pairs = (int)std::min<int64_t>(tiles, n_pairs);
   // column stripes as wide as one wave of pairs spread over every row block: a wave then
   // shares its few W rows across all of X (measured on the LLaMA-7B shapes: 4 column blocks
@@ -438,8 +572,8 @@ cudaError_t launch_linear_pair(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
   const int64_t row_blocks = (T + kPairRows - 1) / kPairRows;
   const int group = (int)std::max<int64_t>(1, pairs / row_blocks);
 #define ZO_PAIR_Y(NN, RR)                                                                     \
-  launch_pair_nr<NN, RR>(tm_x, tm_w, tm_s, tm_u, tm_y, (int)T, (int)m, k_steps, u_row0, group, \
-                         pairs, d_status, s)
+  launch_pair_nr<NN, RR>(tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk, (int)T, (int)m, k_steps, u_row0,  \
+                         group, s_hl, s_count, epoch, inject_wait, pairs, d_status, s)
   switch (N * 64 + r) {
     case 256 * 64 + 16: return ZO_PAIR_Y(256, 16);
     case 256 * 64 + 32: return ZO_PAIR_Y(256, 32);

@@ -45,6 +45,42 @@ def test_expired_wait_reports_timeout_and_the_context_recovers(lib, gpu, r):
     z.close()
 
 
+def test_linear_pair_wait_reports_timeout_and_the_context_recovers(lib, gpu):
+    """The SM-pair perturbed-linear launch: with the hook armed its Y tiles wait for S rows
+    that are never counted as written (the row-block counters' epoch is one ahead); every
+    such wait gives up after ~0.1 s, the launch reports a timeout, zo_sync_status zeroes the
+    counters, and the next call is exact again."""
+    import torch
+    from paper_2608_15665_gb300 import binding as zb
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    from oracle import subzero
+    from gpu_util import f32
+    from test_gpu_linear import _check, _tokens
+    base, seed = 50, 7070
+    z = SubZeroPlus([make_weight(304, 520, "bf16", 4, gpu)], 32, 2, seed, matrix_index_base=base)
+    z.init_subspace(0)
+    zb.zo_linear_prepare(z.ctx, 3, 0, 1.0, 1, -1.0, 1e-2)
+    X = _tokens(700, 520, 12, gpu)
+    Y = torch.empty((700, 304), dtype=torch.bfloat16, device=gpu)
+    zb.zo_linear_perturbed(z.ctx, 0, X, Y)          # a normal call first: counters in use
+    z.sync()
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_TEST_WAIT_TIMEOUT, 1)
+    zb.zo_linear_perturbed(z.ctx, 0, X, Y)
+    assert zb.zo_linear_tiling(z.ctx) >= 4
+    with pytest.raises(zb.ZoError) as e:
+        z.sync()
+    assert e.value.status == zb.ZO_ERR_TIMEOUT
+    z.sync()                                         # cleared; the hook was one-shot
+    before = snapshot(z)
+    Y.fill_(float("nan"))
+    zb.zo_linear_perturbed(z.ctx, 0, X, Y)
+    z.sync()
+    C = subzero.perturb_coeff(seed, base, 3, 32, [(0, 1.0), (1, -1.0)], f32(1e-2))
+    _check(Y, X, before["W"][0], before["U"][0], before["V"][0], C, 2.0 * f32(1e-2),
+           "perturbed linear after the expired wait")
+    z.close()
+
+
 def test_wait_hook_needs_the_tensor_core_pass(lib, gpu):
     from paper_2608_15665_gb300 import binding as zb
     from paper_2608_15665_gb300.schedule import SubZeroPlus
