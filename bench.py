@@ -45,8 +45,8 @@ TRAFFIC_BY_SOURCE = {
     # launch, from an ncu capture on a small case of the same workload, scaled by weights
     # profiles/wpass_tc_r32_llama7b_2layers.md: 1.5779 GB on the 2-layer subset, x16.0
     ("a733f29ccdac1cbd", "llama7b_bf16_r32"): 25.25e9,
-    # profiles/wpass_pair_r128_llama7b_2layers.md: 1.6390 GB on the 2-layer subset, x16.0
-    ("541634a914c93b6a", "llama7b_bf16_r128_q99"): 26.22e9,
+    # profiles/wpass_pair_r128_llama7b_2layers.md: 1.6392 GB on the 2-layer subset, x16.0
+    ("45f2d025ab358fe7", "llama7b_bf16_r128_q99"): 26.23e9,
     # profiles/wpass_tmem_r64_dense32b_1layer.md: 1.9271 GB on the 1-layer subset, x64.0
     ("5d6c6cd8669a0a74", "dense32b_bf16_r64"): 123.33e9,
 }
