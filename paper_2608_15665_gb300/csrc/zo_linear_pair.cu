@@ -73,6 +73,12 @@ struct PairLin {
   static constexpr int kTmemCols = 512;
   static constexpr int kChunks = N / 16;                      // 16-column chunks of a row
   static constexpr size_t kSmem = (size_t)kStages * kStageBytes + kOutBytes + 1024 + 1024;
+  // an S tile's stage: as many 64-element panels of X and of P_K's r rows as fit a stage
+  // (its stages are fewer than a Y tile's, so that it ends before the Y tiles need S)
+  template <int R>
+  static constexpr int s_panels() {
+    return kStageBytes / (kAPanel + R * 128) < 4 ? kStageBytes / (kAPanel + R * 128) : 4;
+  }
   static_assert(kStages >= 3, "operand ring");
   static_assert(kSmem <= 227 * 1024, "shared memory per CTA");
   static_assert(kAccStride + N <= kTmemCols, "two accumulators in TMEM");
@@ -196,6 +202,8 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
                    long long wait_cycles) {
   using Cfg = PairLin<N>;
   constexpr int S = Cfg::kStages;
+  constexpr int kSP = Cfg::template s_panels<R>();            // panels per S-tile stage
+  static_assert(kSP >= 2, "S-tile stage");
   static_assert(sizeof(LinPairShared) <= 1024, "barrier block");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -211,6 +219,7 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
   const int tiles_n = (cols + N - 1) / N;
   const int row_blocks = (rows + kPairRows - 1) / kPairRows;
   const int64_t n_tiles = (int64_t)row_blocks * (tiles_n + 1);
+  const int s_stages = (k_steps + kSP - 1) / kSP;              // an S tile's stages
   const PairTiles tiles{row_blocks,
                         StripeOrder{tiles_n, row_blocks, group < 1 || group > tiles_n ? tiles_n : group}};
   const volatile int* abort = &sh.abort_flag;
@@ -252,7 +261,7 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
       const bool s_tile = tiles.decode(tile, tb, nb);
       const int y_a = tb * kPairRows + kBM * (int)rank;
       const int y_b = nb * N + Cfg::kHalfN * (int)rank;
-      for (int k = 0; k < k_stages + (s_tile ? 0 : 1); ++k) {
+      for (int k = 0; k < (s_tile ? s_stages : k_stages + 1); ++k) {
         if (!mbar_wait_bounded(&sh.empty[s], ph ^ 1u, abort, wait_cycles)) {
           ok = false;
           break;
@@ -260,13 +269,15 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
         uint8_t* a_dst = st_smem + s * Cfg::kStageBytes;
         uint8_t* b_dst = a_dst + Cfg::kABytes;
         if (s_tile) {
-          // X panels and this CTA's R rows of P_K (P_hi in CTA 0, P_lo in CTA 1)
-          if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * Cfg::kPanels * (Cfg::kAPanel + R * 128));
+          // kSP panels of X, then this CTA's R rows of P_K for each (P_hi in CTA 0, P_lo in
+          // CTA 1); panels past n read TMA's zero fill
+          if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * kSP * (Cfg::kAPanel + R * 128));
 #pragma unroll
-          for (int p = 0; p < Cfg::kPanels; ++p) {
-            const int x = 64 * (Cfg::kPanels * k + p);
+          for (int p = 0; p < kSP; ++p) {
+            const int x = 64 * (kSP * k + p);
             tma_load_2d_to_leader(a_dst + p * Cfg::kAPanel, &tm_x, x, y_a, &sh.full[s]);
-            tma_load_2d_to_leader(b_dst + p * Cfg::kBPanel, &tm_pk, x, R * (int)rank, &sh.full[s]);
+            tma_load_2d_to_leader(a_dst + kSP * Cfg::kAPanel + p * R * 128, &tm_pk, x, R * (int)rank,
+                                  &sh.full[s]);
           }
         } else if (k < k_stages) {
           // panels past n read TMA's zero fill
@@ -322,7 +333,7 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
       }
       tc_fence_after();                          // the epilogue's reads of this accumulator
       const uint32_t d = tmem + (uint32_t)(acc * Cfg::kAccStride);
-      for (int k = 0; k < k_stages + (s_tile ? 0 : 1); ++k) {
+      for (int k = 0; k < (s_tile ? s_stages : k_stages + 1); ++k) {
         // the operands arrive by TMA on this barrier: its wait orders the MMAs' reads
         if (!mbar_wait_bounded(&sh.full[s], ph, abort, wait_cycles)) {
           ok = false;
@@ -331,13 +342,14 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
         const uint64_t a0 = sdesc_k_sw128(smem_u32(st_smem + s * Cfg::kStageBytes));
         const uint64_t b0 = sdesc_k_sw128(smem_u32(st_smem + s * Cfg::kStageBytes + Cfg::kABytes));
         if (s_tile) {
-          // D[:, :R] = X P_hi^T, D[:, R:2R] = X P_lo^T
+          // D[:, :R] = X P_hi^T, D[:, R:2R] = X P_lo^T; the P_K panels follow the kSP X panels
+          const uint64_t bs = a0 + kSP * kPanelA;
 #pragma unroll
-          for (int p = 0; p < Cfg::kPanels; ++p)
+          for (int p = 0; p < kSP; ++p)
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-              mma_pair_ss(d, a0 + p * kPanelA + kk * kStepK, b0 + p * kPanelB + kk * kStepK, idesc_s,
-                          (k > 0 || p > 0 || kk > 0) ? 1u : 0u);
+              mma_pair_ss(d, a0 + p * kPanelA + kk * kStepK, bs + p * (R * 128 >> 4) + kk * kStepK,
+                          idesc_s, (k > 0 || p > 0 || kk > 0) ? 1u : 0u);
         } else if (k < k_stages) {
 #pragma unroll
           for (int p = 0; p < Cfg::kPanels; ++p)
