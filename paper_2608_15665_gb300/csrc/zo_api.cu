@@ -1073,8 +1073,26 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
   }
   const int32_t r = c->r;
   const int64_t HLW = zo::tc_hl_width(r);
+  // the Y GEMM's tiling: automatic = the pair tiling whose busiest pair has the least
+  // operand traffic (the single-CTA tilings if no cluster of the pair kernel fits), or the
+  // one ZO_OPTION_LINEAR_TILE names
+  if (c->linear_pairs < 0) c->linear_pairs = std::max(0, (int)zo::linear_pair_max_pairs());
+  int32_t tiling = c->linear_tile;
+  if (tiling == 0)
+    tiling = c->linear_pairs > 0 ? zo::linear_pair_tiling(T, m, n, c->r, c->linear_pairs)
+                                 : zo::linear_y_tiling(T, m, c->sms, 0);
+  const int32_t pair_n = zo::linear_pair_cols(tiling);
+  if (pair_n > 0 && c->linear_pairs <= 0) {
+    g_last_error = "zo_linear_perturbed: no cluster of the SM-pair GEMM fits on this device";
+    return ZO_ERR_UNSUPPORTED;
+  }
+  // S's K split: the single-CTA route's S kernel, or the pair launch's S tiles; each writes
+  // k_split x T x r fp32 partials
   int32_t k_split = 1, k_chunk = 1;
-  zo::linear_s_split(T, n, c->sms, &k_split, &k_chunk);
+  if (pair_n > 0)
+    zo::linear_pair_s_split(T, n, c->linear_pairs, &k_split, &k_chunk);
+  else
+    zo::linear_s_split(T, n, c->sms, &k_split, &k_chunk);
   const int64_t part = (int64_t)k_split * T * r;
   if (T > c->s_cap || part > c->part_cap) {
     ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
@@ -1087,15 +1105,16 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
       c->d_s_flags = nullptr;
       c->s_cap = 0;
       const int64_t cap = (T + 127) / 128 * 128;
+      const int64_t n_flags = (cap / 256 + 1) * zo::kLinearPairCounters;
       ZO_CUDA(cudaMalloc(&c->d_s_hl, sizeof(__nv_bfloat16) * cap * HLW), "cudaMalloc(S_HL)");
       ZO_CUDA(cudaMalloc(&c->d_s_count, sizeof(uint32_t) * (cap / 32)), "cudaMalloc(S counters)");
-      ZO_CUDA(cudaMalloc(&c->d_s_flags, sizeof(uint32_t) * (cap / 256 + 1)),
+      ZO_CUDA(cudaMalloc(&c->d_s_flags, sizeof(uint32_t) * n_flags),
               "cudaMalloc(S row-block counters)");
       // on the context's stream: a plain cudaMemset runs on the legacy default stream,
       // which a non-blocking stream's kernels are not ordered after
       ZO_CUDA(cudaMemsetAsync(c->d_s_count, 0, sizeof(uint32_t) * (cap / 32), c->stream),
               "zero S counters");
-      ZO_CUDA(cudaMemsetAsync(c->d_s_flags, 0, sizeof(uint32_t) * (cap / 256 + 1), c->stream),
+      ZO_CUDA(cudaMemsetAsync(c->d_s_flags, 0, sizeof(uint32_t) * n_flags, c->stream),
               "zero S row-block counters");
       c->lin_epoch = 0;
       c->s_cap = cap;
@@ -1107,18 +1126,6 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
       ZO_CUDA(cudaMalloc(&c->d_s_part, sizeof(float) * part), "cudaMalloc(partial S)");
       c->part_cap = part;
     }
-  }
-  // the Y GEMM's tiling: automatic = the pair tiling with the fewest waves (the single-CTA
-  // tilings if no cluster of the pair kernel fits), or the one ZO_OPTION_LINEAR_TILE names
-  if (c->linear_pairs < 0) c->linear_pairs = std::max(0, (int)zo::linear_pair_max_pairs());
-  int32_t tiling = c->linear_tile;
-  if (tiling == 0)
-    tiling = c->linear_pairs > 0 ? zo::linear_pair_tiling(T, m, c->r, c->linear_pairs)
-                                 : zo::linear_y_tiling(T, m, c->sms, 0);
-  const int32_t pair_n = zo::linear_pair_cols(tiling);
-  if (pair_n > 0 && c->linear_pairs <= 0) {
-    g_last_error = "zo_linear_perturbed: no cluster of the SM-pair GEMM fits on this device";
-    return ZO_ERR_UNSUPPORTED;
   }
   const bool narrow_y = pair_n == 0 && zo::linear_y_tile_cols(tiling) % 64 != 0;
   CUtensorMap tm_x{}, tm_pk{}, tm_s{}, tm_y{}, tm_w{}, tm_u{}, tm_pk_half{};
@@ -1149,7 +1156,9 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     // one launch: S = X P^T in its S tiles (one per 256 rows), then Y = X W^T + S U^T
     if (c->lin_epoch + 1 >= zo::kLinearPairEpochs) {
       // the epochs start again: no counter may hold an old call's complete count
-      ZO_CUDA(cudaMemsetAsync(c->d_s_flags, 0, sizeof(uint32_t) * (c->s_cap / 256 + 1), c->stream),
+      ZO_CUDA(cudaMemsetAsync(c->d_s_flags, 0,
+                              sizeof(uint32_t) * (c->s_cap / 256 + 1) * zo::kLinearPairCounters,
+                              c->stream),
               "zero S row-block counters");
       c->lin_epoch = 0;
     }
@@ -1158,7 +1167,8 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     c->inject_wait = false;
     ZO_CUDA(zo::launch_linear_pair(tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk_half, T, m, n,
                                    c->h_tc[mat].u_row0, r, tiling, c->linear_pairs, c->d_s_hl,
-                                   c->d_s_flags, c->lin_epoch, inject, c->d_status, c->stream),
+                                   c->d_s_part, c->d_s_flags, c->lin_epoch, inject, c->d_status,
+                                   c->stream),
             "perturbed linear kernel (SM pairs)");
     c->launches += 1;
   } else {
@@ -1212,7 +1222,9 @@ zo_status zo_sync_status(zo_ctx* c) {
       ZO_CUDA(cudaMemsetAsync(c->d_s_count, 0, sizeof(uint32_t) * (c->s_cap / 32), c->stream),
               "zero S counters");
     if ((s & zo::kDevTimeout) && c->d_s_flags) {
-      ZO_CUDA(cudaMemsetAsync(c->d_s_flags, 0, sizeof(uint32_t) * (c->s_cap / 256 + 1), c->stream),
+      ZO_CUDA(cudaMemsetAsync(c->d_s_flags, 0,
+                              sizeof(uint32_t) * (c->s_cap / 256 + 1) * zo::kLinearPairCounters,
+                              c->stream),
               "zero S row-block counters");
       c->lin_epoch = 0;
     }

@@ -201,24 +201,30 @@ cudaError_t launch_linear_y(const CUtensorMap& tm_x, const CUtensorMap* d_w_map,
 constexpr int32_t kLinearPairTiling0 = 4;
 int32_t linear_pair_cols(int32_t tiling);        // N of a pair tiling, 0 for the others
 int32_t linear_pair_max_pairs();                 // co-resident clusters (0 if unknown)
+// The S tiles' split of K = n into s_split ranges of s_chunk 64-element panels (about one S
+// tile per pair, at most 15 ranges; the same for every pair tiling).
+void linear_pair_s_split(int64_t T, int64_t n, int32_t n_pairs, int32_t* s_split,
+                         int32_t* s_chunk);
 // The pair tiling whose busiest pair has the least work (S and Y tiles dealt round-robin).
-int32_t linear_pair_tiling(int64_t T, int64_t m, int32_t r, int32_t n_pairs);
+int32_t linear_pair_tiling(int64_t T, int64_t m, int64_t n, int32_t r, int32_t n_pairs);
 // One launch computes S = X P^T (S tiles, written to s_hl as S_HL rows) and Y = X W^T +
 // S U^T.  tm_x over X (box 64 x 128), tm_w over W_i (box 64 x N/2), tm_s over s_hl (box
 // 64 x 128), tm_u over the bf16 U operand (box 64 x N/2; W_i's rows from u_row0), tm_y over
-// Y (box 16 x 32, 32-byte swizzle), tm_pk over P_K (box 64 x r).  s_count: one counter per
-// 256 rows of X (zero before the first call), epoch: 1 .. kLinearPairEpochs - 1, a new one
-// per call (the counters of a launch cut short by a wait timeout must be zeroed before
-// the epochs start again).  inject_wait (test hook): the Y tiles wait for a count that
+// Y (box 16 x 32, 32-byte swizzle), tm_pk over P_K (box 64 x r).  s_part: s_split x T x r
+// floats (linear_pair_s_split).  s_count: kLinearPairCounters counters per 256 rows of X
+// (zero before the first call), epoch: 1 .. kLinearPairEpochs - 1, a new one per call (the
+// counters of a launch cut short by a wait timeout must be zeroed before the epochs start
+// again).  inject_wait (test hook): the Y tiles wait for a count that
 // never comes, with the short test limit; the launch then reports kDevTimeout.
 cudaError_t launch_linear_pair(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
                                const CUtensorMap& tm_s, const CUtensorMap& tm_u,
                                const CUtensorMap& tm_y, const CUtensorMap& tm_pk, int64_t T,
                                int64_t m, int64_t n, int32_t u_row0, int32_t r, int32_t tiling,
-                               int32_t n_pairs, __nv_bfloat16* s_hl, uint32_t* s_count,
-                               uint32_t epoch, bool inject_wait, uint32_t* d_status,
-                               cudaStream_t s);
-constexpr uint32_t kLinearPairCountsPerCall = 8;   // S-tile epilogue warps of a pair
+                               int32_t n_pairs, __nv_bfloat16* s_hl, float* s_part,
+                               uint32_t* s_count, uint32_t epoch, bool inject_wait,
+                               uint32_t* d_status, cudaStream_t s);
+constexpr uint32_t kLinearPairCountsPerCall = 8;   // 32-row groups of a 256-row block
+constexpr int32_t kLinearPairCounters = 16;        // counters per 256-row block
 constexpr uint32_t kLinearPairEpochs = 1u << 28;
 
 // ---- refresh of tall panels at r = 16 ... 128: CholeskyQR2 (zo_cholqr.cu) ----------

@@ -92,20 +92,23 @@ struct LinPairShared {
   int abort_flag;
 };
 
-// Row-block counters of the S tiles: (call epoch << 4) | finished S-tile epilogue warps.
-// A warp of call e moves the counter to (e, count + 1), or to (e, 1) from an older call's
-// value (release, GPU scope); the Y tiles of call e wait for (e, 8) (acquire).  Calls
-// whose T covers fewer row blocks leave the others' counters behind, which the epoch
-// makes harmless.
-__device__ __forceinline__ void count_s_warp(uint32_t* f, uint32_t epoch) {
+// Counters of the S tiles, kLinearPairCounters per row block: [0] the row block's ready
+// count (32-row groups whose S_HL rows are written; the Y tiles wait for all 8), [1 + 4 c
+// + g] the K ranges of 32-row group g of CTA c whose fp32 partial rows are written.  Each
+// holds (call epoch << 4) | count: call e moves it to (e, count + 1), or to (e, 1) from an
+// older call's value, with acquire-release semantics at GPU scope (the release publishes
+// the caller's writes, the acquire shows the others' to the one that completes a group).
+// Calls whose T covers fewer row blocks leave the others' counters behind, which the epoch
+// makes harmless.  Returns the new count.
+__device__ __forceinline__ uint32_t count_epoch(uint32_t* f, uint32_t epoch) {
   uint32_t cur;
   asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(cur) : "l"(f) : "memory");
   for (;;) {
     const uint32_t want = (cur >> 4) == epoch ? cur + 1 : (epoch << 4) + 1;
     uint32_t prev;
-    asm volatile("atom.release.gpu.global.cas.b32 %0, [%1], %2, %3;"
+    asm volatile("atom.acq_rel.gpu.global.cas.b32 %0, [%1], %2, %3;"
                  : "=r"(prev) : "l"(f), "r"(cur), "r"(want) : "memory");
-    if (prev == cur) return;
+    if (prev == cur) return want & 15u;
     cur = prev;
   }
 }
@@ -144,8 +147,6 @@ __device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&v)
       : "r"(taddr));
 }
 
-// The launch's tiles: first one S tile per row block (S = X P^T for its 256 rows, written
-// to S_HL), then the Y tiles in stripe order.
 // Pair tile t -> (row block tb, column block nb): column stripes of `group` column blocks,
 // each walked row block by row block (group = the column blocks: plain row-major order).
 // Stripes about one wave of tiles wide keep the wave's W rows few enough to stay in L2
@@ -168,18 +169,21 @@ struct StripeOrder {
   }
 };
 
-// The launch's tiles: first one S tile per row block (S = X P^T for its 256 rows, written
-// to S_HL), then the Y tiles in stripe order.
+// The launch's tiles: first s_split S tiles per row block (S = X P^T for its 256 rows over
+// one of s_split K ranges: with one range its S_HL rows directly, else fp32 partial rows
+// that the last range of each 32-row group sums), then the Y tiles in stripe order.
 struct PairTiles {
-  int row_blocks;
+  int row_blocks, s_split;
   StripeOrder order;
-  __device__ bool decode(int64_t t, int& tb, int& nb) const {   // true: an S tile
-    if (t < row_blocks) {
-      tb = (int)t;
-      nb = 0;
+  // true: an S tile of row block tb over K range nb
+  __device__ bool decode(int64_t t, int& tb, int& nb) const {
+    const int64_t n_s = (int64_t)row_blocks * s_split;
+    if (t < n_s) {
+      tb = (int)(t % row_blocks);
+      nb = (int)(t / row_blocks);
       return true;
     }
-    order.decode(t - row_blocks, tb, nb);
+    order.decode(t - n_s, tb, nb);
     return false;
   }
 };
@@ -188,7 +192,10 @@ struct PairTiles {
 // route's U operand (box 64 x N/2; this matrix's rows from u_row0), tm_y: Y (box 16 x 32,
 // 32-byte swizzle), tm_pk: P_K = [P_hi ; P_lo] (box 64 x R: CTA c loads rows R c ..).
 // rows = T, cols = m, k_steps = ceil(n / 64).  s_hl: the S_HL rows the S tiles write;
-// s_count[tb]: the row block's counter (count_s_warp); epoch: this call's (1 .. 2^28 - 1),
+// s_split K ranges of s_chunk 64-element panels each (the same for every N, so that every
+// pair tiling sums S alike); s_part: s_split x rows x R fp32 partial
+// rows (s_split > 1); s_count: kLinearPairCounters per row block (count_epoch); epoch: this
+// call's (1 .. 2^28 - 1),
 // which its S tiles write; wait_epoch: the one its Y tiles wait for (= epoch; the test hook
 // passes one that never comes, so that every Y tile's bounded wait runs out).
 template <int N, int R>
@@ -196,8 +203,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairLin<N>::kThreads
 linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
                    const __grid_constant__ CUtensorMap tm_s, const __grid_constant__ CUtensorMap tm_u,
                    const __grid_constant__ CUtensorMap tm_y, const __grid_constant__ CUtensorMap tm_pk,
-                   int rows, int cols, int k_steps, int u_row0, int group,
-                   __nv_bfloat16* __restrict__ s_hl, uint32_t* __restrict__ s_count,
+                   int rows, int cols, int k_steps, int u_row0, int group, int s_split,
+                   int s_chunk, __nv_bfloat16* __restrict__ s_hl, float* __restrict__ s_part,
+                   uint32_t* __restrict__ s_count,
                    uint32_t epoch, uint32_t wait_epoch, uint32_t* __restrict__ status,
                    long long wait_cycles) {
   using Cfg = PairLin<N>;
@@ -218,9 +226,8 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
   const int64_t pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
   const int tiles_n = (cols + N - 1) / N;
   const int row_blocks = (rows + kPairRows - 1) / kPairRows;
-  const int64_t n_tiles = (int64_t)row_blocks * (tiles_n + 1);
-  const int s_stages = (k_steps + kSP - 1) / kSP;              // an S tile's stages
-  const PairTiles tiles{row_blocks,
+  const int64_t n_tiles = (int64_t)row_blocks * (tiles_n + s_split);
+  const PairTiles tiles{row_blocks, s_split,
                         StripeOrder{tiles_n, row_blocks, group < 1 || group > tiles_n ? tiles_n : group}};
   const volatile int* abort = &sh.abort_flag;
 
@@ -261,7 +268,12 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
       const bool s_tile = tiles.decode(tile, tb, nb);
       const int y_a = tb * kPairRows + kBM * (int)rank;
       const int y_b = nb * N + Cfg::kHalfN * (int)rank;
-      for (int k = 0; k < (s_tile ? s_stages : k_stages + 1); ++k) {
+      // an S tile's K range (nb = the range; stages of up to kSP panels) or a Y tile's K
+      // steps and its rank-r step
+      const int p_lo = s_tile ? nb * s_chunk : 0;
+      const int p_hi = s_tile ? min(k_steps, p_lo + s_chunk) : 0;
+      const int n_k = s_tile ? (p_hi - p_lo + kSP - 1) / kSP : k_stages + 1;
+      for (int k = 0; k < n_k; ++k) {
         if (!mbar_wait_bounded(&sh.empty[s], ph ^ 1u, abort, wait_cycles)) {
           ok = false;
           break;
@@ -271,10 +283,10 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
         if (s_tile) {
           // kSP panels of X, then this CTA's R rows of P_K for each (P_hi in CTA 0, P_lo in
           // CTA 1); panels past n read TMA's zero fill
-          if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * kSP * (Cfg::kAPanel + R * 128));
-#pragma unroll
-          for (int p = 0; p < kSP; ++p) {
-            const int x = 64 * (kSP * k + p);
+          const int pb = p_lo + kSP * k, np = min(kSP, p_hi - pb);
+          if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * np * (Cfg::kAPanel + R * 128));
+          for (int p = 0; p < np; ++p) {
+            const int x = 64 * (pb + p);
             tma_load_2d_to_leader(a_dst + p * Cfg::kAPanel, &tm_x, x, y_a, &sh.full[s]);
             tma_load_2d_to_leader(a_dst + kSP * Cfg::kAPanel + p * R * 128, &tm_pk, x, R * (int)rank,
                                   &sh.full[s]);
@@ -291,7 +303,8 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
         } else {                               // the rank-r step: S_HL rows, U operand rows
           // this row block's S rows: written by its S tile (both CTAs' epilogues) earlier in
           // this launch
-          if (!wait_s_rows(s_count + tb, wait_epoch, abort, wait_cycles)) {
+          if (!wait_s_rows(s_count + (int64_t)tb * kLinearPairCounters, wait_epoch, abort,
+                           wait_cycles)) {
             ok = false;
             break;
           }
@@ -333,7 +346,10 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
       }
       tc_fence_after();                          // the epilogue's reads of this accumulator
       const uint32_t d = tmem + (uint32_t)(acc * Cfg::kAccStride);
-      for (int k = 0; k < (s_tile ? s_stages : k_stages + 1); ++k) {
+      const int p_lo = s_tile ? nb * s_chunk : 0;
+      const int p_hi = s_tile ? min(k_steps, p_lo + s_chunk) : 0;
+      const int n_k = s_tile ? (p_hi - p_lo + kSP - 1) / kSP : k_stages + 1;
+      for (int k = 0; k < n_k; ++k) {
         // the operands arrive by TMA on this barrier: its wait orders the MMAs' reads
         if (!mbar_wait_bounded(&sh.full[s], ph, abort, wait_cycles)) {
           ok = false;
@@ -344,8 +360,8 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
         if (s_tile) {
           // D[:, :R] = X P_hi^T, D[:, R:2R] = X P_lo^T; the P_K panels follow the kSP X panels
           const uint64_t bs = a0 + kSP * kPanelA;
-#pragma unroll
-          for (int p = 0; p < kSP; ++p)
+          const int np = min(kSP, p_hi - (p_lo + kSP * k));
+          for (int p = 0; p < np; ++p)
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
               mma_pair_ss(d, a0 + p * kPanelA + kk * kStepK, bs + p * (R * 128 >> 4) + kk * kStepK,
@@ -402,8 +418,10 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
       const int y = tb * kPairRows + kBM * (int)rank + 32 * g;
       const uint32_t t_base = tmem + lane_base + (uint32_t)(acc * Cfg::kAccStride);
       if (s_tile) {
-        // S = D[:, :R] + D[:, R:2R] for this lane's row, written as its S_HL row; four warps
-        // per CTA (one per TMEM lane group), then each counts itself done for the row block
+        // this K range's S = D[:, :R] + D[:, R:2R] for this lane's row; four warps per CTA
+        // (one per TMEM lane group).  One range: the S_HL row directly.  Several: the fp32
+        // partial row, and the warp that completes its 32-row group's ranges sums them in
+        // range order and writes the S_HL rows.  Then the group counts as ready.
         if (h == 0) {
           uint32_t v[32];
           tmem_ld_32x32b_x32(t_base, v);
@@ -413,20 +431,58 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
             tmem_ld_32x32b_x32(t_base + 32u, w);
             tmem_ld_wait();
 #pragma unroll
-            for (int q = 0; q < R; ++q) x[q] = 0.f + (__uint_as_float(v[q]) + __uint_as_float(w[q]));
+            for (int q = 0; q < R; ++q) x[q] = __uint_as_float(v[q]) + __uint_as_float(w[q]);
           } else {
             tmem_ld_wait();
 #pragma unroll
-            for (int q = 0; q < R; ++q) x[q] = 0.f + (__uint_as_float(v[q]) + __uint_as_float(v[R + q]));
+            for (int q = 0; q < R; ++q) x[q] = __uint_as_float(v[q]) + __uint_as_float(v[R + q]);
           }
           tc_fence_before();
           __syncwarp();
           if (lane == 0) arrive_leader(&sh.acc_empty[acc]);
-          if (y + lane < rows) write_s_row<R>(s_hl, y + lane, x);
-          fence_async_global();
-          __threadfence();
-          __syncwarp();
-          if (lane == 0) count_s_warp(s_count + tb, epoch);
+          const int row = y + lane;
+          uint32_t* cnt = s_count + (int64_t)tb * kLinearPairCounters;
+          bool last = true;
+          if (s_split > 1) {
+            if (row < rows) {
+              float4* dst = reinterpret_cast<float4*>(s_part + ((int64_t)nb * rows + row) * R);
+#pragma unroll
+              for (int j = 0; j < R / 4; ++j)
+                dst[j] = make_float4(x[4 * j], x[4 * j + 1], x[4 * j + 2], x[4 * j + 3]);
+            }
+            __threadfence();
+            __syncwarp();
+            uint32_t n_done = 0;
+            if (lane == 0) n_done = count_epoch(cnt + 1 + 4 * (int)rank + g, epoch);
+            n_done = __shfl_sync(0xffffffffu, n_done, 0);
+            last = n_done == (uint32_t)s_split;
+            if (last && row < rows) {
+#pragma unroll
+              for (int q = 0; q < R; ++q) x[q] = 0.f;
+              for (int ks = 0; ks < s_split; ++ks) {
+                const float4* src =
+                    reinterpret_cast<const float4*>(s_part + ((int64_t)ks * rows + row) * R);
+#pragma unroll
+                for (int j = 0; j < R / 4; ++j) {
+                  const float4 p4 = __ldcg(src + j);
+                  x[4 * j] += p4.x;
+                  x[4 * j + 1] += p4.y;
+                  x[4 * j + 2] += p4.z;
+                  x[4 * j + 3] += p4.w;
+                }
+              }
+            }
+          } else {
+#pragma unroll
+            for (int q = 0; q < R; ++q) x[q] = 0.f + x[q];
+          }
+          if (last) {
+            if (row < rows) write_s_row<R>(s_hl, row, x);
+            fence_async_global();
+            __threadfence();
+            __syncwarp();
+            if (lane == 0) count_epoch(cnt, epoch);
+          }
         } else {
           __syncwarp();
           if (lane == 0) arrive_leader(&sh.acc_empty[acc]);
@@ -483,16 +539,16 @@ template <int N, int R>
 cudaError_t launch_pair_nr(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
                            const CUtensorMap& tm_s, const CUtensorMap& tm_u,
                            const CUtensorMap& tm_y, const CUtensorMap& tm_pk, int rows, int cols,
-                           int k_steps, int u_row0, int group, __nv_bfloat16* s_hl,
-                           uint32_t* s_count, uint32_t epoch, bool inject_wait, int n_pairs,
-                           uint32_t* d_status, cudaStream_t s) {
+                           int k_steps, int u_row0, int group, int s_split, int s_chunk,
+                           __nv_bfloat16* s_hl, float* s_part, uint32_t* s_count, uint32_t epoch,
+                           bool inject_wait, int n_pairs, uint32_t* d_status, cudaStream_t s) {
   using Cfg = PairLin<N>;
   cudaError_t e = cudaFuncSetAttribute(linear_pair_kernel<N, R>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::kSmem);
   if (e != cudaSuccess) return e;
   linear_pair_kernel<N, R><<<2 * n_pairs, Cfg::kThreads, Cfg::kSmem, s>>>(
-      tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk, rows, cols, k_steps, u_row0, group, s_hl, s_count,
-      epoch, inject_wait ? epoch + 1 : epoch, d_status, inject_wait ? kTestWaitCycles : kWaitCycles);
+      tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk, rows, cols, k_steps, u_row0, group, s_split, s_chunk,
+      s_hl, s_part, s_count, epoch, inject_wait ? epoch + 1 : epoch, d_status, inject_wait ? kTestWaitCycles : kWaitCycles);
   return cudaGetLastError();
 }
 
@@ -540,22 +596,55 @@ int32_t linear_pair_max_pairs() {
   return p;
 }
 
-int32_t linear_pair_tiling(int64_t T, int64_t m, int32_t r, int32_t n_pairs) {
-  // the busiest pair's work, tiles dealt round-robin (the row blocks' S tiles first); a tile
-  // costs the bytes an SM takes in per 128 elements of K, at ~64 B per cycle the rate that
-  // bounds these tiles: 32 KB of X plus N/2 rows of W (Y tiles), or r rows of P_K (S tiles)
+namespace {
+// panels of X and P_K per S-tile stage (PairLin<N>::s_panels<r>() on the host)
+int s_panels_host(int64_t N, int32_t r) {
+  const int64_t stage = 2 * (kBM * 128 + N / 2 * 128);
+  return (int)std::min<int64_t>(4, stage / (kBM * 128 + (int64_t)r * 128));
+}
+int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+}  // namespace
+
+void linear_pair_s_split(int64_t T, int64_t n, int32_t n_pairs, int32_t* s_split,
+                         int32_t* s_chunk) {
+  // about one S tile per pair: K ranges of s_chunk 64-element panels (a multiple of 6, so
+  // that stages of 2 or 3 panels divide them, where K allows), every range non-empty, at most
+  // 15 (the counters' count field); independent of the tile width
+  const int64_t panels = ceil_div(n, 64);
+  const int64_t row_blocks = ceil_div(T, kPairRows);
+  const int64_t want = std::max<int64_t>(
+      1, std::min<int64_t>({std::max<int32_t>(1, n_pairs) / row_blocks, panels, 15}));
+  int64_t chunk = ceil_div(panels, want);
+  if (chunk > 6) chunk = ceil_div(chunk, 6) * 6;
+  *s_chunk = (int32_t)chunk;
+  *s_split = (int32_t)ceil_div(panels, chunk);
+}
+
+int32_t linear_pair_tiling(int64_t T, int64_t m, int64_t n, int32_t r, int32_t n_pairs) {
+  // the busiest pair's work, tiles dealt round-robin (the S tiles first); a tile costs the
+  // bytes an SM takes in, the rate that bounds these tiles (~64 B per cycle): per 128
+  // elements of K 32 KB of X plus N/2 rows of W (Y tiles: all of K and the rank-r step),
+  // per S-tile stage its panels of X and r rows of P_K (S tiles: their K range)
   int32_t best = kLinearPairTiling0;
   int64_t c_best = -1;
-  const int64_t row_blocks = (T + kPairRows - 1) / kPairRows;
+  const int64_t row_blocks = ceil_div(T, kPairRows);
   const int64_t pairs = std::max<int32_t>(1, n_pairs);
+  const int64_t k_stages = ceil_div(ceil_div(n, 64), 2);
   for (int i = 0; i < 5; ++i) {
     const int64_t N = kPairCols[i];
-    const int64_t total = row_blocks * ((m + N - 1) / N + 1);
+    int32_t s_split = 1, s_chunk = 1;
+    linear_pair_s_split(T, n, n_pairs, &s_split, &s_chunk);
+    const int64_t n_s = row_blocks * s_split;
+    const int64_t total = n_s + row_blocks * ceil_div(m, N);
+    const int64_t cost_y = (k_stages + 1) * 2 * (kBM * 128 + N / 2 * 128);
+    // an S tile's panels, rounded up to whole stages of s_panels_host(N, r) panels
+    const int64_t cost_s = ceil_div(s_chunk, s_panels_host(N, r)) * s_panels_host(N, r) *
+                           (kBM * 128 + (int64_t)r * 128);
     int64_t c = 0;
     for (int64_t p = 0; p < std::min(pairs, total); ++p) {
       const int64_t n_tiles = (total - p + pairs - 1) / pairs;      // tiles p, p + pairs, ...
-      const int64_t n_s = p < row_blocks ? (row_blocks - p + pairs - 1) / pairs : 0;
-      c = std::max(c, n_s * (512 + 4 * r) + (n_tiles - n_s) * (512 + 2 * N));
+      const int64_t n_sp = p < n_s ? (n_s - p + pairs - 1) / pairs : 0;
+      c = std::max(c, n_sp * cost_s + (n_tiles - n_sp) * cost_y);
     }
     if (c_best < 0 || c < c_best) {
       c_best = c;
@@ -569,23 +658,26 @@ cudaError_t launch_linear_pair(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
                                const CUtensorMap& tm_s, const CUtensorMap& tm_u,
                                const CUtensorMap& tm_y, const CUtensorMap& tm_pk, int64_t T,
                                int64_t m, int64_t n, int32_t u_row0, int32_t r, int32_t tiling,
-                               int32_t n_pairs, __nv_bfloat16* s_hl, uint32_t* s_count,
-                               uint32_t epoch, bool inject_wait, uint32_t* d_status,
-                               cudaStream_t s) {
+                               int32_t n_pairs, __nv_bfloat16* s_hl, float* s_part,
+                               uint32_t* s_count, uint32_t epoch, bool inject_wait,
+                               uint32_t* d_status, cudaStream_t s) {
   const int32_t N = linear_pair_cols(tiling);
   if (N == 0 || n_pairs <= 0 || (r != 16 && r != 32)) return cudaErrorInvalidValue;
-  const int k_steps = (int)((n + 63) / 64);
-  const int64_t tiles = (T + kPairRows - 1) / kPairRows * ((m + N - 1) / N + 1);
+  const int k_steps = (int)ceil_div(n, 64);
+  int32_t s_split = 1, s_chunk = 1;
+  linear_pair_s_split(T, n, n_pairs, &s_split, &s_chunk);
+  const int64_t row_blocks = ceil_div(T, kPairRows);
+  const int64_t tiles = row_blocks * (ceil_div(m, N) + s_split);
   const int pairs = (int)std::min<int64_t>(tiles, n_pairs);
   // column stripes as wide as one wave of pairs spread over every row block: a wave then
   // shares its few W rows across all of X (measured on the LLaMA-7B shapes: 4 column blocks
   // per stripe at 4096 tokens beat row-major order by 4% (4096 x 4096), 15% (11008 x 4096)
   // and 2% (4096 x 11008))
-  const int64_t row_blocks = (T + kPairRows - 1) / kPairRows;
   const int group = (int)std::max<int64_t>(1, pairs / row_blocks);
 #define ZO_PAIR_Y(NN, RR)                                                                     \
   launch_pair_nr<NN, RR>(tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk, (int)T, (int)m, k_steps, u_row0,  \
-                         group, s_hl, s_count, epoch, inject_wait, pairs, d_status, s)
+                         group, s_split, s_chunk, s_hl, s_part, s_count, epoch, inject_wait,   \
+                         pairs, d_status, s)
   switch (N * 64 + r) {
     case 256 * 64 + 16: return ZO_PAIR_Y(256, 16);
     case 256 * 64 + 32: return ZO_PAIR_Y(256, 32);
