@@ -564,10 +564,17 @@ def run_ours(args):
     z.close()
     if (world == 1 and args.method == "subzero" and args.workload == "llama7b_bf16_r32"
             and not args.layers and not args.no_secondary):
-        # the second shape the weight pass is held to: the 32B-shaped set (r = 64, q = 8)
+        # the second shape the weight pass is held to: the 32B-shaped set (r = 64, q = 8); the
+        # paper's default scale on the 7B shapes (r = 128, K = 99 queries); the linear layers
+        # of one 7B layer evaluated at the perturbed weights without a weight pass
         del weights, z
         torch.cuda.empty_cache()
-        line["secondary"] = {"dense32b_bf16_r64": secondary_32b(dev, local, peak)}
+        line["secondary"] = {
+            "dense32b_bf16_r64": secondary_weight_pass(dev, local, peak, "dense32b_bf16_r64", 2),
+            "llama7b_bf16_r128_q99": secondary_weight_pass(dev, local, peak,
+                                                           "llama7b_bf16_r128_q99", 1),
+            "perturbed_linear_llama7b_4096tok": secondary_linear(dev, local),
+        }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl0, args.scheme)
     if rank == 0:
@@ -577,20 +584,21 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-def secondary_32b(dev, local, peak):
-    """A short measurement of the weight pass on the 32B-shaped set (448 bf16 matrices,
-    31.2 G parameters, r = 64, q = 8, central scheme: 17 passes per step, refresh every 5):
-    one warm-up step (with its refresh), then 2 timed steps with the weight-pass launches
-    timed by CUDA events, and one refresh timed on its own."""
+def secondary_weight_pass(dev, local, peak, name, K):
+    """A short measurement of the weight pass on a second workload -- the 32B-shaped set
+    (448 bf16 matrices, 31.2 G parameters, r = 64, q = 8: 17 passes per step, refresh every
+    5), or the 7B set at the paper's default scale (r = 128, q = 99: 199 passes per step,
+    refresh every 50; the SM-pair kernel): one warm-up step (with its refresh), then K
+    timed steps with the weight-pass launches timed by CUDA events, and one refresh timed
+    on its own."""
     import torch
     from paper_2608_15665_gb300 import binding as zb
     from paper_2608_15665_gb300 import workloads
     from paper_2608_15665_gb300.schedule import SubZeroPlus, step_plan
-    wl = workloads.get("dense32b_bf16_r64")
+    wl = workloads.get(name)
     weights = [workloads.init_weight(wl, i, dev) for i in range(wl.n_mats)]
     z = SubZeroPlus(weights, wl.r, wl.q, wl.seed)
     calls, (rq, rc) = step_plan("central", wl.q)
-    K = 2
     table = torch.from_numpy(workloads.loss_table(wl, "central", steps=1 + K)).to(dev)
 
     def do_step(t):
@@ -633,7 +641,8 @@ def secondary_32b(dev, local, peak):
     step_ms = window_ms / K + refresh_ms / wl.F
     return {"workload": wl.name, "matrices": wl.n_mats, "params": wl.params, "r": wl.r, "q": wl.q,
             "passes_per_step": 2 * wl.q + 1, "refresh_every": wl.F, "steps_timed": K,
-            "kernel": {2: "wpass_tmem", 1: "wpass_fma"}.get(path, "?"),
+            "kernel": {2: "wpass_pair" if wl.r == 128 else "wpass_tmem" if wl.r == 64
+                       else "wpass_tc", 1: "wpass_fma"}.get(path, "?"),
             "avg_launch_ms": avg_s * 1e3, "launches_timed": wpass_n,
             "algorithmic_bytes_per_launch": wl.bytes_per_pass(),
             "achieved_gbs": achieved, "peak_gbs": peak, "frac": achieved / peak,
@@ -642,28 +651,21 @@ def secondary_32b(dev, local, peak):
             "clocks": clk}
 
 
-def run_linear(args):
-    """The linear layers of the first `--layers` (default 1) layers of the workload at the
-    perturbed weights, Y_i = X_i (W_i + U_i C V_i^T)^T with no weight pass (the forward
-    route of one loss evaluation: C_i and P_i once, then S = X P^T and X W^T + S U^T per
-    layer).
-    X_i: --tokens x n_i bf16 activations, N(0, 1), resident.  A step is one
-    zo_linear_prepare and the layer's zo_linear_perturbed calls.  value = TFLOP/s of the
-    exact-arithmetic work 2 T (m n + r (m + n)) per layer; roofline against the measured
-    bf16 tensor peak.  For context, the same GEMMs without the perturbation (torch, i.e.
-    cuBLAS) and the weight-pass route (one zo_perturb pass over the layer, then those
-    GEMMs) are timed too."""
+def linear_measure(dev, wl, T, K, W, compare=True, e2e=True):
+    """The linear layers of `wl` (one layer's matrices) at the perturbed weights,
+    Y_i = X_i (W_i + U_i C V_i^T)^T with no weight pass (the forward route of one loss
+    evaluation: C_i and P_i once, then S = X P^T and X W^T + S U^T per layer), on
+    X_i: T x n_i bf16 activations, N(0, 1), resident.  A step is one zo_linear_prepare and
+    the layer's zo_linear_perturbed calls; W untimed warm-up steps, K timed ones (CUDA
+    events).  With compare: the same route on single-CTA tiles, the same GEMMs without the
+    perturbation (torch, i.e. cuBLAS) and the weight-pass route (one zo_perturb pass over
+    the layer, then those GEMMs).  With e2e: the route with the activations copied from
+    pinned host memory every step and one output row read back."""
     import torch
-    torch.cuda.set_device(0)
-    dev = torch.device("cuda", 0)
-    from paper_2608_15665_gb300 import build
-    build.build()
     from paper_2608_15665_gb300 import binding as zb
     from paper_2608_15665_gb300 import workloads
     from paper_2608_15665_gb300.schedule import SubZeroPlus
 
-    wl = subset(workloads.get(args.workload), args.layers or 1)
-    T = args.tokens
     weights = [workloads.init_weight(wl, i, dev) for i in range(wl.n_mats)]
     z = SubZeroPlus(weights, wl.r, wl.q, wl.seed)
     z.init_subspace(0)
@@ -671,7 +673,7 @@ def run_linear(args):
     X = {n: torch.randn(T, n, generator=g, device=dev).to(torch.bfloat16)
          for n in sorted({n for _, n in wl.shapes})}
     Y = [torch.empty(T, m, dtype=torch.bfloat16, device=dev) for m, _ in wl.shapes]
-    flops = sum(2.0 * T * (m * n + wl.r * (m + n)) for m, n in wl.shapes)
+    out = {"flops": sum(2.0 * T * (m * n + wl.r * (m + n)) for m, n in wl.shapes)}
 
     def fused(t):
         zb.zo_linear_prepare(z.ctx, t, 0, 1.0, -1, 0.0, wl.eps)
@@ -692,85 +694,127 @@ def run_linear(args):
         torch.cuda.synchronize()
         return e0.elapsed_time(e1) / K
 
-    K, W = args.steps, args.warmup
     for k in range(W):
         fused(k)
         plain()
     z.sync()
     launches0 = zb.zo_kernel_launches(z.ctx)
-    clocks = ClockSampler(0)
+    clocks = ClockSampler(dev.index or 0)
     clocks.start()
-    fused_ms = timed(fused, K)
-    clk = clocks.stop()
-    launches = zb.zo_kernel_launches(z.ctx) - launches0
+    out["fused_ms"] = timed(fused, K)
+    out["clocks"] = clocks.stop()
+    out["launches"] = zb.zo_kernel_launches(z.ctx) - launches0
     z.sync()
     names = {1: "128x256", 2: "256x256", 3: "256x224", 4: "256x256 pair", 5: "256x240 pair",
              6: "256x224 pair", 7: "256x192 pair", 8: "256x128 pair"}
-    tiling = []
+    out["tiling"] = []
     for i, (m, n) in enumerate(wl.shapes):
         zb.zo_linear_perturbed(z.ctx, i, X[n], Y[i])
-        tiling.append(names[zb.zo_linear_tiling(z.ctx)])
-    # for context: the same route with the single-CTA 128 x 256 and 256 x 224 tiles throughout
-    zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 1)
-    fused128_ms = timed(fused, K)
-    zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 3)
-    fused224_ms = timed(fused, K)
-    zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 0)
-    z.sync()
-    plain_ms = timed(lambda k: plain(), K)
-    wpass_ms = timed(lambda k: (z.perturb(k, 0, 1.0, -1, 0.0, wl.eps), plain()), K)
-    z.sync()
+        out["tiling"].append(names[zb.zo_linear_tiling(z.ctx)])
+    if compare:
+        # the same route with the single-CTA 128 x 256 and 256 x 224 tiles throughout
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 1)
+        out["fused128_ms"] = timed(fused, K)
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 3)
+        out["fused224_ms"] = timed(fused, K)
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 0)
+        z.sync()
+        out["plain_ms"] = timed(lambda k: plain(), K)
+        out["wpass_ms"] = timed(lambda k: (z.perturb(k, 0, 1.0, -1, 0.0, wl.eps), plain()), K)
+        z.sync()
+    if e2e:
+        host = {n: x.cpu().pin_memory() for n, x in X.items()}
+        out_row = torch.empty(wl.shapes[-1][0], dtype=torch.bfloat16).pin_memory()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for k in range(K):
+            for n, h in host.items():
+                X[n].copy_(h, non_blocking=True)
+            fused(k)
+            out_row.copy_(Y[-1][0])
+        torch.cuda.synchronize()
+        out["e2e_s"] = (time.perf_counter() - t0) / K
+        out["h2d"] = sum(h.numel() * 2 for h in host.values())
+        out["d2h"] = int(out_row.numel() * 2)
+    z.close()
+    del weights, X, Y, z
+    torch.cuda.empty_cache()
+    return out
 
-    # end to end: the activations copied from pinned host memory every step, one output row
-    # read back
-    host = {n: x.cpu().pin_memory() for n, x in X.items()}
-    out_row = torch.empty(wl.shapes[-1][0], dtype=torch.bfloat16).pin_memory()
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    for k in range(K):
-        for n, h in host.items():
-            X[n].copy_(h, non_blocking=True)
-        fused(k)
-        out_row.copy_(Y[-1][0])
-    torch.cuda.synchronize()
-    e2e_s = (time.perf_counter() - t0) / K
-    h2d = sum(h.numel() * 2 for h in host.values())
 
-    peak = None
+def linear_peak():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             mp = json.load(f)
         # the layer's GEMMs run back to back for tens of ms: the sustained figure
         peak = float(mp.get("bf16_tflops_sustained") or 0.0) or None
-        peak_kind = "measured (cuBLAS bf16, sustained)"
+        if peak:
+            return peak, "measured (cuBLAS bf16, sustained)"
     except Exception:
-        peak_kind = "unavailable"
-    if peak is None:
-        peak, peak_kind = 1700.0, "fallback (sustained)"
-    achieved = flops / (fused_ms / 1e3) / 1e12
+        pass
+    return 1700.0, "fallback (sustained)"
+
+
+def secondary_linear(dev, local):
+    """The perturbed-linear route (zo_linear_perturbed, no weight pass) on one LLaMA-7B
+    layer's seven matrices at 4096 tokens, r = 32: 10 timed steps after 2 warm-up ones,
+    with the weight-pass route and the plain cuBLAS GEMMs timed beside it."""
+    from paper_2608_15665_gb300 import workloads
+    wl = subset(workloads.get("llama7b_bf16_r32"), 1)
+    T = 4096
+    m = linear_measure(dev, wl, T, K=10, W=2, compare=True, e2e=False)
+    peak, peak_kind = linear_peak()
+    achieved = m["flops"] / (m["fused_ms"] / 1e3) / 1e12
+    return {"workload": wl.name, "tokens": T, "r": wl.r, "tiles": m["tiling"],
+            "ms_per_step": m["fused_ms"], "tflops": achieved, "peak_tflops": peak,
+            "frac": achieved / peak, "peak_kind": peak_kind,
+            "kernel": "linear_pair_kernel" if any("pair" in t for t in m["tiling"])
+            else "linear_kernel",
+            "weight_pass_route_ms": m["wpass_ms"], "plain_gemm_ms": m["plain_ms"],
+            "single_cta_256x224_ms": m["fused224_ms"], "clocks": m["clocks"]}
+
+
+def run_linear(args):
+    """bench.py --method linear: the linear layers of the first `--layers` (default 1)
+    layers of the workload at the perturbed weights (linear_measure), --tokens rows of
+    activations.  value = TFLOP/s of the exact-arithmetic work 2 T (m n + r (m + n)) per
+    layer; roofline against the measured bf16 tensor peak."""
+    import torch
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    from paper_2608_15665_gb300 import build
+    build.build()
+    from paper_2608_15665_gb300 import workloads
+
+    wl = subset(workloads.get(args.workload), args.layers or 1)
+    T = args.tokens
+    K, W = args.steps, args.warmup
+    m = linear_measure(dev, wl, T, K, W)
+    peak, peak_kind = linear_peak()
+    flops = m["flops"]
+    achieved = flops / (m["fused_ms"] / 1e3) / 1e12
     line = {
         "metric": "perturbed linear forward TFLOP/s (zo_linear_perturbed, LLaMA-7B layer shapes, 1 GB300)",
         "value": achieved, "unit": "TFLOP/s", "n_gpus": 1, "steps": K, "warmup": W,
-        "ms_per_step": fused_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "ms_per_step": m["fused_ms"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic",
         "config": {"workload": wl.name, "matrices": wl.n_mats, "tokens": T, "r": wl.r,
-                   "method": "linear", "tiles": tiling,
-                   "l2": "inputs larger than L2 (%.0f MB of weights)" % (sum(m * n for m, n in wl.shapes) * 2 / 1e6),
+                   "method": "linear", "tiles": m["tiling"],
+                   "l2": "inputs larger than L2 (%.0f MB of weights)" % (sum(mm * n for mm, n in wl.shapes) * 2 / 1e6),
                    "parallelism": "single GPU"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "peak_kind": peak_kind, "traffic": None,
-                     "kernel": "linear_pair_kernel" if any("pair" in t for t in tiling)
+                     "kernel": "linear_pair_kernel" if any("pair" in t for t in m["tiling"])
                      else "linear_kernel", "algorithmic_flops_per_step": flops},
-        "tile128_ms": fused128_ms,
-        "tile224_single_cta_ms": fused224_ms,
-        "plain_gemm_ms": plain_ms,
-        "weight_pass_route_ms": wpass_ms,
-        "e2e": {"value": flops / e2e_s / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": int(h2d),
-                "d2h_bytes_per_step": int(out_row.numel() * 2)},
-        "clocks": clk,
-        "gpu_launches": int(launches),
+        "tile128_ms": m["fused128_ms"],
+        "tile224_single_cta_ms": m["fused224_ms"],
+        "plain_gemm_ms": m["plain_ms"],
+        "weight_pass_route_ms": m["wpass_ms"],
+        "e2e": {"value": flops / m["e2e_s"] / 1e12, "unit": "TFLOP/s",
+                "h2d_bytes_per_step": int(m["h2d"]), "d2h_bytes_per_step": m["d2h"]},
+        "clocks": m["clocks"],
+        "gpu_launches": int(m["launches"]),
     }
-    z.close()
     print(json.dumps(line), flush=True)
 
 
