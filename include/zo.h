@@ -118,7 +118,7 @@ enum {
                                128 on SM pairs (M = 256 MMAs across a 2-CTA cluster, S in
                                the same launch).  The tilings of one family give
                                bit-identical Y; the two families may differ in the last
-                               bits of S (one K range against split-K partial sums). */
+                               bits of S (each splits S's K in ranges of its own). */
   ZO_OPTION_PAIR_MMA = 4    /* tensor-core weight pass at r = 128: 1 (default) = M = 256 MMAs
                                across the two SMs of a cluster (each SM holds and reads half
                                of every P tile), 0 = the single-SM kernel.  Both give

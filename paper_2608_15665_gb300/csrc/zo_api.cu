@@ -1035,15 +1035,11 @@ zo_status zo_linear_prepare(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t
   ZO_CUDA(zo::launch_coeff(c->d_mats, c->n_mats, p, c->stream), "coefficient kernel");
   ZO_CUDA(zo::launch_split_c(c->d_mats, c->n_mats, r, c->d_amax, c->d_c_hl, c->d_pinv, c->stream),
           "split C");
-  ZO_CUDA(zo::launch_project_tc(c->tm_v, c->tm_c, c->tm_p, c->d_tc, c->d_proj_units,
-                                c->n_proj_units, std::min<int32_t>(c->n_proj_units, c->sms), r,
-                                c->d_status, c->stream),
-          "tensor-core projection kernel");
-  ZO_CUDA(zo::launch_transpose_p(c->d_p_hl, c->d_tc, c->d_proj_units, c->n_proj_units,
-                                 c->d_pk_off, c->d_pinv, (int32_t)zo::tc_hl_width(r), r, c->d_pk,
-                                 c->stream),
-          "P transpose");
-  c->launches += 4;
+  ZO_CUDA(zo::launch_project_tc_pk(c->tm_v, c->tm_c, c->d_tc, c->d_proj_units, c->n_proj_units,
+                                   std::min<int32_t>(c->n_proj_units, c->sms), r, c->d_pinv,
+                                   c->d_pk_off, c->d_pk, c->d_status, c->stream),
+          "tensor-core projection kernel (P_K)");
+  c->launches += 3;
   c->linear_ready = true;
   return ZO_OK;
 }

@@ -156,6 +156,12 @@ cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
                               const CUtensorMap& tm_p, const TcMat* d_tc, const int2* d_units,
                               int32_t n_units, int32_t grid, int32_t r, uint32_t* d_status,
                               cudaStream_t s);
+// The same projection writing, instead of P_HL, P_K = the K-major bf16 pair [P_hi ; P_lo]
+// of P_i at p_k + pk_off[i] (rows of n_i rounded up to 64; r in {16, 32}), from pinv.
+cudaError_t launch_project_tc_pk(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
+                                 const TcMat* d_tc, const int2* d_units, int32_t n_units,
+                                 int32_t grid, int32_t r, const float* pinv, const int64_t* pk_off,
+                                 __nv_bfloat16* p_k, uint32_t* d_status, cudaStream_t s);
 
 // ---- a linear layer at the perturbed weights, without a weight pass (zo_linear.cu) -----
 // Y = X (W + U C V^T)^T = X W^T + S U^T, S = X P^T, for bf16 contexts at r in {16, 32}.
@@ -170,11 +176,6 @@ int32_t linear_y_tile_rows(int32_t tiling);
 int32_t linear_y_tile_cols(int32_t tiling);
 // Elements of matrix i's P_K: 2r rows of n rounded up to 64.
 int64_t linear_pk_elems(int64_t n, int32_t r);
-// P_K of every matrix ([P_hi ; P_lo], the bf16 pair of P) from P_HL and pinv (units = the
-// projection units, pk_off = element offsets).
-cudaError_t launch_transpose_p(const uint16_t* p_hl, const TcMat* d_tc, const int2* d_units,
-                               int32_t n_units, const int64_t* d_pk_off, const float* d_pinv,
-                               int32_t hl_width, int32_t r, __nv_bfloat16* p_k, cudaStream_t s);
 // Kernels launch_linear_s launches for a split of k_split K ranges (1, or 2 with the
 // separate reduction).
 int32_t linear_s_launches(int32_t k_split);

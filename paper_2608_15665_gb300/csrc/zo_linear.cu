@@ -32,8 +32,8 @@
 //           columns at a time through 64-byte-swizzled boxes): 4096 columns make 19 of
 //           them, so 16 or 8 row blocks make exactly two or one wave on 152 SMs.
 //           linear_y_tiling picks the tiling with the fewest waves of tile work.
-// P_K is P_HL (the projection's rows [P_hi(j, :) | P_lo(j, :)], j < n) transposed by
-// transpose_p_kernel, for every matrix once per loss evaluation (zo_linear_prepare).
+// P_K, the K-major bf16 pair [P_hi ; P_lo] of P, is written by the tensor-core projection
+// (zo_project_tc.cu) for every matrix once per loss evaluation (zo_linear_prepare).
 // Ragged edges: TMA zero-fills loads past T, n and m; Y's stores are clipped to T rows and
 // m columns (m a multiple of 8, so that no 16-byte chunk reaches past Y's columns).
 //
@@ -443,46 +443,6 @@ linear_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ 
   }
 }
 
-// P_K of every matrix: rows [P_hi ; P_lo] of the bf16 pair of P_i (P_hi = bf16(P),
-// P_lo = bf16(P - P_hi)), K-major: P_K_i[k][j] and P_K_i[r + k][j] for k < r, j < n_i, at
-// pk_off[i] with row stride ld_i = n_i rounded up to 64.  P comes from the projection's
-// scaled fp16 pair, P = (hi + lo) pinv[i] (exact in fp32 up to the pair's rounding).  One
-// CTA per projection unit (matrix, 128 columns j), through shared memory.
-__global__ void __launch_bounds__(256)
-transpose_p_kernel(const uint16_t* __restrict__ p_hl, const TcMat* __restrict__ tcm,
-                   const int2* __restrict__ units, const int64_t* __restrict__ pk_off,
-                   const float* __restrict__ pinv, int hl_width, int r2,
-                   __nv_bfloat16* __restrict__ p_k) {
-  __shared__ __nv_bfloat16 t[128][66];
-  const int2 u = units[blockIdx.x];
-  const int64_t n = tcm[u.x].n;
-  const int64_t p_row0 = tcm[u.x].p_row0;
-  const int64_t ld = (n + 63) / 64 * 64;
-  const int64_t j0 = u.y;
-  const int r = r2 / 2;
-  const float unscale = pinv[u.x];
-  __nv_bfloat16* dst = p_k + pk_off[u.x];
-  for (int e = threadIdx.x; e < 128 * 32; e += blockDim.x) {
-    const int jj = e / 32, k = e % 32;
-    if (k < r) {
-      float x = 0.f;
-      if (j0 + jj < n) {
-        const uint16_t* row = p_hl + (p_row0 + j0 + jj) * hl_width;
-        x = (__half2float(__ushort_as_half(row[k])) + __half2float(__ushort_as_half(row[r + k]))) *
-            unscale;
-      }
-      const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-      t[jj][k] = hi;
-      t[jj][r + k] = __float2bfloat16_rn(x - __bfloat162float(hi));
-    }
-  }
-  __syncthreads();
-  for (int e = threadIdx.x; e < 128 * 64; e += blockDim.x) {
-    const int k = e / 128, jj = e % 128;
-    if (k < r2 && j0 + jj < n) dst[(int64_t)k * ld + j0 + jj] = t[jj][k];
-  }
-}
-
 // S_HL[row] = [hi | lo | 0] of the sum over the K ranges of the fp32 partial rows of S
 // (k_split > kFusedSplits): thread (row, g) adds columns 8 g .. 8 g + 7 in K-range order.
 template <int R>
@@ -563,15 +523,6 @@ int32_t linear_y_tile_rows(int32_t tiling) { return tiling == 1 ? 128 : 256; }
 int32_t linear_y_tile_cols(int32_t tiling) { return tiling == 3 ? 224 : 256; }
 
 int64_t linear_pk_elems(int64_t n, int32_t r) { return 2 * (int64_t)r * ((n + 63) / 64 * 64); }
-
-cudaError_t launch_transpose_p(const uint16_t* p_hl, const TcMat* d_tc, const int2* d_units,
-                               int32_t n_units, const int64_t* d_pk_off, const float* d_pinv,
-                               int32_t hl_width, int32_t r, __nv_bfloat16* p_k, cudaStream_t s) {
-  if (n_units <= 0 || r > 32) return n_units <= 0 ? cudaSuccess : cudaErrorInvalidValue;
-  transpose_p_kernel<<<n_units, 256, 0, s>>>(p_hl, d_tc, d_units, d_pk_off, d_pinv, hl_width, 2 * r,
-                                             p_k);
-  return cudaGetLastError();
-}
 
 cudaError_t launch_linear_s(const CUtensorMap& tm_x, const CUtensorMap& tm_pk, int64_t T,
                             int64_t n, int32_t r, int32_t k_split, int32_t k_chunk, float* part,

@@ -22,6 +22,10 @@
 //                   the fp32 row of D, scale and split it into fp16 hi/lo, write them as 32 x 64
 //                   boxes of P_HL into shared memory (128-byte swizzle) and TMA-store
 //                   them, 64 columns of D at a time (one hi and one lo box staged).
+//                   For the perturbed-linear route (kPK, r <= 32) it writes instead the
+//                   K-major bf16 pair [P_hi ; P_lo] of P (P_K): the exact fp32 P of D (a
+//                   power-of-two rescale) split into bf16 hi = bf16(P), lo = bf16(P - hi),
+//                   row k of P_K taking column j from lane j (64 contiguous bytes a warp).
 // Every mbarrier wait is bounded; on expiry the kernel records kDevTimeout in the
 // status word, lets the other roles stop, drains its copies and frees TMEM.
 #include <cuda.h>
@@ -86,12 +90,16 @@ __device__ __forceinline__ void proj_give_up(ProjShared& sh, uint32_t* status) {
   *reinterpret_cast<volatile int*>(&sh.abort_flag) = 1;
 }
 
-template <int R>
+// kPK: write P_K at p_k + pk_off[i] (rows of n_i rounded up to 64) from pinv (2^-(e_P,i),
+// written by the C split) instead of P_HL.
+template <int R, bool kPK>
 __global__ void __launch_bounds__(kProjThreads, 1)
 project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_c,
                   const __grid_constant__ CUtensorMap tm_p, const TcMat* __restrict__ mats,
                   const int2* __restrict__ units, int n_units, uint32_t* __restrict__ status,
-                  long long wait_cycles) {
+                  long long wait_cycles, __nv_bfloat16* __restrict__ p_k,
+                  const int64_t* __restrict__ pk_off, const float* __restrict__ pinv) {
+  static_assert(!kPK || R <= 32, "P_K exists for r <= 32");
   using Cfg = ProjCfg<R>;
   static_assert(sizeof(ProjShared) <= 1024, "barrier block");
   static_assert(Cfg::kSmem <= 227 * 1024, "shared memory per CTA");
@@ -246,7 +254,29 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
       // the previous unit's stores have finished reading this warp's boxes
       if (lane == 0) bulk_wait_read_all();
       __syncwarp();
-      if constexpr (R <= 32) {
+      if constexpr (kPK) {
+        uint32_t v[R];
+        if constexpr (R == 32)
+          tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R), v);
+        else
+          tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)(acc * R), v);
+        tmem_ld_wait();
+        // D 2^-(kUVScaleExp + e_C,i) = P exactly (both factors powers of two)
+        const float unscale = p_scale * pinv[un.x];
+        const int64_t n = mats[un.x].n;
+        const int64_t ld = (n + 63) / 64 * 64;
+        const int64_t j = un.y + 32 * g + lane;
+        if (j < n) {
+          __nv_bfloat16* dst = p_k + pk_off[un.x] + j;
+#pragma unroll
+          for (int k = 0; k < R; ++k) {
+            const float x = __uint_as_float(v[k]) * unscale;
+            const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+            dst[k * ld] = hi;
+            dst[(R + k) * ld] = __float2bfloat16_rn(x - __bfloat162float(hi));
+          }
+        }
+      } else if constexpr (R <= 32) {
         // one 64-wide box per row: hi at columns 8 j, lo at R + 8 j, zeros past 2R
         uint32_t v[R];
         if constexpr (R == 32)
@@ -386,16 +416,19 @@ split_rows_kernel(const MatDesc* __restrict__ mats, const TcMat* __restrict__ tc
   }
 }
 
-template <int R>
+template <int R, bool kPK>
 cudaError_t launch_project_tc_r(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
                                 const CUtensorMap& tm_p, const TcMat* d_tc, const int2* d_units,
-                                int32_t n_units, int32_t grid, uint32_t* d_status, cudaStream_t s) {
+                                int32_t n_units, int32_t grid, uint32_t* d_status, cudaStream_t s,
+                                __nv_bfloat16* p_k = nullptr, const int64_t* pk_off = nullptr,
+                                const float* pinv = nullptr) {
   const size_t smem = ProjCfg<R>::kSmem;
-  cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<R>,
+  cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<R, kPK>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  project_tc_kernel<R><<<grid, kProjThreads, smem, s>>>(tm_v, tm_c, tm_p, d_tc, d_units, n_units,
-                                                        d_status, kWaitCycles);
+  project_tc_kernel<R, kPK><<<grid, kProjThreads, smem, s>>>(tm_v, tm_c, tm_p, d_tc, d_units,
+                                                             n_units, d_status, kWaitCycles, p_k,
+                                                             pk_off, pinv);
   return cudaGetLastError();
 }
 
@@ -447,10 +480,22 @@ cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
                               cudaStream_t s) {
   if (n_units <= 0) return cudaSuccess;
   switch (r) {
-    case 16: return launch_project_tc_r<16>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
-    case 32: return launch_project_tc_r<32>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
-    case 64: return launch_project_tc_r<64>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
-    case 128: return launch_project_tc_r<128>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
+    case 16: return launch_project_tc_r<16, false>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
+    case 32: return launch_project_tc_r<32, false>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
+    case 64: return launch_project_tc_r<64, false>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
+    case 128: return launch_project_tc_r<128, false>(tm_v, tm_c, tm_p, d_tc, d_units, n_units, grid, d_status, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_project_tc_pk(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
+                                 const TcMat* d_tc, const int2* d_units, int32_t n_units,
+                                 int32_t grid, int32_t r, const float* pinv, const int64_t* pk_off,
+                                 __nv_bfloat16* p_k, uint32_t* d_status, cudaStream_t s) {
+  if (n_units <= 0) return cudaSuccess;
+  switch (r) {
+    case 16: return launch_project_tc_r<16, true>(tm_v, tm_c, tm_v, d_tc, d_units, n_units, grid, d_status, s, p_k, pk_off, pinv);
+    case 32: return launch_project_tc_r<32, true>(tm_v, tm_c, tm_v, d_tc, d_units, n_units, grid, d_status, s, p_k, pk_off, pinv);
     default: return cudaErrorInvalidValue;
   }
 }

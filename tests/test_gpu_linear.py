@@ -88,7 +88,8 @@ def test_perturbed_linear_matches_oracle_and_leaves_W(lib, gpu, case, eps):
                 out[tiling] = Ybuf[:, :m]
             # the tilings of one family sum each output in the same order: the single-CTA
             # ones take S from the split-K S kernel, the SM-pair ones from their own S tiles
-            # (one K range), so the two families may differ in S's last bits
+            # (K ranges of 64-element panels, the same for every pair tiling), so the two
+            # families may differ in S's last bits
             for tiling in TILINGS:
                 ref = 2 if tiling <= 3 else 6
                 assert torch.equal(out[tiling].view(torch.int16), out[ref].view(torch.int16)), tiling
