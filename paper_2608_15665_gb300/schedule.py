@@ -9,7 +9,11 @@ loss -- and the restore term handed to zo_step:
     +Z_0 | -2 Z_0 | +Z_0 +Z_1 | -2 Z_1 | ... | -2 Z_(q-1)   then restore +Z_(q-1)
 * forward scheme (Alg. 3, Eq. (6)): evaluate at W + eps Z_k (after one at W):
     +Z_0 | +Z_1 -Z_0 | ... | +Z_(q-1) -Z_(q-2)              then restore -Z_(q-1)
-Each entry is ((qa, ca), (qb, cb) or None).  No arithmetic happens here.
+Each entry is ((qa, ca), (qb, cb) or None).  ``linear_plan`` lists the same evaluation
+points for the route that never writes the perturbation into W (zo_linear_prepare /
+zo_linear_perturbed feed W + eps U Z V^T straight into the forward GEMMs): there each entry
+is the absolute perturbation of one loss evaluation, and zo_step then has nothing to
+restore.  No arithmetic happens here.
 """
 
 import torch
@@ -31,6 +35,16 @@ def step_plan(scheme, q):
         calls = [((0, 1.0), None)] + [((k, 1.0), (k - 1, -1.0)) for k in range(1, q)]
         return calls, (q - 1, -1.0)
     raise ValueError(f"no pass plan for scheme {scheme!r}")
+
+
+def linear_plan(scheme, q):
+    """The loss evaluations of one step on the perturbed-linear route: ((qa, ca), None) for
+    the evaluation at W + eps ca Z_qa (ca = 0: at W itself)."""
+    if scheme == "central":
+        return [((k, c), None) for k in range(q) for c in (1.0, -1.0)]
+    if scheme == "forward":
+        return [((0, 0.0), None)] + [((k, 1.0), None) for k in range(q)]
+    raise ValueError(f"no evaluation plan for scheme {scheme!r}")
 
 
 class SubZeroPlus:
@@ -65,6 +79,20 @@ class SubZeroPlus:
         zb.zo_step(self.ctx, t, adam_t, losses, SCHEMES[scheme], eps, lr, beta1, beta2, eps_adam,
                    restore_query, restore_coef, optimizer, gamma_out)
 
+    def linear_prepare(self, t, qa, ca, qb=-1, cb=0.0, eps=1e-3):
+        """Prepare the linear layers' evaluation at W + eps (ca Z_qa + cb Z_qb) (every W
+        left as it is)."""
+        zb.zo_linear_prepare(self.ctx, t, qa, ca, qb, cb, eps)
+
+    def linear_perturbed(self, i, X, Y=None):
+        """Y = X (W_i + U_i C V_i^T)^T for the prepared C (bf16 X of T x n_i; Y allocated
+        as T x m_i bf16 if not given)."""
+        if Y is None:
+            Y = torch.empty(X.shape[0], self.weights[i].shape[0], dtype=torch.bfloat16,
+                            device=X.device)
+        zb.zo_linear_perturbed(self.ctx, i, X, Y)
+        return Y
+
     def mezo_perturb(self, t, coef):
         """Full-space SPSA pass of Eq. (1): every W_i <- rnd(W_i + coef Z_i)."""
         zb.zo_mezo_perturb(self.ctx, t, coef)
@@ -96,5 +124,19 @@ class SubZeroPlus:
             self.perturb(t, qa, ca, qb, cb, eps)
             losses.append(loss_fn(t, len(losses)))
         self.step(t, adam_t, losses, scheme, eps, lr, beta1, beta2, eps_adam, rq, rc, optimizer,
+                  gamma_out)
+        return losses
+
+    def run_step_linear(self, t, adam_t, loss_fn, scheme, eps, lr, beta1, beta2, eps_adam,
+                        optimizer=zb.ZO_OPT_ADAM, gamma_out=None):
+        """Alg. 3 for one step with every loss evaluated at the perturbed weights inside the
+        forward GEMMs: before each ``loss_fn(t, index)`` (whose forward calls
+        ``linear_perturbed``) the evaluation point is prepared; W is written once, by
+        zo_step's update (nothing to restore)."""
+        losses = []
+        for (qa, ca), _ in linear_plan(scheme, self.q):
+            self.linear_prepare(t, qa, ca, -1, 0.0, eps)
+            losses.append(loss_fn(t, len(losses)))
+        self.step(t, adam_t, losses, scheme, eps, lr, beta1, beta2, eps_adam, -1, 0.0, optimizer,
                   gamma_out)
         return losses

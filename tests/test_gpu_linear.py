@@ -192,3 +192,60 @@ def test_perturbed_linear_rejections(lib, gpu):
     with pytest.raises(RuntimeError):                                             # FMA path
         zb.zo_linear_prepare(zf.ctx, 0, 0, 1.0, -1, 0.0, 1e-3)
     zf.close()
+
+
+@pytest.mark.parametrize("scheme", ["central", "forward"])
+def test_linear_route_step_matches_oracle(lib, gpu, scheme):
+    """One whole Alg. 3 step on the perturbed-linear route (SubZeroPlus.run_step_linear):
+    every loss comes from zo_linear_perturbed outputs while W stays as it is; each
+    evaluation's Y matches the oracle's layer, element by element, at the point the scheme
+    defines (Eq. (3): W + eps Z_k, W - eps Z_k; Eq. (6): W, then W + eps Z_k; eps large
+    enough that most outputs move); and zo_step (nothing to restore) leaves W and the
+    moments at the oracle's single update from the losses."""
+    from gpu_util import oracle_step
+    from parity import assert_moments, assert_weights, gabs
+    z, base = _context(gpu, "r32", seed=777)
+    r, spec, _ = LINEAR_CASES["r32"]
+    eps, lr, b1, b2, ea, t = 0.5, 1e-3, 0.9, 0.95, 1e-8, 3
+    T = 48
+    X = [_tokens(T, n, 100 + i, gpu) for i, (m, n, _) in enumerate(spec)]
+    gw = [torch.randn(T, m, generator=torch.Generator().manual_seed(200 + i)).double().numpy()
+          for i, (m, n, _) in enumerate(spec)]
+    if scheme == "central":
+        points = [(k, c) for k in range(z.q) for c in (1.0, -1.0)]
+    else:
+        points = [(0, 0.0)] + [(k, 1.0) for k in range(z.q)]
+    before = snapshot(z)
+    W_bits = [W.detach().clone() for W in z.weights]
+
+    def loss_fn(t_, idx):
+        for W, Wb in zip(z.weights, W_bits):           # the evaluations never write W
+            assert torch.equal(W.view(torch.int16), Wb.view(torch.int16))
+        k, c = points[idx]
+        loss = 2.0
+        for i in range(len(spec)):
+            Y = z.linear_perturbed(i, X[i])
+            z.sync()
+            # element by element at the point the scheme defines (the bound of _check)
+            C = subzero.perturb_coeff(z.seed, base + i, t_, r, [(k, c)], f32(eps))
+            want = _check(Y, X[i], before["W"][i], before["U"][i], before["V"][i], C,
+                          abs(f32(eps) * c), f"{scheme} evaluation {idx}, matrix {i}")
+            if c != 0.0:                                # the perturbation is visible
+                plain = rounding.round_to_bf16(to_f64(X[i]) @ before["W"][i].T)
+                assert (plain != want).mean() > 0.5
+            loss += float((to_f64(Y) * gw[i]).mean())
+        return loss
+
+    losses = z.run_step_linear(t, 1, loss_fn, scheme, eps, lr, b1, b2, ea)
+    assert len(losses) == len(points)
+    after = snapshot(z)
+    z.sync()
+    rho = subzero.rho_from_losses(np.asarray(losses, np.float32), scheme, f32(eps), z.q)
+    for i in range(len(spec)):
+        Wo, Mo, Vmo, G, Tm = oracle_step(before, i, "bf16", z.seed, base + i, t, r, z.q, losses,
+                                         scheme, eps, lr, b1, b2, ea, 1, [])
+        assert_moments(after["M"][i], after["Vm"][i], Mo, Vmo, before["M"][i], before["Vm"][i],
+                       gabs(z.seed, base + i, t, r, rho), b1, b2, f"linear route {i}")
+        assert_weights(after["W"][i], Wo, "bf16", f"linear-route step, matrix {i}",
+                       before=before["W"][i], terms=Tm)
+    z.close()
