@@ -55,3 +55,24 @@ def test_call_plan_matches_the_oracle_plan(lib, scheme, q):
         mine = [(qa, ca)] + ([second] if second is not None else [])
         assert sorted(mine) == sorted(terms)
     assert [restore] == orestore
+
+
+@pytest.mark.parametrize("q", [1, 2, 5])
+def test_linear_plan_visits_the_scheme_points(lib, q):
+    # the perturbed-linear route evaluates each loss at an absolute point: Eq. (3) pairs
+    # W + eps Z_k, W - eps Z_k; Eq. (6) W itself, then W + eps Z_k -- the same points the
+    # weight-pass plan reaches by accumulating its passes
+    from paper_2608_15665_gb300.schedule import linear_plan, step_plan
+    for scheme in ("central", "forward"):
+        pts = [(k, c) for (k, c), second in linear_plan(scheme, q) if second is None]
+        assert len(pts) == len(linear_plan(scheme, q))
+        calls, _ = step_plan(scheme, q)
+        acc, visited = {}, [] if scheme == "central" else [{}]
+        for (qa, ca), second in calls:
+            for kk, cc in [(qa, ca)] + ([second] if second else []):
+                acc[kk] = acc.get(kk, 0.0) + cc
+            visited.append({k: c for k, c in acc.items() if c != 0.0})
+        want = [{k: c} if c != 0.0 else {} for k, c in pts]
+        assert visited == want, scheme
+    with pytest.raises(ValueError):
+        linear_plan("direct", q)
