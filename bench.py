@@ -566,7 +566,8 @@ def run_ours(args):
             and not args.layers and not args.no_secondary):
         # the second shape the weight pass is held to: the 32B-shaped set (r = 64, q = 8); the
         # paper's default scale on the 7B shapes (r = 128, K = 99 queries); the linear layers
-        # of one 7B layer evaluated at the perturbed weights without a weight pass
+        # of one 7B layer evaluated at the perturbed weights without a weight pass (r = 32 and
+        # r = 128)
         del weights, z
         torch.cuda.empty_cache()
         line["secondary"] = {
@@ -574,6 +575,8 @@ def run_ours(args):
             "llama7b_bf16_r128_q99": secondary_weight_pass(dev, local, peak,
                                                            "llama7b_bf16_r128_q99", 1),
             "perturbed_linear_llama7b_4096tok": secondary_linear(dev, local),
+            "perturbed_linear_llama7b_4096tok_r128": secondary_linear(dev, local,
+                                                                     "llama7b_bf16_r128_q99"),
         }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl0, args.scheme)
@@ -712,13 +715,15 @@ def linear_measure(dev, wl, T, K, W, compare=True, e2e=True):
         zb.zo_linear_perturbed(z.ctx, i, X[n], Y[i])
         out["tiling"].append(names[zb.zo_linear_tiling(z.ctx)])
     if compare:
-        # the same route with the single-CTA 128 x 256 and 256 x 224 tiles throughout
-        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 1)
-        out["fused128_ms"] = timed(fused, K)
-        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 3)
-        out["fused224_ms"] = timed(fused, K)
-        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 0)
-        z.sync()
+        if wl.r <= 32:
+            # the same route with the single-CTA 128 x 256 and 256 x 224 tiles throughout
+            # (r <= 32 only)
+            zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 1)
+            out["fused128_ms"] = timed(fused, K)
+            zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 3)
+            out["fused224_ms"] = timed(fused, K)
+            zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 0)
+            z.sync()
         out["plain_ms"] = timed(lambda k: plain(), K)
         out["wpass_ms"] = timed(lambda k: (z.perturb(k, 0, 1.0, -1, 0.0, wl.eps), plain()), K)
         z.sync()
@@ -755,12 +760,13 @@ def linear_peak():
     return 1700.0, "fallback (sustained)"
 
 
-def secondary_linear(dev, local):
+def secondary_linear(dev, local, name="llama7b_bf16_r32"):
     """The perturbed-linear route (zo_linear_perturbed, no weight pass) on one LLaMA-7B
-    layer's seven matrices at 4096 tokens, r = 32: 10 timed steps after 2 warm-up ones,
-    with the weight-pass route and the plain cuBLAS GEMMs timed beside it."""
+    layer's seven matrices at 4096 tokens (r = 32, or the paper's r = 128): 10 timed steps
+    after 2 warm-up ones, with the weight-pass route and the plain cuBLAS GEMMs timed
+    beside it."""
     from paper_2608_15665_gb300 import workloads
-    wl = subset(workloads.get("llama7b_bf16_r32"), 1)
+    wl = subset(workloads.get(name), 1)
     T = 4096
     m = linear_measure(dev, wl, T, K=10, W=2, compare=True, e2e=False)
     peak, peak_kind = linear_peak()
@@ -771,7 +777,7 @@ def secondary_linear(dev, local):
             "kernel": "linear_pair_kernel" if any("pair" in t for t in m["tiling"])
             else "linear_kernel",
             "weight_pass_route_ms": m["wpass_ms"], "plain_gemm_ms": m["plain_ms"],
-            "single_cta_256x224_ms": m["fused224_ms"], "clocks": m["clocks"]}
+            "single_cta_256x224_ms": m.get("fused224_ms"), "clocks": m["clocks"]}
 
 
 def run_linear(args):
@@ -806,8 +812,8 @@ def run_linear(args):
                      "frac": achieved / peak, "peak_kind": peak_kind, "traffic": None,
                      "kernel": "linear_pair_kernel" if any("pair" in t for t in m["tiling"])
                      else "linear_kernel", "algorithmic_flops_per_step": flops},
-        "tile128_ms": m["fused128_ms"],
-        "tile224_single_cta_ms": m["fused224_ms"],
+        "tile128_ms": m.get("fused128_ms"),
+        "tile224_single_cta_ms": m.get("fused224_ms"),
         "plain_gemm_ms": m["plain_ms"],
         "weight_pass_route_ms": m["wpass_ms"],
         "e2e": {"value": flops / m["e2e_s"] / 1e12, "unit": "TFLOP/s",

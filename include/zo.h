@@ -118,7 +118,9 @@ enum {
                                128 on SM pairs (M = 256 MMAs across a 2-CTA cluster, S in
                                the same launch).  The tilings of one family give
                                bit-identical Y; the two families may differ in the last
-                               bits of S (each splits S's K in ranges of its own). */
+                               bits of S (each splits S's K in ranges of its own).  At
+                               r in {64, 128} only the SM-pair tilings exist: a call with
+                               1 .. 3 set returns ZO_ERR_UNSUPPORTED. */
   ZO_OPTION_PAIR_MMA = 4    /* tensor-core weight pass at r = 128: 1 (default) = M = 256 MMAs
                                across the two SMs of a cluster (each SM holds and reads half
                                of every P tile), 0 = the single-SM kernel.  Both give
@@ -233,7 +235,7 @@ ZO_API zo_status zo_mezo_perturb(zo_ctx* ctx, uint32_t t, float coef);
  * Linear layers at the perturbed weights WITHOUT a weight pass: the forward of a loss
  * evaluation of Alg. 3 at W_i' = W_i + U_i C_i V_i^T (Eq. (4) form) with every W_i left as
  * it is, for contexts on the tensor-core path (every W bf16, n a multiple of 8) with r in
- * {16, 32}; otherwise ZO_ERR_UNSUPPORTED.
+ * {16, 32, 64, 128}; otherwise ZO_ERR_UNSUPPORTED.
  *
  * zo_linear_prepare -- once per loss evaluation: C_i = eps (ca Z_i^(qa) + cb Z_i^(qb)) at
  *   step t (qb = -1: one term) for every matrix -- the coefficient zo_perturb(ctx, t, qa,
@@ -246,8 +248,8 @@ ZO_API zo_status zo_mezo_perturb(zo_ctx* ctx, uint32_t t, float coef);
  *   multiple of 8, else ZO_ERR_SHAPE).  The dense product is exact in bf16 with fp32
  *   accumulation; the rank-r term carries the bf16 hi/lo split's ~2^-16 relative error;
  *   Y is rounded to bf16 once.  W_i is read, never written.  Asynchronous; device errors
- *   go to the status word.  The GEMM's tiling follows ZO_OPTION_LINEAR_TILE (all tilings
- *   give the same Y bits); the context keeps an S workspace sized for the most tokens
+ *   go to the status word.  The GEMM's tiling follows ZO_OPTION_LINEAR_TILE (the tilings
+ *   of one family give the same Y bits); the context keeps an S workspace sized for the most tokens
  *   seen so far, and a call with more synchronises the stream to grow it.
  */
 ZO_API zo_status zo_linear_prepare(zo_ctx* ctx, uint32_t t, int32_t qa, float ca, int32_t qb,

@@ -960,7 +960,7 @@ zo_status zo_linear_prepare(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t
   if (!c) return ZO_ERR_INVALID_ARG;
   DeviceGuard guard(c->device);
   if (!c->tc_ok || !zo::linear_supported(c->r)) {
-    g_last_error = "zo_linear_prepare needs the tensor-core path with r in {16, 32}";
+    g_last_error = "zo_linear_prepare needs the tensor-core path with r in {16, 32, 64, 128}";
     return ZO_ERR_UNSUPPORTED;
   }
   if (qa < 0 || qa >= c->q || qb < -1 || qb >= c->q || !std::isfinite(ca) || !std::isfinite(cb) ||
@@ -993,7 +993,8 @@ zo_status zo_linear_prepare(zo_ctx* c, uint32_t t, int32_t qa, float ca, int32_t
     c->d_pk_off = pk_off;
   }
   if (!c->d_u_lin) {
-    // the route's U operand: the bf16 pair of U in rows laid out like d_u_op's (r <= 32)
+    // the route's U operand: the bf16 pair of U in rows of tc_hl_width(r), stacked like
+    // d_u_op's at r <= 32
     const int64_t HLW = zo::tc_hl_width(r);
     const size_t bytes = sizeof(__nv_bfloat16) * (size_t)c->u_rows * HLW;
     __nv_bfloat16* u_lin = nullptr;
@@ -1075,11 +1076,16 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
   if (c->linear_pairs < 0) c->linear_pairs = std::max(0, (int)zo::linear_pair_max_pairs());
   int32_t tiling = c->linear_tile;
   if (tiling == 0)
-    tiling = c->linear_pairs > 0 ? zo::linear_pair_tiling(T, m, n, c->r, c->linear_pairs)
-                                 : zo::linear_y_tiling(T, m, c->sms, 0);
+    tiling = c->linear_pairs > 0 || !zo::linear_single_cta_supported(r)
+                 ? zo::linear_pair_tiling(T, m, n, r, c->linear_pairs)
+                 : zo::linear_y_tiling(T, m, c->sms, 0);
   const int32_t pair_n = zo::linear_pair_cols(tiling);
   if (pair_n > 0 && c->linear_pairs <= 0) {
     g_last_error = "zo_linear_perturbed: no cluster of the SM-pair GEMM fits on this device";
+    return ZO_ERR_UNSUPPORTED;
+  }
+  if (pair_n == 0 && !zo::linear_single_cta_supported(r)) {
+    g_last_error = "zo_linear_perturbed: the single-CTA tilings 1..3 take r in {16, 32}";
     return ZO_ERR_UNSUPPORTED;
   }
   // S's K split: the single-CTA route's S kernel, or the pair launch's S tiles; each writes

@@ -111,8 +111,9 @@ int64_t tc_u_operand_bytes(int32_t r, int64_t rows);
 // into Tensor Memory (zo_wpass_tmem.cu).
 cudaError_t launch_split_u(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                            int32_t n_units, int32_t r, void* u_op, cudaStream_t s);
-// The perturbed-linear route's U operand (r in {16, 32}): rows [hi | lo | 0] of the bf16
-// pair of U, unscaled, laid out as the r <= 32 U operand above.
+// The perturbed-linear route's U operand (r in {16, 32, 64, 128}): rows [hi | lo | 0] of
+// the bf16 pair of U, unscaled, tc_hl_width(r) elements per row, rows as the r <= 32 U
+// operand above.
 cudaError_t launch_split_u_bf16(const MatDesc* d_mats, const TcMat* d_tc, const int2* d_units,
                                 int32_t n_units, int32_t r, __nv_bfloat16* u_lin, cudaStream_t s);
 // tm_a is used for r <= 32, u_op for r >= 64; d_pinv[i] = 2^-(e_P,i) from launch_split_c.
@@ -157,15 +158,18 @@ cudaError_t launch_project_tc(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
                               int32_t n_units, int32_t grid, int32_t r, uint32_t* d_status,
                               cudaStream_t s);
 // The same projection writing, instead of P_HL, P_K = the K-major bf16 pair [P_hi ; P_lo]
-// of P_i at p_k + pk_off[i] (rows of n_i rounded up to 64; r in {16, 32}), from pinv.
+// of P_i at p_k + pk_off[i] (rows of n_i rounded up to 64; r in {16, 32, 64, 128}), from pinv.
 cudaError_t launch_project_tc_pk(const CUtensorMap& tm_v, const CUtensorMap& tm_c,
                                  const TcMat* d_tc, const int2* d_units, int32_t n_units,
                                  int32_t grid, int32_t r, const float* pinv, const int64_t* pk_off,
                                  __nv_bfloat16* p_k, uint32_t* d_status, cudaStream_t s);
 
 // ---- a linear layer at the perturbed weights, without a weight pass (zo_linear.cu) -----
-// Y = X (W + U C V^T)^T = X W^T + S U^T, S = X P^T, for bf16 contexts at r in {16, 32}.
+// Y = X (W + U C V^T)^T = X W^T + S U^T, S = X P^T, for bf16 contexts at r in
+// {16, 32, 64, 128}; the single-CTA tilings (this file) at r in {16, 32}, the SM-pair ones
+// (zo_linear_pair.cu) at every r.
 bool linear_supported(int32_t r);
+bool linear_single_cta_supported(int32_t r);
 // The S GEMM's split of K = n into k_split ranges of k_chunk steps of 64 (~ one wave).
 void linear_s_split(int64_t T, int64_t n, int32_t sms, int32_t* k_split, int32_t* k_chunk);
 // Tiling of the Y GEMM: 1 = 128 x 256, 2 = 256 x 256, 3 = 256 x 224 (rows of X x columns
@@ -208,9 +212,10 @@ void linear_pair_s_split(int64_t T, int64_t n, int32_t n_pairs, int32_t* s_split
                          int32_t* s_chunk);
 // The pair tiling whose busiest pair has the least work (S and Y tiles dealt round-robin).
 int32_t linear_pair_tiling(int64_t T, int64_t m, int64_t n, int32_t r, int32_t n_pairs);
-// One launch computes S = X P^T (S tiles, written to s_hl as S_HL rows) and Y = X W^T +
-// S U^T.  tm_x over X (box 64 x 128), tm_w over W_i (box 64 x N/2), tm_s over s_hl (box
-// 64 x 128), tm_u over the bf16 U operand (box 64 x N/2; W_i's rows from u_row0), tm_y over
+// One launch computes S = X P^T (S tiles, written to s_hl as S_HL rows of tc_hl_width(r))
+// and Y = X W^T + S U^T, r in {16, 32, 64, 128}.  tm_x over X (box 64 x 128), tm_w over
+// W_i (box 64 x N/2), tm_s over s_hl (box 64 x 128), tm_u over the bf16 U operand (box
+// 64 x N/2; W_i's rows from u_row0), tm_y over
 // Y (box 16 x 32, 32-byte swizzle), tm_pk over P_K (box 64 x r).  s_part: s_split x T x r
 // floats (linear_pair_s_split).  s_count: kLinearPairCounters counters per 256 rows of X
 // (zero before the first call), epoch: 1 .. kLinearPairEpochs - 1, a new one per call (the

@@ -491,7 +491,8 @@ cudaError_t launch_linear_r(const CUtensorMap& tm_a, const CUtensorMap& tm_b,
 
 }  // namespace
 
-bool linear_supported(int32_t r) { return r == 16 || r == 32; }
+bool linear_supported(int32_t r) { return r == 16 || r == 32 || r == 64 || r == 128; }
+bool linear_single_cta_supported(int32_t r) { return r == 16 || r == 32; }
 
 void linear_s_split(int64_t T, int64_t n, int32_t sms, int32_t* k_split, int32_t* k_chunk) {
   const int64_t k_steps = (n + 63) / 64;

@@ -11,10 +11,12 @@
 // the pair's next tile accumulate into the other one.
 //
 // K steps: n / 64 steps of X and W (single bf16 products, both operands exact in bf16),
-// then one step of the rank-r term from S_HL = [S_hi | S_lo | 0] (A) and the U operand
-// [U_hi | U_lo | 0] (B) with the three products S_hi U_hi + S_hi U_lo + S_lo U_hi -- the
-// same MMAs, in the same order, as the single-CTA kernels of zo_linear.cu, so each 128-row
-// half of a pair tile gets the bits those kernels give.
+// then the rank-r term from S_HL = [S_hi | S_lo | 0] (A) and the U operand
+// [U_hi | U_lo | 0] (B) with the three products S_hi U_hi + S_hi U_lo + S_lo U_hi.  For
+// r <= 32 that is one operand stage holding one 64-wide panel of each, the same MMAs, in
+// the same order, as the single-CTA kernels of zo_linear.cu, so each 128-row half of a
+// pair tile gets the bits those kernels give; r = 64 takes one stage of two panels (hi,
+// lo), r = 128 three stages of two panels (S_hi U_hi, S_hi U_lo, S_lo U_hi).
 // N (a multiple of 16, 128 .. 256) is chosen by the host so that the tiles fill whole
 // waves of the resident pairs (224 for 4096 columns at 4096 tokens: 19 x 16 = 304 tiles =
 // 4 waves of 76 pairs; 240 for 11008 columns).
@@ -73,12 +75,16 @@ struct PairLin {
   static constexpr int kTmemCols = 512;
   static constexpr int kChunks = N / 16;                      // 16-column chunks of a row
   static constexpr size_t kSmem = (size_t)kStages * kStageBytes + kOutBytes + 1024 + 1024;
-  // an S tile's stage: as many 64-element panels of X and of P_K's r rows as fit a stage
-  // (its stages are fewer than a Y tile's, so that it ends before the Y tiles need S)
+  // an S tile's stage: as many 64-element panels of X and of P_K's r rows as fit a stage,
+  // at most 4 (its stages are fewer than a Y tile's, so that it ends before the Y tiles
+  // need S)
   template <int R>
   static constexpr int s_panels() {
     return kStageBytes / (kAPanel + R * 128) < 4 ? kStageBytes / (kAPanel + R * 128) : 4;
   }
+  // operand stages of a Y tile's rank-r step
+  template <int R>
+  static constexpr int ext_stages() { return R == 128 ? 3 : 1; }
   static_assert(kStages >= 3, "operand ring");
   static_assert(kSmem <= 227 * 1024, "shared memory per CTA");
   static_assert(kAccStride + N <= kTmemCols, "two accumulators in TMEM");
@@ -147,6 +153,25 @@ __device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&v)
       : "r"(taddr));
 }
 
+// Columns kC j .. kC j + kC - 1 of S for this thread's row (kC = min(R, 32)): the sum of
+// the accumulator's X P_hi^T and X P_lo^T columns.  Warp-collective.
+template <int R>
+__device__ __forceinline__ void load_s_chunk(uint32_t t_base, int j, float (&x)[R < 32 ? R : 32]) {
+  uint32_t v[32];
+  tmem_ld_32x32b_x32(t_base + (uint32_t)(32 * j), v);
+  if constexpr (R == 16) {
+    tmem_ld_wait();
+#pragma unroll
+    for (int q = 0; q < 16; ++q) x[q] = __uint_as_float(v[q]) + __uint_as_float(v[16 + q]);
+  } else {
+    uint32_t w[32];
+    tmem_ld_32x32b_x32(t_base + (uint32_t)(R + 32 * j), w);
+    tmem_ld_wait();
+#pragma unroll
+    for (int q = 0; q < 32; ++q) x[q] = __uint_as_float(v[q]) + __uint_as_float(w[q]);
+  }
+}
+
 // Pair tile t -> (row block tb, column block nb): column stripes of `group` column blocks,
 // each walked row block by row block (group = the column blocks: plain row-major order).
 // Stripes about one wave of tiles wide keep the wave's W rows few enough to stay in L2
@@ -211,7 +236,10 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
   using Cfg = PairLin<N>;
   constexpr int S = Cfg::kStages;
   constexpr int kSP = Cfg::template s_panels<R>();            // panels per S-tile stage
-  static_assert(kSP >= 2, "S-tile stage");
+  constexpr int kExt = Cfg::template ext_stages<R>();         // stages of the rank-r step
+  static_assert(R == 16 || R == 32 || R == 64 || R == 128, "rank");
+  static_assert(kSP >= 1, "S-tile stage");
+  static_assert(2 * R <= Cfg::kAccStride, "an S tile's 2 r accumulator columns");
   static_assert(sizeof(LinPairShared) <= 1024, "barrier block");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -272,7 +300,7 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
       // steps and its rank-r step
       const int p_lo = s_tile ? nb * s_chunk : 0;
       const int p_hi = s_tile ? min(k_steps, p_lo + s_chunk) : 0;
-      const int n_k = s_tile ? (p_hi - p_lo + kSP - 1) / kSP : k_stages + 1;
+      const int n_k = s_tile ? (p_hi - p_lo + kSP - 1) / kSP : k_stages + kExt;
       for (int k = 0; k < n_k; ++k) {
         if (!mbar_wait_bounded(&sh.empty[s], ph ^ 1u, abort, wait_cycles)) {
           ok = false;
@@ -301,17 +329,36 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
             tma_load_2d_to_leader(b_dst + p * Cfg::kBPanel, &tm_w, x, y_b, &sh.full[s]);
           }
         } else {                               // the rank-r step: S_HL rows, U operand rows
-          // this row block's S rows: written by its S tile (both CTAs' epilogues) earlier in
-          // this launch
-          if (!wait_s_rows(s_count + (int64_t)tb * kLinearPairCounters, wait_epoch, abort,
-                           wait_cycles)) {
-            ok = false;
-            break;
+          const int j = k - k_stages;
+          if (j == 0) {
+            // this row block's S rows: written by its S tile (both CTAs' epilogues) earlier
+            // in this launch
+            if (!wait_s_rows(s_count + (int64_t)tb * kLinearPairCounters, wait_epoch, abort,
+                             wait_cycles)) {
+              ok = false;
+              break;
+            }
+            fence_async_global();
           }
-          fence_async_global();
-          if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * (Cfg::kAPanel + Cfg::kBPanel));
-          tma_load_2d_to_leader(a_dst, &tm_s, 0, y_a, &sh.full[s]);
-          tma_load_2d_to_leader(b_dst, &tm_u, 0, u_row0 + y_b, &sh.full[s]);
+          if constexpr (R <= 32) {
+            // one 64-wide panel of each: [hi | lo | 0]
+            if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * (Cfg::kAPanel + Cfg::kBPanel));
+            tma_load_2d_to_leader(a_dst, &tm_s, 0, y_a, &sh.full[s]);
+            tma_load_2d_to_leader(b_dst, &tm_u, 0, u_row0 + y_b, &sh.full[s]);
+          } else {
+            // two panels of each, from S_HL columns sx, sx + 64 and U columns ux, ux + 64:
+            // r = 64 the hi and the lo panel of both; r = 128 the hi panels (stage 0), the
+            // hi panels of S and the lo ones of U (stage 1), the lo ones of S and the hi ones
+            // of U (stage 2)
+            const int sx = j == 2 ? R : 0, ux = j == 1 ? R : 0;
+            if (leader) mbar_arrive_expect_tx(&sh.full[s], 2u * Cfg::kStageBytes);
+#pragma unroll
+            for (int p = 0; p < 2; ++p) {
+              tma_load_2d_to_leader(a_dst + p * Cfg::kAPanel, &tm_s, sx + 64 * p, y_a, &sh.full[s]);
+              tma_load_2d_to_leader(b_dst + p * Cfg::kBPanel, &tm_u, ux + 64 * p, u_row0 + y_b,
+                                    &sh.full[s]);
+            }
+          }
         }
         ++n_st;
         if (++s == S) { s = 0; ph ^= 1u; }
@@ -348,7 +395,7 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
       const uint32_t d = tmem + (uint32_t)(acc * Cfg::kAccStride);
       const int p_lo = s_tile ? nb * s_chunk : 0;
       const int p_hi = s_tile ? min(k_steps, p_lo + s_chunk) : 0;
-      const int n_k = s_tile ? (p_hi - p_lo + kSP - 1) / kSP : k_stages + 1;
+      const int n_k = s_tile ? (p_hi - p_lo + kSP - 1) / kSP : k_stages + kExt;
       for (int k = 0; k < n_k; ++k) {
         // the operands arrive by TMA on this barrier: its wait orders the MMAs' reads
         if (!mbar_wait_bounded(&sh.full[s], ph, abort, wait_cycles)) {
@@ -373,7 +420,7 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
             for (int kk = 0; kk < 4; ++kk)
               mma_pair_ss(d, a0 + p * kPanelA + kk * kStepK, b0 + p * kPanelB + kk * kStepK, idesc,
                           (k > 0 || p > 0 || kk > 0) ? 1u : 0u);
-        } else {
+        } else if constexpr (R <= 32) {
           // hi chunk kk at element 16 kk of an operand row, lo chunk at R + 16 kk
 #pragma unroll
           for (int kk = 0; kk < R / 16; ++kk) {
@@ -382,6 +429,23 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
             mma_pair_ss(d, a0 + hi, b0 + lo, idesc, 1u);
             mma_pair_ss(d, a0 + lo, b0 + hi, idesc, 1u);
           }
+        } else if constexpr (R == 64) {
+          // panel 0 holds the hi chunks, panel 1 the lo ones
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t st = kk * kStepK;
+            mma_pair_ss(d, a0 + st, b0 + st, idesc, 1u);
+            mma_pair_ss(d, a0 + st, b0 + kPanelB + st, idesc, 1u);
+            mma_pair_ss(d, a0 + kPanelA + st, b0 + st, idesc, 1u);
+          }
+        } else {
+          // one of the three products over its 128 elements of K
+#pragma unroll
+          for (int p = 0; p < 2; ++p)
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              mma_pair_ss(d, a0 + p * kPanelA + kk * kStepK, b0 + p * kPanelB + kk * kStepK,
+                          idesc, 1u);
         }
         commit_both(&sh.empty[s]);
         ++n_st;
@@ -423,33 +487,35 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
         // partial row, and the warp that completes its 32-row group's ranges sums them in
         // range order and writes the S_HL rows.  Then the group counts as ready.
         if (h == 0) {
-          uint32_t v[32];
-          tmem_ld_32x32b_x32(t_base, v);
-          float x[R];
-          if constexpr (R == 32) {
-            uint32_t w[32];
-            tmem_ld_32x32b_x32(t_base + 32u, w);
-            tmem_ld_wait();
-#pragma unroll
-            for (int q = 0; q < R; ++q) x[q] = __uint_as_float(v[q]) + __uint_as_float(w[q]);
-          } else {
-            tmem_ld_wait();
-#pragma unroll
-            for (int q = 0; q < R; ++q) x[q] = __uint_as_float(v[q]) + __uint_as_float(v[R + q]);
-          }
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) arrive_leader(&sh.acc_empty[acc]);
+          // kC columns of S at a time (D[:, kC j ..] + D[:, R + kC j ..])
+          constexpr int kC = R < 32 ? R : 32;
           const int row = y + lane;
           uint32_t* cnt = s_count + (int64_t)tb * kLinearPairCounters;
+          float* part_row = s_part + ((int64_t)nb * rows + row) * R;
+#pragma unroll 1
+          for (int j = 0; j < R / kC; ++j) {
+            float x[kC];
+            load_s_chunk<R>(t_base, j, x);
+            if (j == R / kC - 1) {                   // this warp's last read of the accumulator
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) arrive_leader(&sh.acc_empty[acc]);
+            }
+            if (row < rows) {
+              if (s_split > 1) {
+                float4* dst = reinterpret_cast<float4*>(part_row + kC * j);
+#pragma unroll
+                for (int q = 0; q < kC / 4; ++q)
+                  dst[q] = make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3]);
+              } else {
+#pragma unroll
+                for (int q = 0; q < kC; ++q) x[q] = 0.f + x[q];
+                write_s_chunk<R>(s_hl, row, j, x);
+              }
+            }
+          }
           bool last = true;
           if (s_split > 1) {
-            if (row < rows) {
-              float4* dst = reinterpret_cast<float4*>(s_part + ((int64_t)nb * rows + row) * R);
-#pragma unroll
-              for (int j = 0; j < R / 4; ++j)
-                dst[j] = make_float4(x[4 * j], x[4 * j + 1], x[4 * j + 2], x[4 * j + 3]);
-            }
             __threadfence();
             __syncwarp();
             uint32_t n_done = 0;
@@ -457,27 +523,29 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
             n_done = __shfl_sync(0xffffffffu, n_done, 0);
             last = n_done == (uint32_t)s_split;
             if (last && row < rows) {
+#pragma unroll 1
+              for (int j = 0; j < R / kC; ++j) {
+                float x[kC];
 #pragma unroll
-              for (int q = 0; q < R; ++q) x[q] = 0.f;
-              for (int ks = 0; ks < s_split; ++ks) {
-                const float4* src =
-                    reinterpret_cast<const float4*>(s_part + ((int64_t)ks * rows + row) * R);
+                for (int q = 0; q < kC; ++q) x[q] = 0.f;
+                for (int ks = 0; ks < s_split; ++ks) {
+                  const float4* src = reinterpret_cast<const float4*>(
+                      s_part + ((int64_t)ks * rows + row) * R + kC * j);
 #pragma unroll
-                for (int j = 0; j < R / 4; ++j) {
-                  const float4 p4 = __ldcg(src + j);
-                  x[4 * j] += p4.x;
-                  x[4 * j + 1] += p4.y;
-                  x[4 * j + 2] += p4.z;
-                  x[4 * j + 3] += p4.w;
+                  for (int q = 0; q < kC / 4; ++q) {
+                    const float4 p4 = __ldcg(src + q);
+                    x[4 * q] += p4.x;
+                    x[4 * q + 1] += p4.y;
+                    x[4 * q + 2] += p4.z;
+                    x[4 * q + 3] += p4.w;
+                  }
                 }
+                write_s_chunk<R>(s_hl, row, j, x);
               }
             }
-          } else {
-#pragma unroll
-            for (int q = 0; q < R; ++q) x[q] = 0.f + x[q];
           }
           if (last) {
-            if (row < rows) write_s_row<R>(s_hl, row, x);
+            if (row < rows) zero_s_pad<R>(s_hl, row);
             fence_async_global();
             __threadfence();
             __syncwarp();
@@ -629,14 +697,15 @@ int32_t linear_pair_tiling(int64_t T, int64_t m, int64_t n, int32_t r, int32_t n
   int64_t c_best = -1;
   const int64_t row_blocks = ceil_div(T, kPairRows);
   const int64_t pairs = std::max<int32_t>(1, n_pairs);
-  const int64_t k_stages = ceil_div(ceil_div(n, 64), 2);
+  // a Y tile's operand stages: K in steps of 128, then the rank-r step's
+  const int64_t y_stages = ceil_div(ceil_div(n, 64), 2) + (r == 128 ? 3 : 1);
   for (int i = 0; i < 5; ++i) {
     const int64_t N = kPairCols[i];
     int32_t s_split = 1, s_chunk = 1;
     linear_pair_s_split(T, n, n_pairs, &s_split, &s_chunk);
     const int64_t n_s = row_blocks * s_split;
     const int64_t total = n_s + row_blocks * ceil_div(m, N);
-    const int64_t cost_y = (k_stages + 1) * 2 * (kBM * 128 + N / 2 * 128);
+    const int64_t cost_y = y_stages * 2 * (kBM * 128 + N / 2 * 128);
     // an S tile's panels, rounded up to whole stages of s_panels_host(N, r) panels
     const int64_t cost_s = ceil_div(s_chunk, s_panels_host(N, r)) * s_panels_host(N, r) *
                            (kBM * 128 + (int64_t)r * 128);
@@ -662,7 +731,8 @@ cudaError_t launch_linear_pair(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
                                uint32_t* s_count, uint32_t epoch, bool inject_wait,
                                uint32_t* d_status, cudaStream_t s) {
   const int32_t N = linear_pair_cols(tiling);
-  if (N == 0 || n_pairs <= 0 || (r != 16 && r != 32)) return cudaErrorInvalidValue;
+  if (N == 0 || n_pairs <= 0 || (r != 16 && r != 32 && r != 64 && r != 128))
+    return cudaErrorInvalidValue;
   const int k_steps = (int)ceil_div(n, 64);
   int32_t s_split = 1, s_chunk = 1;
   linear_pair_s_split(T, n, n_pairs, &s_split, &s_chunk);
@@ -678,19 +748,20 @@ cudaError_t launch_linear_pair(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
   launch_pair_nr<NN, RR>(tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk, (int)T, (int)m, k_steps, u_row0,  \
                          group, s_split, s_chunk, s_hl, s_part, s_count, epoch, inject_wait,   \
                          pairs, d_status, s)
-  switch (N * 64 + r) {
-    case 256 * 64 + 16: return ZO_PAIR_Y(256, 16);
-    case 256 * 64 + 32: return ZO_PAIR_Y(256, 32);
-    case 240 * 64 + 16: return ZO_PAIR_Y(240, 16);
-    case 240 * 64 + 32: return ZO_PAIR_Y(240, 32);
-    case 224 * 64 + 16: return ZO_PAIR_Y(224, 16);
-    case 224 * 64 + 32: return ZO_PAIR_Y(224, 32);
-    case 192 * 64 + 16: return ZO_PAIR_Y(192, 16);
-    case 192 * 64 + 32: return ZO_PAIR_Y(192, 32);
-    case 128 * 64 + 16: return ZO_PAIR_Y(128, 16);
-    case 128 * 64 + 32: return ZO_PAIR_Y(128, 32);
+#define ZO_PAIR_RANKS(NN)                                 \
+  case NN * 256 + 16: return ZO_PAIR_Y(NN, 16);           \
+  case NN * 256 + 32: return ZO_PAIR_Y(NN, 32);           \
+  case NN * 256 + 64: return ZO_PAIR_Y(NN, 64);           \
+  case NN * 256 + 128: return ZO_PAIR_Y(NN, 128);
+  switch (N * 256 + r) {
+    ZO_PAIR_RANKS(256)
+    ZO_PAIR_RANKS(240)
+    ZO_PAIR_RANKS(224)
+    ZO_PAIR_RANKS(192)
+    ZO_PAIR_RANKS(128)
     default: return cudaErrorInvalidValue;
   }
+#undef ZO_PAIR_RANKS
 #undef ZO_PAIR_Y
 }
 

@@ -1,8 +1,9 @@
 // The U operand of the r <= 32 tensor-core weight pass (zo_wpass_tc.cu): rows
 // [hi(U s) | lo(U s) | 0 ...] in fp16 with s = 2^kUVScaleExp (zo_tc_common.cuh), formed once
 // per refresh, stacked per matrix in 128-row blocks and read by TMA.  The perturbed-linear
-// route (zo_linear.cu) reads the same rows as a bf16 pair, hi = bf16(x), lo = bf16(x - hi),
-// unscaled, from a buffer of its own: there U meets the bf16 X and W in one accumulator.
+// route (zo_linear.cu, zo_linear_pair.cu; every r) reads rows of the same layout as a bf16
+// pair, hi = bf16(x), lo = bf16(x - hi), unscaled, from a buffer of its own: there U meets
+// the bf16 X and W in one accumulator.
 // Also the dispatch of the split by rank (r >= 64: the chunk-major U of zo_wpass_tmem.cu).
 // P^T = V C^T, the other operand, comes from the tensor-core projection (zo_project_tc.cu).
 #include "zo_kernels.h"
@@ -13,7 +14,8 @@ namespace {
 
 using namespace tc;
 
-// The split kernel below (U rows, r <= 32) handles 128 consecutive rows of one matrix
+// The split kernel below (U rows; r <= 32 for the weight pass, every r for the
+// perturbed-linear route) handles 128 consecutive rows of one matrix
 // per CTA: each thread splits one row into 16-byte chunks of hi and lo, staged
 // in shared memory with the chunk index XOR (row & 7) so a quarter-warp's stores hit
 // distinct banks; the CTA then writes its rows, which are contiguous in the stacked
@@ -94,6 +96,8 @@ cudaError_t launch_split_u_bf16(const MatDesc* d_mats, const TcMat* d_tc, const 
   switch (r) {
     case 16: return launch_split_u_r<16, false>(d_mats, d_tc, d_units, n_units, reinterpret_cast<uint16_t*>(u_lin), s);
     case 32: return launch_split_u_r<32, false>(d_mats, d_tc, d_units, n_units, reinterpret_cast<uint16_t*>(u_lin), s);
+    case 64: return launch_split_u_r<64, false>(d_mats, d_tc, d_units, n_units, reinterpret_cast<uint16_t*>(u_lin), s);
+    case 128: return launch_split_u_r<128, false>(d_mats, d_tc, d_units, n_units, reinterpret_cast<uint16_t*>(u_lin), s);
     default: return cudaErrorInvalidValue;
   }
 }

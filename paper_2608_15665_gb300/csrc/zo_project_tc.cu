@@ -22,7 +22,7 @@
 //                   the fp32 row of D, scale and split it into fp16 hi/lo, write them as 32 x 64
 //                   boxes of P_HL into shared memory (128-byte swizzle) and TMA-store
 //                   them, 64 columns of D at a time (one hi and one lo box staged).
-//                   For the perturbed-linear route (kPK, r <= 32) it writes instead the
+//                   For the perturbed-linear route (kPK) it writes instead the
 //                   K-major bf16 pair [P_hi ; P_lo] of P (P_K): the exact fp32 P of D (a
 //                   power-of-two rescale) split into bf16 hi = bf16(P), lo = bf16(P - hi),
 //                   row k of P_K taking column j from lane j (64 contiguous bytes a warp).
@@ -99,7 +99,6 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
                   const int2* __restrict__ units, int n_units, uint32_t* __restrict__ status,
                   long long wait_cycles, __nv_bfloat16* __restrict__ p_k,
                   const int64_t* __restrict__ pk_off, const float* __restrict__ pinv) {
-  static_assert(!kPK || R <= 32, "P_K exists for r <= 32");
   using Cfg = ProjCfg<R>;
   static_assert(sizeof(ProjShared) <= 1024, "barrier block");
   static_assert(Cfg::kSmem <= 227 * 1024, "shared memory per CTA");
@@ -255,25 +254,30 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constan
       if (lane == 0) bulk_wait_read_all();
       __syncwarp();
       if constexpr (kPK) {
-        uint32_t v[R];
-        if constexpr (R == 32)
-          tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R), v);
-        else
-          tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)(acc * R), v);
-        tmem_ld_wait();
-        // D 2^-(kUVScaleExp + e_C,i) = P exactly (both factors powers of two)
+        // D 2^-(kUVScaleExp + e_C,i) = P exactly (both factors powers of two); kC columns
+        // of D at a time
+        constexpr int kC = R < 32 ? R : 32;
         const float unscale = p_scale * pinv[un.x];
         const int64_t n = mats[un.x].n;
         const int64_t ld = (n + 63) / 64 * 64;
         const int64_t j = un.y + 32 * g + lane;
-        if (j < n) {
-          __nv_bfloat16* dst = p_k + pk_off[un.x] + j;
+        __nv_bfloat16* dst = p_k + pk_off[un.x] + j;
+#pragma unroll 1
+        for (int c = 0; c < R / kC; ++c) {
+          uint32_t v[kC];
+          if constexpr (kC == 32)
+            tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(acc * R + 32 * c), v);
+          else
+            tmem_ld_32x32b_x16(tmem + lane_base + (uint32_t)(acc * R), v);
+          tmem_ld_wait();
+          if (j < n) {
 #pragma unroll
-          for (int k = 0; k < R; ++k) {
-            const float x = __uint_as_float(v[k]) * unscale;
-            const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-            dst[k * ld] = hi;
-            dst[(R + k) * ld] = __float2bfloat16_rn(x - __bfloat162float(hi));
+            for (int k = 0; k < kC; ++k) {
+              const float x = __uint_as_float(v[k]) * unscale;
+              const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+              dst[(kC * c + k) * ld] = hi;
+              dst[(R + kC * c + k) * ld] = __float2bfloat16_rn(x - __bfloat162float(hi));
+            }
           }
         }
       } else if constexpr (R <= 32) {
@@ -496,6 +500,8 @@ cudaError_t launch_project_tc_pk(const CUtensorMap& tm_v, const CUtensorMap& tm_
   switch (r) {
     case 16: return launch_project_tc_r<16, true>(tm_v, tm_c, tm_v, d_tc, d_units, n_units, grid, d_status, s, p_k, pk_off, pinv);
     case 32: return launch_project_tc_r<32, true>(tm_v, tm_c, tm_v, d_tc, d_units, n_units, grid, d_status, s, p_k, pk_off, pinv);
+    case 64: return launch_project_tc_r<64, true>(tm_v, tm_c, tm_v, d_tc, d_units, n_units, grid, d_status, s, p_k, pk_off, pinv);
+    case 128: return launch_project_tc_r<128, true>(tm_v, tm_c, tm_v, d_tc, d_units, n_units, grid, d_status, s, p_k, pk_off, pinv);
     default: return cudaErrorInvalidValue;
   }
 }

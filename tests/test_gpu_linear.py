@@ -19,14 +19,24 @@ from parity import NORMAL_ABS, to_f64
 pytestmark = pytest.mark.gpu
 
 # ZO_OPTION_LINEAR_TILE values: 1..3 single-CTA tiles (with the separate S = X P^T
-# kernel), 4..8 SM-pair tiles (N = 256, 240, 224, 192, 128 columns of Y; S in the same launch)
+# kernel; r <= 32), 4..8 SM-pair tiles (N = 256, 240, 224, 192, 128 columns of Y; S in the
+# same launch; every r)
 TILINGS = (1, 2, 3, 4, 5, 6, 7, 8)
+PAIR_TILINGS = (4, 5, 6, 7, 8)
 
-# (r, [(m, n, ldw)], token counts)
+# (r, [(m, n, ldw)], token counts).  r = 64 and 128 (the paper's rank): the rank-r step in
+# one operand stage of two panels and in three, S tiles with 128 and 256 accumulator
+# columns and one or two K panels per stage; ragged row blocks, column blocks and K panels.
 LINEAR_CASES = {
     "r32": (32, [(304, 520, None), (264, 2048, None), (1032, 72, 80)], (1, 130, 300)),
     "r16": (16, [(304, 520, 528), (136, 1000, 1008), (64, 136, None)], (7, 257)),
+    "r64": (64, [(392, 648, None), (136, 2056, 2064)], (5, 300)),
+    "r128": (128, [(520, 1032, None), (264, 264, 272)], (3, 513)),
 }
+
+
+def _tilings(r):
+    return TILINGS if r <= 32 else PAIR_TILINGS
 
 
 def _context(gpu, case, seed, base=31):
@@ -77,7 +87,7 @@ def test_perturbed_linear_matches_oracle_and_leaves_W(lib, gpu, case, eps):
             ldy = (m + 7) // 8 * 8
             out = {}
             # 128x256, 256x256, 256x224 on single CTAs; 256 x (256, 240, 224, 192, 128) on SM pairs
-            for tiling in TILINGS:
+            for tiling in _tilings(r):
                 zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, tiling)
                 Ybuf = torch.full((T, ldy), float("nan"), dtype=torch.bfloat16, device=gpu)
                 zb.zo_linear_perturbed(z.ctx, i, X, Ybuf[:, :m])
@@ -90,18 +100,30 @@ def test_perturbed_linear_matches_oracle_and_leaves_W(lib, gpu, case, eps):
             # ones take S from the split-K S kernel, the SM-pair ones from their own S tiles
             # (K ranges of 64-element panels, the same for every pair tiling), so the two
             # families may differ in S's last bits
-            for tiling in TILINGS:
+            for tiling in _tilings(r):
                 ref = 2 if tiling <= 3 else 6
                 assert torch.equal(out[tiling].view(torch.int16), out[ref].view(torch.int16)), tiling
             C = subzero.perturb_coeff(z.seed, base + i, 5, r, terms, f32(eps))
             zc = abs(f32(eps)) * 2.0
-            for Y in (out[3], out[6]):
+            for Y in [out[k] for k in (3, 6) if k in out]:
                 want = _check(Y, X, before["W"][i], before["U"][i], before["V"][i], C, zc,
                               f"{case} matrix {i} T={T} eps={eps}")
             if eps == 1e-1:
                 # the perturbation is visible: most outputs differ from the plain layer's
                 plain = rounding.round_to_bf16(to_f64(X) @ before["W"][i].T)
                 assert (plain != want).mean() > 0.5
+    if r > 32:
+        # the single-CTA tilings take r <= 32; the automatic choice is an SM-pair one
+        m, n, _ = spec[0]
+        X = _tokens(8, n, 1, gpu)
+        Y = torch.empty((8, m), dtype=torch.bfloat16, device=gpu)
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 2)
+        with pytest.raises(RuntimeError):
+            zb.zo_linear_perturbed(z.ctx, 0, X, Y)
+        zb.zo_set_option(z.ctx, zb.ZO_OPTION_LINEAR_TILE, 0)
+        zb.zo_linear_perturbed(z.ctx, 0, X, Y)
+        z.sync()
+        assert zb.zo_linear_tiling(z.ctx) >= 4
     for W, Wb in zip(z.weights, W_bits):
         assert torch.equal(W.view(torch.int16), Wb.view(torch.int16))
     z.close()
@@ -194,8 +216,9 @@ def test_perturbed_linear_rejections(lib, gpu):
     zf.close()
 
 
-@pytest.mark.parametrize("scheme", ["central", "forward"])
-def test_linear_route_step_matches_oracle(lib, gpu, scheme):
+@pytest.mark.parametrize("scheme,case", [("central", "r32"), ("forward", "r32"),
+                                         ("central", "r128")])
+def test_linear_route_step_matches_oracle(lib, gpu, scheme, case):
     """One whole Alg. 3 step on the perturbed-linear route (SubZeroPlus.run_step_linear):
     every loss comes from zo_linear_perturbed outputs while W stays as it is; each
     evaluation's Y matches the oracle's layer, element by element, at the point the scheme
@@ -204,8 +227,8 @@ def test_linear_route_step_matches_oracle(lib, gpu, scheme):
     moments at the oracle's single update from the losses."""
     from gpu_util import oracle_step
     from parity import assert_moments, assert_weights, gabs
-    z, base = _context(gpu, "r32", seed=777)
-    r, spec, _ = LINEAR_CASES["r32"]
+    z, base = _context(gpu, case, seed=777)
+    r, spec, _ = LINEAR_CASES[case]
     eps, lr, b1, b2, ea, t = 0.5, 1e-3, 0.9, 0.95, 1e-8, 3
     T = 48
     X = [_tokens(T, n, 100 + i, gpu) for i, (m, n, _) in enumerate(spec)]
