@@ -1088,13 +1088,20 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     g_last_error = "zo_linear_perturbed: the single-CTA tilings 1..3 take r in {16, 32}";
     return ZO_ERR_UNSUPPORTED;
   }
-  // S's K split: the single-CTA route's S kernel, or the pair launch's S tiles; each writes
-  // k_split x T x r fp32 partials
+  // S's K split: the single-CTA route's S kernel, or the pair launch's plan (contributor
+  // tiles, or S tiles); each split writes k_split x T x r fp32 partials
   int32_t k_split = 1, k_chunk = 1;
-  if (pair_n > 0)
-    zo::linear_pair_s_split(T, n, c->linear_pairs, &k_split, &k_chunk);
-  else
+  zo::LinearPairPlan plan{};
+  if (pair_n > 0) {
+    plan = zo::linear_pair_plan(T, m, n, r, tiling, c->linear_pairs);
+    if (plan.pairs <= 0) {
+      g_last_error = "zo_linear_perturbed: no SM-pair plan for this shape";
+      return ZO_ERR_UNSUPPORTED;
+    }
+    k_split = std::max<int32_t>(1, plan.s_split);
+  } else {
     zo::linear_s_split(T, n, c->sms, &k_split, &k_chunk);
+  }
   const int64_t part = (int64_t)k_split * T * r;
   if (T > c->s_cap || part > c->part_cap) {
     ZO_CUDA(cudaStreamSynchronize(c->stream), "stream synchronize");
@@ -1130,7 +1137,7 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     }
   }
   const bool narrow_y = pair_n == 0 && zo::linear_y_tile_cols(tiling) % 64 != 0;
-  CUtensorMap tm_x{}, tm_pk{}, tm_s{}, tm_y{}, tm_w{}, tm_u{}, tm_pk_half{};
+  CUtensorMap tm_x{}, tm_pk{}, tm_s{}, tm_y{}, tm_w{}, tm_u{}, tm_pk_half{}, tm_ps{};
   bool enc =
       encode_bf16_2d(&tm_x, const_cast<void*>(X), n, T, ldx * 2, 64, 128) &&
       encode_bf16_2d(&tm_pk, c->d_pk + c->h_pk_off[mat], n, 2 * r, (n + 63) / 64 * 64 * 2, 64,
@@ -1142,9 +1149,12 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     enc = enc && encode_bf16_2d(&tm_w, md.W, n, m, md.ldw * 2, 64, (uint32_t)(pair_n / 2)) &&
           encode_bf16_2d(&tm_u, c->d_u_lin, HLW, c->u_rows, HLW * 2, 64, (uint32_t)(pair_n / 2)) &&
           encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 16, 32, CU_TENSOR_MAP_SWIZZLE_32B) &&
-          // P_K in boxes of r rows: CTA 0 of a pair loads P_hi, CTA 1 P_lo
+          // P_K in boxes of r rows: CTA 0 of a pair loads P_hi, CTA 1 P_lo; and in boxes of a
+          // contributor's slice rows
           encode_bf16_2d(&tm_pk_half, c->d_pk + c->h_pk_off[mat], n, 2 * r, (n + 63) / 64 * 64 * 2,
-                         64, (uint32_t)r);
+                         64, (uint32_t)r) &&
+          encode_bf16_2d(&tm_ps, c->d_pk + c->h_pk_off[mat], n, 2 * r, (n + 63) / 64 * 64 * 2,
+                         64, (uint32_t)(plan.n_contrib > 0 ? plan.s_cols / 2 : r));
   } else {
     enc = enc && (narrow_y ? encode_bf16_2d(&tm_y, Y, m, T, ldy * 2, 32, 32,
                                             CU_TENSOR_MAP_SWIZZLE_64B)
@@ -1155,7 +1165,7 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     return ZO_ERR_CUDA;
   }
   if (pair_n > 0) {
-    // one launch: S = X P^T in its S tiles (one per 256 rows), then Y = X W^T + S U^T
+    // one launch: S = X P^T (in contributor tiles or S tiles) and Y = X W^T + S U^T
     if (c->lin_epoch + 1 >= zo::kLinearPairEpochs) {
       // the epochs start again: no counter may hold an old call's complete count
       ZO_CUDA(cudaMemsetAsync(c->d_s_flags, 0,
@@ -1167,10 +1177,9 @@ zo_status zo_linear_perturbed(zo_ctx* c, int32_t mat, const void* X, int64_t T, 
     ++c->lin_epoch;
     const bool inject = c->inject_wait;    // the test hook is one-shot
     c->inject_wait = false;
-    ZO_CUDA(zo::launch_linear_pair(tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk_half, T, m, n,
-                                   c->h_tc[mat].u_row0, r, tiling, c->linear_pairs, c->d_s_hl,
-                                   c->d_s_part, c->d_s_flags, c->lin_epoch, inject, c->d_status,
-                                   c->stream),
+    ZO_CUDA(zo::launch_linear_pair(tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk_half, tm_ps, T, m, n,
+                                   c->h_tc[mat].u_row0, r, tiling, plan, c->d_s_hl, c->d_s_part,
+                                   c->d_s_flags, c->lin_epoch, inject, c->d_status, c->stream),
             "perturbed linear kernel (SM pairs)");
     c->launches += 1;
   } else {

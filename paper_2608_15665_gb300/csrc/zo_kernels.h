@@ -206,32 +206,42 @@ cudaError_t launch_linear_y(const CUtensorMap& tm_x, const CUtensorMap* d_w_map,
 constexpr int32_t kLinearPairTiling0 = 4;
 int32_t linear_pair_cols(int32_t tiling);        // N of a pair tiling, 0 for the others
 int32_t linear_pair_max_pairs();                 // co-resident clusters (0 if unknown)
-// The S tiles' split of K = n into s_split ranges of s_chunk 64-element panels (about one S
-// tile per pair, at most 15 ranges; the same for every pair tiling).
-void linear_pair_s_split(int64_t T, int64_t n, int32_t n_pairs, int32_t* s_split,
-                         int32_t* s_chunk);
-// The pair tiling whose busiest pair has the least work (S and Y tiles dealt round-robin).
+// How one call computes S = X P^T and walks its tiles: n_contrib > 0 -- the first n_contrib
+// Y tiles (column blocks) of each row block also compute s_cols / 2 of S's columns each
+// (r <= 64, where the accumulator has spare columns); else s_split S tiles per row block
+// over K ranges of s_chunk 64-element panels (one range at r <= 64, about one S tile per
+// pair at r = 128; at most 15).  pairs: clusters launched; group: column blocks per stripe
+// of the tile order.  pairs = 0: no plan (bad arguments).
+struct LinearPairPlan {
+  int32_t pairs, group, n_contrib, s_cols, s_split, s_chunk;
+};
+LinearPairPlan linear_pair_plan(int64_t T, int64_t m, int64_t n, int32_t r, int32_t tiling,
+                                int32_t n_pairs);
+// The pair tiling whose busiest pair has the least work (tiles dealt round-robin).
 int32_t linear_pair_tiling(int64_t T, int64_t m, int64_t n, int32_t r, int32_t n_pairs);
-// One launch computes S = X P^T (S tiles, written to s_hl as S_HL rows of tc_hl_width(r))
-// and Y = X W^T + S U^T, r in {16, 32, 64, 128}.  tm_x over X (box 64 x 128), tm_w over
-// W_i (box 64 x N/2), tm_s over s_hl (box 64 x 128), tm_u over the bf16 U operand (box
-// 64 x N/2; W_i's rows from u_row0), tm_y over
-// Y (box 16 x 32, 32-byte swizzle), tm_pk over P_K (box 64 x r).  s_part: s_split x T x r
-// floats (linear_pair_s_split).  s_count: kLinearPairCounters counters per 256 rows of X
-// (zero before the first call), epoch: 1 .. kLinearPairEpochs - 1, a new one per call (the
-// counters of a launch cut short by a wait timeout must be zeroed before the epochs start
-// again).  inject_wait (test hook): the Y tiles wait for a count that
-// never comes, with the short test limit; the launch then reports kDevTimeout.
+// One launch computes S (written to s_hl as S_HL rows of tc_hl_width(r)) and Y = X W^T +
+// S U^T, r in {16, 32, 64, 128}, as plan (linear_pair_plan) says.  tm_x over X (box
+// 64 x 128), tm_w over W_i (box 64 x N/2), tm_s over s_hl (box 64 x 128), tm_u over the
+// bf16 U operand (box 64 x N/2; W_i's rows from u_row0), tm_y over Y (box 16 x 32, 32-byte
+// swizzle), tm_pk over P_K (box 64 x r), tm_ps over P_K (box 64 x s_cols / 2; any box when
+// n_contrib = 0).  s_part: s_split x T x r floats (s_split > 1).  s_count:
+// kLinearPairCounters counters per 256 rows of X (zero before the first call), epoch:
+// 1 .. kLinearPairEpochs - 1, a new one per call (the counters of a launch cut short by a
+// wait timeout must be zeroed before the epochs start again).  inject_wait (test hook):
+// the Y tiles wait for a count that never comes, with the short test limit; the launch
+// then reports kDevTimeout.
 cudaError_t launch_linear_pair(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
                                const CUtensorMap& tm_s, const CUtensorMap& tm_u,
-                               const CUtensorMap& tm_y, const CUtensorMap& tm_pk, int64_t T,
-                               int64_t m, int64_t n, int32_t u_row0, int32_t r, int32_t tiling,
-                               int32_t n_pairs, __nv_bfloat16* s_hl, float* s_part,
+                               const CUtensorMap& tm_y, const CUtensorMap& tm_pk,
+                               const CUtensorMap& tm_ps, int64_t T, int64_t m, int64_t n,
+                               int32_t u_row0, int32_t r, int32_t tiling,
+                               const LinearPairPlan& plan, __nv_bfloat16* s_hl, float* s_part,
                                uint32_t* s_count, uint32_t epoch, bool inject_wait,
                                uint32_t* d_status, cudaStream_t s);
 constexpr uint32_t kLinearPairCountsPerCall = 8;   // 32-row groups of a 256-row block
-constexpr int32_t kLinearPairCounters = 16;        // counters per 256-row block
-constexpr uint32_t kLinearPairEpochs = 1u << 28;
+                                                   // (S_HL writes per S slice)
+constexpr int32_t kLinearPairCounters = 40;        // flags and counters per 256-row block
+constexpr uint32_t kLinearPairEpochs = 1u << 26;
 
 // ---- refresh of tall panels at r = 16 ... 128: CholeskyQR2 (zo_cholqr.cu) ----------
 constexpr int32_t kCqChunkRows = 1024;   // rows per partial Gram matrix
