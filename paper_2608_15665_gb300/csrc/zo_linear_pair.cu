@@ -6,9 +6,10 @@
 // holds rows 128 c .. 128 c + 127 of the tile (its half of the A operand, its accumulator
 // lanes) and rows N/2 c .. N/2 c + N/2 - 1 of the B operand (W rows, then U operand rows);
 // the leader's MMAs read both halves of B.  Each SM then stages 128 x 64 + N/2 x 64 bf16
-// per K step for 128 x N x 64 multiply-adds, and holds a 128 x N fp32 accumulator -- two
-// of them fit its Tensor Memory (N <= 256), so a tile's epilogue runs while the MMAs of
-// the pair's next tile accumulate into the other one.
+// per 64 elements of K for 128 x N x 64 multiply-adds (two such panels per operand stage,
+// three stages), and holds a 128 x N fp32 accumulator -- two of them fit its Tensor Memory
+// (N <= 256), so a tile's epilogue runs while the MMAs of the pair's next tile accumulate
+// into the other one.
 //
 // K steps: n / 64 steps of X and W (single bf16 products, both operands exact in bf16),
 // then the rank-r term from S_HL = [S_hi | S_lo | 0] (A) and the U operand
@@ -17,9 +18,10 @@
 // the same order, as the single-CTA kernels of zo_linear.cu, so each 128-row half of a
 // pair tile gets the bits those kernels give; r = 64 takes one stage of two panels (hi,
 // lo), r = 128 three stages of two panels (S_hi U_hi, S_hi U_lo, S_lo U_hi).
-// N (a multiple of 16, 128 .. 256) is chosen by the host so that the tiles fill whole
-// waves of the resident pairs (224 for 4096 columns at 4096 tokens: 19 x 16 = 304 tiles =
-// 4 waves of 76 pairs; 240 for 11008 columns).
+// S = X P^T comes from S tiles or from contributor tiles in the same launch (see the
+// kernel's comment), its rows published through per-writer ready flags.  N (256, 240,
+// 224, 192 or 128) is chosen by the host by simulating the launch's schedule
+// (linear_pair_tiling).
 //
 // Roles (320 threads per CTA, one CTA per SM):
 //   warp 0, lane 0: TMA producer of this CTA's halves, kStages stages; both halves of a
@@ -30,9 +32,10 @@
 //   warps 2..9:     epilogue of this CTA's 128 rows: warp w reads TMEM lanes 32 (w % 4) ..
 //                   + 31, every other 16-column chunk, rounds to bf16 and stores 32 x 16
 //                   boxes of Y (32-byte swizzle) by TMA.
-// Barriers: in each CTA empty[s] and acc_full[a] (arrived in both CTAs by the leader's
-// multicast commits); in the leader full[s] (bytes of both halves) and acc_empty[a] (the
-// sixteen epilogue warps of the pair, the peer's through its shared::cluster address).
+// Barriers: in each CTA empty[s], acc_full[a] and s_full[a] (a contributor's S columns;
+// arrived in both CTAs by the leader's multicast commits); in the leader full[s] (bytes
+// of both halves) and acc_empty[a] (the sixteen epilogue warps of the pair, the peer's
+// through its shared::cluster address).
 // Every wait is bounded; a give-up sets the abort flag of both CTAs and kDevTimeout in
 // the status word, the producers wait (bounded) for the leader's release of every stage
 // they filled, the MMA thread for its last MMAs, and TMEM is freed after a cluster barrier.
