@@ -379,6 +379,12 @@ linear_pair_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_consta
   cluster_sync_all();                         // both CTAs' barriers and TMEM exist
   tc_fence_after();
   const uint32_t tmem = sh.tmem_base;
+  // launched as a programmatic dependent of the stream's previous kernel: the prologue
+  // above overlaps that kernel's tail; everything below reads or writes memory it may use
+  // (X, S_HL, the flags, Y), so wait for its completion.  Then let the stream's next
+  // kernel be scheduled as SMs free up (it waits the same way).
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------ TMA producer (each CTA)
@@ -759,10 +765,25 @@ cudaError_t launch_pair_nr(const CUtensorMap& tm_x, const CUtensorMap& tm_w,
   cudaError_t e = cudaFuncSetAttribute(linear_pair_kernel<N, R>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::kSmem);
   if (e != cudaSuccess) return e;
-  linear_pair_kernel<N, R><<<2 * plan.pairs, Cfg::kThreads, Cfg::kSmem, s>>>(
-      tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk, tm_ps, rows, cols, k_steps, u_row0, plan.group,
-      plan.s_split, plan.s_chunk, plan.n_contrib, plan.s_cols, s_hl, s_part, s_count, epoch,
-      inject_wait ? epoch + 1 : epoch, d_status, inject_wait ? kTestWaitCycles : kWaitCycles);
+  // a programmatic dependent launch: the kernel's prologue may start before the stream's
+  // previous kernel ends (the kernel waits for it before touching memory)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * plan.pairs, 1, 1);
+  cfg.blockDim = dim3(Cfg::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const uint32_t wait_epoch = inject_wait ? epoch + 1 : epoch;
+  const long long wait_limit = inject_wait ? kTestWaitCycles : kWaitCycles;
+  e = cudaLaunchKernelEx(&cfg, linear_pair_kernel<N, R>, tm_x, tm_w, tm_s, tm_u, tm_y, tm_pk,
+                         tm_ps, rows, cols, k_steps, u_row0, (int)plan.group, (int)plan.s_split,
+                         (int)plan.s_chunk, (int)plan.n_contrib, (int)plan.s_cols, s_hl, s_part,
+                         s_count, epoch, wait_epoch, d_status, wait_limit);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
