@@ -154,6 +154,37 @@ def test_perturbed_linear_single_query_and_repeat(lib, gpu):
     z.close()
 
 
+def test_perturbed_linear_back_to_back_calls_read_each_others_output(lib, gpu):
+    """Two calls on the context's stream with no synchronisation between them, the second
+    reading the first's Y as its X: each pair launch starts as a programmatic dependent of
+    the stream's previous kernel and must wait for it before touching memory.  Y1 starts
+    as NaN, so a second launch that read it early would not match the oracle."""
+    from paper_2608_15665_gb300 import binding as zb
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    base = 5
+    w = [make_weight(520, 520, "bf16", 910, gpu)]
+    z = SubZeroPlus(w, 32, 4, 77, matrix_index_base=base)
+    z.init_subspace(0)
+    zb.zo_linear_prepare(z.ctx, 2, 3, 1.0, -1, 0.0, 1e-2)
+    before = snapshot(z)
+    C = subzero.perturb_coeff(z.seed, base, 2, 32, [(3, 1.0)], f32(1e-2))
+    X = _tokens(600, 520, 8, gpu)
+    Y1 = torch.full((600, 520), float("nan"), dtype=torch.bfloat16, device=gpu)
+    Y2 = torch.empty_like(Y1)
+    torch.cuda.synchronize()
+    for _ in range(3):
+        zb.zo_linear_perturbed(z.ctx, 0, X, Y1)
+        zb.zo_linear_perturbed(z.ctx, 0, Y1, Y2)
+        z.sync()
+        assert torch.isfinite(Y2.float()).all()
+        _check(Y1, X, before["W"][0], before["U"][0], before["V"][0], C, 2.0 * f32(1e-2), "first")
+        _check(Y2, Y1, before["W"][0], before["U"][0], before["V"][0], C, 2.0 * f32(1e-2),
+               "second, reading the first's output")
+        Y1.fill_(float("nan"))
+        torch.cuda.synchronize()
+    z.close()
+
+
 def test_perturbed_linear_long_token_block(lib, gpu):
     """S = X P^T's three ways to S_HL: 257 and 300 tokens split K over many ranges (a
     separate reduction kernel); 5000 tokens (40 row blocks) over 3 ranges, which the S
