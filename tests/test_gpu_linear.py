@@ -27,10 +27,13 @@ PAIR_TILINGS = (4, 5, 6, 7, 8)
 # (r, [(m, n, ldw)], token counts).  r = 64 and 128 (the paper's rank): the rank-r step in
 # one operand stage of two panels and in three, S tiles with 128 and 256 accumulator
 # columns and one or two K panels per stage; ragged row blocks, column blocks and K panels.
+# S comes from S tiles or from contributor tiles depending on the tiling (every pair tiling
+# must give the same bits); 2000 and 3000 tokens put several row blocks' contributors in
+# one wave of tiles.
 LINEAR_CASES = {
-    "r32": (32, [(304, 520, None), (264, 2048, None), (1032, 72, 80)], (1, 130, 300)),
+    "r32": (32, [(304, 520, None), (264, 2048, None), (1032, 72, 80)], (1, 130, 300, 2000)),
     "r16": (16, [(304, 520, 528), (136, 1000, 1008), (64, 136, None)], (7, 257)),
-    "r64": (64, [(392, 648, None), (136, 2056, 2064)], (5, 300)),
+    "r64": (64, [(392, 648, None), (136, 2056, 2064)], (5, 300, 3000)),
     "r128": (128, [(520, 1032, None), (264, 264, 272)], (3, 513)),
 }
 
