@@ -570,14 +570,16 @@ def run_ours(args):
         # r = 128)
         del weights, z
         torch.cuda.empty_cache()
-        line["secondary"] = {
-            "dense32b_bf16_r64": secondary_weight_pass(dev, local, peak, "dense32b_bf16_r64", 2),
-            "llama7b_bf16_r128_q99": secondary_weight_pass(dev, local, peak,
-                                                           "llama7b_bf16_r128_q99", 1),
-            "perturbed_linear_llama7b_4096tok": secondary_linear(dev, local),
-            "perturbed_linear_llama7b_4096tok_r128": secondary_linear(dev, local,
-                                                                     "llama7b_bf16_r128_q99"),
-        }
+        # (the short linear measurements first: the long weight-pass ones run under the
+        # power cap and leave the clocks lowered for a while; each records its own clocks)
+        sec = {}
+        sec["perturbed_linear_llama7b_4096tok"] = secondary_linear(dev, local)
+        sec["perturbed_linear_llama7b_4096tok_r128"] = secondary_linear(dev, local,
+                                                                        "llama7b_bf16_r128_q99")
+        sec["dense32b_bf16_r64"] = secondary_weight_pass(dev, local, peak, "dense32b_bf16_r64", 2)
+        sec["llama7b_bf16_r128_q99"] = secondary_weight_pass(dev, local, peak,
+                                                             "llama7b_bf16_r128_q99", 1)
+        line["secondary"] = sec
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl0, args.scheme)
     if rank == 0:
