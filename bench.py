@@ -577,6 +577,7 @@ def run_ours(args):
         sec["perturbed_linear_llama7b_4096tok_r128"] = secondary_linear(dev, local,
                                                                         "llama7b_bf16_r128_q99")
         sec["dense32b_bf16_r64"] = secondary_weight_pass(dev, local, peak, "dense32b_bf16_r64", 2)
+        sec["mezo_llama7b_bf16"] = secondary_mezo(dev, local, peak)
         sec["llama7b_bf16_r128_q99"] = secondary_weight_pass(dev, local, peak,
                                                              "llama7b_bf16_r128_q99", 1)
         line["secondary"] = sec
@@ -654,6 +655,62 @@ def secondary_weight_pass(dev, local, peak, name, K):
             "traffic": TRAFFIC_BY_SOURCE.get((kernel_source_hash(wl.r), wl.name)),
             "zo_steps_s": 1e3 / step_ms, "ms_per_step": step_ms, "refresh_ms": refresh_ms,
             "clocks": clk}
+
+
+def secondary_mezo(dev, local, peak, K=3):
+    """MeZO's full-space SPSA step (Eq. (1)) on the LLaMA-7B set: three zo_mezo_perturb
+    passes per step (+eps, -2 eps, then +eps fused with the SGD update from the step's loss
+    pair); one warm-up step, then K timed steps with the passes timed by CUDA events.
+    Roofline: bound by instruction issue (thread instructions per weight from the ncu
+    count of the kernel, against 152 SMs x 128 lanes x 2.07 GHz)."""
+    import torch
+    from paper_2608_15665_gb300 import binding as zb
+    from paper_2608_15665_gb300 import workloads
+    from paper_2608_15665_gb300.schedule import SubZeroPlus
+    wl = workloads.get("llama7b_bf16_r32")
+    weights = [workloads.init_weight(wl, i, dev) for i in range(wl.n_mats)]
+    z = SubZeroPlus(weights, wl.r, wl.q, wl.seed)
+    table = workloads.loss_table(wl, "central", steps=1 + K)
+
+    def do_step(t):
+        rho = (float(table[t][0]) - float(table[t][1])) / (2.0 * wl.eps)
+        z.mezo_perturb(t, wl.eps)
+        z.mezo_perturb(t, -2.0 * wl.eps)
+        z.mezo_perturb(t, wl.eps - wl.lr * rho)
+
+    do_step(0)
+    z.sync()
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_TIMING, 1)
+    clocks = ClockSampler(local)
+    clocks.start()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for t in range(1, 1 + K):
+        do_step(t)
+    e1.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    window_ms = e0.elapsed_time(e1)
+    pass_ms, n = zb.zo_get_timing(z.ctx)
+    zb.zo_set_option(z.ctx, zb.ZO_OPTION_TIMING, 0)
+    z.sync()
+    z.close()
+    del weights, z
+    torch.cuda.empty_cache()
+    avg_s = (pass_ms / n) / 1e3
+    ipw = INSTR_PER_WEIGHT_BY_SOURCE.get(mezo_source_hash())
+    issue_peak = 152 * 128 * 2.07e9 / 1e12
+    ach = ipw * wl.params / avg_s / 1e12 if ipw else None
+    return {"workload": wl.name, "params": wl.params, "passes_per_step": 3, "steps_timed": K,
+            "kernel": "mezo_kernel", "avg_launch_ms": avg_s * 1e3, "launches_timed": n,
+            "mezo_steps_s": 1e3 * K / window_ms, "ms_per_step": window_ms / K,
+            "roofline": {"bound": "alu", "achieved": ach, "peak": issue_peak,
+                         "unit": "T thread-instructions/s",
+                         "frac": ach / issue_peak if ach else None,
+                         "instructions_per_weight": ipw},
+            "weight_gbs": wl.bytes_per_pass() / avg_s / 1e9,
+            "weight_gbs_frac_of_hbm": wl.bytes_per_pass() / avg_s / 1e9 / peak, "clocks": clk}
 
 
 def linear_measure(dev, wl, T, K, W, compare=True, e2e=True):
